@@ -1,0 +1,223 @@
+/* libabcd -- GB300 (sm_103a) hot path of ABCD, Alpha-Composited Block Coordinate Descent.
+ *
+ * ABCD trains one spatial block of 3D Gaussians at a time (Section 2).  The frozen blocks
+ * that lie in front of / behind the active partition, seen from a camera, are collapsed by
+ * associativity of alpha compositing into two premultiplied RGBA images F and B; every
+ * training step renders only the active block A and composites F over A over B, evaluates
+ * the reconstruction loss and backpropagates into the active block only.  The renderer is
+ * 3D Gaussian Splatting (Section 1, last paragraph).
+ *
+ * Conventions for every call:
+ *  - Tensor arguments are DEVICE pointers owned by the caller, fp32 unless stated, C order.
+ *  - Struct arguments (camera, options, pointer bundles) are HOST structs read during the
+ *    call; nothing keeps a reference to them after it returns.
+ *  - Every compute call is asynchronous on the context's CUDA stream and returns a status.
+ *    Argument errors are reported before anything is launched (ABCD_ERR_INVALID_ARG).
+ *    Errors found on the device (tile-list capacity, bounds) are OR-ed into a device status
+ *    word that abcd_sync() reads.  No call allocates device memory, synchronizes the
+ *    device, throws, traps or exits; scratch comes from the caller's workspace.
+ *  - The library never touches parameters outside the active block it is given.
+ */
+#ifndef ABCD_H
+#define ABCD_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ABCD_OK = 0,
+  ABCD_ERR_INVALID_ARG = 1,   /* bad pointer / size / option; nothing launched */
+  ABCD_ERR_CUDA = 2,          /* a CUDA runtime call or launch failed (see abcd_last_error) */
+  ABCD_ERR_CAPACITY = 3,      /* device: tile pairs K exceeded abcd_tiles.capacity */
+  ABCD_ERR_TIMEOUT = 4,       /* device: a bounded wait gave up (reserved) */
+  ABCD_ERR_WORKSPACE = 5      /* workspace missing or smaller than abcd_workspace_size() */
+} abcd_status;
+
+typedef struct abcd_ctx abcd_ctx;
+
+/* Pinhole camera: x_cam = R * x_world + t (R row-major), x right, y down, z forward;
+ * pixel (i, j) covers [i, i+1) x [j, j+1), so its centre is (i + 0.5, j + 0.5) and a camera
+ * point projects to (fx x/z + cx, fy y/z + cy). */
+typedef struct {
+  float R[9];
+  float t[3];
+  float fx, fy, cx, cy;
+  int width, height;
+} abcd_camera;
+
+/* Renderer constants of 3D Gaussian Splatting.  Pass NULL for the defaults in brackets. */
+typedef struct {
+  float near_z;     /* cull Gaussians with camera depth <= near_z [0.2] */
+  float dilation;   /* added to the diagonal of the 2-D covariance [0.3] */
+  float guard;      /* Jacobian uses x/z, y/z clamped to guard * tan(fov/2) [1.3] */
+  float alpha_max;  /* alpha = min(alpha_max, o exp(-sigma)) [0.99] */
+  float alpha_min;  /* contributions with alpha < alpha_min are skipped [1/255] */
+  float t_min;      /* a pixel stops before a Gaussian that would take T below t_min [1e-4] */
+} abcd_render_opts;
+
+/* Parameters of the active block (SoA, device).  Shapes: means [n][3], log_scales [n][3],
+ * quats [n][4] as (w, x, y, z), not necessarily unit, opacity_logits [n],
+ * sh [n][D][3] with D = (sh_degree + 1)^2 and coefficient index l*l + l + m (real SH,
+ * Condon-Shortley phase).  The same struct carries gradients and Adam moments. */
+typedef struct {
+  float* means;
+  float* log_scales;
+  float* quats;
+  float* opacity_logits;
+  float* sh;
+  int n;
+  int sh_degree;    /* 0..3 */
+} abcd_gaussians;
+
+/* Output of abcd_project (device, length n each).  A Gaussian is visible iff radius > 0. */
+typedef struct {
+  float* uv;             /* [n][2] pixel-space mean */
+  float* conic_opacity;  /* [n][4] (a, b, c, opacity): inverse 2-D covariance [[a,b],[b,c]] */
+  float* rgb;            /* [n][3] view-dependent colour, clamped at 0 */
+  float* depth;          /* [n] camera-space depth (sort key) */
+  int* radius;           /* [n] ceil(3 sqrt(lambda_max)) in pixels, 0 = culled */
+  unsigned* tiles_touched; /* [n] 16x16 tiles met by the square of half-side radius */
+} abcd_projected;
+
+/* Per-tile Gaussian lists (device).  For tile t = ty * tiles_x + tx (16x16 tiles,
+ * tiles_x = ceil(W/16)), ids[ranges[2t] .. ranges[2t+1]) are the Gaussians whose square
+ * meets the tile, front to back by (fp32 depth, id). */
+typedef struct {
+  unsigned* ids;         /* [capacity] */
+  unsigned* ranges;      /* [tiles_x * tiles_y][2] */
+  long long capacity;    /* entries available in ids (<= the workspace's max_pairs) */
+  long long* count;      /* device scalar: K, the number of (tile, Gaussian) pairs.  If
+                            K > capacity, ABCD_ERR_CAPACITY is raised, ranges are all empty
+                            and *count still holds the required K. */
+} abcd_tiles;
+
+/* Per-pixel state saved by the forward pass for the backward pass (device). */
+typedef struct {
+  float* A_T;            /* [H][W][4]: active premultiplied rgb and its final transmittance */
+  unsigned* n_last;      /* [H][W]: list positions walked up to the last contributor */
+} abcd_fwd_state;
+
+enum { ABCD_F16 = 0, ABCD_F32 = 1 };   /* element type of F, B and cached layers */
+
+/* ---- context, stream, workspace ------------------------------------------------------ */
+abcd_status abcd_create(abcd_ctx** ctx, int device, void* cuda_stream);
+abcd_status abcd_destroy(abcd_ctx* ctx);
+abcd_status abcd_set_stream(abcd_ctx* ctx, void* cuda_stream);
+/* Bytes of device scratch for blocks of up to max_gaussians, up to max_pairs tile pairs
+ * and images of up to max_pixels pixels. */
+abcd_status abcd_workspace_size(int max_gaussians, long long max_pairs, long long max_pixels,
+                                size_t* bytes);
+/* Hands the context a caller-owned device buffer (>= abcd_workspace_size bytes, 256-byte
+ * aligned).  Clears the device status word (asynchronously, on the context's stream). */
+abcd_status abcd_set_workspace(abcd_ctx* ctx, void* device_ptr, size_t bytes,
+                               int max_gaussians, long long max_pairs, long long max_pixels);
+/* Waits for the stream, then returns the first device-detected error (sticky) or ABCD_OK. */
+abcd_status abcd_sync(abcd_ctx* ctx);
+abcd_status abcd_clear_status(abcd_ctx* ctx);
+const char* abcd_last_error(const abcd_ctx* ctx);
+/* Number of kernels this context has launched since creation (instrumentation). */
+long long abcd_launch_count(const abcd_ctx* ctx);
+
+/* ---- the hot path (Section 2: one step renders only the active block) ----------------- */
+
+/* K2. EWA projection of the active block for one camera (3DGS): camera-space mean, world
+ * covariance R(q) diag(exp(2 log_scale)) R(q)^T, 2-D covariance J W Sigma W^T J^T +
+ * dilation*I, its inverse, the 3-sigma radius, SH colour + 0.5 clamped at 0 and
+ * opacity = sigmoid(logit).  Writes every field of out. */
+abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_camera* cam,
+                         const abcd_render_opts* opts, abcd_projected* out);
+
+/* K3 + K4. Tile binning and depth sort: every visible Gaussian is listed in each tile its
+ * square [u-r, u+r] x [v-r, v+r] meets; lists are ordered by the fp32 depth, ties by id.
+ * n must equal the n given to abcd_project. */
+abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, int n,
+                          const abcd_camera* cam, abcd_tiles* out);
+
+/* K5. Front-to-back blend of the active block per pixel (alpha = min(alpha_max,
+ * o exp(-sigma)), skip alpha < alpha_min, stop before T < t_min), giving the premultiplied
+ * A = (sum T_i alpha_i c_i, 1 - T_final); then out = F over (A over B), over meaning
+ * X + (1 - X.a) Y on premultiplied RGBA, and out.rgb += (1 - out.a) * bg.
+ * F, B: [H][W][4] of fb_dtype, or NULL for transparent.  bg: 3 host floats or NULL (0).
+ * out_rgba: [H][W][4] fp32 (may be NULL).  state: may be NULL (no backward).
+ * refresh_f16: optional [H][W][4] fp16 receiving A alone (the cache refresh of Section 2). */
+abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camera* cam,
+                                      const abcd_render_opts* opts, const abcd_projected* proj,
+                                      const abcd_tiles* tiles, const void* F, const void* B,
+                                      int fb_dtype, const float* bg, float* out_rgba,
+                                      abcd_fwd_state* state, void* refresh_f16);
+
+/* K6. Reconstruction loss (1 - lambda) mean|x - y| + lambda (1 - mean SSIM(x, y)) over the
+ * rgb of out_rgba [H][W][4] against gt_rgb [H][W][3]; SSIM with an 11x11 Gaussian window
+ * (sigma 1.5), zero padding, C1 = 0.01^2, C2 = 0.03^2.  loss_out: device float scalar.
+ * dL_dout: [H][W][3] receives dL/d(out.rgb). */
+abcd_status abcd_loss(abcd_ctx* ctx, const float* out_rgba, const float* gt_rgb, int width,
+                      int height, float lambda_ssim, float* loss_out, float* dL_dout);
+
+/* K7. Backward of the blend + composite for one image: given dL/d(final rgb) [H][W][3],
+ * writes grad2d [n][9] = dL/d(u, v, a, b, c, opacity, r, g, b) per Gaussian (overwritten).
+ * The alpha of the active layer also receives -(1 - F.a) <g, B.rgb + (1 - B.a) bg>. */
+abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* cam,
+                                 const abcd_render_opts* opts, const abcd_projected* proj,
+                                 const abcd_tiles* tiles, const void* F, const void* B,
+                                 int fb_dtype, const float* bg, const abcd_fwd_state* state,
+                                 const float* dL_dout, int n, float* grad2d);
+
+/* K8. Chain rule from grad2d [n][9] to the parameters of theta (overwrites grads; culled
+ * Gaussians get 0). */
+abcd_status abcd_project_backward(abcd_ctx* ctx, const abcd_gaussians* theta,
+                                  const abcd_camera* cam, const abcd_render_opts* opts,
+                                  const float* grad2d, abcd_gaussians* grads);
+
+/* K6 + K7 + K8: the backward pass of one step into the active block only.  With gt_rgb,
+ * evaluates the loss into loss_out and uses its gradient; with gt_rgb == NULL, dL_dout is
+ * the given upstream gradient.  grad2d and dL/dout live in the workspace. */
+abcd_status abcd_backward(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_camera* cam,
+                          const abcd_render_opts* opts, const abcd_projected* proj,
+                          const abcd_tiles* tiles, const void* F, const void* B, int fb_dtype,
+                          const float* bg, const float* out_rgba, const abcd_fwd_state* state,
+                          const float* gt_rgb, float lambda_ssim, float* loss_out,
+                          const float* dL_dout, abcd_gaussians* grads);
+
+/* K9. Adam with bias correction (torch semantics), dense over the active block only:
+ * m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2; theta -= lr m/(1-b1^t) / (sqrt(v/(1-b2^t)) + eps).
+ * lr[6] per group: means, log_scales, quats, opacity_logits, sh degree 0, sh degree >= 1.
+ * step is 1-based. */
+abcd_status abcd_adam_active(abcd_ctx* ctx, abcd_gaussians* theta, const abcd_gaussians* grads,
+                             abcd_gaussians* m, abcd_gaussians* v, const float lr[6],
+                             float beta1, float beta2, float eps, int step);
+
+/* K1. Depth-ordered over-compositing of cached per-partition renders (Section 2: "cached
+ * renders from frozen partitions are composited into F and B according to depth
+ * ordering").  layers: host array of L device pointers to [H][W][4] premultiplied RGBA of
+ * layer_dtype; order: host array of L indices, front to back; split: position in order of
+ * the active partition (its layer is skipped and may be NULL), or L for "all in front".
+ * F_out = fold over order[0 .. split), B_out = fold over order[split+1 .. L), each a left
+ * fold of X over Y from transparent, accumulated in fp32 and rounded once to out_dtype.
+ * L <= 256.  Either output may be NULL. */
+abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* layers, int L,
+                                 int layer_dtype, const int* order, int split, int width,
+                                 int height, void* F_out, void* B_out, int out_dtype);
+
+/* ---- host-side partition logic (Section 2: regular grid, assignment by mean) --------- */
+
+/* cell[i] = linear id (i + gx (j + gy k)) of the grid cell holding means[i] (host array,
+ * [n][3] float), clamped into the grid. */
+abcd_status abcd_assign_cells(const float* means_host, int n, const double origin[3],
+                              double side, const int dims[3], int* cell);
+
+/* Front-to-back order of the frozen partitions seen from campos and the split at the active
+ * partition.  A cell's key is its Manhattan distance (in cells) from the camera's cell (not
+ * clamped into the grid); along any ray the key grows strictly from cell to cell, so every
+ * cell with a smaller key than the active one that shares a ray with it lies in front.
+ * front/back: capacity for gx*gy*gz entries; ascending (key, id); equal keys go behind. */
+abcd_status abcd_partition_split(const int dims[3], const double origin[3], double side,
+                                 const double campos[3], int active, int* front, int* n_front,
+                                 int* back, int* n_back);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

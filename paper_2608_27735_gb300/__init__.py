@@ -1,5 +1,416 @@
 """GB300-native (sm_103a) ABCD active-block hot path.
 
-The compute lives in ``libabcd.so`` (hand-written CUDA behind a C ABI, declared in
-``include/abcd.h``); this package is a thin ctypes binding with the same names.
+The compute lives in ``libabcd.so`` (hand-written CUDA behind the C ABI declared in
+``include/abcd.h``).  This module is the thin binding: ctypes structures mirroring the
+header, functions with the same names (argument marshalling only), and small containers
+that allocate the caller-owned device buffers with torch.  There is no CPU fallback: if the
+library is missing or no GPU is present, every call raises.
 """
+from __future__ import annotations
+
+import ctypes as C
+import os
+import re
+import threading
+from dataclasses import dataclass
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "libabcd.so")
+HEADER = os.path.join(os.path.dirname(HERE), "include", "abcd.h")
+
+ABCD_OK, ABCD_ERR_INVALID_ARG, ABCD_ERR_CUDA, ABCD_ERR_CAPACITY, ABCD_ERR_TIMEOUT, \
+    ABCD_ERR_WORKSPACE = range(6)
+ABCD_F16, ABCD_F32 = 0, 1
+STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "CUDA", 3: "CAPACITY", 4: "TIMEOUT", 5: "WORKSPACE"}
+TILE = 16
+
+
+class AbcdError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"abcd status {STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+# ---------------------------------------------------------------------------------------
+# ctypes mirrors of include/abcd.h
+
+class abcd_camera(C.Structure):
+    _fields_ = [("R", C.c_float * 9), ("t", C.c_float * 3), ("fx", C.c_float), ("fy", C.c_float),
+                ("cx", C.c_float), ("cy", C.c_float), ("width", C.c_int), ("height", C.c_int)]
+
+
+class abcd_render_opts(C.Structure):
+    _fields_ = [(k, C.c_float) for k in ("near_z", "dilation", "guard", "alpha_max",
+                                         "alpha_min", "t_min")]
+
+
+class abcd_gaussians(C.Structure):
+    _fields_ = [("means", C.c_void_p), ("log_scales", C.c_void_p), ("quats", C.c_void_p),
+                ("opacity_logits", C.c_void_p), ("sh", C.c_void_p), ("n", C.c_int),
+                ("sh_degree", C.c_int)]
+
+
+class abcd_projected(C.Structure):
+    _fields_ = [(k, C.c_void_p) for k in ("uv", "conic_opacity", "rgb", "depth", "radius",
+                                          "tiles_touched")]
+
+
+class abcd_tiles(C.Structure):
+    _fields_ = [("ids", C.c_void_p), ("ranges", C.c_void_p), ("capacity", C.c_longlong),
+                ("count", C.c_void_p)]
+
+
+class abcd_fwd_state(C.Structure):
+    _fields_ = [("A_T", C.c_void_p), ("n_last", C.c_void_p)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+_SIGS = {
+    "abcd_create": [C.POINTER(C.c_void_p), C.c_int, C.c_void_p],
+    "abcd_destroy": [C.c_void_p],
+    "abcd_set_stream": [C.c_void_p, C.c_void_p],
+    "abcd_workspace_size": [C.c_int, C.c_longlong, C.c_longlong, C.POINTER(C.c_size_t)],
+    "abcd_set_workspace": [C.c_void_p, C.c_void_p, C.c_size_t, C.c_int, C.c_longlong, C.c_longlong],
+    "abcd_sync": [C.c_void_p],
+    "abcd_clear_status": [C.c_void_p],
+    "abcd_project": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p],
+    "abcd_bin_sort": [C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p],
+    "abcd_render_composite_fwd": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                  C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p,
+                                  C.c_void_p, C.c_void_p],
+    "abcd_loss": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_float, C.c_void_p,
+                  C.c_void_p],
+    "abcd_render_backward": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                             C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p,
+                             C.c_void_p, C.c_int, C.c_void_p],
+    "abcd_project_backward": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                              C.c_void_p],
+    "abcd_backward": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                      C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p,
+                      C.c_void_p, C.c_float, C.c_void_p, C.c_void_p, C.c_void_p],
+    "abcd_adam_active": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                         C.c_float, C.c_float, C.c_float, C.c_int],
+    "abcd_composite_cache": [C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p, C.c_int,
+                             C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int],
+    "abcd_assign_cells": [C.c_void_p, C.c_int, C.c_void_p, C.c_double, C.c_void_p, C.c_void_p],
+    "abcd_partition_split": [C.c_void_p, C.c_void_p, C.c_double, C.c_void_p, C.c_int,
+                             C.c_void_p, C.POINTER(C.c_int), C.c_void_p, C.POINTER(C.c_int)],
+}
+
+
+def build(force: bool = False) -> str:
+    from . import _build
+    return _build.build(force=force)
+
+
+def lib():
+    """The loaded libabcd.so.  Raises if it has not been built (no fallback)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"libabcd.so is not built ({LIB_PATH}); run "
+                                   "paper_2608_27735_gb300.build() (nvcc, sm_103a)")
+            L = C.CDLL(LIB_PATH)
+            for name, args in _SIGS.items():
+                f = getattr(L, name)
+                f.argtypes = args
+                f.restype = C.c_int
+            L.abcd_last_error.argtypes = [C.c_void_p]
+            L.abcd_last_error.restype = C.c_char_p
+            L.abcd_launch_count.argtypes = [C.c_void_p]
+            L.abcd_launch_count.restype = C.c_longlong
+            _lib = L
+    return _lib
+
+
+def header_functions():
+    """Names of the functions include/abcd.h declares."""
+    txt = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:abcd_status|const char\*|long long)\s+(abcd_\w+)\s*\(",
+                                 txt, flags=re.M)))
+
+
+# ---------------------------------------------------------------------------------------
+# device buffers (torch is the allocator; pointers only cross the ABI)
+
+def _torch():
+    import torch
+    return torch
+
+
+def _p(t):
+    if t is None:
+        return None
+    assert t.is_cuda and t.is_contiguous(), "ABI arguments must be contiguous CUDA tensors"
+    return C.c_void_p(t.data_ptr())
+
+
+@dataclass
+class Gaussians:
+    """Active-block parameters (or gradients / Adam moments) as CUDA float32 tensors."""
+    means: object
+    log_scales: object
+    quats: object
+    opacity_logits: object
+    sh: object
+    sh_degree: int
+
+    @property
+    def n(self):
+        return int(self.means.shape[0])
+
+    def c(self):
+        return abcd_gaussians(_p(self.means), _p(self.log_scales), _p(self.quats),
+                              _p(self.opacity_logits), _p(self.sh), self.n, self.sh_degree)
+
+    def tensors(self):
+        return (self.means, self.log_scales, self.quats, self.opacity_logits, self.sh)
+
+    @classmethod
+    def from_numpy(cls, g, device="cuda"):
+        torch = _torch()
+        f = lambda a: torch.as_tensor(a, dtype=torch.float32).contiguous().to(device)
+        return cls(f(g.means), f(g.log_scales), f(g.quats), f(g.opacity_logits), f(g.sh),
+                   int(g.sh_degree))
+
+    @classmethod
+    def zeros_like(cls, o):
+        torch = _torch()
+        return cls(*(torch.zeros_like(t) for t in o.tensors()), o.sh_degree)
+
+
+@dataclass
+class Projected:
+    uv: object
+    conic_opacity: object
+    rgb: object
+    depth: object
+    radius: object
+    tiles_touched: object
+
+    @classmethod
+    def alloc(cls, n, device="cuda"):
+        torch = _torch()
+        f = lambda *s, dt=torch.float32: torch.empty(*s, dtype=dt, device=device)
+        return cls(f(n, 2), f(n, 4), f(n, 3), f(n), f(n, dt=torch.int32), f(n, dt=torch.int32))
+
+    def c(self):
+        return abcd_projected(_p(self.uv), _p(self.conic_opacity), _p(self.rgb), _p(self.depth),
+                              _p(self.radius), _p(self.tiles_touched))
+
+
+@dataclass
+class Tiles:
+    ids: object
+    ranges: object
+    count: object
+    capacity: int
+
+    @classmethod
+    def alloc(cls, capacity, width, height, device="cuda"):
+        torch = _torch()
+        nt = ((width + TILE - 1) // TILE) * ((height + TILE - 1) // TILE)
+        return cls(torch.empty(max(1, capacity), dtype=torch.int32, device=device),
+                   torch.zeros(nt, 2, dtype=torch.int32, device=device),
+                   torch.zeros(1, dtype=torch.int64, device=device), int(capacity))
+
+    def c(self):
+        return abcd_tiles(_p(self.ids), _p(self.ranges), self.capacity, _p(self.count))
+
+
+@dataclass
+class FwdState:
+    A_T: object
+    n_last: object
+
+    @classmethod
+    def alloc(cls, width, height, device="cuda"):
+        torch = _torch()
+        return cls(torch.empty(height, width, 4, dtype=torch.float32, device=device),
+                   torch.empty(height, width, dtype=torch.int32, device=device))
+
+    def c(self):
+        return abcd_fwd_state(_p(self.A_T), _p(self.n_last))
+
+
+def camera(cam) -> abcd_camera:
+    """abcd_camera from any object with R, t, fx, fy, cx, cy, width, height."""
+    import numpy as np
+    c = abcd_camera()
+    c.R[:] = [float(v) for v in np.asarray(cam.R, dtype=np.float32).reshape(-1)]
+    c.t[:] = [float(v) for v in np.asarray(cam.t, dtype=np.float32).reshape(-1)]
+    c.fx, c.fy, c.cx, c.cy = float(cam.fx), float(cam.fy), float(cam.cx), float(cam.cy)
+    c.width, c.height = int(cam.width), int(cam.height)
+    return c
+
+
+def render_opts(near_z=0.2, dilation=0.3, guard=1.3, alpha_max=0.99, alpha_min=1.0 / 255.0,
+                t_min=1e-4) -> abcd_render_opts:
+    return abcd_render_opts(near_z, dilation, guard, alpha_max, alpha_min, t_min)
+
+
+class Context:
+    """An abcd_ctx bound to a device and a CUDA stream, plus its caller-owned workspace."""
+
+    def __init__(self, device=0, stream=None):
+        torch = _torch()
+        if not torch.cuda.is_available():
+            raise RuntimeError("libabcd needs a CUDA device; there is no CPU fallback")
+        self.device = device
+        self.stream = stream if stream is not None else torch.cuda.current_stream(device)
+        h = C.c_void_p()
+        st = lib().abcd_create(C.byref(h), device, C.c_void_p(self.stream.cuda_stream))
+        if st != ABCD_OK:
+            raise AbcdError(st, "abcd_create failed")
+        self.h = h
+        self.workspace = None
+        self.limits = (0, 0, 0)
+
+    def __del__(self):
+        try:
+            if getattr(self, "h", None):
+                lib().abcd_destroy(self.h)
+                self.h = None
+        except Exception:
+            pass
+
+    def check(self, st):
+        if st != ABCD_OK:
+            raise AbcdError(st, lib().abcd_last_error(self.h).decode(errors="replace"))
+
+    def reserve(self, max_gaussians, max_pairs, max_pixels):
+        """(Re)allocates the workspace if the limits grew."""
+        torch = _torch()
+        mg, mp, mx = (max(a, b) for a, b in zip((max_gaussians, max_pairs, max_pixels), self.limits))
+        if self.workspace is not None and (mg, mp, mx) == self.limits:
+            return
+        nbytes = C.c_size_t()
+        self.check(lib().abcd_workspace_size(mg, mp, mx, C.byref(nbytes)))
+        ws = torch.empty(nbytes.value + 256, dtype=torch.uint8, device=self.device)
+        off = (-ws.data_ptr()) % 256
+        self.workspace = ws
+        self.check(lib().abcd_set_workspace(self.h, C.c_void_p(ws.data_ptr() + off), nbytes.value,
+                                            mg, mp, mx))
+        self.limits = (mg, mp, mx)
+
+    def sync(self):
+        self.check(lib().abcd_sync(self.h))
+
+    def clear_status(self):
+        self.check(lib().abcd_clear_status(self.h))
+
+    def launches(self):
+        return int(lib().abcd_launch_count(self.h))
+
+
+# ---------------------------------------------------------------------------------------
+# the ABI, same names (each raises AbcdError on a non-OK status)
+
+def _opt(o):
+    return None if o is None else C.byref(o)
+
+
+def abcd_project(ctx: Context, theta: Gaussians, cam: abcd_camera, opts, out: Projected):
+    g = theta.c(); o = out.c()
+    ctx.check(lib().abcd_project(ctx.h, C.byref(g), C.byref(cam), _opt(opts), C.byref(o)))
+
+
+def abcd_bin_sort(ctx: Context, proj: Projected, n: int, cam: abcd_camera, out: Tiles):
+    p = proj.c(); t = out.c()
+    ctx.check(lib().abcd_bin_sort(ctx.h, C.byref(p), int(n), C.byref(cam), C.byref(t)))
+
+
+def _bg(bg):
+    if bg is None:
+        return None
+    return (C.c_float * 3)(*[float(v) for v in bg])
+
+
+def abcd_render_composite_fwd(ctx: Context, cam, opts, proj: Projected, tiles: Tiles, F=None,
+                              B=None, fb_dtype=ABCD_F16, bg=None, out_rgba=None,
+                              state: FwdState = None, refresh_f16=None):
+    p = proj.c(); t = tiles.c()
+    s = state.c() if state is not None else None
+    ctx.check(lib().abcd_render_composite_fwd(
+        ctx.h, C.byref(cam), _opt(opts), C.byref(p), C.byref(t), _p(F), _p(B), int(fb_dtype),
+        _bg(bg), _p(out_rgba), C.byref(s) if s is not None else None, _p(refresh_f16)))
+
+
+def abcd_loss(ctx: Context, out_rgba, gt_rgb, width, height, lambda_ssim, loss_out, dL_dout):
+    ctx.check(lib().abcd_loss(ctx.h, _p(out_rgba), _p(gt_rgb), int(width), int(height),
+                              float(lambda_ssim), _p(loss_out), _p(dL_dout)))
+
+
+def abcd_render_backward(ctx: Context, cam, opts, proj: Projected, tiles: Tiles, F, B, fb_dtype,
+                         bg, state: FwdState, dL_dout, n, grad2d):
+    p = proj.c(); t = tiles.c(); s = state.c()
+    ctx.check(lib().abcd_render_backward(ctx.h, C.byref(cam), _opt(opts), C.byref(p), C.byref(t),
+                                         _p(F), _p(B), int(fb_dtype), _bg(bg), C.byref(s),
+                                         _p(dL_dout), int(n), _p(grad2d)))
+
+
+def abcd_project_backward(ctx: Context, theta: Gaussians, cam, opts, grad2d, grads: Gaussians):
+    g = theta.c(); d = grads.c()
+    ctx.check(lib().abcd_project_backward(ctx.h, C.byref(g), C.byref(cam), _opt(opts),
+                                          _p(grad2d), C.byref(d)))
+
+
+def abcd_backward(ctx: Context, theta: Gaussians, cam, opts, proj: Projected, tiles: Tiles, F, B,
+                  fb_dtype, bg, out_rgba, state: FwdState, gt_rgb, lambda_ssim, loss_out,
+                  dL_dout, grads: Gaussians):
+    g = theta.c(); p = proj.c(); t = tiles.c(); s = state.c(); d = grads.c()
+    ctx.check(lib().abcd_backward(ctx.h, C.byref(g), C.byref(cam), _opt(opts), C.byref(p),
+                                  C.byref(t), _p(F), _p(B), int(fb_dtype), _bg(bg), _p(out_rgba),
+                                  C.byref(s), _p(gt_rgb), float(lambda_ssim), _p(loss_out),
+                                  _p(dL_dout), C.byref(d)))
+
+
+def abcd_adam_active(ctx: Context, theta: Gaussians, grads: Gaussians, m: Gaussians, v: Gaussians,
+                     lr, beta1, beta2, eps, step):
+    a, g, mm, vv = theta.c(), grads.c(), m.c(), v.c()
+    lrs = (C.c_float * 6)(*[float(x) for x in lr])
+    ctx.check(lib().abcd_adam_active(ctx.h, C.byref(a), C.byref(g), C.byref(mm), C.byref(vv), lrs,
+                                     float(beta1), float(beta2), float(eps), int(step)))
+
+
+def abcd_composite_cache(ctx: Context, layers, order, split, width, height, F_out, B_out,
+                         layer_dtype=ABCD_F16, out_dtype=ABCD_F16):
+    """layers: list of CUDA tensors (or None at the active position); order: list of ints."""
+    L = len(layers)
+    arr = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in layers])
+    ordr = (C.c_int * max(1, L))(*[int(k) for k in order])
+    ctx.check(lib().abcd_composite_cache(ctx.h, arr, L, int(layer_dtype), ordr, int(split),
+                                         int(width), int(height), _p(F_out), _p(B_out),
+                                         int(out_dtype)))
+
+
+def abcd_assign_cells(means_np, origin, side, dims):
+    import numpy as np
+    m = np.ascontiguousarray(means_np, dtype=np.float32)
+    n = m.shape[0]
+    cell = np.zeros(n, np.int32)
+    o = (C.c_double * 3)(*[float(v) for v in origin])
+    d = (C.c_int * 3)(*[int(v) for v in dims])
+    st = lib().abcd_assign_cells(m.ctypes.data_as(C.c_void_p), n, o, float(side), d,
+                                 cell.ctypes.data_as(C.c_void_p))
+    if st != ABCD_OK:
+        raise AbcdError(st, "abcd_assign_cells")
+    return cell
+
+
+def abcd_partition_split(dims, origin, side, campos, active):
+    import numpy as np
+    total = int(np.prod(dims))
+    front, back = np.zeros(total, np.int32), np.zeros(total, np.int32)
+    nf, nb = C.c_int(), C.c_int()
+    st = lib().abcd_partition_split((C.c_int * 3)(*[int(v) for v in dims]),
+                                    (C.c_double * 3)(*[float(v) for v in origin]), float(side),
+                                    (C.c_double * 3)(*[float(v) for v in campos]), int(active),
+                                    front.ctypes.data_as(C.c_void_p), C.byref(nf),
+                                    back.ctypes.data_as(C.c_void_p), C.byref(nb))
+    if st != ABCD_OK:
+        raise AbcdError(st, "abcd_partition_split")
+    return front[:nf.value].copy(), back[:nb.value].copy()

@@ -1,0 +1,81 @@
+// Internal declarations shared by the libabcd translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/abcd.h"
+
+namespace abcd {
+
+constexpr int kTile = 16;                 // tile edge (pixels)
+constexpr int kTileThreads = kTile * kTile;
+constexpr int kRadixBits = 8;
+constexpr int kRadixBins = 1 << kRadixBits;
+constexpr int kMaxRadixBlocks = 1024;     // upper bound used to size the histogram scratch
+constexpr int kLossTile = 32;             // loss output tile edge
+constexpr int kMaxLossBlocks = 1 << 16;
+constexpr int kMaxLayers = 256;
+
+// Device status bits (OR-ed into the status word; abcd_sync reports the lowest set code).
+constexpr unsigned kStatusCapacity = 1u << ABCD_ERR_CAPACITY;
+constexpr unsigned kStatusTimeout = 1u << ABCD_ERR_TIMEOUT;
+
+struct Cam {               // camera as the kernels read it (by value)
+  float R[9], t[3];
+  float fx, fy, cx, cy;
+  float campos[3];         // -R^T t (host fp64, rounded)
+  float limx, limy;        // guard * tan(fov/2)
+  int width, height, tiles_x, tiles_y;
+};
+
+struct Opts {
+  float near_z, dilation, alpha_max, alpha_min, t_min, guard;
+};
+
+struct SHConst { float k[16]; };    // normalisation factors of the real SH basis
+
+struct Workspace {
+  unsigned* status;                 // [0] status word, [1] loss ticket
+  unsigned long long* dsort[2];     // depth sort items [max_g]
+  unsigned long long* pairs[2];     // (tile << 32 | id) items [max_pairs]
+  unsigned* hist;                   // [kRadixBins][kMaxRadixBlocks]
+  unsigned long long* block_sums;   // [kMaxRadixBlocks + 1]
+  float* grad2d;                    // [max_g][9]
+  float* dl_dout;                   // [max_pixels][3]
+  float* loss_partials;             // [kMaxLossBlocks][2]
+};
+
+}  // namespace abcd
+
+struct abcd_ctx {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  int num_sms = 0;
+  int radix_blocks = 0;
+  char* ws_base = nullptr;
+  size_t ws_bytes = 0;
+  int max_g = 0;
+  long long max_pairs = 0;
+  long long max_pixels = 0;
+  abcd::Workspace ws{};
+  abcd::SHConst sh{};
+  long long launches = 0;
+  char err[512] = {0};
+};
+
+namespace abcd {
+
+abcd_status fail(abcd_ctx* ctx, abcd_status code, const char* fmt, ...);
+abcd_status check_launch(abcd_ctx* ctx, const char* what);
+bool has_workspace(const abcd_ctx* ctx);
+Cam make_cam(const abcd_camera* c, const abcd_render_opts* o);
+Opts make_opts(const abcd_render_opts* o);
+void sh_constants(SHConst* out);
+
+// translation-unit entry points used by the composite calls
+abcd_status loss_launch(abcd_ctx* ctx, const float* out_rgba, const float* gt_rgb, int width,
+                        int height, float lambda_ssim, float* loss_out, float* dL_dout);
+
+}  // namespace abcd

@@ -1,0 +1,166 @@
+// K1: depth-ordered over-compositing of cached per-partition RGBA renders into F and B
+// (Section 2: "cached renders from frozen partitions are composited into F and B according
+// to depth ordering"; by associativity of 'over' the frozen blocks in front of the active
+// partition collapse into F, those behind into B).
+//
+// Pure streaming work: every layer is read once (16-byte streaming loads, evict-first), the
+// accumulator stays in registers across layers, F and B are written once.  Four layers are
+// loaded before they are folded so each thread keeps 64 bytes in flight.  The grid is a
+// multiple of the SM count and strides over pixel pairs.
+#include "abcd_internal.cuh"
+
+namespace abcd {
+namespace {
+
+struct LayerTable {
+  const void* p[kMaxLayers];   // front layers in order, then back layers in order
+};
+
+__device__ __forceinline__ void unpack_h8(uint4 r, float* f) {
+  const unsigned w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float2 v = __half22float2(*reinterpret_cast<const __half2*>(&w[k]));
+    f[2 * k] = v.x;
+    f[2 * k + 1] = v.y;
+  }
+}
+
+__device__ __forceinline__ void unpack_h4(uint2 r, float* f) {
+  const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&r.x));
+  const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&r.y));
+  f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
+}
+
+// acc (premultiplied RGBA x PIX pixels) = acc over layer
+template <int PIX>
+__device__ __forceinline__ void fold(float* acc, const float* L) {
+#pragma unroll
+  for (int q = 0; q < PIX; ++q) {
+    const float k = 1.f - acc[4 * q + 3];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[4 * q + c] = __fmaf_rn(k, L[4 * q + c], acc[4 * q + c]);
+  }
+}
+
+// Loads PIX pixels (4 channels each) of layer `ptr` at pixel group g into f.
+template <int PIX, bool F16>
+__device__ __forceinline__ void load_group(const void* ptr, long long g, float* f) {
+  if (F16) {
+    if (PIX == 2) unpack_h8(__ldcs(reinterpret_cast<const uint4*>(ptr) + g), f);
+    else unpack_h4(__ldcs(reinterpret_cast<const uint2*>(ptr) + g), f);
+  } else {
+#pragma unroll
+    for (int q = 0; q < PIX; ++q) {
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(ptr) + g * PIX + q);
+      f[4 * q] = v.x; f[4 * q + 1] = v.y; f[4 * q + 2] = v.z; f[4 * q + 3] = v.w;
+    }
+  }
+}
+
+template <int PIX, bool F16>
+__device__ __forceinline__ void fold_range(const LayerTable& lt, int k0, int k1, long long g,
+                                           float* acc) {
+  int k = k0;
+  for (; k + 4 <= k1; k += 4) {
+    float v[4][4 * PIX];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) load_group<PIX, F16>(lt.p[k + j], g, v[j]);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) fold<PIX>(acc, v[j]);
+  }
+  for (; k < k1; ++k) {
+    float v[4 * PIX];
+    load_group<PIX, F16>(lt.p[k], g, v);
+    fold<PIX>(acc, v);
+  }
+}
+
+template <int PIX>
+__device__ __forceinline__ void store_group(void* out, int f16, long long g, const float* acc) {
+  if (!out) return;
+  if (f16) {
+    unsigned w[2 * PIX];
+#pragma unroll
+    for (int k = 0; k < 2 * PIX; ++k) {
+      const __half2 h = __floats2half2_rn(acc[2 * k], acc[2 * k + 1]);
+      w[k] = *reinterpret_cast<const unsigned*>(&h);
+    }
+    if (PIX == 2) reinterpret_cast<uint4*>(out)[g] = make_uint4(w[0], w[1], w[2], w[3]);
+    else reinterpret_cast<uint2*>(out)[g] = make_uint2(w[0], w[1]);
+  } else {
+#pragma unroll
+    for (int q = 0; q < PIX; ++q)
+      reinterpret_cast<float4*>(out)[g * PIX + q] =
+          make_float4(acc[4 * q], acc[4 * q + 1], acc[4 * q + 2], acc[4 * q + 3]);
+  }
+}
+
+template <int PIX, bool F16>
+__global__ void __launch_bounds__(256)
+composite_kernel(const __grid_constant__ LayerTable lt, int nf, int nb, long long groups,
+                 void* Fout, void* Bout, int out_f16) {
+  for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < groups;
+       g += (long long)gridDim.x * blockDim.x) {
+    float acc[4 * PIX];
+    if (Fout) {
+#pragma unroll
+      for (int c = 0; c < 4 * PIX; ++c) acc[c] = 0.f;
+      fold_range<PIX, F16>(lt, 0, nf, g, acc);
+      store_group<PIX>(Fout, out_f16, g, acc);
+    }
+    if (Bout) {
+#pragma unroll
+      for (int c = 0; c < 4 * PIX; ++c) acc[c] = 0.f;
+      fold_range<PIX, F16>(lt, nf, nf + nb, g, acc);
+      store_group<PIX>(Bout, out_f16, g, acc);
+    }
+  }
+}
+
+}  // namespace
+}  // namespace abcd
+
+using namespace abcd;
+
+extern "C" abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* layers, int L,
+                                            int layer_dtype, const int* order, int split,
+                                            int width, int height, void* F_out, void* B_out,
+                                            int out_dtype) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (L < 0 || L > kMaxLayers || (L > 0 && (!layers || !order)) || split < 0 || split > L ||
+      width <= 0 || height <= 0)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache: bad layer list, split or size");
+  if ((layer_dtype != ABCD_F16 && layer_dtype != ABCD_F32) || (out_dtype != ABCD_F16 && out_dtype != ABCD_F32))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache: bad dtype");
+  LayerTable lt;
+  int nf = 0, nb = 0;
+  bool al16 = true;
+  for (int k = 0; k < L; ++k) {
+    if (k == split) continue;
+    if (order[k] < 0 || order[k] >= L) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache: order[%d] out of range", k);
+    const void* p = layers[order[k]];
+    if (!p) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache: layer %d is NULL", order[k]);
+    if ((uintptr_t)p & 15) al16 = false;
+    if ((uintptr_t)p & (layer_dtype == ABCD_F16 ? 7 : 15))
+      return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache: layer %d misaligned", order[k]);
+    if (k < split) lt.p[nf++] = p;
+  }
+  for (int k = split + 1; k < L; ++k) lt.p[nf + nb++] = layers[order[k]];
+  const long long npix = (long long)width * height;
+  const uintptr_t oal = out_dtype == ABCD_F16 ? 7 : 15;
+  if (((uintptr_t)F_out & oal) || ((uintptr_t)B_out & oal))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache: misaligned output");
+  if (((uintptr_t)F_out & 15) || ((uintptr_t)B_out & 15)) al16 = false;
+  if (!F_out && !B_out) return ABCD_OK;
+  const int grid = ctx->num_sms * 8;
+  const bool pairs = al16 && (npix % 2 == 0);
+  if (layer_dtype == ABCD_F16) {
+    if (pairs) composite_kernel<2, true><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix / 2, F_out, B_out, out_dtype == ABCD_F16);
+    else composite_kernel<1, true><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix, F_out, B_out, out_dtype == ABCD_F16);
+  } else {
+    if (pairs) composite_kernel<2, false><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix / 2, F_out, B_out, out_dtype == ABCD_F16);
+    else composite_kernel<1, false><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix, F_out, B_out, out_dtype == ABCD_F16);
+  }
+  return check_launch(ctx, "composite_kernel");
+}

@@ -1,0 +1,351 @@
+// K5 (blend + composite forward, also the cache refresh K10) and K7 (its backward).
+//
+// Per pixel, front to back over its tile's list (3DGS blending): sigma = 1/2 d^T Q d with
+// d = pixel centre - uv, alpha = min(alpha_max, o exp(-sigma)), skip alpha < alpha_min (and
+// sigma < 0), stop before T (1 - alpha) < t_min; A = (sum T_i alpha_i c_i, 1 - T).  Then the
+// frozen partitions enter through out = F over (A over B) (Section 2), over meaning
+// X + (1 - X.a) Y on premultiplied RGBA, and out.rgb += (1 - out.a) bg.
+//
+// One CTA per 16x16 tile, one thread per pixel; batches of 256 list entries are staged in
+// shared memory; a CTA leaves as soon as every pixel has terminated (__syncthreads_count),
+// a warp as soon as its lanes have.  Every quantity that decides a branch (sigma, alpha, T)
+// is computed with explicit round-to-nearest intrinsics in one shared function, so the
+// backward kernel retraces exactly the forward's contributors.
+#include "abcd_internal.cuh"
+
+namespace abcd {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kHalfLog2e = 0.7213475204444817f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Conic scaled for base-2 exponentials: (a/2, b, c/2) * log2(e), opacity kept.
+__device__ __forceinline__ float4 scaled_conic(float4 c) {
+  return make_float4(__fmul_rn(kHalfLog2e, c.x), __fmul_rn(kLog2e, c.y), __fmul_rn(kHalfLog2e, c.z), c.w);
+}
+
+// sigma * log2(e) = dx (a/2 dx + b dy) + c/2 dy^2 in log2 units; dx, dy returned.
+__device__ __forceinline__ float sigma2(float4 s, float2 m, float fx, float fy, float& dx, float& dy) {
+  dx = __fsub_rn(fx, m.x);
+  dy = __fsub_rn(fy, m.y);
+  return __fmaf_rn(dx, __fmaf_rn(s.x, dx, __fmul_rn(s.y, dy)), __fmul_rn(__fmul_rn(s.z, dy), dy));
+}
+
+__device__ __forceinline__ float4 load_px(const void* img, int dtype, long long p) {
+  if (dtype == ABCD_F16) {
+    const uint2 r = reinterpret_cast<const uint2*>(img)[p];
+    const __half2 a = *reinterpret_cast<const __half2*>(&r.x);
+    const __half2 b = *reinterpret_cast<const __half2*>(&r.y);
+    const float2 fa = __half22float2(a), fb = __half22float2(b);
+    return make_float4(fa.x, fa.y, fb.x, fb.y);
+  }
+  return reinterpret_cast<const float4*>(img)[p];
+}
+
+struct FwdArgs {
+  Cam cam;
+  Opts op;
+  const float2* uv;
+  const float4* co;
+  const float* rgb;
+  const unsigned* ids;
+  const uint2* ranges;
+  const void* F;
+  const void* B;
+  int fb_dtype;
+  float bg[3];
+  float4* out;
+  float4* state_at;
+  unsigned* n_last;
+  uint2* refresh;      // fp16 x4 per pixel
+};
+
+__global__ void __launch_bounds__(kTileThreads) render_fwd_kernel(FwdArgs a) {
+  __shared__ float2 s_uv[kTileThreads];
+  __shared__ float4 s_co[kTileThreads];
+  __shared__ float4 s_rgb[kTileThreads];
+  const int tile = blockIdx.x;
+  const int tx = tile % a.cam.tiles_x, ty = tile / a.cam.tiles_x;
+  const int px = tx * kTile + (threadIdx.x & (kTile - 1));
+  const int py = ty * kTile + (threadIdx.x / kTile);
+  const bool inside = px < a.cam.width && py < a.cam.height;
+  const uint2 rg = a.ranges[tile];
+  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
+  const float fx = (float)px + 0.5f, fy = (float)py + 0.5f;
+  float T = 1.f, c0 = 0.f, c1 = 0.f, c2 = 0.f;
+  unsigned last = 0;
+  bool done = !inside;
+  for (int base = 0; base < n; base += kTileThreads) {
+    if (__syncthreads_count(done) == kTileThreads) break;
+    const int k = base + threadIdx.x;
+    if (k < n) {
+      const unsigned g = a.ids[rg.x + k];
+      s_uv[threadIdx.x] = a.uv[g];
+      s_co[threadIdx.x] = scaled_conic(a.co[g]);
+      s_rgb[threadIdx.x] = make_float4(a.rgb[3 * g], a.rgb[3 * g + 1], a.rgb[3 * g + 2], 0.f);
+    }
+    __syncthreads();
+    const int cnt = min(kTileThreads, n - base);
+    if (!done) {
+      for (int j = 0; j < cnt; ++j) {
+        float dx, dy;
+        const float4 s = s_co[j];
+        const float sig = sigma2(s, s_uv[j], fx, fy, dx, dy);
+        if (!(sig >= 0.f)) continue;
+        const float alpha = fminf(a.op.alpha_max, __fmul_rn(s.w, ex2_approx(-sig)));
+        if (alpha < a.op.alpha_min) continue;
+        const float test = __fmul_rn(T, __fsub_rn(1.f, alpha));
+        if (test < a.op.t_min) { done = true; break; }
+        const float w = __fmul_rn(alpha, T);
+        const float4 col = s_rgb[j];
+        c0 = __fmaf_rn(w, col.x, c0);
+        c1 = __fmaf_rn(w, col.y, c1);
+        c2 = __fmaf_rn(w, col.z, c2);
+        T = test;
+        last = (unsigned)(base + j + 1);
+      }
+    }
+  }
+  if (!inside) return;
+  const long long p = (long long)py * a.cam.width + px;
+  const float Aa = 1.f - T;
+  if (a.refresh) {
+    const __half2 lo = __floats2half2_rn(c0, c1), hi = __floats2half2_rn(c2, Aa);
+    uint2 r;
+    r.x = *reinterpret_cast<const unsigned*>(&lo);
+    r.y = *reinterpret_cast<const unsigned*>(&hi);
+    a.refresh[p] = r;
+  }
+  if (a.state_at) {
+    a.state_at[p] = make_float4(c0, c1, c2, T);
+    a.n_last[p] = last;
+  }
+  if (a.out) {
+    const float4 Bv = a.B ? load_px(a.B, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 Fv = a.F ? load_px(a.F, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float kb = 1.f - Aa;      // A over B
+    const float m0 = c0 + kb * Bv.x, m1 = c1 + kb * Bv.y, m2 = c2 + kb * Bv.z, ma = Aa + kb * Bv.w;
+    const float kf = 1.f - Fv.w;    // F over (A over B)
+    float4 o = make_float4(Fv.x + kf * m0, Fv.y + kf * m1, Fv.z + kf * m2, Fv.w + kf * ma);
+    const float kg = 1.f - o.w;
+    o.x += kg * a.bg[0];
+    o.y += kg * a.bg[1];
+    o.z += kg * a.bg[2];
+    a.out[p] = o;
+  }
+}
+
+struct BwdArgs {
+  Cam cam;
+  Opts op;
+  const float2* uv;
+  const float4* co;
+  const float* rgb;
+  const unsigned* ids;
+  const uint2* ranges;
+  const void* F;
+  const void* B;
+  int fb_dtype;
+  float bg[3];
+  const float4* state_at;
+  const unsigned* n_last;
+  const float* dl_dout;
+  float* grad2d;
+};
+
+__global__ void __launch_bounds__(kTileThreads) render_bwd_kernel(BwdArgs a) {
+  __shared__ float2 s_uv[kTileThreads];
+  __shared__ float4 s_co[kTileThreads];
+  __shared__ float4 s_rgb[kTileThreads];
+  __shared__ unsigned s_id[kTileThreads];
+  __shared__ unsigned s_max;
+  const int tile = blockIdx.x;
+  const int tx = tile % a.cam.tiles_x, ty = tile / a.cam.tiles_x;
+  const int px = tx * kTile + (threadIdx.x & (kTile - 1));
+  const int py = ty * kTile + (threadIdx.x / kTile);
+  const int lane = threadIdx.x & 31;
+  const bool inside = px < a.cam.width && py < a.cam.height;
+  const uint2 rg = a.ranges[tile];
+  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
+  const float fx = (float)px + 0.5f, fy = (float)py + 0.5f;
+  unsigned last = 0;
+  float Gr = 0.f, Gg = 0.f, Gb = 0.f, Ga = 0.f, Tf = 1.f, A0 = 0.f, A1 = 0.f, A2 = 0.f;
+  if (inside) {
+    const long long p = (long long)py * a.cam.width + px;
+    last = min(a.n_last[p], (unsigned)n);
+    const float4 at = a.state_at[p];
+    A0 = at.x; A1 = at.y; A2 = at.z; Tf = at.w;
+    const float g0 = a.dl_dout[3 * p], g1 = a.dl_dout[3 * p + 1], g2 = a.dl_dout[3 * p + 2];
+    const float4 Fv = a.F ? load_px(a.F, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 Bv = a.B ? load_px(a.B, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float kf = 1.f - Fv.w;
+    Gr = kf * g0; Gg = kf * g1; Gb = kf * g2;
+    // d final / d A.a = -(1 - F.a) (B.rgb + (1 - B.a) bg)
+    Ga = -kf * (g0 * (Bv.x + (1.f - Bv.w) * a.bg[0]) + g1 * (Bv.y + (1.f - Bv.w) * a.bg[1]) +
+                g2 * (Bv.z + (1.f - Bv.w) * a.bg[2]));
+  }
+  if (threadIdx.x == 0) s_max = 0;
+  __syncthreads();
+  const unsigned wmax = __reduce_max_sync(0xffffffffu, last);
+  if (lane == 0) atomicMax(&s_max, wmax);
+  __syncthreads();
+  const int span = (int)s_max;
+  float T = 1.f, c0 = 0.f, c1 = 0.f, c2 = 0.f;
+  for (int base = 0; base < span; base += kTileThreads) {
+    __syncthreads();
+    const int k = base + threadIdx.x;
+    if (k < span) {
+      const unsigned g = a.ids[rg.x + k];
+      s_id[threadIdx.x] = g;
+      s_uv[threadIdx.x] = a.uv[g];
+      s_co[threadIdx.x] = scaled_conic(a.co[g]);
+      s_rgb[threadIdx.x] = make_float4(a.rgb[3 * g], a.rgb[3 * g + 1], a.rgb[3 * g + 2], 0.f);
+    }
+    __syncthreads();
+    const int cnt = min(kTileThreads, span - base);
+    for (int j = 0; j < cnt; ++j) {
+      float v[9];
+#pragma unroll
+      for (int q = 0; q < 9; ++q) v[q] = 0.f;
+      bool contrib = false;
+      if ((unsigned)(base + j) < last) {
+        float dx, dy;
+        const float4 s = s_co[j];
+        const float sig = sigma2(s, s_uv[j], fx, fy, dx, dy);
+        if (sig >= 0.f) {
+          const float G = ex2_approx(-sig);
+          const float raw = __fmul_rn(s.w, G);
+          const float alpha = fminf(a.op.alpha_max, raw);
+          if (alpha >= a.op.alpha_min) {
+            contrib = true;
+            const float4 col = s_rgb[j];
+            const float w = __fmul_rn(alpha, T);
+            c0 = __fmaf_rn(w, col.x, c0);
+            c1 = __fmaf_rn(w, col.y, c1);
+            c2 = __fmaf_rn(w, col.z, c2);
+            const float ioma = 1.f / (1.f - alpha);
+            // R = colour accumulated behind this Gaussian = A - (sum up to and including it)
+            const float dalpha = Gr * (T * col.x - (A0 - c0) * ioma) +
+                                 Gg * (T * col.y - (A1 - c1) * ioma) +
+                                 Gb * (T * col.z - (A2 - c2) * ioma) + Ga * Tf * ioma;
+            v[6] = Gr * w; v[7] = Gg * w; v[8] = Gb * w;
+            if (raw <= a.op.alpha_max) {          // derivative of min() is 0 once clamped
+              v[5] = dalpha * G;                   // d alpha / d opacity = exp(-sigma)
+              const float dsig = -dalpha * raw;    // d alpha / d sigma = -alpha
+              const float ca = 2.f * kLn2 * s.x, cb = kLn2 * s.y, cc = 2.f * kLn2 * s.z;
+              v[0] = -dsig * (ca * dx + cb * dy);  // d = pixel - uv
+              v[1] = -dsig * (cb * dx + cc * dy);
+              v[2] = 0.5f * dsig * dx * dx;
+              v[3] = dsig * dx * dy;
+              v[4] = 0.5f * dsig * dy * dy;
+            }
+            T = __fmul_rn(T, __fsub_rn(1.f, alpha));
+          }
+        }
+      }
+      if (__any_sync(0xffffffffu, contrib)) {
+#pragma unroll
+        for (int q = 0; q < 9; ++q)
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) v[q] += __shfl_xor_sync(0xffffffffu, v[q], o);
+        float mine = 0.f;
+#pragma unroll
+        for (int q = 0; q < 9; ++q) mine = (lane == q) ? v[q] : mine;
+        if (lane < 9) atomicAdd(&a.grad2d[9 * (size_t)s_id[j] + lane], mine);
+      }
+    }
+  }
+}
+
+bool fb_ok(const void* F, const void* B, int dtype) {
+  if (dtype != ABCD_F16 && dtype != ABCD_F32) return false;
+  const uintptr_t al = dtype == ABCD_F16 ? 7 : 15;
+  return (((uintptr_t)F & al) == 0) && (((uintptr_t)B & al) == 0);
+}
+
+bool proj_ok(const abcd_projected* p) {
+  return p && p->uv && p->conic_opacity && p->rgb && ((uintptr_t)p->uv & 7) == 0 &&
+         ((uintptr_t)p->conic_opacity & 15) == 0;
+}
+
+}  // namespace
+}  // namespace abcd
+
+using namespace abcd;
+
+extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camera* cam,
+                                                 const abcd_render_opts* opts,
+                                                 const abcd_projected* proj,
+                                                 const abcd_tiles* tiles, const void* F,
+                                                 const void* B, int fb_dtype, const float* bg,
+                                                 float* out_rgba, abcd_fwd_state* state,
+                                                 void* refresh_f16) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!cam || cam->width <= 0 || cam->height <= 0 || !tiles || !tiles->ids || !tiles->ranges)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_composite_fwd: bad camera or tiles");
+  if (!proj_ok(proj)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_composite_fwd: bad projected buffers");
+  if (!fb_ok(F, B, fb_dtype)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_composite_fwd: bad F/B dtype or alignment");
+  if (state && (!state->A_T || !state->n_last || ((uintptr_t)state->A_T & 15)))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_composite_fwd: bad state buffers");
+  if (((uintptr_t)out_rgba & 15) || ((uintptr_t)refresh_f16 & 7))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_composite_fwd: misaligned output");
+  FwdArgs a;
+  a.cam = make_cam(cam, opts);
+  a.op = make_opts(opts);
+  a.uv = (const float2*)proj->uv;
+  a.co = (const float4*)proj->conic_opacity;
+  a.rgb = proj->rgb;
+  a.ids = tiles->ids;
+  a.ranges = (const uint2*)tiles->ranges;
+  a.F = F; a.B = B; a.fb_dtype = fb_dtype;
+  for (int c = 0; c < 3; ++c) a.bg[c] = bg ? bg[c] : 0.f;
+  a.out = (float4*)out_rgba;
+  a.state_at = state ? (float4*)state->A_T : nullptr;
+  a.n_last = state ? state->n_last : nullptr;
+  a.refresh = (uint2*)refresh_f16;
+  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y;
+  render_fwd_kernel<<<n_tiles, kTileThreads, 0, ctx->stream>>>(a);
+  return check_launch(ctx, "render_fwd_kernel");
+}
+
+extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* cam,
+                                            const abcd_render_opts* opts,
+                                            const abcd_projected* proj, const abcd_tiles* tiles,
+                                            const void* F, const void* B, int fb_dtype,
+                                            const float* bg, const abcd_fwd_state* state,
+                                            const float* dL_dout, int n, float* grad2d) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!cam || cam->width <= 0 || cam->height <= 0 || !tiles || !tiles->ids || !tiles->ranges)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_backward: bad camera or tiles");
+  if (!proj_ok(proj)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_backward: bad projected buffers");
+  if (!fb_ok(F, B, fb_dtype)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_backward: bad F/B dtype or alignment");
+  if (!state || !state->A_T || !state->n_last || !dL_dout || n < 0 || (n > 0 && !grad2d))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_backward: null state, gradient or output");
+  if (n == 0) return ABCD_OK;
+  cudaError_t e = cudaMemsetAsync(grad2d, 0, sizeof(float) * 9 * (size_t)n, ctx->stream);
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "grad2d memset: %s", cudaGetErrorString(e));
+  BwdArgs a;
+  a.cam = make_cam(cam, opts);
+  a.op = make_opts(opts);
+  a.uv = (const float2*)proj->uv;
+  a.co = (const float4*)proj->conic_opacity;
+  a.rgb = proj->rgb;
+  a.ids = tiles->ids;
+  a.ranges = (const uint2*)tiles->ranges;
+  a.F = F; a.B = B; a.fb_dtype = fb_dtype;
+  for (int c = 0; c < 3; ++c) a.bg[c] = bg ? bg[c] : 0.f;
+  a.state_at = (const float4*)state->A_T;
+  a.n_last = state->n_last;
+  a.dl_dout = dL_dout;
+  a.grad2d = grad2d;
+  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y;
+  render_bwd_kernel<<<n_tiles, kTileThreads, 0, ctx->stream>>>(a);
+  return check_launch(ctx, "render_bwd_kernel");
+}

@@ -1,0 +1,35 @@
+// abcd_backward: the backward pass of one active-block step (Section 2: the reconstruction
+// loss is evaluated and gradients are backpropagated only through theta_active):
+// K6 loss (optional) -> K7 blend/composite backward -> K8 projection backward.
+#include "abcd_internal.cuh"
+
+using namespace abcd;
+
+extern "C" abcd_status abcd_backward(abcd_ctx* ctx, const abcd_gaussians* theta,
+                                     const abcd_camera* cam, const abcd_render_opts* opts,
+                                     const abcd_projected* proj, const abcd_tiles* tiles,
+                                     const void* F, const void* B, int fb_dtype, const float* bg,
+                                     const float* out_rgba, const abcd_fwd_state* state,
+                                     const float* gt_rgb, float lambda_ssim, float* loss_out,
+                                     const float* dL_dout, abcd_gaussians* grads) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!has_workspace(ctx)) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_backward: no workspace");
+  if (!theta || !cam) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_backward: null theta or camera");
+  if (theta->n > ctx->max_g) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_backward: n exceeds workspace");
+  const long long npix = (long long)cam->width * cam->height;
+  const float* g = dL_dout;
+  abcd_status s;
+  if (gt_rgb) {
+    if (npix > ctx->max_pixels) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_backward: image exceeds workspace");
+    if ((s = loss_launch(ctx, out_rgba, gt_rgb, cam->width, cam->height, lambda_ssim, loss_out,
+                         ctx->ws.dl_dout)))
+      return s;
+    g = ctx->ws.dl_dout;
+  } else if (!g) {
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_backward: need gt_rgb or dL_dout");
+  }
+  if ((s = abcd_render_backward(ctx, cam, opts, proj, tiles, F, B, fb_dtype, bg, state, g,
+                                theta->n, ctx->ws.grad2d)))
+    return s;
+  return abcd_project_backward(ctx, theta, cam, opts, ctx->ws.grad2d, grads);
+}

@@ -1,0 +1,232 @@
+"""Parity machinery: CUDA path (fp32) versus the fp64 oracle, element by element.
+
+Where an fp32 computation decides something discrete (a radius, a tile boundary, whether a
+Gaussian is skipped at a pixel, where a pixel's blend stops), both outcomes are correct when
+the exact (fp64) value lies within fp32 rounding reach of the threshold.  This module derives
+those ambiguous decisions from the oracle's own values with a stated uncertainty model, and
+enumerates the oracle's result for every combination of them; the GPU must equal one of the
+valid results (within the float tolerance) and everything else exactly.
+
+Uncertainty model (u = 2^-24, unit roundoff of fp32):
+  * camera-space mean:   dt_k = 8u (sum_j |R_kj mu_j| + |t_k|)
+  * pixel-space mean:    du = fx (dt_x + |t_x/t_z| dt_z)/t_z + 8u (|fx t_x/t_z| + |cx|), same for v
+  * conic (relative):    64u (1 + lambda_max/lambda_min)
+  * radius (relative):   1e-5 on 3 sqrt(lambda_max)
+  * sigma (relative, w.r.t. its absolute terms): 64u;   alpha: 4e-6;   transmittance step: 8u
+"""
+from __future__ import annotations
+
+import itertools
+import math
+
+import numpy as np
+
+import oracle
+
+U = 2.0 ** -24
+TOL_PIX = 1e-4
+K_ARITH = 64 * U
+EPS_ALPHA = 4e-6
+EPS_STEP = 8 * U
+
+
+def margins(g, cam, P):
+    """Per-Gaussian absolute uncertainty of (u, v) and relative uncertainty of the conic."""
+    R = np.asarray(cam.R, np.float64).reshape(3, 3)
+    t = np.asarray(cam.t, np.float64)
+    mu = np.asarray(g.means, np.float64)
+    terms = np.abs(mu[:, None, :] * R[None, :, :]).sum(-1) + np.abs(t)[None, :]   # [n,3]
+    dt = 8 * U * terms
+    tc = mu @ R.T + t
+    tz = np.where(np.abs(tc[:, 2]) > 1e-9, tc[:, 2], 1e-9)
+    du = cam.fx * (dt[:, 0] + np.abs(tc[:, 0] / tz) * dt[:, 2]) / np.abs(tz) + \
+        8 * U * (np.abs(cam.fx * tc[:, 0] / tz) + abs(cam.cx))
+    dv = cam.fy * (dt[:, 1] + np.abs(tc[:, 1] / tz) * dt[:, 2]) / np.abs(tz) + \
+        8 * U * (np.abs(cam.fy * tc[:, 1] / tz) + abs(cam.cy))
+    lam = P["eig"]
+    kappa = np.where(lam[:, 1] > 0, lam[:, 0] / np.maximum(lam[:, 1], 1e-30), 1.0)
+    m_uv = np.stack([du, dv], -1)
+    m_conic = 64 * U * (1 + kappa)
+    return m_uv, m_conic
+
+
+def splats_with_margins(g, cam, P):
+    m_uv, m_c = margins(g, cam, P)
+    return oracle.SplatSet.from_proj(P, m_uv=m_uv, m_conic=m_c, k_arith=K_ARITH,
+                                     eps_alpha=EPS_ALPHA, eps_step=EPS_STEP)
+
+
+def rect_bounds(P, cam, m_uv, tile=16):
+    """Smallest and largest tile rectangle any admissible fp32 rounding can give."""
+    tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
+    n = P["visible"].shape[0]
+    lo = np.zeros((n, 4), np.int64)
+    hi = np.zeros((n, 4), np.int64)
+    amb_radius = np.zeros(n, bool)
+    for i in range(n):
+        if P["depth"][i] <= 0.2 or P["radius_exact"][i] == 0:
+            continue
+        re = P["radius_exact"][i]
+        rs = {math.ceil(re * (1 - 1e-5)), math.ceil(re * (1 + 1e-5))}
+        amb_radius[i] = len(rs) > 1
+        u, v = P["uv"][i]
+        du, dv = m_uv[i]
+        cands = []
+        for r in rs:
+            for uu in (u - du, u + du):
+                for vv in (v - dv, v + dv):
+                    x0 = min(max(math.floor((uu - r) / tile), 0), tx)
+                    y0 = min(max(math.floor((vv - r) / tile), 0), ty)
+                    x1 = min(max(math.floor((uu + r) / tile) + 1, 0), tx)
+                    y1 = min(max(math.floor((vv + r) / tile) + 1, 0), ty)
+                    cands.append((x0, y0, x1, y1))
+        c = np.array(cands)
+        lo[i] = [c[:, 0].max(), c[:, 1].max(), c[:, 2].min(), c[:, 3].min()]
+        hi[i] = [c[:, 0].min(), c[:, 1].min(), c[:, 2].max(), c[:, 3].max()]
+    return lo, hi, amb_radius
+
+
+def _in(rect, x, y):
+    return rect[0] <= x < rect[2] and rect[1] <= y < rect[3]
+
+
+def optional_members(P, lo, hi, cam, tile=16):
+    """tile -> set of Gaussians that may or may not be listed there."""
+    tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
+    opt = {}
+    diff = np.where(np.any(lo != hi, axis=1) & (P["depth"] > 0.2))[0]
+    for i in diff:
+        for y in range(hi[i, 1], hi[i, 3]):
+            for x in range(hi[i, 0], hi[i, 2]):
+                if not _in(lo[i], x, y):
+                    opt.setdefault(y * tx + x, set()).add(int(i))
+    return opt
+
+
+def check_tile_lists(gpu_ranges, gpu_ids, off, ids, P, opt, n_tiles):
+    """GPU lists == oracle lists up to optional members, sorted by (fp32 depth, id)."""
+    keys = P["depth_key"].astype(np.int64)
+    for t in range(n_tiles):
+        s, e = int(gpu_ranges[t, 0]), int(gpu_ranges[t, 1])
+        L = [int(v) for v in gpu_ids[s:e]] if e > s else []
+        O = [int(v) for v in ids[off[t]:off[t + 1]]]
+        o = opt.get(t, set())
+        assert [g for g in L if g not in o] == [g for g in O if g not in o], f"tile {t}"
+        assert set(L) <= set(O) | o, f"tile {t}: unexpected members"
+        k = [(keys[g], g) for g in L]
+        assert k == sorted(k), f"tile {t}: not sorted by (depth, id)"
+
+
+def pixel_alternatives(sp, lst_full, labels, px, py, events, F, B, bg, opts, max_toggles=4):
+    """All valid (render, list, event flips) of one pixel: every subset of its ambiguous
+    decisions flipped.  labels[k] is "in" (certain member), "opt_in" / "opt_out" (optional
+    member, present / absent in the oracle's nominal list)."""
+    toggles = [("m", g) for g, m in zip(lst_full, labels) if m != "in"]
+    toggles += [("e", ev) for ev in events]
+    if len(toggles) > max_toggles:
+        return None
+    outs = []
+    for k in range(len(toggles) + 1):
+        for sub in itertools.combinations(toggles, k):
+            mem_flip = {g for kind, g in sub if kind == "m"}
+            ev_flip = [ev for kind, ev in sub if kind == "e"]
+            lst = [g for g, m in zip(lst_full, labels)
+                   if m == "in" or (m == "opt_in") != (g in mem_flip)]
+            r = oracle.render_pixel(sp, lst, px, py, F=F, B=B, bg=bg, toggles=ev_flip, opts=opts)
+            outs.append((r, lst, ev_flip))
+    return outs
+
+
+def tile_candidates(t, off, ids, P, opt):
+    """Oracle's list of tile t merged with its optional members, with membership labels."""
+    O = [int(v) for v in ids[off[t]:off[t + 1]]]
+    o = opt.get(t, set())
+    allg = sorted(set(O) | o, key=lambda g: (int(P["depth_key"][g]), g))
+    lab = []
+    for g in allg:
+        if g in o:
+            lab.append("opt_in" if g in O else "opt_out")
+        else:
+            lab.append("in")
+    return allg, lab
+
+
+def compare_render(gpu_out, gpu_T, R, sp, off, ids, P, opt, cam, F=None, B=None, bg=None,
+                   opts=None, tol=TOL_PIX, tile=16):
+    """Returns the number of pixels resolved through alternatives; asserts parity."""
+    H, W = cam.height, cam.width
+    tx, _ = oracle.tiles_xy(W, H, tile)
+    ref = R["out"]
+    flagged = R["n_ev"] > 0
+    for t in opt:
+        y0, x0 = (t // tx) * tile, (t % tx) * tile
+        flagged[y0:y0 + tile, x0:x0 + tile] = True
+    ok = ~flagged
+    err = np.abs(gpu_out[ok] - ref[ok]).max() if ok.any() else 0.0
+    assert err <= tol, f"max |gpu - oracle| on unambiguous pixels = {err}"
+    errT = np.abs(gpu_T[ok] - R["T_final"][ok]).max() if ok.any() else 0.0
+    assert errT <= tol, f"max |T_gpu - T_oracle| = {errT}"
+    n_alt = 0
+    for py, px in zip(*np.nonzero(flagged)):
+        t = (py // tile) * tx + (px // tile)
+        allg, lab = tile_candidates(t, off, ids, P, opt)
+        evs = [tuple(e) for e in R["ev"][py, px][:min(R["n_ev"][py, px], R["ev"].shape[2])]]
+        Fp = None if F is None else F[py, px]
+        Bp = None if B is None else B[py, px]
+        alts = pixel_alternatives(sp, allg, lab, px, py, evs, Fp, Bp, bg, opts)
+        assert alts is not None, f"pixel {(px, py)}: too many ambiguous decisions"
+        best = min(np.abs(gpu_out[py, px] - a[0]["out"]).max() for a in alts)
+        assert best <= tol, f"pixel {(px, py)} matches no valid alternative ({best})"
+        n_alt += 1
+    return n_alt
+
+
+def grad_envelope(sp, off, ids, P, opt, R, cam, G, F=None, B=None, bg=None, opts=None, tile=16):
+    """Per-Gaussian [lo, hi] offsets of grad2d over the alternatives of ambiguous pixels."""
+    H, W = cam.height, cam.width
+    tx, _ = oracle.tiles_xy(W, H, tile)
+    n = sp.s.n
+    lo = np.zeros((n, 9))
+    hi = np.zeros((n, 9))
+    flagged = R["n_ev"] > 0
+    for t in opt:
+        y0, x0 = (t // tx) * tile, (t % tx) * tile
+        flagged[y0:y0 + tile, x0:x0 + tile] = True
+    pix = list(zip(*np.nonzero(flagged)))
+    for py, px in pix:
+        t = (py // tile) * tx + (px // tile)
+        allg, lab = tile_candidates(t, off, ids, P, opt)
+        evs = [tuple(e) for e in R["ev"][py, px][:min(R["n_ev"][py, px], R["ev"].shape[2])]]
+        Fp = None if F is None else F[py, px]
+        Bp = None if B is None else B[py, px]
+        alts = pixel_alternatives(sp, allg, lab, px, py, evs, Fp, Bp, bg, opts)
+        assert alts is not None
+        nominal_lst = [int(v) for v in ids[off[t]:off[t + 1]]]
+        base = oracle.backward_pixel(sp, nominal_lst, px, py, G[py, px], F=Fp, B=Bp, bg=bg,
+                                     opts=opts)
+        deltas = []
+        for _, lst, evf in alts:
+            g = oracle.backward_pixel(sp, lst, px, py, G[py, px], F=Fp, B=Bp, bg=bg,
+                                      toggles=evf, opts=opts)
+            deltas.append(g - base)
+        D = np.stack(deltas)
+        lo += D.min(0)
+        hi += D.max(0)
+    return lo, hi, len(pix)
+
+
+def assert_grad_close(gpu, ref, lo=None, hi=None, rtol=1e-3, atol=1e-5, what="grad"):
+    gpu = np.asarray(gpu, np.float64)
+    ref = np.asarray(ref, np.float64)
+    if lo is None:
+        lo = np.zeros_like(ref)
+        hi = np.zeros_like(ref)
+    tol = np.maximum(rtol * np.abs(ref), atol)
+    below = gpu < ref + lo - tol
+    above = gpu > ref + hi + tol
+    bad = below | above
+    if bad.any():
+        idx = np.argwhere(bad)[:8]
+        det = [(tuple(i), float(gpu[tuple(i)]), float(ref[tuple(i)])) for i in idx]
+        raise AssertionError(f"{what}: {int(bad.sum())} of {bad.size} entries out of tolerance; "
+                             f"first: {det}")

@@ -1,0 +1,407 @@
+"""CUDA path (libabcd.so through its C ABI) versus the fp64 oracle on seeded inputs.
+
+Tolerances: tile lists and sort order bit-exact (up to decisions the oracle proves are within
+fp32 rounding of their threshold, see tests/_parity.py); pixels 1e-4 absolute; gradients 1e-3
+relative or 1e-5 absolute; loss 1e-5 relative; fp16 outputs bit-exact except where the exact
+value lies within fp32 accumulation error of an fp16 rounding midpoint.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2608_27735_gb300 as ab
+from paper_2608_27735_gb300 import scenegen as sg
+from tests import _parity as par
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    ab.build()
+    c = ab.Context(0)
+    c.reserve(200_000, 8_000_000, 2_100_000)
+    return c
+
+
+class Case:
+    """One seeded workload: the active block, a camera, F/B from the frozen partitions."""
+
+    def __init__(self, scene, cam_idx, active=0, fb=True, fb_dtype="f16"):
+        self.scene = scene
+        self.cam = scene.cameras[cam_idx]
+        g = scene.gaussians
+        cells = oracle.assign_cells(g.means, scene.grid.origin, scene.grid.side, scene.grid.dims)
+        self.g = g.subset(np.nonzero(cells == active)[0])
+        self.F = self.B = None
+        if fb:
+            front, back = oracle.partition_split(scene.grid.dims, scene.grid.origin,
+                                                 scene.grid.side, self.cam.position, active)
+            layers = {}
+            for p in list(front) + list(back):
+                gp = g.subset(np.nonzero(cells == p)[0])
+                P = oracle.project(gp, self.cam)
+                off, ids = oracle.tile_lists(P, self.cam.width, self.cam.height)
+                layers[p] = oracle.render(oracle.SplatSet.from_proj(P), off, ids,
+                                          self.cam.width, self.cam.height)["out"]
+            H, W = self.cam.height, self.cam.width
+            keys = sorted(layers)
+            st = np.stack([layers[k] for k in keys]) if keys else np.zeros((0, H, W, 4))
+            idx = {k: i for i, k in enumerate(keys)}
+            F64 = oracle.composite_layers(st, [idx[k] for k in front]) if len(front) else np.zeros((H, W, 4))
+            B64 = oracle.composite_layers(st, [idx[k] for k in back]) if len(back) else np.zeros((H, W, 4))
+            dt = np.float16 if fb_dtype == "f16" else np.float32
+            self.F = F64.astype(dt)
+            self.B = B64.astype(dt)
+        self.P = oracle.project(self.g, self.cam)
+        self.off, self.ids = oracle.tile_lists(self.P, self.cam.width, self.cam.height)
+        self.m_uv, _ = par.margins(self.g, self.cam, self.P)
+        self.lo, self.hi, self.amb_r = par.rect_bounds(self.P, self.cam, self.m_uv)
+        self.opt = par.optional_members(self.P, self.lo, self.hi, self.cam)
+        self.sp = par.splats_with_margins(self.g, self.cam, self.P)
+
+    def F64(self):
+        return None if self.F is None else self.F.astype(np.float64)
+
+    def B64(self):
+        return None if self.B is None else self.B.astype(np.float64)
+
+
+def run_forward(ctx, case, bg=None, opts=None, want_state=True, refresh=False):
+    cam = ab.camera(case.cam)
+    theta = ab.Gaussians.from_numpy(case.g)
+    proj = ab.Projected.alloc(theta.n)
+    ab.abcd_project(ctx, theta, cam, opts, proj)
+    tiles = ab.Tiles.alloc(4_000_000, case.cam.width, case.cam.height)
+    ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+    H, W = case.cam.height, case.cam.width
+    out = torch.empty(H, W, 4, device="cuda")
+    st = ab.FwdState.alloc(W, H) if want_state else None
+    Ft = None if case.F is None else torch.from_numpy(case.F).cuda()
+    Bt = None if case.B is None else torch.from_numpy(case.B).cuda()
+    fbd = ab.ABCD_F16 if (case.F is None or case.F.dtype == np.float16) else ab.ABCD_F32
+    rf = torch.empty(H, W, 4, dtype=torch.float16, device="cuda") if refresh else None
+    ab.abcd_render_composite_fwd(ctx, cam, opts, proj, tiles, Ft, Bt, fbd, bg, out, st, rf)
+    ctx.sync()
+    return dict(cam=cam, theta=theta, proj=proj, tiles=tiles, out=out, state=st, F=Ft, B=Bt,
+                fbd=fbd, refresh=rf)
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    return sg.tiny_scene()
+
+
+@pytest.fixture(scope="module")
+def ragged():
+    # ragged image (150x100: partial tiles on both axes), SH degree 3
+    s = sg.grid_scene((2, 2, 1), 5.0, 1500, 3, seed=77)
+    s.cameras = sg.ring_cameras(3, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 150, 100, seed=77,
+                                height_jitter=1.0)
+    return s
+
+
+# ----------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("cam_idx", [0, 1, 2, 3])
+def test_project_matches_oracle(ctx, tiny, cam_idx):
+    case = Case(tiny, cam_idx, fb=False)
+    r = run_forward(ctx, case, want_state=False)
+    pr = r["proj"]
+    P = case.P
+    depth = pr.depth.cpu().numpy()
+    np.testing.assert_array_equal(depth.view(np.uint32)[P["depth"] > 0.2], P["depth_key"][P["depth"] > 0.2])
+    rad = pr.radius.cpu().numpy()
+    vis = P["visible"] == 1
+    exact = ~case.amb_r & vis & np.all(case.lo == case.hi, axis=1)
+    np.testing.assert_array_equal(rad[exact], P["radius"][exact])
+    assert np.all((rad > 0) == vis) or np.all(((rad > 0) != vis) <= ~np.all(case.lo == case.hi, axis=1))
+    uv = pr.uv.cpu().numpy()
+    co = pr.conic_opacity.cpu().numpy()
+    rgb = pr.rgb.cpu().numpy()
+    both = vis & (rad > 0)
+    np.testing.assert_allclose(uv[both], P["uv"][both], rtol=0, atol=1e-3)
+    np.testing.assert_allclose(co[both, 3], P["opacity"][both], rtol=1e-6, atol=1e-7)
+    np.testing.assert_allclose(rgb[both], P["rgb"][both], rtol=1e-5, atol=1e-6)
+    # conic: relative to its own scale (|a| + |c|)
+    scale = (np.abs(P["conic"][both, 0]) + np.abs(P["conic"][both, 2]))[:, None]
+    assert np.all(np.abs(co[both, :3] - P["conic"][both]) <= 1e-4 * scale)
+    tt = pr.tiles_touched.cpu().numpy()
+    nom = (P["rect"][:, 2] - P["rect"][:, 0]) * (P["rect"][:, 3] - P["rect"][:, 1])
+    np.testing.assert_array_equal(tt[exact], nom[exact])
+
+
+@pytest.mark.parametrize("cam_idx", [0, 1, 2, 3])
+def test_bin_sort_matches_oracle(ctx, tiny, cam_idx):
+    case = Case(tiny, cam_idx, fb=False)
+    r = run_forward(ctx, case, want_state=False)
+    K = int(r["tiles"].count.item())
+    rng = r["tiles"].ranges.cpu().numpy().astype(np.int64)
+    ids = r["tiles"].ids.cpu().numpy()[:K]
+    tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
+    par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt, tx * ty)
+    n_opt = sum(len(v) for v in case.opt.values())
+    assert abs(K - len(case.ids)) <= n_opt
+
+
+def test_bin_sort_ragged_and_sh3(ctx, ragged):
+    for ci in range(3):
+        case = Case(ragged, ci, fb=False)
+        r = run_forward(ctx, case, want_state=False)
+        K = int(r["tiles"].count.item())
+        rng = r["tiles"].ranges.cpu().numpy().astype(np.int64)
+        ids = r["tiles"].ids.cpu().numpy()[:K]
+        tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
+        par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt, tx * ty)
+
+
+@pytest.mark.parametrize("cam_idx,bg,fbdt", [(0, None, "f16"), (1, (0.2, 0.5, 0.9), "f16"),
+                                             (2, None, "f32"), (3, (1.0, 1.0, 1.0), "f16")])
+def test_render_composite_fwd_matches_oracle(ctx, tiny, cam_idx, bg, fbdt):
+    case = Case(tiny, cam_idx, fb=True, fb_dtype=fbdt)
+    r = run_forward(ctx, case, bg=bg)
+    R = oracle.render(case.sp, case.off, case.ids, case.cam.width, case.cam.height,
+                      F=case.F64(), B=case.B64(), bg=bg)
+    gout = r["out"].cpu().numpy()
+    gT = r["state"].A_T.cpu().numpy()[..., 3]
+    n_alt = par.compare_render(gout, gT, R, case.sp, case.off, case.ids, case.P, case.opt,
+                               case.cam, F=case.F64(), B=case.B64(), bg=bg)
+    assert n_alt < 0.01 * case.cam.width * case.cam.height
+    # the saved active layer A also matches (state used by the backward pass)
+    A = r["state"].A_T.cpu().numpy()[..., :3]
+    ok = (R["n_ev"] == 0)
+    tx, _ = oracle.tiles_xy(case.cam.width, case.cam.height)
+    for t in case.opt:
+        ok[(t // tx) * 16:(t // tx) * 16 + 16, (t % tx) * 16:(t % tx) * 16 + 16] = False
+    assert np.abs(A[ok] - R["A"][..., :3][ok]).max() <= 1e-4
+    nl = r["state"].n_last.cpu().numpy()
+    assert np.all(nl[ok] == R["n_used"][ok])
+
+
+def test_render_ragged_no_fb(ctx, ragged):
+    case = Case(ragged, 1, fb=False)
+    r = run_forward(ctx, case)
+    R = oracle.render(case.sp, case.off, case.ids, case.cam.width, case.cam.height)
+    par.compare_render(r["out"].cpu().numpy(), r["state"].A_T.cpu().numpy()[..., 3], R, case.sp,
+                       case.off, case.ids, case.P, case.opt, case.cam)
+
+
+def test_refresh_fp16_matches_oracle(ctx, tiny):
+    """Cache refresh (Section 2): the active layer alone, premultiplied, rounded to fp16."""
+    case = Case(tiny, 0, fb=False)
+    r = run_forward(ctx, case, refresh=True)
+    R = oracle.render(case.sp, case.off, case.ids, case.cam.width, case.cam.height)
+    got = r["refresh"].cpu().numpy()
+    ref = R["A"]
+    ok = R["n_ev"] == 0
+    tx, _ = oracle.tiles_xy(case.cam.width, case.cam.height)
+    for t in case.opt:
+        ok[(t // tx) * 16:(t // tx) * 16 + 16, (t % tx) * 16:(t % tx) * 16 + 16] = False
+    # fp16 of the fp32 value: equal to the RNE rounding of the exact value unless the exact
+    # value is within 1e-4 (the fp32 pixel tolerance) of an fp16 rounding midpoint
+    lo = (ref - 1e-4).astype(np.float16)
+    hi = (ref + 1e-4).astype(np.float16)
+    g = got.astype(np.float64)
+    assert np.all((g[ok] >= lo[ok].astype(np.float64)) & (g[ok] <= hi[ok].astype(np.float64)))
+    exact = ok[..., None] & (lo == hi)
+    assert np.all(got[exact] == ref.astype(np.float16)[exact])
+
+
+@pytest.mark.parametrize("cam_idx", [0, 2])
+def test_render_backward_matches_oracle(ctx, tiny, cam_idx):
+    case = Case(tiny, cam_idx, fb=True)
+    bg = (0.1, 0.2, 0.3)
+    r = run_forward(ctx, case, bg=bg)
+    H, W = case.cam.height, case.cam.width
+    rng = np.random.default_rng(100 + cam_idx)
+    G = (rng.normal(size=(H, W, 3)) / (3.0 * H * W)).astype(np.float32)
+    grad2d = torch.empty(case.g.n, 9, device="cuda")
+    ab.abcd_render_backward(ctx, r["cam"], None, r["proj"], r["tiles"], r["F"], r["B"], r["fbd"],
+                            bg, r["state"], torch.from_numpy(G).cuda(), case.g.n, grad2d)
+    ctx.sync()
+    ref = oracle.backward(case.sp, case.off, case.ids, W, H, G.astype(np.float64), F=case.F64(),
+                          B=case.B64(), bg=bg)
+    R = oracle.render(case.sp, case.off, case.ids, W, H, F=case.F64(), B=case.B64(), bg=bg)
+    lo, hi, npx = par.grad_envelope(case.sp, case.off, case.ids, case.P, case.opt, R, case.cam,
+                                    G.astype(np.float64), F=case.F64(), B=case.B64(), bg=bg)
+    # absolute floor: 1e-5 of each component's largest magnitude (G is scaled like a loss
+    # gradient, so this is stricter than a fixed 1e-5)
+    scale = np.abs(ref).max(0, keepdims=True)
+    par.assert_grad_close(grad2d.cpu().numpy(), ref, lo, hi, rtol=1e-3, atol=1e-5 * scale,
+                          what="grad2d")
+
+
+def test_project_backward_matches_oracle(ctx, ragged):
+    case = Case(ragged, 0, fb=False)
+    theta = ab.Gaussians.from_numpy(case.g)
+    rng = np.random.default_rng(5)
+    vis = case.P["visible"] == 1
+    g2 = (rng.normal(size=(case.g.n, 9)) * vis[:, None]).astype(np.float32)
+    g2[:, 2:5] *= 10.0
+    grads = ab.Gaussians.zeros_like(theta)
+    ab.abcd_project_backward(ctx, theta, ab.camera(case.cam), None, torch.from_numpy(g2).cuda(), grads)
+    ctx.sync()
+    ref = oracle.project_backward(case.g, case.cam, g2.astype(np.float64))
+    clamp_near = np.any(np.abs(case.P["rgb_raw"]) < 1e-5, axis=1)
+    keep = ~clamp_near
+    for name, t in zip(("means", "log_scales", "quats", "opacity_logits", "sh"), grads.tensors()):
+        got = t.cpu().numpy()[keep]
+        r = ref[name][keep]
+        s = np.abs(r).max()
+        par.assert_grad_close(got, r, rtol=1e-3, atol=1e-5 * max(s, 1.0), what=name)
+
+
+def test_loss_matches_oracle(ctx):
+    for (H, W, lam, seed) in [(64, 64, 0.2, 1), (100, 150, 0.2, 2), (37, 53, 0.0, 3), (128, 96, 1.0, 4)]:
+        x = sg.random_image(H, W, 4, seed)
+        y = np.clip(x[..., :3] + sg.random_image(H, W, 3, seed + 50, -0.2, 0.2), 0, 1).astype(np.float32)
+        L, g = oracle.loss(x[..., :3].astype(np.float64), y.astype(np.float64), lam)
+        lt = torch.zeros(1, device="cuda")
+        gt = torch.empty(H, W, 3, device="cuda")
+        ab.abcd_loss(ctx, torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda(), W, H, lam, lt, gt)
+        ctx.sync()
+        assert abs(lt.item() - L) <= 1e-5 * abs(L), (H, W, lam, lt.item(), L)
+        got = gt.cpu().numpy().astype(np.float64)
+        tol = 1e-3 * np.abs(g) + 1e-6 * np.abs(g).max()
+        assert np.all(np.abs(got - g) <= tol), (H, W, lam, np.abs(got - g).max())
+
+
+@pytest.mark.parametrize("dtype,out_dtype,H,W,L", [("f16", "f16", 48, 64, 9), ("f16", "f16", 37, 29, 5),
+                                                    ("f32", "f32", 40, 40, 7), ("f16", "f32", 17, 33, 12)])
+def test_composite_cache_matches_oracle(ctx, dtype, out_dtype, H, W, L):
+    st = sg.premultiplied_layers(L, H, W, seed=L)
+    order = list(sg.random_permutation(L, seed=H))
+    ldt = np.float16 if dtype == "f16" else np.float32
+    layers_np = st.astype(ldt)
+    layers = [torch.from_numpy(layers_np[k]).cuda() for k in range(L)]
+    for split in (0, L // 2, L - 1, L):
+        odt = torch.float16 if out_dtype == "f16" else torch.float32
+        Fo = torch.empty(H, W, 4, dtype=odt, device="cuda")
+        Bo = torch.empty(H, W, 4, dtype=odt, device="cuda")
+        lay = list(layers)
+        if split < L:
+            lay[order[split]] = None        # the active partition's own layer is skipped
+        ab.abcd_composite_cache(ctx, lay, order, split, W, H, Fo, Bo,
+                                ab.ABCD_F16 if dtype == "f16" else ab.ABCD_F32,
+                                ab.ABCD_F16 if out_dtype == "f16" else ab.ABCD_F32)
+        ctx.sync()
+        src = layers_np.astype(np.float64)
+        Fr = oracle.composite_layers(src, order[:split]) if split > 0 else np.zeros((H, W, 4))
+        Br = oracle.composite_layers(src, order[split + 1:]) if split + 1 < L else np.zeros((H, W, 4))
+        for got, ref in ((Fo, Fr), (Bo, Br)):
+            g = got.cpu().numpy()
+            if out_dtype == "f32":
+                assert np.abs(g - ref).max() <= 1e-6
+            else:
+                # fp32 accumulation: each fold rounds a few times (<= L * 4 ulp of 1.0)
+                m = L * 4 * 2.0 ** -24
+                lo, hi = (ref - m).astype(np.float16), (ref + m).astype(np.float16)
+                assert np.all((g >= lo) & (g <= hi))
+                exact = lo == hi
+                assert np.all(g[exact] == ref.astype(np.float16)[exact])
+                assert exact.mean() > 0.99
+
+
+def test_adam_matches_oracle(ctx, ragged):
+    g = ragged.gaussians.subset(slice(0, 3001))
+    theta = ab.Gaussians.from_numpy(g)
+    rng = np.random.default_rng(9)
+    gr = [rng.normal(size=t.shape).astype(np.float32) for t in theta.tensors()]
+    grads = ab.Gaussians(*(torch.from_numpy(a).cuda() for a in gr), g.sh_degree)
+    m = ab.Gaussians.zeros_like(theta)
+    v = ab.Gaussians.zeros_like(theta)
+    lr = [1.6e-4, 5e-3, 1e-3, 0.025, 2.5e-3, 2.5e-3 / 20]
+    ref = [a.astype(np.float64).copy() for a in g.arrays()]
+    mr = [np.zeros_like(a) for a in ref]
+    vr = [np.zeros_like(a) for a in ref]
+    for step in (1, 2, 3):
+        ab.abcd_adam_active(ctx, theta, grads, m, v, lr, 0.9, 0.999, 1e-15, step)
+        for k in range(5):
+            if k < 4:
+                oracle.adam(ref[k], gr[k], mr[k], vr[k], lr[k], 0.9, 0.999, 1e-15, step)
+            else:   # SH: degree-0 coefficients and the rest have their own learning rates
+                for sl, l in ((np.s_[:, :1, :], lr[4]), (np.s_[:, 1:, :], lr[5])):
+                    a, mm, vv = (np.ascontiguousarray(x[sl]) for x in (ref[4], mr[4], vr[4]))
+                    oracle.adam(a, np.ascontiguousarray(gr[4][sl]), mm, vv, l, 0.9, 0.999, 1e-15, step)
+                    ref[4][sl], mr[4][sl], vr[4][sl] = a, mm, vv
+    ctx.sync()
+    for k, t in enumerate(theta.tensors()):
+        np.testing.assert_allclose(t.cpu().numpy(), ref[k], rtol=2e-6, atol=2e-7)
+
+
+def test_full_step_matches_oracle(ctx, tiny):
+    """project -> bin/sort -> render+composite -> L1 + 0.2 D-SSIM -> backward, one camera."""
+    case = Case(tiny, 1, fb=True)
+    H, W = case.cam.height, case.cam.width
+    tgt = sg.perturbed(tiny.gaussians, tiny.grid.side, seed=2002)
+    Pt = oracle.project(tgt, case.cam)
+    ot, it = oracle.tile_lists(Pt, W, H)
+    gt = oracle.render(oracle.SplatSet.from_proj(Pt), ot, it, W, H)["out"][..., :3].astype(np.float32)
+    r = run_forward(ctx, case)
+    loss = torch.zeros(1, device="cuda")
+    grads = ab.Gaussians.zeros_like(r["theta"])
+    ab.abcd_backward(ctx, r["theta"], r["cam"], None, r["proj"], r["tiles"], r["F"], r["B"],
+                     r["fbd"], None, r["out"], r["state"], torch.from_numpy(gt).cuda(), 0.2, loss,
+                     None, grads)
+    ctx.sync()
+    R = oracle.render(case.sp, case.off, case.ids, W, H, F=case.F64(), B=case.B64())
+    L, dL = oracle.loss(R["out"][..., :3], gt.astype(np.float64), 0.2)
+    assert abs(loss.item() - L) <= 1e-5 * L
+    g2 = oracle.backward(case.sp, case.off, case.ids, W, H, dL, F=case.F64(), B=case.B64())
+    ref = oracle.project_backward(case.g, case.cam, g2)
+    # Gaussians whose tiles hold an ambiguous pixel (or its 11x11 SSIM neighbourhood) may
+    # legitimately differ; require them to be few and check the rest element-wise.
+    flagged = R["n_ev"] > 0
+    tx, _ = oracle.tiles_xy(W, H)
+    for t in case.opt:
+        flagged[(t // tx) * 16:(t // tx) * 16 + 16, (t % tx) * 16:(t % tx) * 16 + 16] = True
+    touched = np.zeros(case.g.n, bool)
+    tiles_hit = set()
+    for y, x in zip(*np.nonzero(flagged)):
+        for dy in (-5, 0, 5):
+            for dx in (-5, 0, 5):
+                yy, xx = min(max(y + dy, 0), H - 1), min(max(x + dx, 0), W - 1)
+                tiles_hit.add((yy // 16) * tx + xx // 16)
+    for t in tiles_hit:
+        touched[case.ids[case.off[t]:case.off[t + 1]]] = True
+    assert touched.mean() < 0.2
+    keep = ~touched
+    for name, t in zip(("means", "log_scales", "quats", "opacity_logits", "sh"), grads.tensors()):
+        got = t.cpu().numpy()[keep]
+        rr = ref[name][keep]
+        # spec tolerance (1e-3 relative or 1e-5 absolute), with the absolute floor taken
+        # as 1e-5 of the group's largest gradient when that is smaller
+        atol = min(1e-5, 1e-5 * float(np.abs(ref[name]).max()))
+        par.assert_grad_close(got, rr, rtol=1e-3, atol=atol, what=name)
+
+
+def test_capacity_overflow_reported(ctx, tiny):
+    case = Case(tiny, 0, fb=False)
+    cam = ab.camera(case.cam)
+    theta = ab.Gaussians.from_numpy(case.g)
+    proj = ab.Projected.alloc(theta.n)
+    ab.abcd_project(ctx, theta, cam, None, proj)
+    tiles = ab.Tiles.alloc(100, case.cam.width, case.cam.height)
+    ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+    with pytest.raises(ab.AbcdError) as ei:
+        ctx.sync()
+    assert ei.value.status == ab.ABCD_ERR_CAPACITY
+    assert int(tiles.count.item()) == len(case.ids) or abs(int(tiles.count.item()) - len(case.ids)) <= \
+        sum(len(v) for v in case.opt.values())
+    assert int(tiles.ranges.abs().sum().item()) == 0
+    ctx.clear_status()
+    ctx.sync()
+
+
+def test_invalid_arguments_rejected(ctx):
+    cam = ab.abcd_camera()
+    cam.width = 0
+    theta = ab.Gaussians(*(torch.zeros(1, k, device="cuda") for k in (3, 3, 4, 1, 3)), 0)
+    theta.opacity_logits = torch.zeros(1, device="cuda")
+    with pytest.raises(ab.AbcdError) as ei:
+        ab.abcd_project(ctx, theta, cam, None, ab.Projected.alloc(1))
+    assert ei.value.status == ab.ABCD_ERR_INVALID_ARG
