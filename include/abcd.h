@@ -201,6 +201,23 @@ abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* layers, int L
                                  int layer_dtype, const int* order, int split, int width,
                                  int height, void* F_out, void* B_out, int out_dtype);
 
+/* The loss of abcd_loss without a context or workspace, for callers that cannot allocate
+ * device memory: code running inside a host application that owns every device allocation
+ * (its own pool or arena, with raw cudaMalloc forbidden), or a caller that must not allocate
+ * between set-up and a latency-critical loop.  The paper has no counterpart; it exists only
+ * for those callers.  Same arguments and results as abcd_loss, with an explicit stream.
+ * Its scratch (per-CTA partial sums and a completion counter, about 128 KB) is a static
+ * device array of this library, held by every GPU that loads the library until the process
+ * exits; images may have at most 16384 CTAs of 32x32 pixels (e.g. 4096 x 4096), larger ones
+ * return ABCD_ERR_WORKSPACE.  The first call on a device looks up the array's address (with
+ * that device current), so make it before any stream capture.  All calls on a device share
+ * the array: calls whose kernels overlap on the GPU race and give wrong losses, so order them
+ * (one stream, or events).  The counter is cleared at the start of every call.  Returns
+ * ABCD_ERR_INVALID_ARG for bad pointers, sizes or lambda, ABCD_ERR_CUDA if a launch fails. */
+abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba, const float* gt_rgb,
+                             int width, int height, float lambda_ssim, float* loss_out,
+                             float* dL_dout);
+
 /* ---- host-side partition logic (Section 2: regular grid, assignment by mean) --------- */
 
 /* cell[i] = linear id (i + gx (j + gy k)) of the grid cell holding means[i] (host array,

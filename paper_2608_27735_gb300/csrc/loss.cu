@@ -9,6 +9,8 @@
 // and windows them again: dSSIM_sum/dx(q) = (w*A)(q) + 2 x(q) (w*B)(q) + y(q) (w*C)(q).
 // The scalar is reduced deterministically: per-CTA partial sums, then the last CTA to finish
 // adds them in a fixed order (no waiting on other CTAs).
+#include <mutex>
+
 #include "abcd_internal.cuh"
 
 namespace abcd {
@@ -225,4 +227,65 @@ extern "C" abcd_status abcd_loss(abcd_ctx* ctx, const float* out_rgba, const flo
                                  float* dL_dout) {
   if (!ctx) return ABCD_ERR_INVALID_ARG;
   return abcd::loss_launch(ctx, out_rgba, gt_rgb, width, height, lambda_ssim, loss_out, dL_dout);
+}
+
+// ---------------------------------------------------------------------------------------
+// abcd_loss_static: the same loss kernel with its scratch in this file's static device array
+// instead of the context workspace, for callers that cannot allocate device memory.
+
+namespace abcd {
+namespace {
+
+constexpr int kStaticLossMaxBlocks = 16384;            // 32x32-pixel CTAs: up to 4096 x 4096
+constexpr int kStaticLossWords = 2 * kStaticLossMaxBlocks + 64;   // partial sums, then the ticket
+
+// Device scratch shared by every abcd_loss_static call on a device (held until exit).
+static __device__ __align__(256) unsigned g_loss_static_scratch[kStaticLossWords];
+
+constexpr int kMaxDevices = 256;
+std::mutex g_static_mu;
+unsigned* g_static_ptr[kMaxDevices] = {nullptr};
+
+// Device address of the static scratch on the current device, looked up once per device.
+cudaError_t static_scratch(int device, unsigned** out) {
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_loss_static_scratch);
+    if (e != cudaSuccess) return e;
+    g_static_ptr[device] = static_cast<unsigned*>(p);
+  }
+  *out = g_static_ptr[device];
+  return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace abcd
+
+extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba,
+                                        const float* gt_rgb, int width, int height,
+                                        float lambda_ssim, float* loss_out, float* dL_dout) {
+  using namespace abcd;
+  if (!out_rgba || !gt_rgb || width <= 0 || height <= 0 ||
+      !(lambda_ssim >= 0.f && lambda_ssim <= 1.f))
+    return ABCD_ERR_INVALID_ARG;
+  const dim3 grid((width + T - 1) / T, (height + T - 1) / T);
+  if ((long long)grid.x * grid.y > kStaticLossMaxBlocks) return ABCD_ERR_WORKSPACE;
+  int device = 0;
+  if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices)
+    return ABCD_ERR_CUDA;
+  unsigned* scratch = nullptr;
+  if (static_scratch(device, &scratch) != cudaSuccess) return ABCD_ERR_CUDA;
+  float* partials = reinterpret_cast<float*>(scratch);
+  unsigned* ticket = scratch + 2 * kStaticLossMaxBlocks;
+  cudaStream_t stream = (cudaStream_t)cuda_stream;
+  // the ticket must start at zero whatever an earlier (possibly failed) call left there
+  if (cudaMemsetAsync(ticket, 0, sizeof(unsigned), stream) != cudaSuccess) return ABCD_ERR_CUDA;
+  const size_t smem = sizeof(float) * kSmemFloats;
+  if (cudaFuncSetAttribute(loss_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+      cudaSuccess)
+    return ABCD_ERR_CUDA;
+  loss_kernel<<<grid, kThreads, smem, stream>>>(out_rgba, gt_rgb, width, height, lambda_ssim,
+                                                dL_dout, partials, ticket, loss_out);
+  return cudaGetLastError() == cudaSuccess ? ABCD_OK : ABCD_ERR_CUDA;
 }
