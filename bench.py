@@ -432,10 +432,12 @@ def run_ours(args):
     clk.start()
     time.sleep(0.3)
     l0 = st.ctx.launches()
+    torch.cuda.nvtx.range_push("abcd_timed")
     e0 = torch_event(torch, st.stream)
     for _ in range(args.steps):
         st.run_stage()
     e1 = torch_event(torch, st.stream)
+    torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
     barrier()
     launches = st.ctx.launches() - l0

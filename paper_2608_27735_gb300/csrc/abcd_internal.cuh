@@ -17,6 +17,7 @@ constexpr int kMaxRadixBlocks = 1024;     // upper bound used to size the histog
 constexpr int kLossTile = 32;             // loss output tile edge
 constexpr int kMaxLossBlocks = 1 << 16;
 constexpr int kMaxLayers = 256;
+constexpr long long kMaxDiffCells = 1LL << 20;   // (tiles_x + 1) * (tiles_y + 1)
 
 // Device status bits (OR-ed into the status word; abcd_sync reports the lowest set code).
 constexpr unsigned kStatusCapacity = 1u << ABCD_ERR_CAPACITY;
@@ -40,7 +41,10 @@ struct Workspace {
   unsigned* status;                 // [0] status word, [1] loss ticket
   unsigned long long* dsort[2];     // depth sort items [max_g]
   unsigned long long* pairs[2];     // (tile << 32 | id) items [max_pairs]
-  unsigned* hist;                   // [kRadixBins][kMaxRadixBlocks]
+  unsigned* hist;                   // [kRadixBins][kMaxRadixBlocks], then [kRadixBins] totals
+  int4* rects;                      // [max_g] tile rectangle per Gaussian
+  int* diff;                        // 2-D difference array over the tile grid
+  size_t diff_bytes;
   unsigned long long* block_sums;   // [kMaxRadixBlocks + 1]
   float* grad2d;                    // [max_g][9]
   float* dl_dout;                   // [max_pixels][3]

@@ -126,7 +126,10 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.dsort[1] = (unsigned long long*)take(8ull * (size_t)max_g);
   w.pairs[0] = (unsigned long long*)take(8ull * (size_t)max_pairs);
   w.pairs[1] = (unsigned long long*)take(8ull * (size_t)max_pairs);
-  w.hist = (unsigned*)take(4ull * kRadixBins * kMaxRadixBlocks);
+  w.hist = (unsigned*)take(4ull * kRadixBins * (kMaxRadixBlocks + 1));
+  w.rects = (int4*)take(16ull * (size_t)max_g);
+  w.diff_bytes = 4ull * kMaxDiffCells;
+  w.diff = (int*)take(w.diff_bytes);
   w.block_sums = (unsigned long long*)take(8ull * (kMaxRadixBlocks + 1));
   w.grad2d = (float*)take(4ull * 9 * (size_t)max_g);
   w.dl_dout = (float*)take(4ull * 3 * (size_t)max_pixels);
