@@ -6,11 +6,15 @@
 // frozen partitions enter through out = F over (A over B) (Section 2), over meaning
 // X + (1 - X.a) Y on premultiplied RGBA, and out.rgb += (1 - out.a) bg.
 //
-// One CTA per 16x16 tile, one thread per pixel; batches of 256 list entries are staged in
-// shared memory; a CTA leaves as soon as every pixel has terminated (__syncthreads_count),
-// a warp as soon as its lanes have.  Every quantity that decides a branch (sigma, alpha, T)
-// is computed with explicit round-to-nearest intrinsics in one shared function, so the
-// backward kernel retraces exactly the forward's contributors.
+// One CTA per 8x8 block of pixels (four per 16x16 binning tile), one thread per pixel, so the
+// few heavily covered tiles of a small active block spread over four times as many CTAs and
+// each CTA stops as soon as its own 64 pixels have terminated (__syncthreads_count).  List
+// entries are staged 256 at a time in shared memory; while staging, an entry whose opacity
+// cannot reach alpha_min anywhere on the CTA's pixel-centre box (analytic minimum of the
+// quadratic form over the box, with a margin far above fp32 rounding) is dropped: every pixel
+// would skip it, so results are unchanged.  Every quantity that decides a branch per pixel
+// (sigma, alpha, T) is computed with explicit round-to-nearest intrinsics in one shared
+// function, so the backward kernel retraces exactly the forward's contributors.
 #include "abcd_internal.cuh"
 
 namespace abcd {
@@ -36,6 +40,39 @@ __device__ __forceinline__ float sigma2(float4 s, float2 m, float fx, float fy, 
   dx = __fsub_rn(fx, m.x);
   dy = __fsub_rn(fy, m.y);
   return __fmaf_rn(dx, __fmaf_rn(s.x, dx, __fmul_rn(s.y, dy)), __fmul_rn(__fmul_rn(s.z, dy), dy));
+}
+
+constexpr int kSub = 8;                          // CTA pixel block edge
+constexpr int kSubThreads = kSub * kSub;         // 64
+constexpr int kSubPerTile = (kTile / kSub) * (kTile / kSub);
+constexpr int kRounds = 4;                       // list entries per thread per batch
+constexpr int kBatch = kSubThreads * kRounds;    // 256
+
+// Lower bound of sigma * log2(e) over the box [X0, X1] x [Y0, Y1] of offsets d = pixel - uv:
+// 0 if the box contains d = 0, else the least value on its four edges (convex quadratic).
+__device__ __forceinline__ float box_min_sigma2(float4 s, float X0, float X1, float Y0, float Y1) {
+  if (X0 <= 0.f && X1 >= 0.f && Y0 <= 0.f && Y1 >= 0.f) return 0.f;
+  float best = 3.0e38f;
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const float X = e ? X1 : X0;
+    const float dy = fminf(fmaxf(-s.y * X / (2.f * s.z), Y0), Y1);
+    best = fminf(best, X * (s.x * X + s.y * dy) + s.z * dy * dy);
+    const float Y = e ? Y1 : Y0;
+    const float dx = fminf(fmaxf(-s.y * Y / (2.f * s.x), X0), X1);
+    best = fminf(best, dx * (s.x * dx + s.y * Y) + s.z * Y * Y);
+  }
+  return best;
+}
+
+// True when no pixel centre of the CTA's box can give alpha >= alpha_min: alpha = o 2^-sigma'
+// < alpha_min needs sigma' > log2(o / alpha_min); the margin (0.02 + 0.2% in log2 units) is
+// orders of magnitude above the fp32 error of either evaluation.
+__device__ __forceinline__ bool cull(float4 s, float2 m, float bx0, float by0, float alpha_min) {
+  if (!(s.w >= alpha_min)) return true;
+  const float thr = __log2f(s.w / alpha_min);
+  const float lo = box_min_sigma2(s, bx0 - m.x, bx0 + (kSub - 1) - m.x, by0 - m.y, by0 + (kSub - 1) - m.y);
+  return lo * 0.998f > thr + 0.02f;
 }
 
 __device__ __forceinline__ float4 load_px(const void* img, int dtype, long long p) {
@@ -67,49 +104,91 @@ struct FwdArgs {
   uint2* refresh;      // fp16 x4 per pixel
 };
 
-__global__ void __launch_bounds__(kTileThreads) render_fwd_kernel(FwdArgs a) {
-  __shared__ float2 s_uv[kTileThreads];
-  __shared__ float4 s_co[kTileThreads];
-  __shared__ float4 s_rgb[kTileThreads];
-  const int tile = blockIdx.x;
+// Stages one batch of list entries (positions base .. base + kBatch) and compacts the indices
+// of the entries that survive the CTA-box cull into s_idx; returns the number of survivors.
+template <bool WITH_ID>
+__device__ __forceinline__ int stage_batch(const unsigned* ids, unsigned start, int n, int base,
+                                           const float2* uv, const float4* co, const float* rgb,
+                                           float bx0, float by0, float alpha_min, float2* s_uv,
+                                           float4* s_co, float4* s_rgb, unsigned* s_id,
+                                           unsigned short* s_idx, unsigned* s_ballot) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  bool keep[kRounds];
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const int q = threadIdx.x + r * kSubThreads;
+    keep[r] = false;
+    if (base + q < n) {
+      const unsigned g = ids[start + base + q];
+      const float2 m = uv[g];
+      const float4 sc = scaled_conic(co[g]);
+      keep[r] = !cull(sc, m, bx0, by0, alpha_min);
+      if (keep[r]) {
+        s_uv[q] = m;
+        s_co[q] = sc;
+        s_rgb[q] = make_float4(rgb[3 * g], rgb[3 * g + 1], rgb[3 * g + 2], 0.f);
+        if (WITH_ID) s_id[q] = g;
+      }
+    }
+    const unsigned b = __ballot_sync(0xffffffffu, keep[r]);
+    if (lane == 0) s_ballot[r * 2 + w] = b;
+  }
+  __syncthreads();
+  int total = 0, before_r = 0;
+  const unsigned lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int r = 0; r < kRounds; ++r) {
+    const unsigned b0 = s_ballot[2 * r], b1 = s_ballot[2 * r + 1];
+    const int at = before_r + (w ? __popc(b0) : 0) + __popc((w ? b1 : b0) & lt);
+    if (keep[r]) s_idx[at] = (unsigned short)(threadIdx.x + r * kSubThreads);
+    before_r += __popc(b0) + __popc(b1);
+  }
+  total = before_r;
+  __syncthreads();
+  return total;
+}
+
+__global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
+  __shared__ float2 s_uv[kBatch];
+  __shared__ float4 s_co[kBatch];
+  __shared__ float4 s_rgb[kBatch];
+  __shared__ unsigned short s_idx[kBatch];
+  __shared__ unsigned s_ballot[2 * kRounds];
+  const int tile = blockIdx.x / kSubPerTile, sub = blockIdx.x % kSubPerTile;
   const int tx = tile % a.cam.tiles_x, ty = tile / a.cam.tiles_x;
-  const int px = tx * kTile + (threadIdx.x & (kTile - 1));
-  const int py = ty * kTile + (threadIdx.x / kTile);
+  const int px0 = tx * kTile + (sub % (kTile / kSub)) * kSub;
+  const int py0 = ty * kTile + (sub / (kTile / kSub)) * kSub;
+  const int px = px0 + (threadIdx.x % kSub), py = py0 + (threadIdx.x / kSub);
   const bool inside = px < a.cam.width && py < a.cam.height;
   const uint2 rg = a.ranges[tile];
   const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
   const float fx = (float)px + 0.5f, fy = (float)py + 0.5f;
+  const float bx0 = (float)px0 + 0.5f, by0 = (float)py0 + 0.5f;
   float T = 1.f, c0 = 0.f, c1 = 0.f, c2 = 0.f;
   unsigned last = 0;
   bool done = !inside;
-  for (int base = 0; base < n; base += kTileThreads) {
-    if (__syncthreads_count(done) == kTileThreads) break;
-    const int k = base + threadIdx.x;
-    if (k < n) {
-      const unsigned g = a.ids[rg.x + k];
-      s_uv[threadIdx.x] = a.uv[g];
-      s_co[threadIdx.x] = scaled_conic(a.co[g]);
-      s_rgb[threadIdx.x] = make_float4(a.rgb[3 * g], a.rgb[3 * g + 1], a.rgb[3 * g + 2], 0.f);
-    }
-    __syncthreads();
-    const int cnt = min(kTileThreads, n - base);
+  for (int base = 0; base < n; base += kBatch) {
+    if (__syncthreads_count(done) == kSubThreads) break;
+    const int cnt = stage_batch<false>(a.ids, rg.x, n, base, a.uv, a.co, a.rgb, bx0, by0,
+                                       a.op.alpha_min, s_uv, s_co, s_rgb, nullptr, s_idx, s_ballot);
     if (!done) {
       for (int j = 0; j < cnt; ++j) {
+        const int q = s_idx[j];
         float dx, dy;
-        const float4 s = s_co[j];
-        const float sig = sigma2(s, s_uv[j], fx, fy, dx, dy);
+        const float4 s = s_co[q];
+        const float sig = sigma2(s, s_uv[q], fx, fy, dx, dy);
         if (!(sig >= 0.f)) continue;
         const float alpha = fminf(a.op.alpha_max, __fmul_rn(s.w, ex2_approx(-sig)));
         if (alpha < a.op.alpha_min) continue;
         const float test = __fmul_rn(T, __fsub_rn(1.f, alpha));
         if (test < a.op.t_min) { done = true; break; }
         const float w = __fmul_rn(alpha, T);
-        const float4 col = s_rgb[j];
+        const float4 col = s_rgb[q];
         c0 = __fmaf_rn(w, col.x, c0);
         c1 = __fmaf_rn(w, col.y, c1);
         c2 = __fmaf_rn(w, col.z, c2);
         T = test;
-        last = (unsigned)(base + j + 1);
+        last = (unsigned)(base + q + 1);
       }
     }
   }
@@ -160,21 +239,25 @@ struct BwdArgs {
   float* grad2d;
 };
 
-__global__ void __launch_bounds__(kTileThreads) render_bwd_kernel(BwdArgs a) {
-  __shared__ float2 s_uv[kTileThreads];
-  __shared__ float4 s_co[kTileThreads];
-  __shared__ float4 s_rgb[kTileThreads];
-  __shared__ unsigned s_id[kTileThreads];
+__global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
+  __shared__ float2 s_uv[kBatch];
+  __shared__ float4 s_co[kBatch];
+  __shared__ float4 s_rgb[kBatch];
+  __shared__ unsigned s_id[kBatch];
+  __shared__ unsigned short s_idx[kBatch];
+  __shared__ unsigned s_ballot[2 * kRounds];
   __shared__ unsigned s_max;
-  const int tile = blockIdx.x;
+  const int tile = blockIdx.x / kSubPerTile, sub = blockIdx.x % kSubPerTile;
   const int tx = tile % a.cam.tiles_x, ty = tile / a.cam.tiles_x;
-  const int px = tx * kTile + (threadIdx.x & (kTile - 1));
-  const int py = ty * kTile + (threadIdx.x / kTile);
+  const int px0 = tx * kTile + (sub % (kTile / kSub)) * kSub;
+  const int py0 = ty * kTile + (sub / (kTile / kSub)) * kSub;
+  const int px = px0 + (threadIdx.x % kSub), py = py0 + (threadIdx.x / kSub);
   const int lane = threadIdx.x & 31;
   const bool inside = px < a.cam.width && py < a.cam.height;
   const uint2 rg = a.ranges[tile];
   const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
   const float fx = (float)px + 0.5f, fy = (float)py + 0.5f;
+  const float bx0 = (float)px0 + 0.5f, by0 = (float)py0 + 0.5f;
   unsigned last = 0;
   float Gr = 0.f, Gg = 0.f, Gb = 0.f, Ga = 0.f, Tf = 1.f, A0 = 0.f, A1 = 0.f, A2 = 0.f;
   if (inside) {
@@ -198,34 +281,27 @@ __global__ void __launch_bounds__(kTileThreads) render_bwd_kernel(BwdArgs a) {
   __syncthreads();
   const int span = (int)s_max;
   float T = 1.f, c0 = 0.f, c1 = 0.f, c2 = 0.f;
-  for (int base = 0; base < span; base += kTileThreads) {
+  for (int base = 0; base < span; base += kBatch) {
     __syncthreads();
-    const int k = base + threadIdx.x;
-    if (k < span) {
-      const unsigned g = a.ids[rg.x + k];
-      s_id[threadIdx.x] = g;
-      s_uv[threadIdx.x] = a.uv[g];
-      s_co[threadIdx.x] = scaled_conic(a.co[g]);
-      s_rgb[threadIdx.x] = make_float4(a.rgb[3 * g], a.rgb[3 * g + 1], a.rgb[3 * g + 2], 0.f);
-    }
-    __syncthreads();
-    const int cnt = min(kTileThreads, span - base);
+    const int cnt = stage_batch<true>(a.ids, rg.x, span, base, a.uv, a.co, a.rgb, bx0, by0,
+                                      a.op.alpha_min, s_uv, s_co, s_rgb, s_id, s_idx, s_ballot);
     for (int j = 0; j < cnt; ++j) {
+      const int q = s_idx[j];
       float v[9];
 #pragma unroll
-      for (int q = 0; q < 9; ++q) v[q] = 0.f;
+      for (int k = 0; k < 9; ++k) v[k] = 0.f;
       bool contrib = false;
-      if ((unsigned)(base + j) < last) {
+      if ((unsigned)(base + q) < last) {
         float dx, dy;
-        const float4 s = s_co[j];
-        const float sig = sigma2(s, s_uv[j], fx, fy, dx, dy);
+        const float4 s = s_co[q];
+        const float sig = sigma2(s, s_uv[q], fx, fy, dx, dy);
         if (sig >= 0.f) {
           const float G = ex2_approx(-sig);
           const float raw = __fmul_rn(s.w, G);
           const float alpha = fminf(a.op.alpha_max, raw);
           if (alpha >= a.op.alpha_min) {
             contrib = true;
-            const float4 col = s_rgb[j];
+            const float4 col = s_rgb[q];
             const float w = __fmul_rn(alpha, T);
             c0 = __fmaf_rn(w, col.x, c0);
             c1 = __fmaf_rn(w, col.y, c1);
@@ -252,13 +328,13 @@ __global__ void __launch_bounds__(kTileThreads) render_bwd_kernel(BwdArgs a) {
       }
       if (__any_sync(0xffffffffu, contrib)) {
 #pragma unroll
-        for (int q = 0; q < 9; ++q)
+        for (int k = 0; k < 9; ++k)
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) v[q] += __shfl_xor_sync(0xffffffffu, v[q], o);
+          for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
         float mine = 0.f;
 #pragma unroll
-        for (int q = 0; q < 9; ++q) mine = (lane == q) ? v[q] : mine;
-        if (lane < 9) atomicAdd(&a.grad2d[9 * (size_t)s_id[j] + lane], mine);
+        for (int k = 0; k < 9; ++k) mine = (lane == k) ? v[k] : mine;
+        if (lane < 9) atomicAdd(&a.grad2d[9 * (size_t)s_id[q] + lane], mine);
       }
     }
   }
@@ -311,7 +387,7 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.n_last = state ? state->n_last : nullptr;
   a.refresh = (uint2*)refresh_f16;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y;
-  render_fwd_kernel<<<n_tiles, kTileThreads, 0, ctx->stream>>>(a);
+  render_fwd_kernel<<<n_tiles * kSubPerTile, kSubThreads, 0, ctx->stream>>>(a);
   return check_launch(ctx, "render_fwd_kernel");
 }
 
@@ -346,6 +422,6 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   a.dl_dout = dL_dout;
   a.grad2d = grad2d;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y;
-  render_bwd_kernel<<<n_tiles, kTileThreads, 0, ctx->stream>>>(a);
+  render_bwd_kernel<<<n_tiles * kSubPerTile, kSubThreads, 0, ctx->stream>>>(a);
   return check_launch(ctx, "render_bwd_kernel");
 }
