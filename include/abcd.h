@@ -83,8 +83,8 @@ typedef struct {
 } abcd_projected;
 
 /* Per-tile Gaussian lists (device).  For tile t = ty * tiles_x + tx (16x16 tiles,
- * tiles_x = ceil(W/16)), ids[ranges[2t] .. ranges[2t+1]) are the Gaussians whose square
- * meets the tile, front to back by (fp32 depth, id). */
+ * tiles_x = ceil(W/16)), ids[ranges[2t] .. ranges[2t+1]) are the Gaussians listed on the tile
+ * (see abcd_bin_sort), front to back by (fp32 depth, id). */
 typedef struct {
   unsigned* ids;         /* [capacity] */
   unsigned* ranges;      /* [tiles_x * tiles_y][2] */
@@ -130,11 +130,15 @@ long long abcd_launch_count(const abcd_ctx* ctx);
 abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_camera* cam,
                          const abcd_render_opts* opts, abcd_projected* out);
 
-/* K3 + K4. Tile binning and depth sort: every visible Gaussian is listed in each tile its
- * square [u-r, u+r] x [v-r, v+r] meets; lists are ordered by the fp32 depth, ties by id.
- * n must equal the n given to abcd_project. */
+/* K3 + K4. Tile binning and depth sort: a visible Gaussian is listed in each tile its square
+ * [u-r, u+r] x [v-r, v+r] meets on which it can reach alpha >= alpha_min (the least sigma over
+ * the box of the tile's pixel centres is at most ln(opacity / alpha_min), tested with a margin
+ * of about 0.7% in sigma, so a list may hold a few entries that every pixel of the tile
+ * skips); lists are ordered by the fp32 depth, ties by id.  Leaving out the tiles on which
+ * every pixel would skip the Gaussian does not change any pixel.  n must equal the n given
+ * to abcd_project; opts as there (NULL = defaults; alpha_min is used). */
 abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, int n,
-                          const abcd_camera* cam, abcd_tiles* out);
+                          const abcd_camera* cam, const abcd_render_opts* opts, abcd_tiles* out);
 
 /* K5. Front-to-back blend of the active block per pixel (alpha = min(alpha_max,
  * o exp(-sigma)), skip alpha < alpha_min, stop before T < t_min), giving the premultiplied

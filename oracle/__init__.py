@@ -82,6 +82,9 @@ def lib():
         if _lib is None:
             _lib = C.CDLL(build())
             _lib.orc_tile_lists.restype = C.c_longlong
+            _lib.orc_box_min_sigma.restype = C.c_double
+            _lib.orc_box_min_sigma.argtypes = [C.c_void_p, C.c_double, C.c_double, C.c_double,
+                                               C.c_double]
             _lib.orc_sh_basis.restype = C.c_double
             _lib.orc_sh_basis.argtypes = [C.c_int, C.c_int, C.c_double, C.c_double, C.c_double]
     return _lib
@@ -162,8 +165,10 @@ def tiles_xy(width, height, tile=16):
     return (width + tile - 1) // tile, (height + tile - 1) // tile
 
 
-def tile_lists(proj, width, height, tile=16):
-    """Returns (offsets[n_tiles + 1] int64, ids[K] int32)."""
+def tile_lists(proj, width, height, tile=16, rule="alpha", alpha_min=1.0 / 255.0):
+    """Returns (offsets[n_tiles + 1] int64, ids[K] int32).  rule="alpha" keeps a tile of the
+    3-sigma square only where the Gaussian can reach alpha_min (the renderer's listing rule);
+    rule="square" keeps the whole square (3DGS)."""
     tx, ty = tiles_xy(width, height, tile)
     vis = np.ascontiguousarray(proj["visible"], dtype=np.int32)
     rect = np.ascontiguousarray(proj["rect"], dtype=np.int32)
@@ -173,10 +178,17 @@ def tile_lists(proj, width, height, tile=16):
                      np.maximum(rect[:, 3] - rect[:, 1], 0)))
     offsets = np.zeros(tx * ty + 1, np.int64)
     ids = np.zeros(max(cap, 1), np.int32)
+    sp = SplatSet.from_proj(proj) if rule == "alpha" else None
     K = lib().orc_tile_lists(n, _p(vis), _p(rect), _p(key), tx, ty, _p(offsets), _p(ids),
-                             C.c_longlong(cap))
-    assert K == cap, (K, cap)
+                             C.c_longlong(cap), C.byref(sp.s) if sp is not None else None,
+                             C.c_double(alpha_min), int(tile))
+    assert 0 <= K <= cap, (K, cap)
     return offsets, ids[:K]
+
+
+def box_min_sigma(conic, X0, X1, Y0, Y1):
+    q = _f64(conic)
+    return lib().orc_box_min_sigma(_p(q), float(X0), float(X1), float(Y0), float(Y1))
 
 
 class SplatSet:

@@ -450,16 +450,42 @@ int orc_project_backward(const orc_gaussians* g, const orc_camera* cam, const or
   return 0;
 }
 
+double orc_box_min_sigma(const double* q, double X0, double X1, double Y0, double Y1) {
+  if (X0 <= 0.0 && X1 >= 0.0 && Y0 <= 0.0 && Y1 >= 0.0) return 0.0;
+  auto sig = [q](double dx, double dy) { return 0.5 * (q[0] * dx * dx + q[2] * dy * dy) + q[1] * dx * dy; };
+  double best = HUGE_VAL;
+  for (double X : {X0, X1}) {          // edge dx = X: d sigma / d dy = b X + c dy = 0
+    const double dy = std::min(std::max(-q[1] * X / q[2], Y0), Y1);
+    best = std::min(best, sig(X, dy));
+  }
+  for (double Y : {Y0, Y1}) {          // edge dy = Y: a dx + b Y = 0
+    const double dx = std::min(std::max(-q[1] * Y / q[0], X0), X1);
+    best = std::min(best, sig(dx, Y));
+  }
+  return best;
+}
+
 long long orc_tile_lists(int n, const int* visible, const int* rect, const unsigned* depth_key,
                          int tiles_x, int tiles_y, long long* offsets, int* ids,
-                         long long capacity) {
+                         long long capacity, const orc_splats* s, double alpha_min, int tile) {
   struct Item { long long tile; unsigned key; int id; };
   std::vector<Item> items;
   for (int i = 0; i < n; ++i) {
     if (!visible[i]) continue;
     const int* r = rect + 4 * i;
     for (int y = r[1]; y < r[3]; ++y)
-      for (int x = r[0]; x < r[2]; ++x) items.push_back(Item{(long long)y * tiles_x + x, depth_key[i], i});
+      for (int x = r[0]; x < r[2]; ++x) {
+        if (s) {
+          const double o = s->opacity[i];
+          if (!(o >= alpha_min)) continue;
+          const double u = s->uv[2 * i], v = s->uv[2 * i + 1];
+          const double m = orc_box_min_sigma(s->conic + 3 * i, x * tile + 0.5 - u,
+                                             x * tile + tile - 0.5 - u, y * tile + 0.5 - v,
+                                             y * tile + tile - 0.5 - v);
+          if (m > std::log(o / alpha_min)) continue;
+        }
+        items.push_back(Item{(long long)y * tiles_x + x, depth_key[i], i});
+      }
   }
   std::stable_sort(items.begin(), items.end(), [](const Item& a, const Item& b) {
     if (a.tile != b.tile) return a.tile < b.tile;

@@ -17,7 +17,8 @@
  * Parity status per function (what pins it; see tests/test_oracle_*.py):
  *   orc_project            single-Gaussian closed form, SH vs scipy, brute-force rect
  *   orc_project_backward   central finite differences (fp64)
- *   orc_tile_lists         brute-force per-tile scan + Python sort
+ *   orc_tile_lists         brute-force per-tile scan + Python sort; listing rule against the
+ *                          square rule (identical images) and dense box sampling
  *   orc_render_pixel/image closed form, invariants, associativity identity
  *   orc_backward_pixel/... central finite differences (fp64), incl. the F/B alpha term
  *   orc_composite_layers   constant-layer closed form, split invariance
@@ -59,6 +60,14 @@ typedef struct {
   int sh_degree;                /* 0..3 */
 } orc_gaussians;
 
+typedef struct {               /* screen-space splats the per-pixel renderer reads */
+  int n;
+  const double* uv;            /* [n][2] */
+  const double* conic;         /* [n][3] */
+  const double* opacity;       /* [n] */
+  const double* rgb;           /* [n][3] */
+} orc_splats;
+
 typedef struct {
   int* visible;             /* [n] 1 if z > near and the tile rectangle is non-empty */
   double* depth;            /* [n] camera-space z */
@@ -75,13 +84,6 @@ typedef struct {
   double* view_tan;         /* [n][2] x/z and y/z (to locate the guard clamp) */
 } orc_projected;
 
-typedef struct {               /* screen-space splats the per-pixel renderer reads */
-  int n;
-  const double* uv;            /* [n][2] */
-  const double* conic;         /* [n][3] */
-  const double* opacity;       /* [n] */
-  const double* rgb;           /* [n][3] */
-} orc_splats;
 
 /* Uncertainty model used only to REPORT decisions of the blend loop that lie so close to
  * their threshold that an fp32 implementation may take either branch.  NULL = no events. */
@@ -108,10 +110,18 @@ int orc_project_backward(const orc_gaussians* g, const orc_camera* cam, const or
 
 /* Stable sort of (tile, depth_key) over all visible Gaussians emitted in id order.
  * offsets has n_tiles+1 entries; ids has capacity entries.  Returns K (or -K-1 if
- * K > capacity; nothing is written then). */
+ * K > capacity; nothing is written then).
+ * Listing rule: tile t of Gaussian i's rectangle is kept when s (uv, conic, opacity) is NULL,
+ * else only if the Gaussian can reach alpha >= alpha_min on t: o >= alpha_min and the minimum
+ * of sigma over the box of t's pixel centres [16 tx + 0.5, 16 tx + 15.5] x [...] is
+ * <= ln(o / alpha_min).  Dropped entries are skipped by every pixel of t anyway. */
 long long orc_tile_lists(int n, const int* visible, const int* rect, const unsigned* depth_key,
                          int tiles_x, int tiles_y, long long* offsets, int* ids,
-                         long long capacity);
+                         long long capacity, const orc_splats* s, double alpha_min, int tile);
+
+/* Minimum of sigma(d) = 1/2 (a dx^2 + c dy^2) + b dx dy over the box [X0, X1] x [Y0, Y1]
+ * (convex: 0 if the box holds d = 0, else the least value on its four edges). */
+double orc_box_min_sigma(const double* conic, double X0, double X1, double Y0, double Y1);
 
 /* One pixel: front-to-back blend of list[0..len) then F over (A over B), + (1-out.a)*bg.
  * F, B: 4 doubles (premultiplied RGBA) or NULL (transparent).  toggles: n_toggles pairs

@@ -76,7 +76,7 @@ _SIGS = {
     "abcd_sync": [C.c_void_p],
     "abcd_clear_status": [C.c_void_p],
     "abcd_project": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p],
-    "abcd_bin_sort": [C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p],
+    "abcd_bin_sort": [C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p],
     "abcd_render_composite_fwd": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                   C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p,
                                   C.c_void_p, C.c_void_p],
@@ -318,9 +318,10 @@ def abcd_project(ctx: Context, theta: Gaussians, cam: abcd_camera, opts, out: Pr
     ctx.check(lib().abcd_project(ctx.h, C.byref(g), C.byref(cam), _opt(opts), C.byref(o)))
 
 
-def abcd_bin_sort(ctx: Context, proj: Projected, n: int, cam: abcd_camera, out: Tiles):
+def abcd_bin_sort(ctx: Context, proj: Projected, n: int, cam: abcd_camera, out: Tiles,
+                  opts=None):
     p = proj.c(); t = out.c()
-    ctx.check(lib().abcd_bin_sort(ctx.h, C.byref(p), int(n), C.byref(cam), C.byref(t)))
+    ctx.check(lib().abcd_bin_sort(ctx.h, C.byref(p), int(n), C.byref(cam), _opt(opts), C.byref(t)))
 
 
 def _bg(bg):

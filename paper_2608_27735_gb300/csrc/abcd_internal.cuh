@@ -43,6 +43,7 @@ struct Workspace {
   unsigned long long* pairs[2];     // (tile << 32 | id) items [max_pairs]
   unsigned* hist;                   // [kRadixBins][kMaxRadixBlocks], then [kRadixBins] totals
   int4* rects;                      // [max_g] tile rectangle per Gaussian
+  unsigned* counts;                 // [max_g] listed tiles per Gaussian
   int* diff;                        // 2-D difference array over the tile grid
   size_t diff_bytes;
   unsigned long long* block_sums;   // [kMaxRadixBlocks + 1]

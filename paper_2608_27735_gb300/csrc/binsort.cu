@@ -1,17 +1,23 @@
 // K3 (tile binning) and K4 (sort + tile ranges) of the ABCD active-block step.
 //
 // What is computed (3DGS binning, Section 1 of the paper by citation): every visible Gaussian
-// is listed in each 16x16 tile met by its square [u-r, u+r] x [v-r, v+r]; each tile's list
-// is ordered front to back by (fp32 depth, Gaussian id).
+// is listed in each 16x16 tile met by its square [u-r, u+r] x [v-r, v+r] on which it can
+// reach alpha >= alpha_min (the least sigma over the tile's pixel-centre box is at most
+// ln(o / alpha_min), tested with a small margin, so the lists may hold a few more entries
+// than the exact rule; every pixel skips those); each tile's list is ordered front to back by
+// (fp32 depth, Gaussian id).  Dropping the tiles every pixel would skip leaves the image
+// unchanged and halves the pairs to sort and to walk.
 //
 // How (GB300 design, different from sorting 64-bit (tile | depth) keys):
-//   1. per Gaussian: its tile rectangle (kept in the workspace), a sort key (fp32 depth bits,
-//      all ones when culled) and +-1 at the rectangle's four corners of a 2-D difference
-//      array over the tile grid;
+//   1. per Gaussian: its tile rectangle (kept in the workspace) and a sort key (fp32 depth
+//      bits, all ones when culled); then, one warp per Gaussian, one lane per tile row: the
+//      contiguous run of kept tiles in that row (the kept set is convex), the Gaussian's pair
+//      count, and +-1 at the run's ends in a per-row difference array over the tile grid;
 //   2. stable LSD radix sort of the n Gaussians by the 32 depth bits;
-//   3. exclusive scan of the rectangle areas in that order: K = total pairs; the 2-D prefix
-//      sum of the difference array gives every tile's pair count, hence its range;
-//   4. warp-cooperative emission of (tile << 32 | id) items in depth order;
+//   3. exclusive scan of the pair counts in that order: K = total pairs; the row prefix sums
+//      of the difference array give every tile's pair count, hence its range;
+//   4. emission of (tile << 32 | id) items in depth order (the runs are recomputed with the
+//      same round-to-nearest arithmetic, so they match step 1 bit for bit);
 //   5. stable LSD radix sort of the K items on the tile bits only (ceil(log2 n_tiles) <= 16
 //      bits, 8 per pass), which keeps depth order inside each tile; the last pass writes ids.
 // Radix passes are reduce-then-scan (per-block digit counts, per-digit row scans, stable
@@ -49,10 +55,10 @@ __device__ __forceinline__ int4 tile_rect(float2 m, int r, int tiles_x, int tile
   return q;
 }
 
-// ---- per Gaussian: depth key (bits(depth) << 32 | id, all ones when culled), tile
-// rectangle, and the rectangle's corners in the (tiles_y + 1) x (tiles_x + 1) difference array
+// ---- per Gaussian: depth key (bits(depth) << 32 | id, all ones when culled) and the tile
+// rectangle of its square
 __global__ void keys_rects_kernel(const float* depth, const int* radius, const float2* uv, int n,
-                                  int tiles_x, int tiles_y, u64* items, int4* rects, int* diff) {
+                                  int tiles_x, int tiles_y, u64* items, int4* rects) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   int4 q = make_int4(0, 0, 0, 0);
@@ -63,12 +69,95 @@ __global__ void keys_rects_kernel(const float* depth, const int* radius, const f
   rects[i] = q;
   const unsigned key = vis ? __float_as_uint(depth[i]) : 0xFFFFFFFFu;
   items[i] = ((u64)key << 32) | (unsigned)i;
-  if (vis) {
-    const int W1 = tiles_x + 1;
-    atomicAdd(&diff[q.y * W1 + q.x], 1);
-    atomicAdd(&diff[q.y * W1 + q.z], -1);
-    atomicAdd(&diff[q.w * W1 + q.x], -1);
-    atomicAdd(&diff[q.w * W1 + q.z], 1);
+}
+
+// Least sigma * log2(e) over the offset box [X0, X1] x [Y0, Y1] (convex quadratic with the
+// log2-scaled conic s = (a/2, b, c/2) log2 e): 0 if the box holds 0, else the least value on
+// its edges (the edge minimiser is clamped into the edge; r_a = -b / (2 a'), r_c = -b / (2 c')
+// are precomputed per Gaussian).  Round-to-nearest intrinsics only, so every kernel gets the
+// same bits.
+__device__ __forceinline__ float box_min_rn(float ha, float hb, float hc, float ra, float rc,
+                                            float X0, float X1, float Y0, float Y1) {
+  if (X0 <= 0.f && X1 >= 0.f && Y0 <= 0.f && Y1 >= 0.f) return 0.f;
+  float best = 3.0e38f;
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const float X = e ? X1 : X0;
+    const float dy = fminf(fmaxf(__fmul_rn(rc, X), Y0), Y1);
+    best = fminf(best, __fmaf_rn(X, __fmaf_rn(ha, X, __fmul_rn(hb, dy)), __fmul_rn(__fmul_rn(hc, dy), dy)));
+    const float Y = e ? Y1 : Y0;
+    const float dx = fminf(fmaxf(__fmul_rn(ra, Y), X0), X1);
+    best = fminf(best, __fmaf_rn(dx, __fmaf_rn(ha, dx, __fmul_rn(hb, Y)), __fmul_rn(__fmul_rn(hc, Y), Y)));
+  }
+  return best;
+}
+
+struct Splat {
+  float u, v, ha, hb, hc, ra, rc, lim;   // lim: keep a tile when its least sigma' <= lim
+};
+
+__device__ __forceinline__ Splat load_splat(const float2* uv, const float4* co, unsigned g,
+                                            float alpha_min) {
+  const float2 m = uv[g];
+  const float4 c = co[g];
+  Splat s;
+  s.u = m.x; s.v = m.y;
+  s.ha = __fmul_rn(0.7213475204444817f, c.x);   // log2(e)/2
+  s.hb = __fmul_rn(1.4426950408889634f, c.y);   // log2(e)
+  s.hc = __fmul_rn(0.7213475204444817f, c.z);
+  s.ra = __fmul_rn(-s.hb, __frcp_rn(__fmul_rn(2.f, s.ha)));
+  s.rc = __fmul_rn(-s.hb, __frcp_rn(__fmul_rn(2.f, s.hc)));
+  // alpha = o 2^-sigma' >= alpha_min  <=>  sigma' <= log2(o / alpha_min); margin 0.01 + 0.1%
+  const float thr = c.w >= alpha_min ? log2f(__fdiv_rn(c.w, alpha_min)) : -1.f;
+  s.lim = thr >= 0.f ? __fmul_rn(__fadd_rn(__fmul_rn(thr, 1.001f), 0.01f), 1.001f) : -1.f;
+  return s;
+}
+
+__device__ __forceinline__ bool tile_kept(const Splat& s, int tx, int ty) {
+  const float X0 = __fsub_rn((float)(tx * kTile) + 0.5f, s.u);
+  const float Y0 = __fsub_rn((float)(ty * kTile) + 0.5f, s.v);
+  const float X1 = __fadd_rn(X0, (float)(kTile - 1)), Y1 = __fadd_rn(Y0, (float)(kTile - 1));
+  return box_min_rn(s.ha, s.hb, s.hc, s.ra, s.rc, X0, X1, Y0, Y1) <= s.lim;
+}
+
+// ---- one warp per Gaussian, its rectangle's cells over the lanes in row-major order (32 at a
+// time): the count of kept cells, and +1 / -1 in the per-row difference array at the start /
+// one past the end of every run of kept cells (correct for any pattern of kept cells).
+__global__ void __launch_bounds__(256)
+tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, int tiles_x,
+                 float alpha_min, unsigned* counts, int* diff) {
+  const int lane = threadIdx.x & 31;
+  const int W1 = tiles_x + 1;
+  for (int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; g < n;
+       g += (gridDim.x * blockDim.x) >> 5) {
+    const int4 q = rects[g];
+    const int w = q.z - q.x, area = w * (q.w - q.y);
+    unsigned c = 0;
+    if (area > 0) {
+      const Splat s = load_splat(uv, co, (unsigned)g, alpha_min);
+      bool prev_last = false;                // kept flag of the cell before this word
+      for (int base = 0; base < area; base += 32) {
+        const int k = base + lane;
+        const int ry = k / w, rx = k - ry * w;
+        const bool kept = k < area && tile_kept(s, q.x + rx, q.y + ry);
+        const unsigned b = __ballot_sync(0xffffffffu, kept);
+        c += __popc(b);
+        // neighbours in the same row: the cell before is lane - 1 (or the previous word)
+        const bool left = rx > 0 && (lane > 0 ? ((b >> (lane - 1)) & 1u) : prev_last);
+        const bool right_in_word = lane < 31 ? ((b >> (lane + 1)) & 1u) : false;
+        bool right;
+        if (rx == w - 1) right = false;
+        else if (lane < 31) right = right_in_word;
+        else {                                 // the next cell is the first of the next word
+          const int k2 = k + 1;
+          right = k2 < area && tile_kept(s, q.x + (k2 - (k2 / w) * w), q.y + k2 / w);
+        }
+        if (kept && !left) atomicAdd(&diff[(q.y + ry) * W1 + q.x + rx], 1);
+        if (kept && !right) atomicAdd(&diff[(q.y + ry) * W1 + q.x + rx + 1], -1);
+        prev_last = (b >> 31) & 1u;
+      }
+    }
+    if (lane == 0) counts[g] = c;
   }
 }
 
@@ -184,16 +273,15 @@ radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_sta
   }
 }
 
-// ---- binning: per-block sums of rectangle areas in depth order
-__device__ __forceinline__ unsigned rect_area(int4 q) { return (unsigned)((q.z - q.x) * (q.w - q.y)); }
-
+// ---- binning: per-block sums of pair counts in depth order
 __global__ void __launch_bounds__(256)
-count_kernel(const u64* sorted, int n, const int4* rects, unsigned long long* block_sums, int G) {
+count_kernel(const u64* sorted, int n, const unsigned* counts, unsigned long long* block_sums,
+             int G) {
   long long lo, hi;
   block_range(n, G, &lo, &hi);
   unsigned long long s = 0;
   for (long long i = lo + threadIdx.x; i < hi; i += blockDim.x)
-    s += rect_area(rects[(unsigned)sorted[i]]);
+    s += counts[(unsigned)sorted[i]];
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   __shared__ unsigned long long ws[8];
   if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = s;
@@ -205,20 +293,38 @@ count_kernel(const u64* sorted, int n, const int4* rects, unsigned long long* bl
   }
 }
 
-// ---- tile ranges from the difference array: 2-D prefix sum -> per-tile counts -> exclusive
-// scan (one block).  Empty ranges when K overflowed the capacity.
+__global__ void __launch_bounds__(1024)
+scan_blocks_kernel(unsigned long long* block_sums, int G, long long* count, long long cap,
+                   unsigned* status) {
+  const unsigned long long v = (int)threadIdx.x < G ? block_sums[threadIdx.x] : 0ull;
+  unsigned long long total = 0;
+  const unsigned long long ex = block_exclusive_scan(v, &total);
+  if ((int)threadIdx.x < G) block_sums[threadIdx.x] = ex;
+  if (threadIdx.x == 0) {
+    *count = (long long)total;
+    if ((long long)total > cap) atomicOr(status, kStatusCapacity);
+  }
+}
+
+// ---- tile ranges from the per-row difference array: prefix sums along each row -> per-tile
+// counts -> exclusive scan (one block).  Empty ranges when K overflowed the capacity.
 __global__ void __launch_bounds__(1024)
 ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* count, long long cap,
                         unsigned* ranges) {
   const int W1 = tiles_x + 1;
-  for (int y = threadIdx.x; y < tiles_y; y += blockDim.x) {       // prefix along x
-    int run = 0;
-    for (int x = 0; x < tiles_x; ++x) { run += diff[y * W1 + x]; diff[y * W1 + x] = run; }
-  }
-  __syncthreads();
-  for (int x = threadIdx.x; x < tiles_x; x += blockDim.x) {       // prefix along y
-    int run = 0;
-    for (int y = 0; y < tiles_y; ++y) { run += diff[y * W1 + x]; diff[y * W1 + x] = run; }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (int y = wid; y < tiles_y; y += nw) {                        // prefix along each row
+    int carry = 0;
+    for (int x0 = 0; x0 < tiles_x; x0 += 32) {
+      const int x = x0 + lane;
+      int v = x < tiles_x ? diff[y * W1 + x] : 0;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += u;
+      }
+      if (x < tiles_x) diff[y * W1 + x] = v + carry;
+      carry += __shfl_sync(0xffffffffu, v, 31);
+    }
   }
   __syncthreads();
   const bool ok = *count <= cap;
@@ -236,34 +342,23 @@ ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* co
   }
 }
 
-__global__ void __launch_bounds__(1024)
-scan_blocks_kernel(unsigned long long* block_sums, int G, long long* count, long long cap,
-                   unsigned* status) {
-  const unsigned long long v = (int)threadIdx.x < G ? block_sums[threadIdx.x] : 0ull;
-  unsigned long long total = 0;
-  const unsigned long long ex = block_exclusive_scan(v, &total);
-  if ((int)threadIdx.x < G) block_sums[threadIdx.x] = ex;
-  if (threadIdx.x == 0) {
-    *count = (long long)total;
-    if ((long long)total > cap) atomicOr(status, kStatusCapacity);
-  }
-}
-
-// ---- emission of (tile << 32 | id) in depth order; each warp writes its Gaussians' pairs
-// one Gaussian at a time with all lanes (contiguous, coalesced stores)
+// ---- emission of (tile << 32 | id) in depth order: each warp takes its Gaussians one at a
+// time and spreads the rectangle's cells over the lanes; kept cells are compacted in
+// row-major order with a ballot, so consecutive lanes write consecutive entries.
 __global__ void __launch_bounds__(256)
-emit_kernel(const u64* sorted, int n, const int4* rects, const unsigned long long* block_off,
-            const long long* count, long long cap, int tiles_x, u64* pairs, int G) {
+emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const int4* rects,
+            const unsigned* counts, const unsigned long long* block_off, const long long* count,
+            long long cap, int tiles_x, float alpha_min, u64* pairs, int G) {
   if (*count > cap) return;
   long long lo, hi;
   block_range(n, G, &lo, &hi);
   const int lane = threadIdx.x & 31;
+  const unsigned lt = (1u << lane) - 1u;
   unsigned long long run = block_off[blockIdx.x];
   for (long long base = lo; base < hi; base += blockDim.x) {
     const long long i = base + threadIdx.x;
     unsigned id = 0, t = 0;
-    int4 q = make_int4(0, 0, 0, 0);
-    if (i < hi) { id = (unsigned)sorted[i]; q = rects[id]; t = rect_area(q); }
+    if (i < hi) { id = (unsigned)sorted[i]; t = counts[id]; }
     unsigned long long tot = 0;
     const unsigned long long off = run + block_exclusive_scan(t, &tot);
     for (int j = 0; j < 32; ++j) {
@@ -271,11 +366,19 @@ emit_kernel(const u64* sorted, int n, const int4* rects, const unsigned long lon
       if (tj == 0) continue;
       const unsigned idj = __shfl_sync(0xffffffffu, id, j);
       const unsigned long long oj = __shfl_sync(0xffffffffu, off, j);
-      const int x0 = __shfl_sync(0xffffffffu, q.x, j), y0 = __shfl_sync(0xffffffffu, q.y, j);
-      const int w = __shfl_sync(0xffffffffu, q.z, j) - x0;
-      for (unsigned k = lane; k < tj; k += 32) {
-        const int tile = (y0 + (int)(k / (unsigned)w)) * tiles_x + x0 + (int)(k % (unsigned)w);
-        pairs[oj + k] = ((u64)(unsigned)tile << 32) | idj;
+      const int4 q = rects[idj];
+      const int w = q.z - q.x, area = w * (q.w - q.y);
+      const Splat s = load_splat(uv, co, idj, alpha_min);
+      unsigned done = 0;
+      for (int cb = 0; cb < area && done < tj; cb += 32) {
+        const int k = cb + lane;
+        const int ry = k / w, rx = k - ry * w;
+        const bool kept = k < area && tile_kept(s, q.x + rx, q.y + ry);
+        const unsigned b = __ballot_sync(0xffffffffu, kept);
+        const unsigned at = done + __popc(b & lt);
+        if (kept && at < tj)
+          pairs[oj + at] = ((u64)(unsigned)((q.y + ry) * tiles_x + q.x + rx) << 32) | idj;
+        done += __popc(b);
       }
     }
     run += tot;
@@ -313,7 +416,8 @@ abcd_status radix_sort(abcd_ctx* ctx, u64* a, u64* b, long long n_static, const 
 using namespace abcd;
 
 extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, int n,
-                                     const abcd_camera* cam, abcd_tiles* out) {
+                                     const abcd_camera* cam, const abcd_render_opts* opts,
+                                     abcd_tiles* out) {
   if (!ctx) return ABCD_ERR_INVALID_ARG;
   if (!has_workspace(ctx)) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_bin_sort: no workspace");
   if (!proj || !cam || !out || n < 0 || cam->width <= 0 || cam->height <= 0)
@@ -326,7 +430,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   const long long n_tiles = (long long)tiles_x * tiles_y;
   if (n_tiles >= (1LL << 24)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_bin_sort: too many tiles");
   if (cap >= (1LL << 32)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_bin_sort: capacity must be < 2^32");
-  if (n > 0 && (!proj->depth || !proj->radius || !proj->uv || !proj->tiles_touched))
+  if (n > 0 && (!proj->depth || !proj->radius || !proj->uv || !proj->conic_opacity ||
+                ((uintptr_t)proj->uv & 7) || ((uintptr_t)proj->conic_opacity & 15)))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_bin_sort: null projected field");
   cudaError_t e = cudaSuccess;
   if (n == 0) {
@@ -342,22 +447,33 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   e = cudaMemsetAsync(ctx->ws.diff, 0, diff_bytes, ctx->stream);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "diff memset: %s", cudaGetErrorString(e));
   abcd_status s;
+  const float alpha_min = make_opts(opts).alpha_min;
   keys_rects_kernel<<<(n + 255) / 256, 256, 0, ctx->stream>>>(
       proj->depth, proj->radius, (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
-      ctx->ws.rects, ctx->ws.diff);
+      ctx->ws.rects);
   if ((s = check_launch(ctx, "keys_rects_kernel"))) return s;
+  {
+    const long long warps = std::min<long long>(n, (long long)ctx->num_sms * 64);
+    tile_rows_kernel<<<(int)((warps * 32 + 255) / 256), 256, 0, ctx->stream>>>(
+        (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects, n, tiles_x,
+        alpha_min, ctx->ws.counts, ctx->ws.diff);
+    if ((s = check_launch(ctx, "tile_rows_kernel"))) return s;
+  }
   u64* by_depth = nullptr;
   if ((s = radix_sort(ctx, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64, &by_depth, nullptr)))
     return s;
-  count_kernel<<<G, 256, 0, ctx->stream>>>(by_depth, n, ctx->ws.rects, ctx->ws.block_sums, G);
+  const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
+  count_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, ctx->ws.counts, ctx->ws.block_sums, Ge);
   if ((s = check_launch(ctx, "count_kernel"))) return s;
-  scan_blocks_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.block_sums, G, out->count, cap, ctx->ws.status);
+  scan_blocks_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status);
   if ((s = check_launch(ctx, "scan_blocks_kernel"))) return s;
   ranges_from_diff_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.diff, tiles_x, tiles_y, out->count, cap,
                                                       out->ranges);
   if ((s = check_launch(ctx, "ranges_from_diff_kernel"))) return s;
-  emit_kernel<<<G, 256, 0, ctx->stream>>>(by_depth, n, ctx->ws.rects, ctx->ws.block_sums, out->count,
-                                          cap, tiles_x, ctx->ws.pairs[0], G);
+  emit_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, (const float2*)proj->uv,
+                                           (const float4*)proj->conic_opacity, ctx->ws.rects,
+                                           ctx->ws.counts, ctx->ws.block_sums, out->count, cap,
+                                           tiles_x, alpha_min, ctx->ws.pairs[0], Ge);
   if ((s = check_launch(ctx, "emit_kernel"))) return s;
   int tile_bits = 1;
   while ((1LL << tile_bits) < n_tiles) ++tile_bits;

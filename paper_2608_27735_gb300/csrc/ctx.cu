@@ -128,6 +128,7 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.pairs[1] = (unsigned long long*)take(8ull * (size_t)max_pairs);
   w.hist = (unsigned*)take(4ull * kRadixBins * (kMaxRadixBlocks + 1));
   w.rects = (int4*)take(16ull * (size_t)max_g);
+  w.counts = (unsigned*)take(4ull * (size_t)max_g);
   w.diff_bytes = 4ull * kMaxDiffCells;
   w.diff = (int*)take(w.diff_bytes);
   w.block_sums = (unsigned long long*)take(8ull * (kMaxRadixBlocks + 1));

@@ -75,6 +75,29 @@ __device__ __forceinline__ bool cull(float4 s, float2 m, float bx0, float by0, f
   return lo * 0.998f > thr + 0.02f;
 }
 
+// Adds the warp-wide sums of v[0..9) to dst[0..9).  Transpose reduction: at each step a lane
+// keeps half of its (padded to 16) partial sums and receives the partner's matching half, so
+// 16 shuffles replace the 45 of a butterfly per value; afterwards lanes 2c, 2c + 1 hold the
+// sum of component c = lane / 2 (bits 4..1), and lane 2c adds it to memory.
+__device__ __forceinline__ void warp_sum9_atomic(const float v[9], float* dst, int lane) {
+  float x[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) x[k] = k < 9 ? v[k] : 0.f;
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1) {       // halves of 16, 8, 4, 2 values; lane bits 4..1
+    const bool up = (lane & (2 * w)) != 0;
+#pragma unroll
+    for (int k = 0; k < w; ++k) {
+      const float send = up ? x[k] : x[k + w];
+      const float keep = up ? x[k + w] : x[k];
+      x[k] = keep + __shfl_xor_sync(0xffffffffu, send, 2 * w);
+    }
+  }
+  x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
+  const int c = lane >> 1;
+  if ((lane & 1) == 0 && c < 9) atomicAdd(&dst[c], x[0]);
+}
+
 __device__ __forceinline__ float4 load_px(const void* img, int dtype, long long p) {
   if (dtype == ABCD_F16) {
     const uint2 r = reinterpret_cast<const uint2*>(img)[p];
@@ -306,7 +329,7 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
             c0 = __fmaf_rn(w, col.x, c0);
             c1 = __fmaf_rn(w, col.y, c1);
             c2 = __fmaf_rn(w, col.z, c2);
-            const float ioma = 1.f / (1.f - alpha);
+            const float ioma = __fdividef(1.f, 1.f - alpha);   // gradient scale only
             // R = colour accumulated behind this Gaussian = A - (sum up to and including it)
             const float dalpha = Gr * (T * col.x - (A0 - c0) * ioma) +
                                  Gg * (T * col.y - (A1 - c1) * ioma) +
@@ -326,15 +349,15 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
           }
         }
       }
-      if (__any_sync(0xffffffffu, contrib)) {
+      const unsigned who = __ballot_sync(0xffffffffu, contrib);
+      if (who == 0) continue;
+      float* dst = a.grad2d + 9 * (size_t)s_id[q];
+      if (__popc(who) <= 2) {                   // one or two pixels: add directly
+        if (contrib)
 #pragma unroll
-        for (int k = 0; k < 9; ++k)
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
-        float mine = 0.f;
-#pragma unroll
-        for (int k = 0; k < 9; ++k) mine = (lane == k) ? v[k] : mine;
-        if (lane < 9) atomicAdd(&a.grad2d[9 * (size_t)s_id[q] + lane], mine);
+          for (int k = 0; k < 9; ++k) atomicAdd(&dst[k], v[k]);
+      } else {
+        warp_sum9_atomic(v, dst, lane);
       }
     }
   }

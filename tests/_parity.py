@@ -90,17 +90,40 @@ def _in(rect, x, y):
     return rect[0] <= x < rect[2] and rect[1] <= y < rect[3]
 
 
-def optional_members(P, lo, hi, cam, tile=16):
-    """tile -> set of Gaussians that may or may not be listed there."""
+LOG2E = 1.4426950408889634
+
+
+def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, delta=1e-4):
+    """Entries (Gaussian, tile) the GPU may list or not.
+
+    The oracle lists tile t of Gaussian g when t is in g's square and the least sigma over
+    t's pixel-centre box is <= ln(o / alpha_min).  The GPU tests the same quantity in fp32 in
+    log2 units with a margin: kept when sigma' * 0.999 <= (1.001 thr' + 0.01) * 1.001.
+    Returns (opt_list, opt_render): tile -> set of ids whose listing may differ, and the
+    subset where the Gaussian might still reach alpha_min at a pixel (render alternatives
+    needed); the rest of opt_list is skipped by every pixel either way."""
     tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
-    opt = {}
-    diff = np.where(np.any(lo != hi, axis=1) & (P["depth"] > 0.2))[0]
-    for i in diff:
-        for y in range(hi[i, 1], hi[i, 3]):
-            for x in range(hi[i, 0], hi[i, 2]):
-                if not _in(lo[i], x, y):
-                    opt.setdefault(y * tx + x, set()).add(int(i))
-    return opt
+    opt_list, opt_render = {}, {}
+    for g in np.nonzero(np.any(hi != 0, axis=1) & (P["depth"] > 0.2))[0]:
+        o = P["opacity"][g]
+        u, v = P["uv"][g]
+        thr = math.log(o / alpha_min) * LOG2E if o >= alpha_min else -1.0
+        lim = (thr * 1.001 + 0.01) * 1.001 if thr >= 0 else -1.0
+        for y in range(hi[g, 1], hi[g, 3]):
+            for x in range(hi[g, 0], hi[g, 2]):
+                m = LOG2E * oracle.box_min_sigma(P["conic"][g], x * tile + 0.5 - u,
+                                                 x * tile + tile - 0.5 - u,
+                                                 y * tile + 0.5 - v, y * tile + tile - 0.5 - v)
+                in_sq_certain = _in(lo[g], x, y)
+                keep_certain = thr >= 0 and m <= thr * (1 - delta) - delta
+                keep_possible = thr >= 0 and m * 0.999 <= lim * (1 + delta) + delta
+                if (in_sq_certain and keep_certain) or not keep_possible:
+                    continue
+                t = y * tx + x
+                opt_list.setdefault(t, set()).add(int(g))
+                if thr >= 0 and m <= thr * (1 + delta) + delta:
+                    opt_render.setdefault(t, set()).add(int(g))
+    return opt_list, opt_render
 
 
 def check_tile_lists(gpu_ranges, gpu_ids, off, ids, P, opt, n_tiles):
@@ -137,10 +160,36 @@ def pixel_alternatives(sp, lst_full, labels, px, py, events, F, B, bg, opts, max
     return outs
 
 
-def tile_candidates(t, off, ids, P, opt):
-    """Oracle's list of tile t merged with its optional members, with membership labels."""
+def reaches(P, g, px, py, alpha_min=1.0 / 255.0, delta=1e-4):
+    """Whether Gaussian g might reach alpha_min at pixel (px, py) (exact value, with slack)."""
+    o = P["opacity"][g]
+    if o < alpha_min:
+        return False
+    u, v = P["uv"][g]
+    a, b, c = P["conic"][g]
+    dx, dy = px + 0.5 - u, py + 0.5 - v
+    sig = 0.5 * (a * dx * dx + c * dy * dy) + b * dx * dy
+    return sig <= math.log(o / alpha_min) * (1 + delta) + delta
+
+
+def opt_pixel_mask(P, opt, cam, tile=16):
+    """Pixels where an optional member of their tile might contribute."""
+    tx, _ = oracle.tiles_xy(cam.width, cam.height, tile)
+    mask = np.zeros((cam.height, cam.width), bool)
+    for t, gs in opt.items():
+        y0, x0 = (t // tx) * tile, (t % tx) * tile
+        for py in range(y0, min(y0 + tile, cam.height)):
+            for px in range(x0, min(x0 + tile, cam.width)):
+                if any(reaches(P, g, px, py) for g in gs):
+                    mask[py, px] = True
+    return mask
+
+
+def tile_candidates(t, off, ids, P, opt, px, py):
+    """Oracle's list of tile t merged with the optional members that matter at (px, py),
+    with membership labels."""
     O = [int(v) for v in ids[off[t]:off[t + 1]]]
-    o = opt.get(t, set())
+    o = {g for g in opt.get(t, set()) if reaches(P, g, px, py)}
     allg = sorted(set(O) | o, key=lambda g: (int(P["depth_key"][g]), g))
     lab = []
     for g in allg:
@@ -157,10 +206,7 @@ def compare_render(gpu_out, gpu_T, R, sp, off, ids, P, opt, cam, F=None, B=None,
     H, W = cam.height, cam.width
     tx, _ = oracle.tiles_xy(W, H, tile)
     ref = R["out"]
-    flagged = R["n_ev"] > 0
-    for t in opt:
-        y0, x0 = (t // tx) * tile, (t % tx) * tile
-        flagged[y0:y0 + tile, x0:x0 + tile] = True
+    flagged = (R["n_ev"] > 0) | opt_pixel_mask(P, opt, cam, tile)
     ok = ~flagged
     err = np.abs(gpu_out[ok] - ref[ok]).max() if ok.any() else 0.0
     assert err <= tol, f"max |gpu - oracle| on unambiguous pixels = {err}"
@@ -169,7 +215,7 @@ def compare_render(gpu_out, gpu_T, R, sp, off, ids, P, opt, cam, F=None, B=None,
     n_alt = 0
     for py, px in zip(*np.nonzero(flagged)):
         t = (py // tile) * tx + (px // tile)
-        allg, lab = tile_candidates(t, off, ids, P, opt)
+        allg, lab = tile_candidates(t, off, ids, P, opt, px, py)
         evs = [tuple(e) for e in R["ev"][py, px][:min(R["n_ev"][py, px], R["ev"].shape[2])]]
         Fp = None if F is None else F[py, px]
         Bp = None if B is None else B[py, px]
@@ -188,14 +234,11 @@ def grad_envelope(sp, off, ids, P, opt, R, cam, G, F=None, B=None, bg=None, opts
     n = sp.s.n
     lo = np.zeros((n, 9))
     hi = np.zeros((n, 9))
-    flagged = R["n_ev"] > 0
-    for t in opt:
-        y0, x0 = (t // tx) * tile, (t % tx) * tile
-        flagged[y0:y0 + tile, x0:x0 + tile] = True
+    flagged = (R["n_ev"] > 0) | opt_pixel_mask(P, opt, cam, tile)
     pix = list(zip(*np.nonzero(flagged)))
     for py, px in pix:
         t = (py // tile) * tx + (px // tile)
-        allg, lab = tile_candidates(t, off, ids, P, opt)
+        allg, lab = tile_candidates(t, off, ids, P, opt, px, py)
         evs = [tuple(e) for e in R["ev"][py, px][:min(R["n_ev"][py, px], R["ev"].shape[2])]]
         Fp = None if F is None else F[py, px]
         Bp = None if B is None else B[py, px]

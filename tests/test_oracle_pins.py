@@ -179,7 +179,7 @@ def test_tile_lists_brute_force():
     s = sg.tiny_scene(per_cell=60, res=80, n_cams=1)
     cam = s.cameras[0]
     P = oracle.project(s.gaussians, cam)
-    off, ids = oracle.tile_lists(P, cam.width, cam.height)
+    off, ids = oracle.tile_lists(P, cam.width, cam.height, rule="square")
     tx, ty = oracle.tiles_xy(cam.width, cam.height)
     n = s.gaussians.n
     assert P["visible"].sum() > 0
@@ -202,17 +202,67 @@ def test_tile_lists_brute_force():
     assert np.all(np.abs(z32.astype(np.float64) - P["depth"][vis]) <= 4e-7 * P["depth"][vis])
 
 
+def test_alpha_listing_rule_drops_only_skipped_entries():
+    """The listing rule keeps a tile of the 3-sigma square only where the Gaussian can reach
+    alpha_min: every dropped entry is skipped by all 256 pixel centres of its tile, and the
+    rendered image is bit-identical to the one over the full squares."""
+    s = sg.tiny_scene(per_cell=300, res=96, n_cams=2)
+    for cam in s.cameras:
+        P = oracle.project(s.gaussians, cam)
+        oq, iq = oracle.tile_lists(P, cam.width, cam.height, rule="square")
+        oa, ia = oracle.tile_lists(P, cam.width, cam.height, rule="alpha")
+        tx, ty = oracle.tiles_xy(cam.width, cam.height)
+        assert len(ia) < len(iq)
+        ys, xs = np.mgrid[0:16, 0:16] + 0.5
+        for t in range(tx * ty):
+            full = list(iq[oq[t]:oq[t + 1]])
+            kept = list(ia[oa[t]:oa[t + 1]])
+            assert [g for g in full if g in set(kept)] == kept, t
+            for g in set(full) - set(kept):
+                u, v = P["uv"][g]
+                a, b, c = P["conic"][g]
+                dx, dy = xs + 16 * (t % tx) - u, ys + 16 * (t // tx) - v
+                sig = 0.5 * (a * dx * dx + c * dy * dy) + b * dx * dy
+                assert np.all(P["opacity"][g] * np.exp(-sig) < 1 / 255), (t, g)
+        sp = oracle.SplatSet.from_proj(P)
+        Rq = oracle.render(sp, oq, iq, cam.width, cam.height)
+        Ra = oracle.render(sp, oa, ia, cam.width, cam.height)
+        np.testing.assert_array_equal(Ra["out"], Rq["out"])
+        np.testing.assert_array_equal(Ra["T_final"], Rq["T_final"])
+
+
+def test_box_min_sigma_against_dense_sampling():
+    rng = np.random.default_rng(21)
+    for _ in range(300):
+        L = rng.normal(size=(2, 2))
+        S = L @ L.T + 0.3 * np.eye(2)
+        Q = np.linalg.inv(S) * rng.uniform(0.01, 3.0)
+        conic = [Q[0, 0], Q[0, 1], Q[1, 1]]
+        X0, Y0 = rng.uniform(-30, 30, 2)
+        X1, Y1 = X0 + rng.uniform(0, 15), Y0 + rng.uniform(0, 15)
+        m = oracle.box_min_sigma(conic, X0, X1, Y0, Y1)
+        gx, gy = np.meshgrid(np.linspace(X0, X1, 401), np.linspace(Y0, Y1, 401))
+        sig = 0.5 * (Q[0, 0] * gx * gx + Q[1, 1] * gy * gy) + Q[0, 1] * gx * gy
+        dense = sig.min()
+        h = max(X1 - X0, Y1 - Y0) / 400
+        grad = np.abs(Q).sum() * (max(abs(X0), abs(X1)) + max(abs(Y0), abs(Y1)))
+        assert m <= dense + 1e-12
+        assert dense - m <= grad * h + 1e-12
+    assert oracle.box_min_sigma([1.0, 0.2, 2.0], -1, 1, -3, 2) == 0.0
+
+
 def test_tile_lists_capacity_report():
     s = sg.tiny_scene(per_cell=10, res=48, n_cams=1)
     P = oracle.project(s.gaussians, s.cameras[0])
-    off, ids = oracle.tile_lists(P, 48, 48)
+    off, ids = oracle.tile_lists(P, 48, 48, rule="square")
     import ctypes as C
     K = len(ids)
     o2 = np.zeros_like(off)
     i2 = np.zeros(max(K, 1), np.int32)
     r = oracle.lib().orc_tile_lists(P["visible"].shape[0], oracle._p(P["visible"]),
                                     oracle._p(P["rect"]), oracle._p(P["depth_key"]), 3, 3,
-                                    oracle._p(o2), oracle._p(i2), C.c_longlong(K - 1))
+                                    oracle._p(o2), oracle._p(i2), C.c_longlong(K - 1), None,
+                                    C.c_double(1 / 255), 16)
     assert r == -K - 1
 
 
