@@ -71,30 +71,26 @@ __global__ void keys_rects_kernel(const float* depth, const int* radius, const f
   items[i] = ((u64)key << 32) | (unsigned)i;
 }
 
-// Least sigma * log2(e) over the offset box [X0, X1] x [Y0, Y1] (convex quadratic with the
-// log2-scaled conic s = (a/2, b, c/2) log2 e): 0 if the box holds 0, else the least value on
-// its edges (the edge minimiser is clamped into the edge; r_a = -b / (2 a'), r_c = -b / (2 c')
-// are precomputed per Gaussian).  Round-to-nearest intrinsics only, so every kernel gets the
-// same bits.
-__device__ __forceinline__ float box_min_rn(float ha, float hb, float hc, float ra, float rc,
-                                            float X0, float X1, float Y0, float Y1) {
-  if (X0 <= 0.f && X1 >= 0.f && Y0 <= 0.f && Y1 >= 0.f) return 0.f;
-  float best = 3.0e38f;
-#pragma unroll
-  for (int e = 0; e < 2; ++e) {
-    const float X = e ? X1 : X0;
-    const float dy = fminf(fmaxf(__fmul_rn(rc, X), Y0), Y1);
-    best = fminf(best, __fmaf_rn(X, __fmaf_rn(ha, X, __fmul_rn(hb, dy)), __fmul_rn(__fmul_rn(hc, dy), dy)));
-    const float Y = e ? Y1 : Y0;
-    const float dx = fminf(fmaxf(__fmul_rn(ra, Y), X0), X1);
-    best = fminf(best, __fmaf_rn(dx, __fmaf_rn(ha, dx, __fmul_rn(hb, Y)), __fmul_rn(__fmul_rn(hc, Y), Y)));
-  }
-  return best;
-}
-
+// The tiles of row ty kept for a Gaussian are those whose pixel-centre box meets the ellipse
+// E = {d : sigma'(d) <= lim}, sigma'(d) = ha dx^2 + hb dx dy + hc dy^2 (log2-scaled conic).
+// Over the row's band of centre offsets dy in [Y0, Y1], the x-extent of E is [xl, xr]: the
+// leftmost point of E is (-m, hb m / (2 hc)) with m = sqrt(lim / (ha - hb^2 / (4 hc))), and
+// the left boundary x(dy) = (-hb dy - sqrt(D(dy))) / (2 ha), D = hb^2 dy^2 - 4 ha (hc dy^2 -
+// lim), is convex, so its least value over the band is at the leftmost point's dy clamped into
+// the band (the rightmost side is symmetric).  lim = (1.001 log2(o / alpha_min) + 0.01) 1.001
+// keeps every tile the exact rule keeps.  Round-to-nearest intrinsics only: count and emit
+// kernels get the same bits.
 struct Splat {
-  float u, v, ha, hb, hc, ra, rc, lim;   // lim: keep a tile when its least sigma' <= lim
+  float u, v, ha, hb, hc, lim, det4;   // det4 = 4 ha hc - hb^2 > 0
 };
+
+__device__ __forceinline__ float diff_of_products(float a, float b, float c, float d) {
+  // a b - c d with one rounding error at most (Kahan)
+  const float w = __fmul_rn(c, d);
+  const float e = __fmaf_rn(-c, d, w);
+  const float f = __fmaf_rn(a, b, -w);
+  return __fadd_rn(f, e);
+}
 
 __device__ __forceinline__ Splat load_splat(const float2* uv, const float4* co, unsigned g,
                                             float alpha_min) {
@@ -105,24 +101,43 @@ __device__ __forceinline__ Splat load_splat(const float2* uv, const float4* co, 
   s.ha = __fmul_rn(0.7213475204444817f, c.x);   // log2(e)/2
   s.hb = __fmul_rn(1.4426950408889634f, c.y);   // log2(e)
   s.hc = __fmul_rn(0.7213475204444817f, c.z);
-  s.ra = __fmul_rn(-s.hb, __frcp_rn(__fmul_rn(2.f, s.ha)));
-  s.rc = __fmul_rn(-s.hb, __frcp_rn(__fmul_rn(2.f, s.hc)));
+  s.det4 = diff_of_products(__fmul_rn(4.f, s.ha), s.hc, s.hb, s.hb);
   // alpha = o 2^-sigma' >= alpha_min  <=>  sigma' <= log2(o / alpha_min); margin 0.01 + 0.1%
   const float thr = c.w >= alpha_min ? log2f(__fdiv_rn(c.w, alpha_min)) : -1.f;
-  s.lim = thr >= 0.f ? __fmul_rn(__fadd_rn(__fmul_rn(thr, 1.001f), 0.01f), 1.001f) : -1.f;
+  s.lim = (thr >= 0.f && s.det4 > 0.f) ? __fmul_rn(__fadd_rn(__fmul_rn(thr, 1.001f), 0.01f), 1.001f) : -1.f;
   return s;
 }
 
-__device__ __forceinline__ bool tile_kept(const Splat& s, int tx, int ty) {
-  const float X0 = __fsub_rn((float)(tx * kTile) + 0.5f, s.u);
+// Run [xa, xb) of kept tiles in tile row ty of rectangle q (empty: xa == xb).
+__device__ __forceinline__ int2 row_run(const Splat& s, int4 q, int ty) {
+  if (!(s.lim >= 0.f)) return make_int2(0, 0);
   const float Y0 = __fsub_rn((float)(ty * kTile) + 0.5f, s.v);
-  const float X1 = __fadd_rn(X0, (float)(kTile - 1)), Y1 = __fadd_rn(Y0, (float)(kTile - 1));
-  return box_min_rn(s.ha, s.hb, s.hc, s.ra, s.rc, X0, X1, Y0, Y1) <= s.lim;
+  const float Y1 = __fadd_rn(Y0, (float)(kTile - 1));
+  // |dy| <= ym on E: D(dy) >= 0  <=>  dy^2 (4 ha hc - hb^2) <= 4 ha lim
+  const float ym = __fsqrt_rn(__fdiv_rn(__fmul_rn(__fmul_rn(4.f, s.ha), s.lim), s.det4));
+  const float ylo = fmaxf(Y0, -ym), yhi = fminf(Y1, ym);
+  if (!(ylo <= yhi)) return make_int2(0, 0);
+  // leftmost point of E: dx = -mx, dy = hb mx / (2 hc); mx = sqrt(4 hc lim / det4)
+  const float mx = __fsqrt_rn(__fdiv_rn(__fmul_rn(__fmul_rn(4.f, s.hc), s.lim), s.det4));
+  const float dyl = __fdiv_rn(__fmul_rn(s.hb, mx), __fmul_rn(2.f, s.hc));
+  const float inv2a = __frcp_rn(__fmul_rn(2.f, s.ha));
+  // boundary x at dy: (-hb dy -+ sqrt(D)) / (2 ha), D = 4 ha lim - det4 dy^2
+  const float yl = fminf(fmaxf(dyl, ylo), yhi);
+  const float Dl = fmaxf(__fmaf_rn(-s.det4, __fmul_rn(yl, yl), __fmul_rn(__fmul_rn(4.f, s.ha), s.lim)), 0.f);
+  const float xl = __fmul_rn(__fsub_rn(__fmul_rn(-s.hb, yl), __fsqrt_rn(Dl)), inv2a);
+  const float yr = fminf(fmaxf(-dyl, ylo), yhi);
+  const float Dr = fmaxf(__fmaf_rn(-s.det4, __fmul_rn(yr, yr), __fmul_rn(__fmul_rn(4.f, s.ha), s.lim)), 0.f);
+  const float xr = __fmul_rn(__fadd_rn(__fmul_rn(-s.hb, yr), __fsqrt_rn(Dr)), inv2a);
+  // tiles whose centre box [16 tx + 0.5, 16 tx + 15.5] meets [u + xl, u + xr]
+  const float fa = ceilf(__fmul_rn(__fsub_rn(__fadd_rn(s.u, xl), 15.5f), 1.f / kTile));
+  const float fb = floorf(__fmul_rn(__fsub_rn(__fadd_rn(s.u, xr), 0.5f), 1.f / kTile)) + 1.f;
+  const int xa = (int)fminf(fmaxf(fa, (float)q.x), (float)q.z);
+  const int xb = (int)fminf(fmaxf(fb, (float)xa), (float)q.z);
+  return make_int2(xa, xb);
 }
 
-// ---- one warp per Gaussian, its rectangle's cells over the lanes in row-major order (32 at a
-// time): the count of kept cells, and +1 / -1 in the per-row difference array at the start /
-// one past the end of every run of kept cells (correct for any pattern of kept cells).
+// ---- one warp per Gaussian, lanes over its tile rows: the pair count and +1 / -1 at the ends
+// of every row's run in the per-row difference array
 __global__ void __launch_bounds__(256)
 tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, int tiles_x,
                  float alpha_min, unsigned* counts, int* diff) {
@@ -131,32 +146,19 @@ tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, i
   for (int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; g < n;
        g += (gridDim.x * blockDim.x) >> 5) {
     const int4 q = rects[g];
-    const int w = q.z - q.x, area = w * (q.w - q.y);
     unsigned c = 0;
-    if (area > 0) {
+    if (q.x < q.z) {
       const Splat s = load_splat(uv, co, (unsigned)g, alpha_min);
-      bool prev_last = false;                // kept flag of the cell before this word
-      for (int base = 0; base < area; base += 32) {
-        const int k = base + lane;
-        const int ry = k / w, rx = k - ry * w;
-        const bool kept = k < area && tile_kept(s, q.x + rx, q.y + ry);
-        const unsigned b = __ballot_sync(0xffffffffu, kept);
-        c += __popc(b);
-        // neighbours in the same row: the cell before is lane - 1 (or the previous word)
-        const bool left = rx > 0 && (lane > 0 ? ((b >> (lane - 1)) & 1u) : prev_last);
-        const bool right_in_word = lane < 31 ? ((b >> (lane + 1)) & 1u) : false;
-        bool right;
-        if (rx == w - 1) right = false;
-        else if (lane < 31) right = right_in_word;
-        else {                                 // the next cell is the first of the next word
-          const int k2 = k + 1;
-          right = k2 < area && tile_kept(s, q.x + (k2 - (k2 / w) * w), q.y + k2 / w);
+      for (int ty = q.y + lane; ty < q.w; ty += 32) {
+        const int2 r = row_run(s, q, ty);
+        if (r.y > r.x) {
+          c += (unsigned)(r.y - r.x);
+          atomicAdd(&diff[ty * W1 + r.x], 1);
+          atomicAdd(&diff[ty * W1 + r.y], -1);
         }
-        if (kept && !left) atomicAdd(&diff[(q.y + ry) * W1 + q.x + rx], 1);
-        if (kept && !right) atomicAdd(&diff[(q.y + ry) * W1 + q.x + rx + 1], -1);
-        prev_last = (b >> 31) & 1u;
       }
     }
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
     if (lane == 0) counts[g] = c;
   }
 }
@@ -343,8 +345,8 @@ ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* co
 }
 
 // ---- emission of (tile << 32 | id) in depth order: each warp takes its Gaussians one at a
-// time and spreads the rectangle's cells over the lanes; kept cells are compacted in
-// row-major order with a ballot, so consecutive lanes write consecutive entries.
+// time; lanes compute the row runs, a warp scan places them, and the pairs are written with
+// consecutive lanes on consecutive entries (row of pair k found by a search over the scan).
 __global__ void __launch_bounds__(256)
 emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const int4* rects,
             const unsigned* counts, const unsigned long long* block_off, const long long* count,
@@ -353,7 +355,6 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
   long long lo, hi;
   block_range(n, G, &lo, &hi);
   const int lane = threadIdx.x & 31;
-  const unsigned lt = (1u << lane) - 1u;
   unsigned long long run = block_off[blockIdx.x];
   for (long long base = lo; base < hi; base += blockDim.x) {
     const long long i = base + threadIdx.x;
@@ -367,18 +368,35 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
       const unsigned idj = __shfl_sync(0xffffffffu, id, j);
       const unsigned long long oj = __shfl_sync(0xffffffffu, off, j);
       const int4 q = rects[idj];
-      const int w = q.z - q.x, area = w * (q.w - q.y);
       const Splat s = load_splat(uv, co, idj, alpha_min);
       unsigned done = 0;
-      for (int cb = 0; cb < area && done < tj; cb += 32) {
-        const int k = cb + lane;
-        const int ry = k / w, rx = k - ry * w;
-        const bool kept = k < area && tile_kept(s, q.x + rx, q.y + ry);
-        const unsigned b = __ballot_sync(0xffffffffu, kept);
-        const unsigned at = done + __popc(b & lt);
-        if (kept && at < tj)
-          pairs[oj + at] = ((u64)(unsigned)((q.y + ry) * tiles_x + q.x + rx) << 32) | idj;
-        done += __popc(b);
+      for (int y0 = q.y; y0 < q.w && done < tj; y0 += 32) {
+        const int ty = y0 + lane;
+        int2 r = make_int2(0, 0);
+        if (ty < q.w) r = row_run(s, q, ty);
+        const unsigned c = (unsigned)(r.y - r.x);
+        unsigned incl = c;
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const unsigned total = __shfl_sync(0xffffffffu, incl, 31);
+        for (unsigned k0 = 0; k0 < total; k0 += 32) {     // uniform trip count: every lane
+          const unsigned k = k0 + lane;                      // takes part in the shuffles
+          // row holding pair k: the number of lanes whose inclusive count is <= k
+          int rl = 0;
+          for (int step = 16; step > 0; step >>= 1) {
+            const unsigned v = __shfl_sync(0xffffffffu, incl, rl + step - 1);
+            if (v <= k) rl += step;
+          }
+          rl = min(rl, 31);
+          const unsigned before = __shfl_sync(0xffffffffu, incl - c, rl);
+          const int xa = __shfl_sync(0xffffffffu, r.x, rl);
+          const unsigned at = done + k;
+          if (k < total && at < tj)
+            pairs[oj + at] = ((u64)(unsigned)((y0 + rl) * tiles_x + xa + (int)(k - before)) << 32) | idj;
+        }
+        done += total;
       }
     }
     run += tot;
@@ -440,7 +458,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
     e = cudaMemsetAsync(out->count, 0, sizeof(long long), ctx->stream);
     return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "count memset: %s", cudaGetErrorString(e));
   }
-  const int G = ctx->radix_blocks;
   const size_t diff_bytes = sizeof(int) * (size_t)(tiles_x + 1) * (tiles_y + 1);
   if (diff_bytes > ctx->ws.diff_bytes)
     return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_bin_sort: tile grid exceeds the workspace");
