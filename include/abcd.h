@@ -193,9 +193,9 @@ abcd_status abcd_adam_active(abcd_ctx* ctx, abcd_gaussians* theta, const abcd_ga
                              abcd_gaussians* m, abcd_gaussians* v, const float lr[6],
                              float beta1, float beta2, float eps, int step);
 
-/* K1. Depth-ordered over-compositing of cached per-partition renders (Section 2: "cached
- * renders from frozen partitions are composited into F and B according to depth
- * ordering").  layers: host array of L device pointers to [H][W][4] premultiplied RGBA of
+/* K1. Depth-ordered over-compositing of cached per-partition renders into the foreground F and
+ * background B of one camera (Section 2: the frozen partitions' stored renders, taken in the
+ * camera's depth order, collapse into two RGBA images).  layers: host array of L device pointers to [H][W][4] premultiplied RGBA of
  * layer_dtype; order: host array of L indices, front to back; split: position in order of
  * the active partition (its layer is skipped and may be NULL), or L for "all in front".
  * F_out = fold over order[0 .. split), B_out = fold over order[split+1 .. L), each a left

@@ -7,7 +7,7 @@
  * blocks in front of / behind the active partition collapse into two RGBA images by
  * associativity of alpha compositing), the L1 + D-SSIM reconstruction loss, the gradient
  * back into the active block only, Adam, and the depth-ordered compositing of cached
- * per-partition renders (Section 2, "composited into F and B according to depth ordering").
+ * per-partition renders into F and B (Section 2).
  * The renderer formulas are those of 3D Gaussian Splatting, which the paper instantiates
  * by citation (Section 1, last paragraph); Section 2 fixes the compositing structure.
  *

@@ -1,7 +1,7 @@
-// K1: depth-ordered over-compositing of cached per-partition RGBA renders into F and B
-// (Section 2: "cached renders from frozen partitions are composited into F and B according
-// to depth ordering"; by associativity of 'over' the frozen blocks in front of the active
-// partition collapse into F, those behind into B).
+// K1: depth-ordered over-compositing of cached per-partition RGBA renders into F and B.
+// Section 2 builds, per camera, the foreground and background images from the stored renders
+// of the frozen partitions in the camera's depth order; by associativity of 'over' the frozen
+// blocks in front of the active partition collapse into F, those behind it into B.
 //
 // Pure streaming work: every layer is read once (16-byte streaming loads, evict-first), the
 // accumulator stays in registers across layers, F and B are written once.  Four layers are

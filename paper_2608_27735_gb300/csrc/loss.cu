@@ -1,6 +1,6 @@
 // K6: reconstruction loss of one step, L = (1 - lambda) mean|x - y| + lambda (1 - mean SSIM),
-// and dL/dx, fused in one kernel (the paper's "reconstruction loss is evaluated", Section 2;
-// L1 + D-SSIM as in 3D Gaussian Splatting).
+// and dL/dx, fused in one kernel (each step of Section 2 scores the composited image against
+// the target; the L1 + D-SSIM form is that of 3D Gaussian Splatting).
 //
 // SSIM uses an 11x11 Gaussian window (sigma 1.5) with zero padding.  Per output tile of 32x32
 // pixels and per channel, a CTA stages x, y over the tile plus a 10-pixel halo, computes the

@@ -1,5 +1,5 @@
-// abcd_backward: the backward pass of one active-block step (Section 2: the reconstruction
-// loss is evaluated and gradients are backpropagated only through theta_active):
+// abcd_backward: the backward pass of one active-block step (Section 2: the step's loss is
+// differentiated with respect to the active block's parameters and nothing else):
 // K6 loss (optional) -> K7 blend/composite backward -> K8 projection backward.
 #include "abcd_internal.cuh"
 
