@@ -14,7 +14,6 @@ constexpr int kTileThreads = kTile * kTile;
 constexpr int kRadixBits = 8;
 constexpr int kRadixBins = 1 << kRadixBits;
 constexpr int kMaxRadixBlocks = 1024;     // upper bound used to size the histogram scratch
-constexpr int kLossTile = 32;             // loss output tile edge
 constexpr int kMaxLossBlocks = 1 << 16;
 constexpr int kMaxLayers = 256;
 constexpr long long kMaxDiffCells = 1LL << 20;   // (tiles_x + 1) * (tiles_y + 1)

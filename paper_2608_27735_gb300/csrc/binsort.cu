@@ -136,31 +136,29 @@ __device__ __forceinline__ int2 row_run(const Splat& s, int4 q, int ty) {
   return make_int2(xa, xb);
 }
 
-// ---- one warp per Gaussian, lanes over its tile rows: the pair count and +1 / -1 at the ends
-// of every row's run in the per-row difference array
+// ---- one thread per Gaussian, looping over its tile rows: the pair count and +1 / -1 at the
+// ends of every row's run in the per-row difference array (rows are short; this many threads
+// hide the latency of the per-Gaussian loads)
 __global__ void __launch_bounds__(256)
 tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, int tiles_x,
                  float alpha_min, unsigned* counts, int* diff) {
-  const int lane = threadIdx.x & 31;
+  const int g = blockIdx.x * blockDim.x + threadIdx.x;
+  if (g >= n) return;
   const int W1 = tiles_x + 1;
-  for (int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; g < n;
-       g += (gridDim.x * blockDim.x) >> 5) {
-    const int4 q = rects[g];
-    unsigned c = 0;
-    if (q.x < q.z) {
-      const Splat s = load_splat(uv, co, (unsigned)g, alpha_min);
-      for (int ty = q.y + lane; ty < q.w; ty += 32) {
-        const int2 r = row_run(s, q, ty);
-        if (r.y > r.x) {
-          c += (unsigned)(r.y - r.x);
-          atomicAdd(&diff[ty * W1 + r.x], 1);
-          atomicAdd(&diff[ty * W1 + r.y], -1);
-        }
+  const int4 q = rects[g];
+  unsigned c = 0;
+  if (q.x < q.z) {
+    const Splat s = load_splat(uv, co, (unsigned)g, alpha_min);
+    for (int ty = q.y; ty < q.w; ++ty) {
+      const int2 r = row_run(s, q, ty);
+      if (r.y > r.x) {
+        c += (unsigned)(r.y - r.x);
+        atomicAdd(&diff[ty * W1 + r.x], 1);
+        atomicAdd(&diff[ty * W1 + r.y], -1);
       }
     }
-    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-    if (lane == 0) counts[g] = c;
   }
+  counts[g] = c;
 }
 
 // ---- radix pass, step 1: per-block digit counts hist[d * G + b]
@@ -243,13 +241,20 @@ radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_sta
   const long long wchunk = (hi - lo + W - 1) / W;
   const long long wl = min(hi, lo + w * wchunk), wh = min(hi, wl + wchunk);
   const unsigned lt = (1u << lane) - 1u;
-  for (long long base = wl; base < wh; base += 32) {
-    const long long i = base + lane;
-    const bool valid = i < wh;
-    const unsigned d = valid ? ((unsigned)(in[i] >> shift) & (kRadixBins - 1)) : 0x100u;
-    const unsigned peers = __match_any_sync(0xffffffffu, d);
-    if (valid && (peers & lt) == 0) cnt[w][d] += __popc(peers);
-    __syncwarp();
+  constexpr int U = 4;                        // items per lane per iteration (loads in flight)
+  for (long long b0 = wl; b0 < wh; b0 += 32 * U) {
+    unsigned ds[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const long long i = b0 + 32 * j + lane;
+      ds[j] = i < wh ? ((unsigned)(in[i] >> shift) & (kRadixBins - 1)) : 0x100u;
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const unsigned peers = __match_any_sync(0xffffffffu, ds[j]);
+      if (ds[j] < 0x100u && (peers & lt) == 0) cnt[w][ds[j]] += __popc(peers);
+      __syncwarp();
+    }
   }
   __syncthreads();
   for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) {
@@ -257,21 +262,30 @@ radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_sta
     for (int k = 0; k < W; ++k) { const unsigned c = cnt[k][d]; cnt[k][d] = run; run += c; }
   }
   __syncthreads();
-  for (long long base = wl; base < wh; base += 32) {
-    const long long i = base + lane;
-    const bool valid = i < wh;
-    const u64 x = valid ? in[i] : 0ull;
-    const unsigned d = valid ? ((unsigned)(x >> shift) & (kRadixBins - 1)) : 0x100u;
-    const unsigned peers = __match_any_sync(0xffffffffu, d);
-    unsigned pos = 0;
-    if (valid) pos = cnt[w][d] + __popc(peers & lt);
-    __syncwarp();
-    if (valid) {
-      if (out_ids) out_ids[pos] = (unsigned)x;
-      else out[pos] = x;
-      if ((peers & lt) == 0) cnt[w][d] += __popc(peers);
+  for (long long b0 = wl; b0 < wh; b0 += 32 * U) {
+    u64 xs[U];
+    unsigned ds[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const long long i = b0 + 32 * j + lane;
+      const bool valid = i < wh;
+      xs[j] = valid ? in[i] : 0ull;
+      ds[j] = valid ? ((unsigned)(xs[j] >> shift) & (kRadixBins - 1)) : 0x100u;
     }
-    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const unsigned peers = __match_any_sync(0xffffffffu, ds[j]);
+      const bool valid = ds[j] < 0x100u;
+      unsigned pos = 0;
+      if (valid) pos = cnt[w][ds[j]] + __popc(peers & lt);
+      __syncwarp();
+      if (valid) {
+        if (out_ids) out_ids[pos] = (unsigned)xs[j];
+        else out[pos] = xs[j];
+        if ((peers & lt) == 0) cnt[w][ds[j]] += __popc(peers);
+      }
+      __syncwarp();
+    }
   }
 }
 
@@ -406,8 +420,8 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
 // LSD radix sort of 64-bit items on bits [bit_lo, bit_hi); returns the buffer holding the
 // result, or writes the low 32 bits of the sorted items to ids_out on the last pass.
 abcd_status radix_sort(abcd_ctx* ctx, u64* a, u64* b, long long n_static, const long long* n_dev,
-                       long long cap, int bit_lo, int bit_hi, u64** result, unsigned* ids_out) {
-  const int G = ctx->radix_blocks;
+                       long long cap, int bit_lo, int bit_hi, int G, u64** result,
+                       unsigned* ids_out) {
   unsigned* totals = ctx->ws.hist + kRadixBins * G;
   u64* src = a;
   u64* dst = b;
@@ -470,14 +484,15 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       ctx->ws.rects);
   if ((s = check_launch(ctx, "keys_rects_kernel"))) return s;
   {
-    const long long warps = std::min<long long>(n, (long long)ctx->num_sms * 64);
-    tile_rows_kernel<<<(int)((warps * 32 + 255) / 256), 256, 0, ctx->stream>>>(
+    tile_rows_kernel<<<(n + 255) / 256, 256, 0, ctx->stream>>>(
         (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects, n, tiles_x,
         alpha_min, ctx->ws.counts, ctx->ws.diff);
     if ((s = check_launch(ctx, "tile_rows_kernel"))) return s;
   }
   u64* by_depth = nullptr;
-  if ((s = radix_sort(ctx, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64, &by_depth, nullptr)))
+  const int Gd = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));   // depth sort
+  if ((s = radix_sort(ctx, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64, Gd, &by_depth,
+                      nullptr)))
     return s;
   const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
   count_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, ctx->ws.counts, ctx->ws.block_sums, Ge);
@@ -494,6 +509,7 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if ((s = check_launch(ctx, "emit_kernel"))) return s;
   int tile_bits = 1;
   while ((1LL << tile_bits) < n_tiles) ++tile_bits;
+  // K lives on the device: the tile passes take the largest grid; blocks past K exit at once
   return radix_sort(ctx, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap, 32, 32 + tile_bits,
-                    nullptr, out->ids);
+                    kMaxRadixBlocks, nullptr, out->ids);
 }

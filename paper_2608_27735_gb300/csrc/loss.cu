@@ -2,11 +2,13 @@
 // and dL/dx, fused in one kernel (each step of Section 2 scores the composited image against
 // the target; the L1 + D-SSIM form is that of 3D Gaussian Splatting).
 //
-// SSIM uses an 11x11 Gaussian window (sigma 1.5) with zero padding.  Per output tile of 32x32
+// SSIM uses an 11x11 Gaussian window (sigma 1.5) with zero padding.  Per output tile of 64x32
 // pixels and per channel, a CTA stages x, y over the tile plus a 10-pixel halo, computes the
 // five windowed moments (separably) on the tile plus a 5-pixel halo, the per-pixel partials
 // A = dS/dmu_x - 2 mu_x dS/dsigma_xx - mu_y dS/dsigma_xy, B = dS/dsigma_xx, C = dS/dsigma_xy,
 // and windows them again: dSSIM_sum/dx(q) = (w*A)(q) + 2 x(q) (w*B)(q) + y(q) (w*C)(q).
+// Every window pass is register-blocked: a thread produces 8 consecutive outputs from a
+// sliding run of 18 staged values (about 12 FMAs per shared-memory load).
 // The scalar is reduced deterministically: per-CTA partial sums, then the last CTA to finish
 // adds them in a fixed order (no waiting on other CTAs).
 #include <mutex>
@@ -16,40 +18,48 @@
 namespace abcd {
 namespace {
 
-constexpr int T = kLossTile;      // 32
-constexpr int R0 = T + 20;        // input region edge
-constexpr int R1 = T + 10;        // moment region edge
-constexpr int kThreads = 256;
-constexpr int kSmemFloats = 2 * R0 * R0 + 5 * R0 * R1 + 5 * R1 * R1;
+constexpr int TW = 64;            // output tile (pixels)
+constexpr int TH = 32;
+constexpr int RUN = 8;            // outputs per thread per window pass
+constexpr int IW = TW + 20, IH = TH + 20;    // inputs: tile + 10-pixel halo
+constexpr int MW = TW + 10, MH = TH + 10;    // windowed moments: tile + 5-pixel halo
+constexpr int kThreads = 512;
+// shared memory: x, y [IH][IW]; the five horizontal moment rows [5][IH][MW]; A, B, C
+// [3][MH][MW]; their horizontal windows [3][MH][TW] reuse the moment rows' space
+constexpr int kH5 = 5 * IH * MW;
+constexpr int kABC = 3 * MH * MW;
+constexpr int kSmemFloats = 2 * IH * IW + kH5 + kABC;
+static_assert(3 * MH * TW <= kH5, "windows of A, B, C fit in the moment space");
+
+__device__ __forceinline__ void load_weights(float* w) {
+  float s = 0.f;
+#pragma unroll
+  for (int t = 0; t < 11; ++t) { const float d = (float)t - 5.f; w[t] = expf(-d * d / (2.f * 1.5f * 1.5f)); s += w[t]; }
+#pragma unroll
+  for (int t = 0; t < 11; ++t) w[t] /= s;
+}
 
 __global__ void __launch_bounds__(kThreads)
 loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W, int H,
             float lam, float* __restrict__ grad, float* partials, unsigned* ticket,
             float* loss_out) {
   extern __shared__ float sm[];
-  float* sX = sm;                       // [R0][R0]
-  float* sY = sX + R0 * R0;             // [R0][R0]
-  float* hq = sY + R0 * R0;             // 5 x [R0][R1]; later A, B, C [R1][R1]
-  float* mq = hq + 5 * R0 * R1;         // 5 x [R1][R1]; later 3 x [R1][T]
-  __shared__ float w[11];
+  float* sX = sm;                     // [IH][IW]
+  float* sY = sX + IH * IW;           // [IH][IW]
+  float* h5 = sY + IH * IW;           // [5][IH][MW]
+  float* abc = h5 + kH5;              // [3][MH][MW]
+  float* h3 = h5;                     // [3][MH][TW] (moment rows are consumed by then)
   __shared__ float red[2][kThreads / 32];
-  if (threadIdx.x < 11) {
-    const float d = (float)threadIdx.x - 5.f;
-    w[threadIdx.x] = expf(-d * d / (2.f * 1.5f * 1.5f));
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float s = 0.f;
-    for (int k = 0; k < 11; ++k) s += w[k];
-    for (int k = 0; k < 11; ++k) w[k] /= s;
-  }
-  __syncthreads();
-  const int ox = blockIdx.x * T, oy = blockIdx.y * T;
+  float w[11];
+  load_weights(w);
+  const int ox = blockIdx.x * TW, oy = blockIdx.y * TH;
   const float inv = 1.f / (3.f * (float)W * (float)H);
+  const float C1 = 0.01f * 0.01f, C2 = 0.03f * 0.03f;
   float l1 = 0.f, ssim = 0.f;
   for (int ch = 0; ch < 3; ++ch) {
-    for (int k = threadIdx.x; k < R0 * R0; k += kThreads) {
-      const int r = k / R0, c = k % R0;
+    // ---- inputs with a 10-pixel halo, zero outside the image
+    for (int k = threadIdx.x; k < IH * IW; k += kThreads) {
+      const int r = k / IW, c = k - r * IW;
       const int gy = oy - 10 + r, gx = ox - 10 + c;
       float xv = 0.f, yv = 0.f;
       if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
@@ -61,98 +71,127 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
       sY[k] = yv;
     }
     __syncthreads();
-    // horizontal windows of x, y, x^2, y^2, xy: [R0][R1]
-    for (int k = threadIdx.x; k < R0 * R1; k += kThreads) {
-      const int r = k / R1, c = k % R1;
-      const float* px = sX + r * R0 + c;
-      const float* py = sY + r * R0 + c;
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, a4 = 0.f;
+    // ---- horizontal windows of x, y, x^2, y^2, xy: RUN outputs per item from RUN+10 inputs
+    constexpr int HSEG = (MW + RUN - 1) / RUN;
+    for (int it = threadIdx.x; it < IH * HSEG; it += kThreads) {
+      const int r = it / HSEG, c0 = (it - r * HSEG) * RUN;
+      float xs[RUN + 10], ys[RUN + 10], xx[RUN + 10], yy[RUN + 10], xy[RUN + 10];
 #pragma unroll
-      for (int t = 0; t < 11; ++t) {
-        const float xv = px[t], yv = py[t], wt = w[t];
-        a0 += wt * xv; a1 += wt * yv;
-        a2 += wt * xv * xv; a3 += wt * yv * yv; a4 += wt * xv * yv;
-      }
-      hq[k] = a0; hq[R0 * R1 + k] = a1; hq[2 * R0 * R1 + k] = a2;
-      hq[3 * R0 * R1 + k] = a3; hq[4 * R0 * R1 + k] = a4;
-    }
-    __syncthreads();
-    // vertical windows: moments on [R1][R1]
-    for (int k = threadIdx.x; k < R1 * R1; k += kThreads) {
-      const int r = k / R1, c = k % R1;
-      float a[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int t = 0; t < 11; ++t) {
-        const float wt = w[t];
-#pragma unroll
-        for (int q = 0; q < 5; ++q) a[q] += wt * hq[q * R0 * R1 + (r + t) * R1 + c];
+      for (int t = 0; t < RUN + 10; ++t) {
+        const int c = min(c0 + t, IW - 1);
+        xs[t] = sX[r * IW + c];
+        ys[t] = sY[r * IW + c];
+        xx[t] = xs[t] * xs[t];
+        yy[t] = ys[t] * ys[t];
+        xy[t] = xs[t] * ys[t];
       }
 #pragma unroll
-      for (int q = 0; q < 5; ++q) mq[q * R1 * R1 + k] = a[q];
+      for (int o = 0; o < RUN; ++o) {
+        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, a4 = 0.f;
+#pragma unroll
+        for (int t = 0; t < 11; ++t) {
+          a0 = fmaf(w[t], xs[o + t], a0); a1 = fmaf(w[t], ys[o + t], a1);
+          a2 = fmaf(w[t], xx[o + t], a2); a3 = fmaf(w[t], yy[o + t], a3); a4 = fmaf(w[t], xy[o + t], a4);
+        }
+        if (c0 + o < MW) {
+          const int k = r * MW + c0 + o;
+          h5[k] = a0; h5[IH * MW + k] = a1; h5[2 * IH * MW + k] = a2;
+          h5[3 * IH * MW + k] = a3; h5[4 * IH * MW + k] = a4;
+        }
+      }
     }
     __syncthreads();
-    // per-pixel SSIM and its partials A, B, C (zero outside the image)
-    {
-      const float C1 = 0.01f * 0.01f, C2 = 0.03f * 0.03f;
-      float* A = hq;
-      float* B = hq + R1 * R1;
-      float* Cc = hq + 2 * R1 * R1;
-      for (int k = threadIdx.x; k < R1 * R1; k += kThreads) {
-        const int r = k / R1, c = k % R1;
+    // ---- vertical windows -> moments -> SSIM and its partials A, B, C (zero off-image)
+    constexpr int VSEG = (MH + RUN - 1) / RUN;
+    for (int it = threadIdx.x; it < MW * VSEG; it += kThreads) {
+      const int c = it % MW, r0 = (it / MW) * RUN;
+      float m[5][RUN];
+#pragma unroll
+      for (int q = 0; q < 5; ++q) {
+        float col[RUN + 10];
+#pragma unroll
+        for (int t = 0; t < RUN + 10; ++t) col[t] = h5[q * IH * MW + min(r0 + t, IH - 1) * MW + c];
+#pragma unroll
+        for (int o = 0; o < RUN; ++o) {
+          float a = 0.f;
+#pragma unroll
+          for (int t = 0; t < 11; ++t) a = fmaf(w[t], col[o + t], a);
+          m[q][o] = a;
+        }
+      }
+#pragma unroll
+      for (int o = 0; o < RUN; ++o) {
+        const int r = r0 + o;
+        if (r >= MH) continue;
         const int gy = oy - 5 + r, gx = ox - 5 + c;
-        float av = 0.f, bv = 0.f, cv = 0.f;
+        float A = 0.f, B = 0.f, Cc = 0.f;
         if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
-          const float mx = mq[k], my = mq[R1 * R1 + k];
-          const float vx = mq[2 * R1 * R1 + k] - mx * mx;
-          const float vy = mq[3 * R1 * R1 + k] - my * my;
-          const float cxy = mq[4 * R1 * R1 + k] - mx * my;
+          const float mx = m[0][o], my = m[1][o];
+          const float vx = m[2][o] - mx * mx, vy = m[3][o] - my * my, cxy = m[4][o] - mx * my;
           const float N1 = 2.f * mx * my + C1, N2 = 2.f * cxy + C2;
           const float D1 = mx * mx + my * my + C1, D2 = vx + vy + C2;
           const float iD = 1.f / (D1 * D2);
           const float S = N1 * N2 * iD;
-          const float dmx = (2.f * my * N2 - S * 2.f * mx * D2) * iD;
           const float dvx = -S / D2;
           const float dcxy = 2.f * N1 * iD;
-          av = dmx - 2.f * mx * dvx - my * dcxy;
-          bv = dvx;
-          cv = dcxy;
-          if (r >= 5 && r < 5 + T && c >= 5 && c < 5 + T) ssim += S;
+          A = (2.f * my * N2 - S * 2.f * mx * D2) * iD - 2.f * mx * dvx - my * dcxy;
+          B = dvx;
+          Cc = dcxy;
+          if (r >= 5 && r < 5 + TH && c >= 5 && c < 5 + TW) ssim += S;
         }
-        A[k] = av; B[k] = bv; Cc[k] = cv;
+        const int k = r * MW + c;
+        abc[k] = A; abc[MH * MW + k] = B; abc[2 * MH * MW + k] = Cc;
       }
     }
     __syncthreads();
-    // horizontal windows of A, B, C: [R1][T]
-    for (int k = threadIdx.x; k < R1 * T; k += kThreads) {
-      const int r = k / T, c = k % T;
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f;
+    // ---- horizontal windows of A, B, C: [MH][TW]
+    constexpr int HSEG3 = TW / RUN;
+    for (int it = threadIdx.x; it < MH * HSEG3; it += kThreads) {
+      const int r = it / HSEG3, c0 = (it - r * HSEG3) * RUN;
 #pragma unroll
-      for (int t = 0; t < 11; ++t) {
-        const float wt = w[t];
-        const int idx = r * R1 + c + t;
-        a0 += wt * hq[idx]; a1 += wt * hq[R1 * R1 + idx]; a2 += wt * hq[2 * R1 * R1 + idx];
+      for (int q = 0; q < 3; ++q) {
+        float v[RUN + 10];
+#pragma unroll
+        for (int t = 0; t < RUN + 10; ++t) v[t] = abc[q * MH * MW + r * MW + c0 + t];
+#pragma unroll
+        for (int o = 0; o < RUN; ++o) {
+          float a = 0.f;
+#pragma unroll
+          for (int t = 0; t < 11; ++t) a = fmaf(w[t], v[o + t], a);
+          h3[q * MH * TW + r * TW + c0 + o] = a;
+        }
       }
-      mq[k] = a0; mq[R1 * T + k] = a1; mq[2 * R1 * T + k] = a2;
     }
     __syncthreads();
-    // vertical windows and the gradient on the output tile
-    for (int k = threadIdx.x; k < T * T; k += kThreads) {
-      const int r = k / T, c = k % T;
-      const int gy = oy + r, gx = ox + c;
-      if (gx >= W || gy >= H) continue;
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f;
+    // ---- vertical windows and the gradient on the output tile
+    constexpr int VSEG3 = TH / RUN;
+    for (int it = threadIdx.x; it < TW * VSEG3; it += kThreads) {
+      const int c = it % TW, r0 = (it / TW) * RUN;
+      float g[3][RUN];
 #pragma unroll
-      for (int t = 0; t < 11; ++t) {
-        const float wt = w[t];
-        const int idx = (r + t) * T + c;
-        a0 += wt * mq[idx]; a1 += wt * mq[R1 * T + idx]; a2 += wt * mq[2 * R1 * T + idx];
+      for (int q = 0; q < 3; ++q) {
+        float v[RUN + 10];
+#pragma unroll
+        for (int t = 0; t < RUN + 10; ++t) v[t] = h3[q * MH * TW + (r0 + t) * TW + c];
+#pragma unroll
+        for (int o = 0; o < RUN; ++o) {
+          float a = 0.f;
+#pragma unroll
+          for (int t = 0; t < 11; ++t) a = fmaf(w[t], v[o + t], a);
+          g[q][o] = a;
+        }
       }
-      const float xv = sX[(r + 10) * R0 + c + 10], yv = sY[(r + 10) * R0 + c + 10];
-      const float d = xv - yv;
-      l1 += fabsf(d);
-      const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
-      const float dS = a0 + 2.f * xv * a1 + yv * a2;
-      if (grad) grad[3 * ((long long)gy * W + gx) + ch] = ((1.f - lam) * sgn - lam * dS) * inv;
+#pragma unroll
+      for (int o = 0; o < RUN; ++o) {
+        const int gy = oy + r0 + o, gx = ox + c;
+        if (gx >= W || gy >= H) continue;
+        const float xv = sX[(r0 + o + 10) * IW + c + 10], yv = sY[(r0 + o + 10) * IW + c + 10];
+        const float d = xv - yv;
+        l1 += fabsf(d);
+        const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
+        const float dS = g[0][o] + 2.f * xv * g[1][o] + yv * g[2][o];
+        if (grad) grad[3 * ((long long)gy * W + gx) + ch] = ((1.f - lam) * sgn - lam * dS) * inv;
+      }
     }
     __syncthreads();
   }
@@ -208,7 +247,7 @@ abcd_status loss_launch(abcd_ctx* ctx, const float* out_rgba, const float* gt_rg
   if (!has_workspace(ctx)) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_loss: no workspace");
   if (!out_rgba || !gt_rgb || width <= 0 || height <= 0 || !(lambda_ssim >= 0.f && lambda_ssim <= 1.f))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_loss: bad arguments");
-  const dim3 grid((width + T - 1) / T, (height + T - 1) / T);
+  const dim3 grid((width + TW - 1) / TW, (height + TH - 1) / TH);
   if ((long long)grid.x * grid.y > kMaxLossBlocks)
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_loss: image too large (%d x %d)", width, height);
   const size_t smem = sizeof(float) * kSmemFloats;
@@ -236,7 +275,7 @@ extern "C" abcd_status abcd_loss(abcd_ctx* ctx, const float* out_rgba, const flo
 namespace abcd {
 namespace {
 
-constexpr int kStaticLossMaxBlocks = 16384;            // 32x32-pixel CTAs: up to 4096 x 4096
+constexpr int kStaticLossMaxBlocks = 16384;            // 64x32-pixel CTAs: up to 8192 x 4096
 constexpr int kStaticLossWords = 2 * kStaticLossMaxBlocks + 64;   // partial sums, then the ticket
 
 // Device scratch shared by every abcd_loss_static call on a device (held until exit).
@@ -269,7 +308,7 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
   if (!out_rgba || !gt_rgb || width <= 0 || height <= 0 ||
       !(lambda_ssim >= 0.f && lambda_ssim <= 1.f))
     return ABCD_ERR_INVALID_ARG;
-  const dim3 grid((width + T - 1) / T, (height + T - 1) / T);
+  const dim3 grid((width + TW - 1) / TW, (height + TH - 1) / TH);
   if ((long long)grid.x * grid.y > kStaticLossMaxBlocks) return ABCD_ERR_WORKSPACE;
   int device = 0;
   if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices)
