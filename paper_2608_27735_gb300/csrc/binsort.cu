@@ -81,7 +81,12 @@ __global__ void keys_rects_kernel(const float* depth, const int* radius, const f
 // keeps every tile the exact rule keeps.  Round-to-nearest intrinsics only: count and emit
 // kernels get the same bits.
 struct Splat {
-  float u, v, ha, hb, hc, lim, det4;   // det4 = 4 ha hc - hb^2 > 0
+  float u, v, hb, lim;
+  float ym;        // |dy| <= ym on E
+  float dyl;       // dy of the leftmost point of E (the rightmost is at -dyl)
+  float fal;       // 4 ha lim
+  float det4;      // 4 ha hc - hb^2 > 0
+  float inv2a;     // 1 / (2 ha)
 };
 
 __device__ __forceinline__ float diff_of_products(float a, float b, float c, float d) {
@@ -98,13 +103,24 @@ __device__ __forceinline__ Splat load_splat(const float2* uv, const float4* co, 
   const float4 c = co[g];
   Splat s;
   s.u = m.x; s.v = m.y;
-  s.ha = __fmul_rn(0.7213475204444817f, c.x);   // log2(e)/2
-  s.hb = __fmul_rn(1.4426950408889634f, c.y);   // log2(e)
-  s.hc = __fmul_rn(0.7213475204444817f, c.z);
-  s.det4 = diff_of_products(__fmul_rn(4.f, s.ha), s.hc, s.hb, s.hb);
+  const float ha = __fmul_rn(0.7213475204444817f, c.x);   // log2(e)/2
+  s.hb = __fmul_rn(1.4426950408889634f, c.y);             // log2(e)
+  const float hc = __fmul_rn(0.7213475204444817f, c.z);
+  s.det4 = diff_of_products(__fmul_rn(4.f, ha), hc, s.hb, s.hb);
   // alpha = o 2^-sigma' >= alpha_min  <=>  sigma' <= log2(o / alpha_min); margin 0.01 + 0.1%
   const float thr = c.w >= alpha_min ? log2f(__fdiv_rn(c.w, alpha_min)) : -1.f;
-  s.lim = (thr >= 0.f && s.det4 > 0.f) ? __fmul_rn(__fadd_rn(__fmul_rn(thr, 1.001f), 0.01f), 1.001f) : -1.f;
+  s.lim = (thr >= 0.f && s.det4 > 0.f && ha > 0.f && hc > 0.f)
+              ? __fmul_rn(__fadd_rn(__fmul_rn(thr, 1.001f), 0.01f), 1.001f) : -1.f;
+  s.fal = __fmul_rn(__fmul_rn(4.f, ha), s.lim);
+  s.ym = 0.f; s.dyl = 0.f; s.inv2a = 0.f;
+  if (s.lim >= 0.f) {
+    // |dy| <= ym on E: D(dy) = 4 ha lim - det4 dy^2 >= 0
+    s.ym = __fsqrt_rn(__fdiv_rn(s.fal, s.det4));
+    // leftmost point of E: dx = -mx, dy = hb mx / (2 hc); mx = sqrt(4 hc lim / det4)
+    const float mx = __fsqrt_rn(__fdiv_rn(__fmul_rn(__fmul_rn(4.f, hc), s.lim), s.det4));
+    s.dyl = __fdiv_rn(__fmul_rn(s.hb, mx), __fmul_rn(2.f, hc));
+    s.inv2a = __frcp_rn(__fmul_rn(2.f, ha));
+  }
   return s;
 }
 
@@ -113,21 +129,16 @@ __device__ __forceinline__ int2 row_run(const Splat& s, int4 q, int ty) {
   if (!(s.lim >= 0.f)) return make_int2(0, 0);
   const float Y0 = __fsub_rn((float)(ty * kTile) + 0.5f, s.v);
   const float Y1 = __fadd_rn(Y0, (float)(kTile - 1));
-  // |dy| <= ym on E: D(dy) >= 0  <=>  dy^2 (4 ha hc - hb^2) <= 4 ha lim
-  const float ym = __fsqrt_rn(__fdiv_rn(__fmul_rn(__fmul_rn(4.f, s.ha), s.lim), s.det4));
-  const float ylo = fmaxf(Y0, -ym), yhi = fminf(Y1, ym);
+  const float ylo = fmaxf(Y0, -s.ym), yhi = fminf(Y1, s.ym);
   if (!(ylo <= yhi)) return make_int2(0, 0);
-  // leftmost point of E: dx = -mx, dy = hb mx / (2 hc); mx = sqrt(4 hc lim / det4)
-  const float mx = __fsqrt_rn(__fdiv_rn(__fmul_rn(__fmul_rn(4.f, s.hc), s.lim), s.det4));
-  const float dyl = __fdiv_rn(__fmul_rn(s.hb, mx), __fmul_rn(2.f, s.hc));
-  const float inv2a = __frcp_rn(__fmul_rn(2.f, s.ha));
-  // boundary x at dy: (-hb dy -+ sqrt(D)) / (2 ha), D = 4 ha lim - det4 dy^2
-  const float yl = fminf(fmaxf(dyl, ylo), yhi);
-  const float Dl = fmaxf(__fmaf_rn(-s.det4, __fmul_rn(yl, yl), __fmul_rn(__fmul_rn(4.f, s.ha), s.lim)), 0.f);
-  const float xl = __fmul_rn(__fsub_rn(__fmul_rn(-s.hb, yl), __fsqrt_rn(Dl)), inv2a);
-  const float yr = fminf(fmaxf(-dyl, ylo), yhi);
-  const float Dr = fmaxf(__fmaf_rn(-s.det4, __fmul_rn(yr, yr), __fmul_rn(__fmul_rn(4.f, s.ha), s.lim)), 0.f);
-  const float xr = __fmul_rn(__fadd_rn(__fmul_rn(-s.hb, yr), __fsqrt_rn(Dr)), inv2a);
+  // boundary x at dy: (-hb dy -+ sqrt(D)) / (2 ha), D = 4 ha lim - det4 dy^2; the least x over
+  // the band is at the leftmost point's dy clamped into it, the largest at -dyl clamped
+  const float yl = fminf(fmaxf(s.dyl, ylo), yhi);
+  const float Dl = fmaxf(__fmaf_rn(-s.det4, __fmul_rn(yl, yl), s.fal), 0.f);
+  const float xl = __fmul_rn(__fsub_rn(__fmul_rn(-s.hb, yl), __fsqrt_rn(Dl)), s.inv2a);
+  const float yr = fminf(fmaxf(-s.dyl, ylo), yhi);
+  const float Dr = fmaxf(__fmaf_rn(-s.det4, __fmul_rn(yr, yr), s.fal), 0.f);
+  const float xr = __fmul_rn(__fadd_rn(__fmul_rn(-s.hb, yr), __fsqrt_rn(Dr)), s.inv2a);
   // tiles whose centre box [16 tx + 0.5, 16 tx + 15.5] meets [u + xl, u + xr]
   const float fa = ceilf(__fmul_rn(__fsub_rn(__fadd_rn(s.u, xl), 15.5f), 1.f / kTile));
   const float fb = floorf(__fmul_rn(__fsub_rn(__fadd_rn(s.u, xr), 0.5f), 1.f / kTile)) + 1.f;
@@ -137,28 +148,47 @@ __device__ __forceinline__ int2 row_run(const Splat& s, int4 q, int ty) {
 }
 
 // ---- one thread per Gaussian, looping over its tile rows: the pair count and +1 / -1 at the
-// ends of every row's run in the per-row difference array (rows are short; this many threads
-// hide the latency of the per-Gaussian loads)
+// ends of every row's run in the per-row difference array.  The +-1 go to a block-local copy of
+// the difference array in shared memory first (the same few thousand cells are hit by every
+// block), then only its non-zero cells to the global array.
+constexpr int kSmemDiffCells = 12288;      // 48 KB: tile grids up to ~1900x1500 pixels
+
 __global__ void __launch_bounds__(256)
 tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, int tiles_x,
-                 float alpha_min, unsigned* counts, int* diff) {
-  const int g = blockIdx.x * blockDim.x + threadIdx.x;
-  if (g >= n) return;
+                 int tiles_y, float alpha_min, unsigned* counts, int* diff) {
+  extern __shared__ int sdiff[];
   const int W1 = tiles_x + 1;
-  const int4 q = rects[g];
-  unsigned c = 0;
-  if (q.x < q.z) {
-    const Splat s = load_splat(uv, co, (unsigned)g, alpha_min);
-    for (int ty = q.y; ty < q.w; ++ty) {
-      const int2 r = row_run(s, q, ty);
-      if (r.y > r.x) {
-        c += (unsigned)(r.y - r.x);
-        atomicAdd(&diff[ty * W1 + r.x], 1);
-        atomicAdd(&diff[ty * W1 + r.y], -1);
+  const int cells = W1 * (tiles_y + 1);
+  const bool local = cells <= kSmemDiffCells;
+  if (local) {
+    for (int k = threadIdx.x; k < cells; k += blockDim.x) sdiff[k] = 0;
+    __syncthreads();
+  }
+  int* dst = local ? sdiff : diff;
+  const int g = blockIdx.x * blockDim.x + threadIdx.x;
+  if (g < n) {
+    const int4 q = rects[g];
+    unsigned c = 0;
+    if (q.x < q.z) {
+      const Splat s = load_splat(uv, co, (unsigned)g, alpha_min);
+      for (int ty = q.y; ty < q.w; ++ty) {
+        const int2 r = row_run(s, q, ty);
+        if (r.y > r.x) {
+          c += (unsigned)(r.y - r.x);
+          atomicAdd(&dst[ty * W1 + r.x], 1);
+          atomicAdd(&dst[ty * W1 + r.y], -1);
+        }
       }
     }
+    counts[g] = c;
   }
-  counts[g] = c;
+  if (local) {
+    __syncthreads();
+    for (int k = threadIdx.x; k < cells; k += blockDim.x) {
+      const int v = sdiff[k];
+      if (v != 0) atomicAdd(&diff[k], v);
+    }
+  }
 }
 
 // ---- radix pass, step 1: per-block digit counts hist[d * G + b]
@@ -373,7 +403,13 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
   for (long long base = lo; base < hi; base += blockDim.x) {
     const long long i = base + threadIdx.x;
     unsigned id = 0, t = 0;
-    if (i < hi) { id = (unsigned)sorted[i]; t = counts[id]; }
+    int4 qm = make_int4(0, 0, 0, 0);
+    Splat sm_ = {};
+    if (i < hi) {
+      id = (unsigned)sorted[i];
+      t = counts[id];
+      if (t > 0) { qm = rects[id]; sm_ = load_splat(uv, co, id, alpha_min); }
+    }
     unsigned long long tot = 0;
     const unsigned long long off = run + block_exclusive_scan(t, &tot);
     for (int j = 0; j < 32; ++j) {
@@ -381,8 +417,19 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
       if (tj == 0) continue;
       const unsigned idj = __shfl_sync(0xffffffffu, id, j);
       const unsigned long long oj = __shfl_sync(0xffffffffu, off, j);
-      const int4 q = rects[idj];
-      const Splat s = load_splat(uv, co, idj, alpha_min);
+      // lane j prepared Gaussian j: broadcast its rectangle and ellipse
+      const int4 q = make_int4(__shfl_sync(0xffffffffu, qm.x, j), __shfl_sync(0xffffffffu, qm.y, j),
+                               __shfl_sync(0xffffffffu, qm.z, j), __shfl_sync(0xffffffffu, qm.w, j));
+      Splat s;
+      s.u = __shfl_sync(0xffffffffu, sm_.u, j);
+      s.v = __shfl_sync(0xffffffffu, sm_.v, j);
+      s.hb = __shfl_sync(0xffffffffu, sm_.hb, j);
+      s.lim = __shfl_sync(0xffffffffu, sm_.lim, j);
+      s.ym = __shfl_sync(0xffffffffu, sm_.ym, j);
+      s.dyl = __shfl_sync(0xffffffffu, sm_.dyl, j);
+      s.fal = __shfl_sync(0xffffffffu, sm_.fal, j);
+      s.det4 = __shfl_sync(0xffffffffu, sm_.det4, j);
+      s.inv2a = __shfl_sync(0xffffffffu, sm_.inv2a, j);
       unsigned done = 0;
       for (int y0 = q.y; y0 < q.w && done < tj; y0 += 32) {
         const int ty = y0 + lane;
@@ -484,9 +531,15 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       ctx->ws.rects);
   if ((s = check_launch(ctx, "keys_rects_kernel"))) return s;
   {
-    tile_rows_kernel<<<(n + 255) / 256, 256, 0, ctx->stream>>>(
+    const int cells = (tiles_x + 1) * (tiles_y + 1);
+    const size_t smem = cells <= kSmemDiffCells ? sizeof(int) * cells : 0;
+    if (smem > 48 * 1024) {
+      const cudaError_t e2 = cudaFuncSetAttribute(tile_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile_rows smem: %s", cudaGetErrorString(e2));
+    }
+    tile_rows_kernel<<<(n + 255) / 256, 256, smem, ctx->stream>>>(
         (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects, n, tiles_x,
-        alpha_min, ctx->ws.counts, ctx->ws.diff);
+        tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff);
     if ((s = check_launch(ctx, "tile_rows_kernel"))) return s;
   }
   u64* by_depth = nullptr;
