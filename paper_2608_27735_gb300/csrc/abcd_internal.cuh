@@ -49,7 +49,14 @@ struct Workspace {
   float* grad2d;                    // [max_g][9]
   float* dl_dout;                   // [max_pixels][3]
   float* loss_partials;             // [kMaxLossBlocks][2]
+  unsigned* block_work;             // [max_blocks] per render CTA: list entries its backward walks
+  unsigned* block_order;            // [max_blocks] render CTAs, most work first
+  long long max_blocks;
 };
+
+// Render CTAs (8x8 pixel blocks, four per tile) the workspace orders for images of up to
+// max_pixels pixels with sides up to 16384.
+inline long long max_render_blocks(long long max_pixels) { return 4 * (max_pixels / 256 + 2048); }
 
 }  // namespace abcd
 

@@ -6,15 +6,25 @@
 // frozen partitions enter through out = F over (A over B) (Section 2), over meaning
 // X + (1 - X.a) Y on premultiplied RGBA, and out.rgb += (1 - out.a) bg.
 //
-// One CTA per 8x8 block of pixels (four per 16x16 binning tile), one thread per pixel, so the
-// few heavily covered tiles of a small active block spread over four times as many CTAs and
-// each CTA stops as soon as its own 64 pixels have terminated (__syncthreads_count).  List
-// entries are staged 256 at a time in shared memory; while staging, an entry whose opacity
+// One warp per 8x8 block of pixels (four per 16x16 binning tile), two pixels per lane --
+// (x, y) and (x + 4, y), which share the shared-memory loads and the dy terms of sigma -- so
+// the few heavily covered tiles of a small active block spread over four times as many CTAs,
+// each lane runs two independent blend chains, and each CTA stops as soon as its own 64
+// pixels have terminated.  List entries are staged in shared memory; an entry whose opacity
 // cannot reach alpha_min anywhere on the CTA's pixel-centre box (analytic minimum of the
-// quadratic form over the box, with a margin far above fp32 rounding) is dropped: every pixel
-// would skip it, so results are unchanged.  Every quantity that decides a branch per pixel
+// quadratic form over the box, with a margin far above fp32 rounding) is dropped while
+// staging -- every pixel would skip it, so results are unchanged -- and staging keeps loading
+// groups of 64 entries, all in flight at once, until a batch of survivors is full, so the
+// blocks that walk a long list whose entries mostly miss them are bound by bandwidth rather
+// than by one load round trip per 32 entries.  Every quantity that decides a branch per pixel
 // (sigma, alpha, T) is computed with explicit round-to-nearest intrinsics in one shared
 // function, so the backward kernel retraces exactly the forward's contributors.
+//
+// Work is very uneven across blocks (lists of a few entries next to lists of 15,000), so with
+// a workspace each launch first orders its CTAs by decreasing work -- list length for the
+// forward, the longest contributor walk the forward recorded per block for the backward -- and
+// the longest blocks start in the first wave instead of trailing the launch.  The order
+// changes no result (CTAs are independent; the backward's gradient sums are atomic either way).
 #include "abcd_internal.cuh"
 
 namespace abcd {
@@ -23,6 +33,14 @@ namespace {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kHalfLog2e = 0.7213475204444817f;
 constexpr float kLn2 = 0.6931471805599453f;
+
+constexpr int kSub = 8;                          // CTA pixel block edge
+constexpr int kSubThreads = 32;                  // one warp, two pixels per lane
+constexpr int kSubPerTile = (kTile / kSub) * (kTile / kSub);
+constexpr int kRounds = 2;                       // list entries per lane per staging group
+constexpr int kGroup = kSubThreads * kRounds;    // 64 entries loaded together
+constexpr int kBatch = 2 * kGroup;               // staged survivors per batch (at most)
+constexpr int kOrderBuckets = 256;
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -35,31 +53,33 @@ __device__ __forceinline__ float4 scaled_conic(float4 c) {
   return make_float4(__fmul_rn(kHalfLog2e, c.x), __fmul_rn(kLog2e, c.y), __fmul_rn(kHalfLog2e, c.z), c.w);
 }
 
-// sigma * log2(e) = dx (a/2 dx + b dy) + c/2 dy^2 in log2 units; dx, dy returned.
-__device__ __forceinline__ float sigma2(float4 s, float2 m, float fx, float fy, float& dx, float& dy) {
-  dx = __fsub_rn(fx, m.x);
+// sigma * log2(e) = dx (a/2 dx + b dy) + c/2 dy^2 at the lane's two pixels (fx0, fy) and
+// (fx1, fy); the dy terms are shared.  Both kernels take every branch decision from these bits.
+__device__ __forceinline__ void sigma_pair(float4 s, float2 m, float fx0, float fx1, float fy,
+                                           float& dx0, float& dx1, float& dy, float& s0, float& s1) {
   dy = __fsub_rn(fy, m.y);
-  return __fmaf_rn(dx, __fmaf_rn(s.x, dx, __fmul_rn(s.y, dy)), __fmul_rn(__fmul_rn(s.z, dy), dy));
+  dx0 = __fsub_rn(fx0, m.x);
+  dx1 = __fsub_rn(fx1, m.x);
+  const float bdy = __fmul_rn(s.y, dy);
+  const float cdy2 = __fmul_rn(__fmul_rn(s.z, dy), dy);
+  s0 = __fmaf_rn(dx0, __fmaf_rn(s.x, dx0, bdy), cdy2);
+  s1 = __fmaf_rn(dx1, __fmaf_rn(s.x, dx1, bdy), cdy2);
 }
 
-constexpr int kSub = 8;                          // CTA pixel block edge
-constexpr int kSubThreads = kSub * kSub;         // 64
-constexpr int kSubPerTile = (kTile / kSub) * (kTile / kSub);
-constexpr int kRounds = 4;                       // list entries per thread per batch
-constexpr int kBatch = kSubThreads * kRounds;    // 256
-
 // Lower bound of sigma * log2(e) over the box [X0, X1] x [Y0, Y1] of offsets d = pixel - uv:
-// 0 if the box contains d = 0, else the least value on its four edges (convex quadratic).
+// 0 if the box contains d = 0, else the least value on its four edges (convex quadratic; on
+// each edge the minimiser of the other coordinate is clamped into the box).
 __device__ __forceinline__ float box_min_sigma2(float4 s, float X0, float X1, float Y0, float Y1) {
   if (X0 <= 0.f && X1 >= 0.f && Y0 <= 0.f && Y1 >= 0.f) return 0.f;
+  const float ry = __fdividef(-s.y, 2.f * s.z), rx = __fdividef(-s.y, 2.f * s.x);
   float best = 3.0e38f;
 #pragma unroll
   for (int e = 0; e < 2; ++e) {
     const float X = e ? X1 : X0;
-    const float dy = fminf(fmaxf(-s.y * X / (2.f * s.z), Y0), Y1);
+    const float dy = fminf(fmaxf(ry * X, Y0), Y1);
     best = fminf(best, X * (s.x * X + s.y * dy) + s.z * dy * dy);
     const float Y = e ? Y1 : Y0;
-    const float dx = fminf(fmaxf(-s.y * Y / (2.f * s.x), X0), X1);
+    const float dx = fminf(fmaxf(rx * Y, X0), X1);
     best = fminf(best, dx * (s.x * dx + s.y * Y) + s.z * Y * Y);
   }
   return best;
@@ -70,32 +90,9 @@ __device__ __forceinline__ float box_min_sigma2(float4 s, float X0, float X1, fl
 // orders of magnitude above the fp32 error of either evaluation.
 __device__ __forceinline__ bool cull(float4 s, float2 m, float bx0, float by0, float alpha_min) {
   if (!(s.w >= alpha_min)) return true;
-  const float thr = __log2f(s.w / alpha_min);
+  const float thr = __log2f(__fdividef(s.w, alpha_min));
   const float lo = box_min_sigma2(s, bx0 - m.x, bx0 + (kSub - 1) - m.x, by0 - m.y, by0 + (kSub - 1) - m.y);
   return lo * 0.998f > thr + 0.02f;
-}
-
-// Adds the warp-wide sums of v[0..9) to dst[0..9).  Transpose reduction: at each step a lane
-// keeps half of its (padded to 16) partial sums and receives the partner's matching half, so
-// 16 shuffles replace the 45 of a butterfly per value; afterwards lanes 2c, 2c + 1 hold the
-// sum of component c = lane / 2 (bits 4..1), and lane 2c adds it to memory.
-__device__ __forceinline__ void warp_sum9_atomic(const float v[9], float* dst, int lane) {
-  float x[16];
-#pragma unroll
-  for (int k = 0; k < 16; ++k) x[k] = k < 9 ? v[k] : 0.f;
-#pragma unroll
-  for (int w = 8; w >= 1; w >>= 1) {       // halves of 16, 8, 4, 2 values; lane bits 4..1
-    const bool up = (lane & (2 * w)) != 0;
-#pragma unroll
-    for (int k = 0; k < w; ++k) {
-      const float send = up ? x[k] : x[k + w];
-      const float keep = up ? x[k + w] : x[k];
-      x[k] = keep + __shfl_xor_sync(0xffffffffu, send, 2 * w);
-    }
-  }
-  x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
-  const int c = lane >> 1;
-  if ((lane & 1) == 0 && c < 9) atomicAdd(&dst[c], x[0]);
 }
 
 __device__ __forceinline__ float4 load_px(const void* img, int dtype, long long p) {
@@ -107,6 +104,142 @@ __device__ __forceinline__ float4 load_px(const void* img, int dtype, long long 
     return make_float4(fa.x, fa.y, fb.x, fb.y);
   }
   return reinterpret_cast<const float4*>(img)[p];
+}
+
+// Stages list entries from position `next` on, in groups of kGroup whose loads are all issued
+// before any is used, until more than kBatch - kGroup survivors of the CTA-box cull are staged
+// or position n is reached; survivors are compacted in list order, each with its list
+// position in s_rgb[.].w (bits) and, for the backward, its Gaussian id.  Returns the number
+// staged.  next and the count are warp-uniform.
+template <bool WITH_ID>
+__device__ __forceinline__ int stage_fill(const unsigned* ids, unsigned start, int n, int& next,
+                                          const float2* uv, const float4* co, const float* rgb,
+                                          float bx0, float by0, float alpha_min, float2* s_uv,
+                                          float4* s_co, float4* s_rgb, unsigned* s_id) {
+  const int lane = threadIdx.x & 31;
+  const unsigned lt = (1u << lane) - 1u;
+  int total = 0;
+  while (next < n && total <= kBatch - kGroup) {
+    unsigned g[kRounds];
+    float2 m[kRounds];
+    float4 c[kRounds];
+    float col[kRounds][3];
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) {
+      const int pos = next + lane + r * kSubThreads;
+      g[r] = pos < n ? __ldg(ids + start + pos) : 0xffffffffu;
+    }
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) {
+      if (g[r] != 0xffffffffu) {
+        m[r] = __ldg(uv + g[r]);
+        c[r] = __ldg(co + g[r]);
+        col[r][0] = __ldg(rgb + 3 * g[r]);
+        col[r][1] = __ldg(rgb + 3 * g[r] + 1);
+        col[r][2] = __ldg(rgb + 3 * g[r] + 2);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) {
+      bool keep = false;
+      float4 sc = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (g[r] != 0xffffffffu) {
+        sc = scaled_conic(c[r]);
+        keep = !cull(sc, m[r], bx0, by0, alpha_min);
+      }
+      const unsigned b = __ballot_sync(0xffffffffu, keep);
+      if (keep) {
+        const int slot = total + __popc(b & lt);
+        s_uv[slot] = m[r];
+        s_co[slot] = sc;
+        s_rgb[slot] = make_float4(col[r][0], col[r][1], col[r][2],
+                                  __uint_as_float((unsigned)(next + lane + r * kSubThreads)));
+        if (WITH_ID) s_id[slot] = g[r];
+      }
+      total += __popc(b);
+    }
+    next += kGroup;
+  }
+  __syncwarp();
+  return total;
+}
+
+// Orders n_blocks render CTAs by decreasing work (16 buckets per octave, counting sort in one
+// CTA; within a bucket in no particular order).  work = tile list length for the forward
+// (span == nullptr), else span[block].  Produces a permutation whatever the work values are.
+__global__ void __launch_bounds__(1024) order_kernel(const uint2* ranges, const unsigned* span,
+                                                     int n_blocks, unsigned* order) {
+  __shared__ unsigned hist[kOrderBuckets];
+  const int tid = threadIdx.x, lane = tid & 31;
+  const unsigned lt = (1u << lane) - 1u;
+  for (int i = tid; i < kOrderBuckets; i += blockDim.x) hist[i] = 0;
+  __syncthreads();
+  auto key_of = [&](int i) -> unsigned {
+    if (i >= n_blocks) return kOrderBuckets;
+    unsigned w;
+    if (span) {
+      w = span[i];
+    } else {
+      const uint2 rg = ranges[i / kSubPerTile];
+      w = rg.y > rg.x ? rg.y - rg.x : 0u;
+    }
+    if (w == 0) return kOrderBuckets - 1;
+    const int b = (int)(__log2f((float)w) * 16.f) + 1;
+    return (unsigned)(kOrderBuckets - 1 - min(b, kOrderBuckets - 1));
+  };
+  for (int i0 = 0; i0 < n_blocks; i0 += blockDim.x) {
+    const unsigned key = key_of(i0 + tid);
+    const unsigned peers = __match_any_sync(0xffffffffu, key);
+    if (key < kOrderBuckets && (peers & lt) == 0) atomicAdd(&hist[key], (unsigned)__popc(peers));
+  }
+  __syncthreads();
+  if (tid < 32) {                        // exclusive scan of the 256 counts, 8 per lane
+    constexpr int kPer = kOrderBuckets / 32;
+    unsigned v[kPer], sum = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) { v[k] = hist[tid * kPer + k]; sum += v[k]; }
+    unsigned incl = sum;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const unsigned o = __shfl_up_sync(0xffffffffu, incl, d);
+      if (lane >= d) incl += o;
+    }
+    unsigned run = incl - sum;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) { hist[tid * kPer + k] = run; run += v[k]; }
+  }
+  __syncthreads();
+  for (int i0 = 0; i0 < n_blocks; i0 += blockDim.x) {
+    const unsigned key = key_of(i0 + tid);
+    const unsigned peers = __match_any_sync(0xffffffffu, key);
+    const int leader = __ffs(peers) - 1;
+    unsigned base = 0;
+    if (key < kOrderBuckets && lane == leader) base = atomicAdd(&hist[key], (unsigned)__popc(peers));
+    base = __shfl_sync(0xffffffffu, base, leader);
+    if (key < kOrderBuckets) order[base + __popc(peers & lt)] = (unsigned)(i0 + tid);
+  }
+}
+
+// The CTA's 8x8 pixel block and the lane's two pixels (qx0, py), (qx1 = qx0 + 4, py).
+struct Block {
+  int tile, px0, py0, qx0, qx1, py;
+  bool in0, in1;
+};
+
+__device__ __forceinline__ Block block_of(const Cam& cam, int blk) {
+  Block b;
+  b.tile = blk / kSubPerTile;
+  const int sub = blk % kSubPerTile;
+  const int tx = b.tile % cam.tiles_x, ty = b.tile / cam.tiles_x;
+  b.px0 = tx * kTile + (sub % (kTile / kSub)) * kSub;
+  b.py0 = ty * kTile + (sub / (kTile / kSub)) * kSub;
+  const int lane = threadIdx.x & 31;
+  b.qx0 = b.px0 + (lane & 3);
+  b.qx1 = b.qx0 + 4;
+  b.py = b.py0 + (lane >> 2);
+  b.in0 = b.qx0 < cam.width && b.py < cam.height;
+  b.in1 = b.qx1 < cam.width && b.py < cam.height;
+  return b;
 }
 
 struct FwdArgs {
@@ -125,115 +258,81 @@ struct FwdArgs {
   float4* state_at;
   unsigned* n_last;
   uint2* refresh;      // fp16 x4 per pixel
+  const unsigned* order;   // CTA order (nullptr: launch order)
+  unsigned* block_work;    // per block: max n_last over its pixels (nullptr: not recorded)
 };
 
-// Stages one batch of list entries (positions base .. base + kBatch) and compacts the indices
-// of the entries that survive the CTA-box cull into s_idx; returns the number of survivors.
-template <bool WITH_ID>
-__device__ __forceinline__ int stage_batch(const unsigned* ids, unsigned start, int n, int base,
-                                           const float2* uv, const float4* co, const float* rgb,
-                                           float bx0, float by0, float alpha_min, float2* s_uv,
-                                           float4* s_co, float4* s_rgb, unsigned* s_id,
-                                           unsigned short* s_idx, unsigned* s_ballot) {
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  bool keep[kRounds];
-#pragma unroll
-  for (int r = 0; r < kRounds; ++r) {
-    const int q = threadIdx.x + r * kSubThreads;
-    keep[r] = false;
-    if (base + q < n) {
-      const unsigned g = ids[start + base + q];
-      const float2 m = uv[g];
-      const float4 sc = scaled_conic(co[g]);
-      keep[r] = !cull(sc, m, bx0, by0, alpha_min);
-      if (keep[r]) {
-        s_uv[q] = m;
-        s_co[q] = sc;
-        s_rgb[q] = make_float4(rgb[3 * g], rgb[3 * g + 1], rgb[3 * g + 2], 0.f);
-        if (WITH_ID) s_id[q] = g;
-      }
-    }
-    const unsigned b = __ballot_sync(0xffffffffu, keep[r]);
-    if (lane == 0) s_ballot[r * 2 + w] = b;
-  }
-  __syncthreads();
-  int total = 0, before_r = 0;
-  const unsigned lt = (1u << lane) - 1u;
-#pragma unroll
-  for (int r = 0; r < kRounds; ++r) {
-    const unsigned b0 = s_ballot[2 * r], b1 = s_ballot[2 * r + 1];
-    const int at = before_r + (w ? __popc(b0) : 0) + __popc((w ? b1 : b0) & lt);
-    if (keep[r]) s_idx[at] = (unsigned short)(threadIdx.x + r * kSubThreads);
-    before_r += __popc(b0) + __popc(b1);
-  }
-  total = before_r;
-  __syncthreads();
-  return total;
+// Blend state of one pixel.
+struct PixF {
+  float T, c0, c1, c2;
+  unsigned last;       // one past the list position of the last contributor
+  bool done;
+};
+
+// One staged list entry as the blend loops read it.
+struct Entry {
+  float4 s;            // scaled conic, opacity
+  float2 m;            // uv
+  float4 col;          // rgb, list position (bits)
+};
+
+__device__ __forceinline__ Entry load_entry(const float2* s_uv, const float4* s_co,
+                                            const float4* s_rgb, int j) {
+  Entry e;
+  e.s = s_co[j];
+  e.m = s_uv[j];
+  e.col = s_rgb[j];
+  return e;
 }
 
-__global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
-  __shared__ float2 s_uv[kBatch];
-  __shared__ float4 s_co[kBatch];
-  __shared__ float4 s_rgb[kBatch];
-  __shared__ unsigned short s_idx[kBatch];
-  __shared__ unsigned s_ballot[2 * kRounds];
-  const int tile = blockIdx.x / kSubPerTile, sub = blockIdx.x % kSubPerTile;
-  const int tx = tile % a.cam.tiles_x, ty = tile / a.cam.tiles_x;
-  const int px0 = tx * kTile + (sub % (kTile / kSub)) * kSub;
-  const int py0 = ty * kTile + (sub / (kTile / kSub)) * kSub;
-  const int px = px0 + (threadIdx.x % kSub), py = py0 + (threadIdx.x / kSub);
-  const bool inside = px < a.cam.width && py < a.cam.height;
-  const uint2 rg = a.ranges[tile];
-  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
-  const float fx = (float)px + 0.5f, fy = (float)py + 0.5f;
-  const float bx0 = (float)px0 + 0.5f, by0 = (float)py0 + 0.5f;
-  float T = 1.f, c0 = 0.f, c1 = 0.f, c2 = 0.f;
-  unsigned last = 0;
-  bool done = !inside;
-  for (int base = 0; base < n; base += kBatch) {
-    if (__syncthreads_count(done) == kSubThreads) break;
-    const int cnt = stage_batch<false>(a.ids, rg.x, n, base, a.uv, a.co, a.rgb, bx0, by0,
-                                       a.op.alpha_min, s_uv, s_co, s_rgb, nullptr, s_idx, s_ballot);
-    if (!done) {
-      for (int j = 0; j < cnt; ++j) {
-        const int q = s_idx[j];
-        float dx, dy;
-        const float4 s = s_co[q];
-        const float sig = sigma2(s, s_uv[q], fx, fy, dx, dy);
-        if (!(sig >= 0.f)) continue;
-        const float alpha = fminf(a.op.alpha_max, __fmul_rn(s.w, ex2_approx(-sig)));
-        if (alpha < a.op.alpha_min) continue;
-        const float test = __fmul_rn(T, __fsub_rn(1.f, alpha));
-        if (test < a.op.t_min) { done = true; break; }
-        const float w = __fmul_rn(alpha, T);
-        const float4 col = s_rgb[q];
-        c0 = __fmaf_rn(w, col.x, c0);
-        c1 = __fmaf_rn(w, col.y, c1);
-        c2 = __fmaf_rn(w, col.z, c2);
-        T = test;
-        last = (unsigned)(base + q + 1);
-      }
-    }
-  }
-  if (!inside) return;
-  const long long p = (long long)py * a.cam.width + px;
-  const float Aa = 1.f - T;
+// alpha at the lane's two pixels for one entry and whether each passes the skip tests
+// (sigma >= 0, alpha >= alpha_min).  Independent of the blend state, so the loops evaluate
+// it for several entries before the transmittance chain needs it.
+__device__ __forceinline__ void alpha_pair(const Entry& e, float fx0, float fx1, float fy,
+                                           const Opts& op, float& a0, float& a1, bool& ok0,
+                                           bool& ok1) {
+  float dx0, dx1, dy, sg0, sg1;
+  sigma_pair(e.s, e.m, fx0, fx1, fy, dx0, dx1, dy, sg0, sg1);
+  a0 = fminf(op.alpha_max, __fmul_rn(e.s.w, ex2_approx(-sg0)));
+  a1 = fminf(op.alpha_max, __fmul_rn(e.s.w, ex2_approx(-sg1)));
+  ok0 = sg0 >= 0.f && a0 >= op.alpha_min;
+  ok1 = sg1 >= 0.f && a1 >= op.alpha_min;
+}
+
+// Front-to-back step of one pixel (selects, no branches): a passing entry either ends the
+// pixel (T (1 - alpha) < t_min; it does not contribute) or is blended in.
+__device__ __forceinline__ void blend(PixF& p, float alpha, bool ok, float4 col, const Opts& op) {
+  ok = ok && !p.done;
+  const float test = __fmul_rn(p.T, __fsub_rn(1.f, alpha));
+  const bool term = ok && test < op.t_min;
+  const bool use = ok && !term;
+  const float w = __fmul_rn(alpha, p.T);
+  p.done = p.done || term;
+  p.c0 = use ? __fmaf_rn(w, col.x, p.c0) : p.c0;
+  p.c1 = use ? __fmaf_rn(w, col.y, p.c1) : p.c1;
+  p.c2 = use ? __fmaf_rn(w, col.z, p.c2) : p.c2;
+  p.T = use ? test : p.T;
+  p.last = use ? __float_as_uint(col.w) + 1u : p.last;
+}
+
+__device__ __forceinline__ void store_pixel(const FwdArgs& a, long long p, const PixF& s) {
+  const float Aa = 1.f - s.T;
   if (a.refresh) {
-    const __half2 lo = __floats2half2_rn(c0, c1), hi = __floats2half2_rn(c2, Aa);
+    const __half2 lo = __floats2half2_rn(s.c0, s.c1), hi = __floats2half2_rn(s.c2, Aa);
     uint2 r;
     r.x = *reinterpret_cast<const unsigned*>(&lo);
     r.y = *reinterpret_cast<const unsigned*>(&hi);
     a.refresh[p] = r;
   }
   if (a.state_at) {
-    a.state_at[p] = make_float4(c0, c1, c2, T);
-    a.n_last[p] = last;
+    a.state_at[p] = make_float4(s.c0, s.c1, s.c2, s.T);
+    a.n_last[p] = s.last;
   }
   if (a.out) {
     const float4 Bv = a.B ? load_px(a.B, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
     const float4 Fv = a.F ? load_px(a.F, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
     const float kb = 1.f - Aa;      // A over B
-    const float m0 = c0 + kb * Bv.x, m1 = c1 + kb * Bv.y, m2 = c2 + kb * Bv.z, ma = Aa + kb * Bv.w;
+    const float m0 = s.c0 + kb * Bv.x, m1 = s.c1 + kb * Bv.y, m2 = s.c2 + kb * Bv.z, ma = Aa + kb * Bv.w;
     const float kf = 1.f - Fv.w;    // F over (A over B)
     float4 o = make_float4(Fv.x + kf * m0, Fv.y + kf * m1, Fv.z + kf * m2, Fv.w + kf * ma);
     const float kg = 1.f - o.w;
@@ -242,6 +341,48 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
     o.z += kg * a.bg[2];
     a.out[p] = o;
   }
+}
+
+__global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
+  __shared__ float2 s_uv[kBatch];
+  __shared__ float4 s_co[kBatch];
+  __shared__ float4 s_rgb[kBatch];
+  const int blk = a.order ? (int)a.order[blockIdx.x] : (int)blockIdx.x;
+  const Block bk = block_of(a.cam, blk);
+  const uint2 rg = a.ranges[bk.tile];
+  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
+  const float fx0 = (float)bk.qx0 + 0.5f, fx1 = (float)bk.qx1 + 0.5f, fy = (float)bk.py + 0.5f;
+  const float bx0 = (float)bk.px0 + 0.5f, by0 = (float)bk.py0 + 0.5f;
+  PixF p0 = {1.f, 0.f, 0.f, 0.f, 0u, !bk.in0};
+  PixF p1 = {1.f, 0.f, 0.f, 0.f, 0u, !bk.in1};
+  int next = 0;
+  while (next < n) {
+    if (__all_sync(0xffffffffu, p0.done && p1.done)) break;
+    __syncwarp();
+    const int cnt = stage_fill<false>(a.ids, rg.x, n, next, a.uv, a.co, a.rgb, bx0, by0,
+                                      a.op.alpha_min, s_uv, s_co, s_rgb, nullptr);
+    // two entries per iteration (slot j + 1 <= kBatch - 1 exists; unused when j + 1 == cnt)
+    for (int j = 0; j < cnt; j += 2) {
+      const Entry e0 = load_entry(s_uv, s_co, s_rgb, j);
+      const Entry e1 = load_entry(s_uv, s_co, s_rgb, j + 1);
+      float a00, a01, a10, a11;
+      bool k00, k01, k10, k11;
+      alpha_pair(e0, fx0, fx1, fy, a.op, a00, a01, k00, k01);
+      alpha_pair(e1, fx0, fx1, fy, a.op, a10, a11, k10, k11);
+      const bool v1 = j + 1 < cnt;
+      blend(p0, a00, k00, e0.col, a.op);
+      blend(p1, a01, k01, e0.col, a.op);
+      blend(p0, a10, k10 && v1, e1.col, a.op);
+      blend(p1, a11, k11 && v1, e1.col, a.op);
+      if ((j & 30) == 30 && __all_sync(0xffffffffu, p0.done && p1.done)) break;
+    }
+  }
+  if (a.block_work) {
+    const unsigned span = __reduce_max_sync(0xffffffffu, max(p0.last, p1.last));
+    if ((threadIdx.x & 31) == 0) a.block_work[blk] = span;
+  }
+  if (bk.in0) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx0, p0);
+  if (bk.in1) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx1, p1);
 }
 
 struct BwdArgs {
@@ -260,107 +401,142 @@ struct BwdArgs {
   const unsigned* n_last;
   const float* dl_dout;
   float* grad2d;
+  const unsigned* order;   // CTA order (nullptr: launch order)
 };
 
-__global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
-  __shared__ float2 s_uv[kBatch];
-  __shared__ float4 s_co[kBatch];
-  __shared__ float4 s_rgb[kBatch];
-  __shared__ unsigned s_id[kBatch];
-  __shared__ unsigned short s_idx[kBatch];
-  __shared__ unsigned s_ballot[2 * kRounds];
-  __shared__ unsigned s_max;
-  const int tile = blockIdx.x / kSubPerTile, sub = blockIdx.x % kSubPerTile;
-  const int tx = tile % a.cam.tiles_x, ty = tile / a.cam.tiles_x;
-  const int px0 = tx * kTile + (sub % (kTile / kSub)) * kSub;
-  const int py0 = ty * kTile + (sub / (kTile / kSub)) * kSub;
-  const int px = px0 + (threadIdx.x % kSub), py = py0 + (threadIdx.x / kSub);
-  const int lane = threadIdx.x & 31;
-  const bool inside = px < a.cam.width && py < a.cam.height;
-  const uint2 rg = a.ranges[tile];
-  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
-  const float fx = (float)px + 0.5f, fy = (float)py + 0.5f;
-  const float bx0 = (float)px0 + 0.5f, by0 = (float)py0 + 0.5f;
-  unsigned last = 0;
-  float Gr = 0.f, Gg = 0.f, Gb = 0.f, Ga = 0.f, Tf = 1.f, A0 = 0.f, A1 = 0.f, A2 = 0.f;
-  if (inside) {
-    const long long p = (long long)py * a.cam.width + px;
-    last = min(a.n_last[p], (unsigned)n);
-    const float4 at = a.state_at[p];
-    A0 = at.x; A1 = at.y; A2 = at.z; Tf = at.w;
-    const float g0 = a.dl_dout[3 * p], g1 = a.dl_dout[3 * p + 1], g2 = a.dl_dout[3 * p + 2];
-    const float4 Fv = a.F ? load_px(a.F, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
-    const float4 Bv = a.B ? load_px(a.B, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
-    const float kf = 1.f - Fv.w;
-    Gr = kf * g0; Gg = kf * g1; Gb = kf * g2;
-    // d final / d A.a = -(1 - F.a) (B.rgb + (1 - B.a) bg)
-    Ga = -kf * (g0 * (Bv.x + (1.f - Bv.w) * a.bg[0]) + g1 * (Bv.y + (1.f - Bv.w) * a.bg[1]) +
+// Backward state of one pixel.
+struct PixB {
+  float T, c0, c1, c2;          // transmittance and colour replayed up to the current entry
+  float A0, A1, A2, Tf;         // the forward's final active colour and transmittance
+  float Gr, Gg, Gb, Ga;         // dL/dA.rgb and dL/dA.a
+  unsigned last;                // replay only list positions below this
+};
+
+__device__ __forceinline__ void load_pixel_grad(const BwdArgs& a, long long p, int n, PixB& q) {
+  q.last = min(a.n_last[p], (unsigned)n);
+  const float4 at = a.state_at[p];
+  q.A0 = at.x; q.A1 = at.y; q.A2 = at.z; q.Tf = at.w;
+  const float g0 = a.dl_dout[3 * p], g1 = a.dl_dout[3 * p + 1], g2 = a.dl_dout[3 * p + 2];
+  const float4 Fv = a.F ? load_px(a.F, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4 Bv = a.B ? load_px(a.B, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float kf = 1.f - Fv.w;
+  q.Gr = kf * g0; q.Gg = kf * g1; q.Gb = kf * g2;
+  // d final / d A.a = -(1 - F.a) (B.rgb + (1 - B.a) bg)
+  q.Ga = -kf * (g0 * (Bv.x + (1.f - Bv.w) * a.bg[0]) + g1 * (Bv.y + (1.f - Bv.w) * a.bg[1]) +
                 g2 * (Bv.z + (1.f - Bv.w) * a.bg[2]));
-  }
-  if (threadIdx.x == 0) s_max = 0;
-  __syncthreads();
-  const unsigned wmax = __reduce_max_sync(0xffffffffu, last);
-  if (lane == 0) atomicMax(&s_max, wmax);
-  __syncthreads();
-  const int span = (int)s_max;
-  float T = 1.f, c0 = 0.f, c1 = 0.f, c2 = 0.f;
-  for (int base = 0; base < span; base += kBatch) {
-    __syncthreads();
-    const int cnt = stage_batch<true>(a.ids, rg.x, span, base, a.uv, a.co, a.rgb, bx0, by0,
-                                      a.op.alpha_min, s_uv, s_co, s_rgb, s_id, s_idx, s_ballot);
-    for (int j = 0; j < cnt; ++j) {
-      const int q = s_idx[j];
-      float v[9];
+}
+
+// Backward of one pixel for one list entry (selects, no branches): when the entry contributed
+// to the pixel (live: a position below the pixel's last contributor; sigma >= 0; alpha >=
+// alpha_min) adds d(u, v, a, b, c, opacity, r, g, b) into v and advances the replayed
+// transmittance and colour exactly as the forward did.  Returns whether it contributed.
+__device__ __forceinline__ bool pixel_backward(PixB& p, float4 s, float4 col, float sg, float dx,
+                                               float dy, bool live, const Opts& op, float* v) {
+  const float G = ex2_approx(-sg);
+  const float raw = __fmul_rn(s.w, G);
+  const float alpha = fminf(op.alpha_max, raw);
+  const bool ok = live && sg >= 0.f && alpha >= op.alpha_min;
+  const float w = __fmul_rn(alpha, p.T);
+  const float c0 = __fmaf_rn(w, col.x, p.c0);
+  const float c1 = __fmaf_rn(w, col.y, p.c1);
+  const float c2 = __fmaf_rn(w, col.z, p.c2);
+  const float ioma = __fdividef(1.f, 1.f - alpha);   // gradient scale only
+  // colour accumulated behind this Gaussian = A - (sum up to and including it)
+  const float dalpha = p.Gr * (p.T * col.x - (p.A0 - c0) * ioma) +
+                       p.Gg * (p.T * col.y - (p.A1 - c1) * ioma) +
+                       p.Gb * (p.T * col.z - (p.A2 - c2) * ioma) + p.Ga * p.Tf * ioma;
+  const bool grad_a = ok && raw <= op.alpha_max;      // derivative of min() is 0 once clamped
+  const float wk = ok ? w : 0.f;
+  const float dop = grad_a ? dalpha * G : 0.f;        // d alpha / d opacity = exp(-sigma)
+  const float dsig = grad_a ? -dalpha * raw : 0.f;    // d alpha / d sigma = -alpha
+  v[6] += p.Gr * wk; v[7] += p.Gg * wk; v[8] += p.Gb * wk;
+  v[5] += dop;
+  const float ca = 2.f * kLn2 * s.x, cb = kLn2 * s.y, cc = 2.f * kLn2 * s.z;
+  v[0] -= dsig * (ca * dx + cb * dy);                 // d = pixel - uv
+  v[1] -= dsig * (cb * dx + cc * dy);
+  v[2] += 0.5f * dsig * dx * dx;
+  v[3] += dsig * dx * dy;
+  v[4] += 0.5f * dsig * dy * dy;
+  p.c0 = ok ? c0 : p.c0;
+  p.c1 = ok ? c1 : p.c1;
+  p.c2 = ok ? c2 : p.c2;
+  p.T = ok ? __fmul_rn(p.T, __fsub_rn(1.f, alpha)) : p.T;
+  return ok;
+}
+
+// Warp transpose reduction of 32 per-lane values: at each level a lane keeps half of its
+// values and adds the partner's matching half (31 shuffles in 5 dependent levels); lane l
+// returns the warp-wide sum of x[l].
+__device__ __forceinline__ float warp_sum32(float (&x)[32], int lane) {
 #pragma unroll
-      for (int k = 0; k < 9; ++k) v[k] = 0.f;
-      bool contrib = false;
-      if ((unsigned)(base + q) < last) {
-        float dx, dy;
-        const float4 s = s_co[q];
-        const float sig = sigma2(s, s_uv[q], fx, fy, dx, dy);
-        if (sig >= 0.f) {
-          const float G = ex2_approx(-sig);
-          const float raw = __fmul_rn(s.w, G);
-          const float alpha = fminf(a.op.alpha_max, raw);
-          if (alpha >= a.op.alpha_min) {
-            contrib = true;
-            const float4 col = s_rgb[q];
-            const float w = __fmul_rn(alpha, T);
-            c0 = __fmaf_rn(w, col.x, c0);
-            c1 = __fmaf_rn(w, col.y, c1);
-            c2 = __fmaf_rn(w, col.z, c2);
-            const float ioma = __fdividef(1.f, 1.f - alpha);   // gradient scale only
-            // R = colour accumulated behind this Gaussian = A - (sum up to and including it)
-            const float dalpha = Gr * (T * col.x - (A0 - c0) * ioma) +
-                                 Gg * (T * col.y - (A1 - c1) * ioma) +
-                                 Gb * (T * col.z - (A2 - c2) * ioma) + Ga * Tf * ioma;
-            v[6] = Gr * w; v[7] = Gg * w; v[8] = Gb * w;
-            if (raw <= a.op.alpha_max) {          // derivative of min() is 0 once clamped
-              v[5] = dalpha * G;                   // d alpha / d opacity = exp(-sigma)
-              const float dsig = -dalpha * raw;    // d alpha / d sigma = -alpha
-              const float ca = 2.f * kLn2 * s.x, cb = kLn2 * s.y, cc = 2.f * kLn2 * s.z;
-              v[0] = -dsig * (ca * dx + cb * dy);  // d = pixel - uv
-              v[1] = -dsig * (cb * dx + cc * dy);
-              v[2] = 0.5f * dsig * dx * dx;
-              v[3] = dsig * dx * dy;
-              v[4] = 0.5f * dsig * dy * dy;
-            }
-            T = __fmul_rn(T, __fsub_rn(1.f, alpha));
-          }
-        }
-      }
-      const unsigned who = __ballot_sync(0xffffffffu, contrib);
-      if (who == 0) continue;
-      float* dst = a.grad2d + 9 * (size_t)s_id[q];
-      if (__popc(who) <= 2) {                   // one or two pixels: add directly
-        if (contrib)
+  for (int w = 16; w >= 1; w >>= 1) {
+    const bool up = (lane & w) != 0;
 #pragma unroll
-          for (int k = 0; k < 9; ++k) atomicAdd(&dst[k], v[k]);
-      } else {
-        warp_sum9_atomic(v, dst, lane);
-      }
+    for (int k = 0; k < w; ++k) {
+      const float send = up ? x[k] : x[k + w];
+      const float keep = up ? x[k + w] : x[k];
+      x[k] = keep + __shfl_xor_sync(0xffffffffu, send, w);
     }
   }
+  return x[0];
+}
+
+__global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
+  __shared__ float2 s_uv[kBatch + 2];
+  __shared__ float4 s_co[kBatch + 2];
+  __shared__ float4 s_rgb[kBatch + 2];
+  __shared__ unsigned s_id[kBatch + 2];
+  const int blk = a.order ? (int)a.order[blockIdx.x] : (int)blockIdx.x;
+  const Block bk = block_of(a.cam, blk);
+  const int lane = threadIdx.x & 31;
+  const uint2 rg = a.ranges[bk.tile];
+  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
+  const float fx0 = (float)bk.qx0 + 0.5f, fx1 = (float)bk.qx1 + 0.5f, fy = (float)bk.py + 0.5f;
+  const float bx0 = (float)bk.px0 + 0.5f, by0 = (float)bk.py0 + 0.5f;
+  PixB p0 = {}, p1 = {};
+  p0.T = p1.T = 1.f;
+  if (bk.in0) load_pixel_grad(a, (long long)bk.py * a.cam.width + bk.qx0, n, p0);
+  if (bk.in1) load_pixel_grad(a, (long long)bk.py * a.cam.width + bk.qx1, n, p1);
+  const int span = (int)__reduce_max_sync(0xffffffffu, max(p0.last, p1.last));
+  int next = 0;
+  while (next < span) {
+    __syncwarp();
+    const int cnt = stage_fill<true>(a.ids, rg.x, span, next, a.uv, a.co, a.rgb, bx0, by0,
+                                     a.op.alpha_min, s_uv, s_co, s_rgb, s_id);
+    // three entries per iteration, their 27 gradient components summed over the warp in one
+    // transpose reduction (slots up to j + 2 <= kBatch + 1 exist; unused past cnt)
+    for (int j = 0; j < cnt; j += 3) {
+      float x[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k) x[k] = 0.f;
+      unsigned who[3];
+#pragma unroll
+      for (int i = 0; i < 3; ++i) {
+        const Entry e = load_entry(s_uv, s_co, s_rgb, j + i);
+        const unsigned pos = __float_as_uint(e.col.w);
+        const bool valid = j + i < cnt;
+        float dx0, dx1, dy, sg0, sg1;
+        sigma_pair(e.s, e.m, fx0, fx1, fy, dx0, dx1, dy, sg0, sg1);
+        const bool c0 = pixel_backward(p0, e.s, e.col, sg0, dx0, dy, valid && pos < p0.last, a.op, x + 9 * i);
+        const bool c1 = pixel_backward(p1, e.s, e.col, sg1, dx1, dy, valid && pos < p1.last, a.op, x + 9 * i);
+        who[i] = __ballot_sync(0xffffffffu, c0 || c1);
+      }
+      if ((who[0] | who[1] | who[2]) == 0) continue;
+      const float r = warp_sum32(x, lane);
+      const int ei = lane / 9, comp = lane - 9 * ei;
+      const unsigned wi = ei == 0 ? who[0] : (ei == 1 ? who[1] : who[2]);
+      if (lane < 27 && wi != 0) atomicAdd(a.grad2d + 9 * (size_t)s_id[j + ei] + comp, r);
+    }
+  }
+}
+
+// Orders the launch's CTAs in the workspace when there is room; returns the order or nullptr.
+const unsigned* launch_order(abcd_ctx* ctx, const uint2* ranges, const unsigned* span,
+                             int n_blocks) {
+  if (!has_workspace(ctx) || n_blocks > ctx->ws.max_blocks || n_blocks <= 0) return nullptr;
+  order_kernel<<<1, 1024, 0, ctx->stream>>>(ranges, span, n_blocks, ctx->ws.block_order);
+  if (check_launch(ctx, "order_kernel") != ABCD_OK) return nullptr;
+  return ctx->ws.block_order;
 }
 
 bool fb_ok(const void* F, const void* B, int dtype) {
@@ -409,8 +585,10 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.state_at = state ? (float4*)state->A_T : nullptr;
   a.n_last = state ? state->n_last : nullptr;
   a.refresh = (uint2*)refresh_f16;
-  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y;
-  render_fwd_kernel<<<n_tiles * kSubPerTile, kSubThreads, 0, ctx->stream>>>(a);
+  const int n_blocks = a.cam.tiles_x * a.cam.tiles_y * kSubPerTile;
+  a.order = launch_order(ctx, a.ranges, nullptr, n_blocks);
+  a.block_work = (a.order && a.n_last) ? ctx->ws.block_work : nullptr;
+  render_fwd_kernel<<<n_blocks, kSubThreads, 0, ctx->stream>>>(a);
   return check_launch(ctx, "render_fwd_kernel");
 }
 
@@ -444,7 +622,8 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   a.n_last = state->n_last;
   a.dl_dout = dL_dout;
   a.grad2d = grad2d;
-  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y;
-  render_bwd_kernel<<<n_tiles * kSubPerTile, kSubThreads, 0, ctx->stream>>>(a);
+  const int n_blocks = a.cam.tiles_x * a.cam.tiles_y * kSubPerTile;
+  a.order = launch_order(ctx, a.ranges, ctx->ws_base ? ctx->ws.block_work : nullptr, n_blocks);
+  render_bwd_kernel<<<n_blocks, kSubThreads, 0, ctx->stream>>>(a);
   return check_launch(ctx, "render_bwd_kernel");
 }
