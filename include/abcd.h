@@ -136,7 +136,10 @@ abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_
  * of about 0.7% in sigma, so a list may hold a few entries that every pixel of the tile
  * skips); lists are ordered by the fp32 depth, ties by id.  Leaving out the tiles on which
  * every pixel would skip the Gaussian does not change any pixel.  n must equal the n given
- * to abcd_project; opts as there (NULL = defaults; alpha_min is used). */
+ * to abcd_project; opts as there (NULL = defaults; alpha_min is used).  Also leaves in the
+ * context's workspace the tiles ordered by decreasing list length, tagged with out->ranges;
+ * the render calls given these same ranges launch their longest tiles first (a scheduling
+ * hint only: no result depends on it). */
 abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, int n,
                           const abcd_camera* cam, const abcd_render_opts* opts, abcd_tiles* out);
 

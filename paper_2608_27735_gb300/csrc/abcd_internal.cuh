@@ -49,14 +49,28 @@ struct Workspace {
   float* grad2d;                    // [max_g][9]
   float* dl_dout;                   // [max_pixels][3]
   float* loss_partials;             // [kMaxLossBlocks][2]
-  unsigned* block_work;             // [max_blocks] per render CTA: list entries its backward walks
-  unsigned* block_order;            // [max_blocks] render CTAs, most work first
-  long long max_blocks;
+  unsigned* tile_order;             // [max_tiles] tiles by decreasing list length (bin_sort)
+  long long max_tiles;
 };
 
-// Render CTAs (8x8 pixel blocks, four per tile) the workspace orders for images of up to
-// max_pixels pixels with sides up to 16384.
-inline long long max_render_blocks(long long max_pixels) { return 4 * (max_pixels / 256 + 2048); }
+constexpr int kRenderSubPerTile = 4;      // render CTAs (8x8 pixel blocks) per 16x16 tile
+
+// Mask of the lanes whose value equals this lane's, for values 0..256 (256 marks an unused
+// lane; it matches only other unused lanes).  Nine ballots: the cost does not depend on how
+// many distinct values the warp holds, unlike __match_any_sync's.
+__device__ __forceinline__ unsigned match_byte(unsigned d) {
+  unsigned peers = 0xffffffffu;
+#pragma unroll
+  for (int b = 0; b < 9; ++b) {
+    const unsigned bit = (d >> b) & 1u;
+    const unsigned m = __ballot_sync(0xffffffffu, bit);
+    peers &= bit ? m : ~m;
+  }
+  return peers;
+}
+
+// Tiles the workspace orders for images of up to max_pixels pixels with sides up to 16384.
+inline long long max_order_tiles(long long max_pixels) { return max_pixels / 256 + 2048; }
 
 }  // namespace abcd
 
@@ -71,6 +85,8 @@ struct abcd_ctx {
   long long max_pairs = 0;
   long long max_pixels = 0;
   abcd::Workspace ws{};
+  const void* order_ranges = nullptr;   // tile ranges the order in ws.tile_order belongs to
+  long long order_tiles = 0;
   abcd::SHConst sh{};
   long long launches = 0;
   char err[512] = {0};

@@ -15,13 +15,14 @@
 //      count, and +-1 at the run's ends in a per-row difference array over the tile grid;
 //   2. stable LSD radix sort of the n Gaussians by the 32 depth bits;
 //   3. exclusive scan of the pair counts in that order: K = total pairs; the row prefix sums
-//      of the difference array give every tile's pair count, hence its range;
+//      of the difference array give every tile's pair count, hence its range, and the tiles
+//      sorted by decreasing count (the order the render kernels launch them in);
 //   4. emission of (tile << 32 | id) items in depth order (the runs are recomputed with the
 //      same round-to-nearest arithmetic, so they match step 1 bit for bit);
 //   5. stable LSD radix sort of the K items on the tile bits only (ceil(log2 n_tiles) <= 16
 //      bits, 8 per pass), which keeps depth order inside each tile; the last pass writes ids.
 // Radix passes are reduce-then-scan (per-block digit counts, per-digit row scans, stable
-// scatter): no inter-block waits, so nothing can spin.  Counts that live on the device (K)
+// scatter ranked with ballots): no inter-block waits, so nothing can spin.  Counts that live on the device (K)
 // are read by the kernels themselves; grids are fixed, so the step has no host sync.
 #include <algorithm>
 
@@ -248,7 +249,7 @@ __global__ void __launch_bounds__(1024) radix_rowscan_kernel(unsigned* hist, int
 }
 
 // ---- radix pass, step 3: stable scatter.  Each warp owns a contiguous slice of the block's
-// range; lanes of equal digit are ranked with __match_any_sync.
+// range; lanes of equal digit are ranked with match_byte.
 __global__ void __launch_bounds__(256)
 radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_static,
                      const long long* n_dev, long long cap, int shift, const unsigned* hist,
@@ -281,7 +282,7 @@ radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_sta
     }
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      const unsigned peers = __match_any_sync(0xffffffffu, ds[j]);
+      const unsigned peers = match_byte(ds[j]);
       if (ds[j] < 0x100u && (peers & lt) == 0) cnt[w][ds[j]] += __popc(peers);
       __syncwarp();
     }
@@ -304,7 +305,7 @@ radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_sta
     }
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      const unsigned peers = __match_any_sync(0xffffffffu, ds[j]);
+      const unsigned peers = match_byte(ds[j]);
       const bool valid = ds[j] < 0x100u;
       unsigned pos = 0;
       if (valid) pos = cnt[w][ds[j]] + __popc(peers & lt);
@@ -385,6 +386,107 @@ ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* co
     ranges[2 * t] = ok ? (unsigned)run : 0u;
     ranges[2 * t + 1] = ok ? (unsigned)(run + c) : 0u;
     run += c;
+  }
+}
+
+// ---- the same, with the difference array staged in shared memory (one load round trip
+// instead of a chain of dependent ones), followed by the render order: tiles sorted by
+// decreasing pair count (16 buckets per octave; a counting sort, in no particular order inside
+// a bucket) into tile_order, so that the render kernels start the longest lists first.  The
+// order changes no result.
+constexpr int kOrderBuckets = 256;
+
+__device__ __forceinline__ unsigned count_bucket(unsigned c) {
+  if (c == 0) return kOrderBuckets - 1;
+  const int b = (int)(__log2f((float)c) * 16.f) + 1;
+  return (unsigned)(kOrderBuckets - 1 - min(b, kOrderBuckets - 1));
+}
+
+__global__ void __launch_bounds__(1024)
+ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, const long long* count,
+                    long long cap, unsigned* ranges, unsigned* tile_order) {
+  extern __shared__ int sd[];              // [(tiles_x + 1) (tiles_y + 1)] cells, then [nt] keys
+  __shared__ unsigned hist[kOrderBuckets];
+  const int W1 = tiles_x + 1, cells = W1 * (tiles_y + 1), nt = tiles_x * tiles_y;
+  unsigned char* skey = reinterpret_cast<unsigned char*>(sd + cells);
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const unsigned lt = (1u << lane) - 1u;
+  constexpr int kLoads = 8;
+  for (int i0 = threadIdx.x; i0 < cells; i0 += blockDim.x * kLoads) {
+    int v[kLoads];
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+      const int i = i0 + k * (int)blockDim.x;
+      v[k] = i < cells ? diff[i] : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+      const int i = i0 + k * (int)blockDim.x;
+      if (i < cells) sd[i] = v[k];
+    }
+  }
+  for (int i = threadIdx.x; i < kOrderBuckets; i += blockDim.x) hist[i] = 0;
+  __syncthreads();
+  for (int y = wid; y < tiles_y; y += nw) {                        // prefix along each row
+    int carry = 0;
+    for (int x0 = 0; x0 < tiles_x; x0 += 32) {
+      const int x = x0 + lane;
+      int v = x < tiles_x ? sd[y * W1 + x] : 0;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += u;
+      }
+      if (x < tiles_x) sd[y * W1 + x] = v + carry;
+      carry += __shfl_sync(0xffffffffu, v, 31);
+    }
+  }
+  __syncthreads();
+  const bool ok = *count <= cap;
+  const int per = (nt + blockDim.x - 1) / blockDim.x;
+  const int lo = min(nt, (int)threadIdx.x * per), hi = min(nt, lo + per);
+  unsigned long long s = 0;
+  for (int t = lo; t < hi; ++t) s += (unsigned)sd[(t / tiles_x) * W1 + (t % tiles_x)];
+  unsigned long long run = block_exclusive_scan(s, nullptr);
+  for (int t = lo; t < hi; ++t) {
+    const unsigned c = (unsigned)sd[(t / tiles_x) * W1 + (t % tiles_x)];
+    ranges[2 * t] = ok ? (unsigned)run : 0u;
+    ranges[2 * t + 1] = ok ? (unsigned)(run + c) : 0u;
+    skey[t] = (unsigned char)count_bucket(ok ? c : 0u);
+    run += c;
+  }
+  __syncthreads();
+  for (int i0 = 0; i0 < nt; i0 += blockDim.x) {
+    const int i = i0 + threadIdx.x;
+    const unsigned key = i < nt ? skey[i] : (unsigned)kOrderBuckets;
+    const unsigned peers = __match_any_sync(0xffffffffu, key);
+    if (key < kOrderBuckets && (peers & lt) == 0) atomicAdd(&hist[key], (unsigned)__popc(peers));
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {                  // exclusive scan of the 256 counts, 8 per lane
+    constexpr int kPer = kOrderBuckets / 32;
+    unsigned v[kPer], sum = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) { v[k] = hist[lane * kPer + k]; sum += v[k]; }
+    unsigned incl = sum;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const unsigned o = __shfl_up_sync(0xffffffffu, incl, d);
+      if (lane >= d) incl += o;
+    }
+    unsigned r = incl - sum;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) { hist[lane * kPer + k] = r; r += v[k]; }
+  }
+  __syncthreads();
+  for (int i0 = 0; i0 < nt; i0 += blockDim.x) {
+    const int i = i0 + threadIdx.x;
+    const unsigned key = i < nt ? skey[i] : (unsigned)kOrderBuckets;
+    const unsigned peers = __match_any_sync(0xffffffffu, key);
+    const int leader = __ffs(peers) - 1;
+    unsigned base = 0;
+    if (key < kOrderBuckets && lane == leader) base = atomicAdd(&hist[key], (unsigned)__popc(peers));
+    base = __shfl_sync(0xffffffffu, base, leader);
+    if (key < kOrderBuckets) tile_order[base + __popc(peers & lt)] = (unsigned)i;
   }
 }
 
@@ -552,9 +654,26 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if ((s = check_launch(ctx, "count_kernel"))) return s;
   scan_blocks_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status);
   if ((s = check_launch(ctx, "scan_blocks_kernel"))) return s;
-  ranges_from_diff_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.diff, tiles_x, tiles_y, out->count, cap,
-                                                      out->ranges);
-  if ((s = check_launch(ctx, "ranges_from_diff_kernel"))) return s;
+  {
+    const int cells = (tiles_x + 1) * (tiles_y + 1);
+    ctx->order_ranges = nullptr;
+    if (cells <= kSmemDiffCells && n_tiles <= ctx->ws.max_tiles) {
+      const size_t smem = sizeof(int) * cells + (size_t)n_tiles;
+      if (smem > 48 * 1024) {
+        const cudaError_t e2 = cudaFuncSetAttribute(ranges_order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "ranges smem: %s", cudaGetErrorString(e2));
+      }
+      ranges_order_kernel<<<1, 1024, smem, ctx->stream>>>(ctx->ws.diff, tiles_x, tiles_y, out->count,
+                                                          cap, out->ranges, ctx->ws.tile_order);
+      if ((s = check_launch(ctx, "ranges_order_kernel"))) return s;
+      ctx->order_ranges = out->ranges;           // the order belongs to these ranges
+      ctx->order_tiles = n_tiles;
+    } else {
+      ranges_from_diff_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.diff, tiles_x, tiles_y, out->count,
+                                                          cap, out->ranges);
+      if ((s = check_launch(ctx, "ranges_from_diff_kernel"))) return s;
+    }
+  }
   emit_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, (const float2*)proj->uv,
                                            (const float4*)proj->conic_opacity, ctx->ws.rects,
                                            ctx->ws.counts, ctx->ws.block_sums, out->count, cap,

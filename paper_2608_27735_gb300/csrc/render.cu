@@ -20,11 +20,11 @@
 // (sigma, alpha, T) is computed with explicit round-to-nearest intrinsics in one shared
 // function, so the backward kernel retraces exactly the forward's contributors.
 //
-// Work is very uneven across blocks (lists of a few entries next to lists of 15,000), so with
-// a workspace each launch first orders its CTAs by decreasing work -- list length for the
-// forward, the longest contributor walk the forward recorded per block for the backward -- and
-// the longest blocks start in the first wave instead of trailing the launch.  The order
-// changes no result (CTAs are independent; the backward's gradient sums are atomic either way).
+// Work is very uneven across blocks (lists of a few entries next to lists of 15,000), so both
+// kernels take their tiles in the order bin_sort left in the workspace (decreasing list
+// length) when it was made for the ranges they are given: the longest blocks start in the
+// first wave instead of trailing the launch.  The order changes no result (CTAs are
+// independent; the backward's gradient sums are atomic either way).
 #include "abcd_internal.cuh"
 
 namespace abcd {
@@ -37,10 +37,10 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kSub = 8;                          // CTA pixel block edge
 constexpr int kSubThreads = 32;                  // one warp, two pixels per lane
 constexpr int kSubPerTile = (kTile / kSub) * (kTile / kSub);
+static_assert(kSubPerTile == kRenderSubPerTile, "tile order expands to kRenderSubPerTile CTAs per tile");
 constexpr int kRounds = 2;                       // list entries per lane per staging group
 constexpr int kGroup = kSubThreads * kRounds;    // 64 entries loaded together
 constexpr int kBatch = 2 * kGroup;               // staged survivors per batch (at most)
-constexpr int kOrderBuckets = 256;
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -164,60 +164,12 @@ __device__ __forceinline__ int stage_fill(const unsigned* ids, unsigned start, i
   return total;
 }
 
-// Orders n_blocks render CTAs by decreasing work (16 buckets per octave, counting sort in one
-// CTA; within a bucket in no particular order).  work = tile list length for the forward
-// (span == nullptr), else span[block].  Produces a permutation whatever the work values are.
-__global__ void __launch_bounds__(1024) order_kernel(const uint2* ranges, const unsigned* span,
-                                                     int n_blocks, unsigned* order) {
-  __shared__ unsigned hist[kOrderBuckets];
-  const int tid = threadIdx.x, lane = tid & 31;
-  const unsigned lt = (1u << lane) - 1u;
-  for (int i = tid; i < kOrderBuckets; i += blockDim.x) hist[i] = 0;
-  __syncthreads();
-  auto key_of = [&](int i) -> unsigned {
-    if (i >= n_blocks) return kOrderBuckets;
-    unsigned w;
-    if (span) {
-      w = span[i];
-    } else {
-      const uint2 rg = ranges[i / kSubPerTile];
-      w = rg.y > rg.x ? rg.y - rg.x : 0u;
-    }
-    if (w == 0) return kOrderBuckets - 1;
-    const int b = (int)(__log2f((float)w) * 16.f) + 1;
-    return (unsigned)(kOrderBuckets - 1 - min(b, kOrderBuckets - 1));
-  };
-  for (int i0 = 0; i0 < n_blocks; i0 += blockDim.x) {
-    const unsigned key = key_of(i0 + tid);
-    const unsigned peers = __match_any_sync(0xffffffffu, key);
-    if (key < kOrderBuckets && (peers & lt) == 0) atomicAdd(&hist[key], (unsigned)__popc(peers));
-  }
-  __syncthreads();
-  if (tid < 32) {                        // exclusive scan of the 256 counts, 8 per lane
-    constexpr int kPer = kOrderBuckets / 32;
-    unsigned v[kPer], sum = 0;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) { v[k] = hist[tid * kPer + k]; sum += v[k]; }
-    unsigned incl = sum;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      const unsigned o = __shfl_up_sync(0xffffffffu, incl, d);
-      if (lane >= d) incl += o;
-    }
-    unsigned run = incl - sum;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) { hist[tid * kPer + k] = run; run += v[k]; }
-  }
-  __syncthreads();
-  for (int i0 = 0; i0 < n_blocks; i0 += blockDim.x) {
-    const unsigned key = key_of(i0 + tid);
-    const unsigned peers = __match_any_sync(0xffffffffu, key);
-    const int leader = __ffs(peers) - 1;
-    unsigned base = 0;
-    if (key < kOrderBuckets && lane == leader) base = atomicAdd(&hist[key], (unsigned)__popc(peers));
-    base = __shfl_sync(0xffffffffu, base, leader);
-    if (key < kOrderBuckets) order[base + __popc(peers & lt)] = (unsigned)(i0 + tid);
-  }
+// Render CTA b handles the 8x8 block tile_order[b / 4] * 4 + b % 4 (tile_order: a permutation
+// of the tiles, longest list first), or block b.
+__device__ __forceinline__ int block_index(const unsigned* tile_order) {
+  const int b = (int)blockIdx.x;
+  if (tile_order) return (int)tile_order[b / kSubPerTile] * kSubPerTile + b % kSubPerTile;
+  return b;
 }
 
 // The CTA's 8x8 pixel block and the lane's two pixels (qx0, py), (qx1 = qx0 + 4, py).
@@ -258,8 +210,7 @@ struct FwdArgs {
   float4* state_at;
   unsigned* n_last;
   uint2* refresh;      // fp16 x4 per pixel
-  const unsigned* order;   // CTA order (nullptr: launch order)
-  unsigned* block_work;    // per block: max n_last over its pixels (nullptr: not recorded)
+  const unsigned* tile_order;   // tiles, longest list first (nullptr: launch order)
 };
 
 // Blend state of one pixel.
@@ -347,7 +298,7 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
   __shared__ float2 s_uv[kBatch];
   __shared__ float4 s_co[kBatch];
   __shared__ float4 s_rgb[kBatch];
-  const int blk = a.order ? (int)a.order[blockIdx.x] : (int)blockIdx.x;
+  const int blk = block_index(a.tile_order);
   const Block bk = block_of(a.cam, blk);
   const uint2 rg = a.ranges[bk.tile];
   const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
@@ -377,10 +328,6 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
       if ((j & 30) == 30 && __all_sync(0xffffffffu, p0.done && p1.done)) break;
     }
   }
-  if (a.block_work) {
-    const unsigned span = __reduce_max_sync(0xffffffffu, max(p0.last, p1.last));
-    if ((threadIdx.x & 31) == 0) a.block_work[blk] = span;
-  }
   if (bk.in0) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx0, p0);
   if (bk.in1) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx1, p1);
 }
@@ -401,7 +348,7 @@ struct BwdArgs {
   const unsigned* n_last;
   const float* dl_dout;
   float* grad2d;
-  const unsigned* order;   // CTA order (nullptr: launch order)
+  const unsigned* tile_order;   // tiles, longest list first (nullptr: launch order)
 };
 
 // Backward state of one pixel.
@@ -486,7 +433,7 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
   __shared__ float4 s_co[kBatch + 2];
   __shared__ float4 s_rgb[kBatch + 2];
   __shared__ unsigned s_id[kBatch + 2];
-  const int blk = a.order ? (int)a.order[blockIdx.x] : (int)blockIdx.x;
+  const int blk = block_index(a.tile_order);
   const Block bk = block_of(a.cam, blk);
   const int lane = threadIdx.x & 31;
   const uint2 rg = a.ranges[bk.tile];
@@ -530,13 +477,10 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
   }
 }
 
-// Orders the launch's CTAs in the workspace when there is room; returns the order or nullptr.
-const unsigned* launch_order(abcd_ctx* ctx, const uint2* ranges, const unsigned* span,
-                             int n_blocks) {
-  if (!has_workspace(ctx) || n_blocks > ctx->ws.max_blocks || n_blocks <= 0) return nullptr;
-  order_kernel<<<1, 1024, 0, ctx->stream>>>(ranges, span, n_blocks, ctx->ws.block_order);
-  if (check_launch(ctx, "order_kernel") != ABCD_OK) return nullptr;
-  return ctx->ws.block_order;
+// The tile order bin_sort left in the workspace, if it was made for these ranges.
+const unsigned* tile_order_for(const abcd_ctx* ctx, const abcd_tiles* tiles, long long n_tiles) {
+  return (has_workspace(ctx) && ctx->order_ranges == tiles->ranges && ctx->order_tiles == n_tiles)
+             ? ctx->ws.tile_order : nullptr;
 }
 
 bool fb_ok(const void* F, const void* B, int dtype) {
@@ -585,9 +529,8 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.state_at = state ? (float4*)state->A_T : nullptr;
   a.n_last = state ? state->n_last : nullptr;
   a.refresh = (uint2*)refresh_f16;
-  const int n_blocks = a.cam.tiles_x * a.cam.tiles_y * kSubPerTile;
-  a.order = launch_order(ctx, a.ranges, nullptr, n_blocks);
-  a.block_work = (a.order && a.n_last) ? ctx->ws.block_work : nullptr;
+  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
+  a.tile_order = tile_order_for(ctx, tiles, n_tiles);
   render_fwd_kernel<<<n_blocks, kSubThreads, 0, ctx->stream>>>(a);
   return check_launch(ctx, "render_fwd_kernel");
 }
@@ -622,8 +565,8 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   a.n_last = state->n_last;
   a.dl_dout = dL_dout;
   a.grad2d = grad2d;
-  const int n_blocks = a.cam.tiles_x * a.cam.tiles_y * kSubPerTile;
-  a.order = launch_order(ctx, a.ranges, ctx->ws_base ? ctx->ws.block_work : nullptr, n_blocks);
+  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
+  a.tile_order = tile_order_for(ctx, tiles, n_tiles);
   render_bwd_kernel<<<n_blocks, kSubThreads, 0, ctx->stream>>>(a);
   return check_launch(ctx, "render_bwd_kernel");
 }

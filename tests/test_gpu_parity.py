@@ -159,6 +159,22 @@ def test_bin_sort_ragged_and_sh3(ctx, ragged):
         par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
 
 
+def test_bin_sort_many_gaussians(ctx):
+    """More Gaussians (270,000) than the one-cluster depth sort takes (2^18): the depth order
+    comes from the multi-kernel radix passes instead."""
+    s = sg.grid_scene((1, 1, 1), 5.0, 270_000, 0, seed=91)
+    s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 96, 64, seed=91,
+                                height_jitter=1.0)
+    ctx.reserve(270_000, 8_000_000, 2_100_000)
+    case = Case(s, 0, fb=False)
+    r = run_forward(ctx, case, want_state=False)
+    K = int(r["tiles"].count.item())
+    rng = r["tiles"].ranges.cpu().numpy().astype(np.int64)
+    ids = r["tiles"].ids.cpu().numpy()[:K]
+    tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
+    par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
+
+
 @pytest.mark.parametrize("cam_idx,bg,fbdt", [(0, None, "f16"), (1, (0.2, 0.5, 0.9), "f16"),
                                              (2, None, "f32"), (3, (1.0, 1.0, 1.0), "f16")])
 def test_render_composite_fwd_matches_oracle(ctx, tiny, cam_idx, bg, fbdt):
