@@ -192,18 +192,63 @@ tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, i
   }
 }
 
+// Items per thread (hist) or per lane (scatter) loaded at once.
+constexpr int kRadixLoads = 8;
+
+template <typename T>
+__device__ __forceinline__ void load_items(const T* in, long long b0, long long wh, int lane,
+                                           T (&xs)[kRadixLoads]) {
+#pragma unroll
+  for (int j = 0; j < kRadixLoads; ++j) {
+    const long long i = b0 + 32 * j + lane;
+    xs[j] = i < wh ? in[i] : (T)0;
+  }
+}
+
+// Digit of item j of a round (0x100 past the end of the slice).
+template <typename T>
+__device__ __forceinline__ unsigned digit_of(T x, long long i, long long wh, int shift,
+                                             unsigned mask) {
+  return i < wh ? ((unsigned)(x >> shift) & mask) : 0x100u;
+}
+
+// Lanes holding the same BITS-bit digit as this lane, among the lanes of valid_mask: one
+// ballot per bit (a cost independent of how many distinct digits the warp holds).
+template <int BITS>
+__device__ __forceinline__ unsigned match_digit(unsigned d, unsigned valid_mask) {
+  unsigned peers = valid_mask;
+#pragma unroll
+  for (int b = 0; b < BITS; ++b) {
+    const unsigned bit = (d >> b) & 1u;
+    const unsigned m = __ballot_sync(0xffffffffu, bit);
+    peers &= bit ? m : ~m;
+  }
+  return peers;
+}
+
 // ---- radix pass, step 1: per-block digit counts hist[d * G + b]
+template <typename T>
 __global__ void __launch_bounds__(256)
-radix_hist_kernel(const u64* in, long long n_static, const long long* n_dev, long long cap,
-                  int shift, unsigned* hist, int G) {
+radix_hist_kernel(const T* in, long long n_static, const long long* n_dev, long long cap,
+                  int shift, unsigned mask, unsigned* hist, int G) {
   __shared__ unsigned h[kRadixBins];
   for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) h[d] = 0;
   __syncthreads();
   const long long n = dev_count(n_static, n_dev, cap);
   long long lo, hi;
   block_range(n, G, &lo, &hi);
-  for (long long i = lo + threadIdx.x; i < hi; i += blockDim.x)
-    atomicAdd(&h[(unsigned)(in[i] >> shift) & (kRadixBins - 1)], 1u);
+  constexpr int U = kRadixLoads;
+  for (long long b0 = lo; b0 < hi; b0 += (long long)blockDim.x * U) {
+    unsigned d[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const long long i = b0 + (long long)j * blockDim.x + threadIdx.x;
+      d[j] = i < hi ? ((unsigned)(in[i] >> shift) & mask) : 0x100u;
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j)
+      if (d[j] < 0x100u) atomicAdd(&h[d[j]], 1u);
+  }
   __syncthreads();
   for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) hist[d * G + blockIdx.x] = h[d];
 }
@@ -248,23 +293,27 @@ __global__ void __launch_bounds__(1024) radix_rowscan_kernel(unsigned* hist, int
   if (threadIdx.x == 0) totals[d] = (unsigned)tot;
 }
 
-// ---- radix pass, step 3: stable scatter.  Each warp owns a contiguous slice of the block's
-// range; lanes of equal digit are ranked with match_byte.
+// ---- radix pass, step 3: stable scatter of BITS-bit digits.  Each warp owns a contiguous
+// slice of the block's range; lanes of equal digit are ranked with match_digit, once per item
+// (the masks are kept for the scatter when the slice is one round of loads).
+template <typename T, int BITS>
 __global__ void __launch_bounds__(256)
-radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_static,
+radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
                      const long long* n_dev, long long cap, int shift, const unsigned* hist,
                      const unsigned* totals, int G) {
   constexpr int W = 8;
-  __shared__ unsigned cnt[W][kRadixBins];
+  constexpr unsigned BINS = 1u << BITS, MASK = BINS - 1;
+  __shared__ unsigned cnt[W][BINS];
   __shared__ unsigned base[kRadixBins];
   {
-    // digit bases: exclusive scan of the digit totals (kRadixBins == blockDim.x)
+    // digit bases: exclusive scan of the digit totals (kRadixBins == blockDim.x; the totals of
+    // digits >= BINS are zero)
     const unsigned t = totals[threadIdx.x];
     unsigned long long tot = 0;
     base[threadIdx.x] = (unsigned)block_exclusive_scan(t, &tot);
   }
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  for (int k = threadIdx.x; k < W * kRadixBins; k += blockDim.x) (&cnt[0][0])[k] = 0;
+  for (int k = threadIdx.x; k < W * (int)BINS; k += blockDim.x) (&cnt[0][0])[k] = 0;
   __syncthreads();
   const long long n = dev_count(n_static, n_dev, cap);
   long long lo, hi;
@@ -272,48 +321,48 @@ radix_scatter_kernel(const u64* in, u64* out, unsigned* out_ids, long long n_sta
   const long long wchunk = (hi - lo + W - 1) / W;
   const long long wl = min(hi, lo + w * wchunk), wh = min(hi, wl + wchunk);
   const unsigned lt = (1u << lane) - 1u;
-  constexpr int U = 4;                        // items per lane per iteration (loads in flight)
-  for (long long b0 = wl; b0 < wh; b0 += 32 * U) {
-    unsigned ds[U];
+  constexpr int U = kRadixLoads;
+  // the warp's slice in rounds of 32 U items, all loaded at once; with one round (the usual
+  // case) the items and their peer masks stay in registers for the scatter
+  const int rounds = (int)((wh - wl + 32 * U - 1) / (32 * U));
+  T xs[U];
+  unsigned pm[U];
+  for (int r = 0; r < rounds; ++r) {
+    const long long b0 = wl + (long long)r * 32 * U;
+    load_items(in, b0, wh, lane, xs);
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      const long long i = b0 + 32 * j + lane;
-      ds[j] = i < wh ? ((unsigned)(in[i] >> shift) & (kRadixBins - 1)) : 0x100u;
-    }
-#pragma unroll
-    for (int j = 0; j < U; ++j) {
-      const unsigned peers = match_byte(ds[j]);
-      if (ds[j] < 0x100u && (peers & lt) == 0) cnt[w][ds[j]] += __popc(peers);
+      if (b0 + 32 * j >= wh) break;                // warp-uniform
+      const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, wh, shift, MASK);
+      const unsigned peers = match_digit<BITS>(d, __ballot_sync(0xffffffffu, d < 0x100u));
+      pm[j] = peers;
+      if (d < 0x100u && (peers & lt) == 0) cnt[w][d] += __popc(peers);
       __syncwarp();
     }
   }
   __syncthreads();
-  for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) {
+  for (int d = threadIdx.x; d < (int)BINS; d += blockDim.x) {
     unsigned run = base[d] + hist[d * G + blockIdx.x];
     for (int k = 0; k < W; ++k) { const unsigned c = cnt[k][d]; cnt[k][d] = run; run += c; }
   }
   __syncthreads();
-  for (long long b0 = wl; b0 < wh; b0 += 32 * U) {
-    u64 xs[U];
-    unsigned ds[U];
+  for (int r = 0; r < rounds; ++r) {
+    const long long b0 = wl + (long long)r * 32 * U;
+    if (rounds > 1) load_items(in, b0, wh, lane, xs);
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      const long long i = b0 + 32 * j + lane;
-      const bool valid = i < wh;
-      xs[j] = valid ? in[i] : 0ull;
-      ds[j] = valid ? ((unsigned)(xs[j] >> shift) & (kRadixBins - 1)) : 0x100u;
-    }
-#pragma unroll
-    for (int j = 0; j < U; ++j) {
-      const unsigned peers = match_byte(ds[j]);
-      const bool valid = ds[j] < 0x100u;
+      if (b0 + 32 * j >= wh) break;                // warp-uniform
+      const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, wh, shift, MASK);
+      const bool valid = d < 0x100u;
+      const unsigned peers =
+          rounds > 1 ? match_digit<BITS>(d, __ballot_sync(0xffffffffu, valid)) : pm[j];
       unsigned pos = 0;
-      if (valid) pos = cnt[w][ds[j]] + __popc(peers & lt);
+      if (valid) pos = cnt[w][d] + __popc(peers & lt);
       __syncwarp();
       if (valid) {
-        if (out_ids) out_ids[pos] = (unsigned)xs[j];
+        if (out_ids) out_ids[pos] = (unsigned)xs[j] & id_mask;
         else out[pos] = xs[j];
-        if ((peers & lt) == 0) cnt[w][ds[j]] += __popc(peers);
+        if ((peers & lt) == 0) cnt[w][d] += __popc(peers);
       }
       __syncwarp();
     }
@@ -490,17 +539,29 @@ ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, const long long* 
   }
 }
 
-// ---- emission of (tile << 32 | id) in depth order: each warp takes its Gaussians one at a
-// time; lanes compute the row runs, a warp scan places them, and the pairs are written with
-// consecutive lanes on consecutive entries (row of pair k found by a search over the scan).
-__global__ void __launch_bounds__(256)
+// ---- emission of (tile << id_bits | id) in depth order.  A warp takes 32 consecutive
+// Gaussians of the depth order, whose pairs fill one contiguous range of the output; it builds
+// that range in its shared-memory buffer when it fits (else writes in place) and copies it out
+// with coalesced stores.  A lane writes the pairs of its own Gaussian when it has at most
+// kEmitSmall (its rows one after the other); the warp writes the larger ones together, one at a
+// time: lanes compute the row runs, a warp scan places them, and consecutive lanes take
+// consecutive pairs (the row of pair k found by a search over the scan).
+constexpr int kEmitSmall = 64;
+constexpr int kEmitBufBytes = 8192;             // per warp
+constexpr int kEmitThreads = 256;
+
+template <typename T>
+__global__ void __launch_bounds__(kEmitThreads)
 emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const int4* rects,
             const unsigned* counts, const unsigned long long* block_off, const long long* count,
-            long long cap, int tiles_x, float alpha_min, u64* pairs, int G) {
+            long long cap, int tiles_x, float alpha_min, int id_bits, T* pairs, int G) {
+  constexpr unsigned kBuf = kEmitBufBytes / sizeof(T);
+  extern __shared__ __align__(16) unsigned char emit_smem[];
   if (*count > cap) return;
   long long lo, hi;
   block_range(n, G, &lo, &hi);
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  T* buf = reinterpret_cast<T*>(emit_smem) + (size_t)w * kBuf;
   unsigned long long run = block_off[blockIdx.x];
   for (long long base = lo; base < hi; base += blockDim.x) {
     const long long i = base + threadIdx.x;
@@ -514,11 +575,27 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
     }
     unsigned long long tot = 0;
     const unsigned long long off = run + block_exclusive_scan(t, &tot);
-    for (int j = 0; j < 32; ++j) {
+    run += tot;
+    const unsigned long long off0 = __shfl_sync(0xffffffffu, off, 0);
+    const unsigned R = (unsigned)(__shfl_sync(0xffffffffu, off + t, 31) - off0);
+    const bool staged = R <= kBuf;                   // warp-uniform
+    T* out = staged ? buf : pairs + off0;            // this warp's range, from off0
+    if (t > 0 && t <= (unsigned)kEmitSmall) {
+      unsigned at = (unsigned)(off - off0);
+      const unsigned stop = at + t;
+      for (int ty = qm.y; ty < qm.w && at < stop; ++ty) {
+        const int2 r = row_run(sm_, qm, ty);
+        for (int x = r.x; x < r.y && at < stop; ++x)
+          out[at++] = ((T)(unsigned)(ty * tiles_x + x) << id_bits) | (T)id;
+      }
+    }
+    unsigned big = __ballot_sync(0xffffffffu, t > (unsigned)kEmitSmall);
+    while (big) {
+      const int j = __ffs(big) - 1;
+      big &= big - 1;
       const unsigned tj = __shfl_sync(0xffffffffu, t, j);
-      if (tj == 0) continue;
       const unsigned idj = __shfl_sync(0xffffffffu, id, j);
-      const unsigned long long oj = __shfl_sync(0xffffffffu, off, j);
+      const unsigned oj = (unsigned)(__shfl_sync(0xffffffffu, off, j) - off0);
       // lane j prepared Gaussian j: broadcast its rectangle and ellipse
       const int4 q = make_int4(__shfl_sync(0xffffffffu, qm.x, j), __shfl_sync(0xffffffffu, qm.y, j),
                                __shfl_sync(0xffffffffu, qm.z, j), __shfl_sync(0xffffffffu, qm.w, j));
@@ -557,35 +634,72 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
           const int xa = __shfl_sync(0xffffffffu, r.x, rl);
           const unsigned at = done + k;
           if (k < total && at < tj)
-            pairs[oj + at] = ((u64)(unsigned)((y0 + rl) * tiles_x + xa + (int)(k - before)) << 32) | idj;
+            out[oj + at] = ((T)(unsigned)((y0 + rl) * tiles_x + xa + (int)(k - before)) << id_bits) | (T)idj;
         }
         done += total;
       }
     }
-    run += tot;
+    __syncwarp();
+    if (staged)
+      for (unsigned k = lane; k < R; k += 32) pairs[off0 + k] = buf[k];
+    __syncwarp();                                    // the buffer is reused by the next round
   }
 }
 
-// LSD radix sort of 64-bit items on bits [bit_lo, bit_hi); returns the buffer holding the
-// result, or writes the low 32 bits of the sorted items to ids_out on the last pass.
-abcd_status radix_sort(abcd_ctx* ctx, u64* a, u64* b, long long n_static, const long long* n_dev,
-                       long long cap, int bit_lo, int bit_hi, int G, u64** result,
-                       unsigned* ids_out) {
+constexpr size_t kEmitSmem = (size_t)kEmitBufBytes * (kEmitThreads / 32);
+
+template <typename T>
+abcd_status emit_smem_attr(abcd_ctx* ctx) {
+  const cudaError_t e = cudaFuncSetAttribute(emit_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kEmitSmem);
+  return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "emit smem: %s", cudaGetErrorString(e));
+}
+
+// LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi); returns the buffer holding
+// the result, or writes the bits id_mask of the sorted items to ids_out on the last pass.
+template <typename T>
+abcd_status launch_scatter(abcd_ctx* ctx, int bits, int G, const T* src, T* dst, unsigned* ids,
+                           unsigned id_mask, long long n_static, const long long* n_dev,
+                           long long cap, int shift, const unsigned* totals) {
+#define ABCD_SCATTER(B)                                                                     \
+  case B:                                                                                   \
+    radix_scatter_kernel<T, B><<<G, kRadixBins, 0, ctx->stream>>>(                          \
+        src, dst, ids, id_mask, n_static, n_dev, cap, shift, ctx->ws.hist, totals, G);      \
+    break;
+  switch (bits) {
+    ABCD_SCATTER(4) ABCD_SCATTER(5) ABCD_SCATTER(6) ABCD_SCATTER(7) ABCD_SCATTER(8)
+    default: return fail(ctx, ABCD_ERR_INVALID_ARG, "radix digit of %d bits", bits);
+  }
+#undef ABCD_SCATTER
+  return check_launch(ctx, "radix_scatter_kernel");
+}
+
+// LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi), in the fewest passes of at
+// most 8 bits, of equal width (fewer bits per pass: fewer ballots per ranked item); returns
+// the buffer holding the result, or writes the bits id_mask of the sorted items to ids_out on
+// the last pass.
+template <typename T>
+abcd_status radix_sort(abcd_ctx* ctx, T* a, T* b, long long n_static, const long long* n_dev,
+                       long long cap, int bit_lo, int bit_hi, int G, T** result,
+                       unsigned* ids_out, unsigned id_mask) {
   unsigned* totals = ctx->ws.hist + kRadixBins * G;
-  u64* src = a;
-  u64* dst = b;
-  for (int shift = bit_lo; shift < bit_hi; shift += kRadixBits) {
-    const bool last = shift + kRadixBits >= bit_hi;
-    radix_hist_kernel<<<G, 256, 0, ctx->stream>>>(src, n_static, n_dev, cap, shift, ctx->ws.hist, G);
+  T* src = a;
+  T* dst = b;
+  const int nbits = bit_hi - bit_lo;
+  const int passes = (nbits + kRadixBits - 1) / kRadixBits;
+  const int width = std::max(4, (nbits + passes - 1) / passes);
+  for (int shift = bit_lo; shift < bit_hi; shift += width) {
+    const int bits = std::min(width, bit_hi - shift) < 4 ? 4 : std::min(width, bit_hi - shift);
+    const bool last = shift + width >= bit_hi;
+    radix_hist_kernel<T><<<G, 256, 0, ctx->stream>>>(src, n_static, n_dev, cap, shift,
+                                                     (1u << bits) - 1u, ctx->ws.hist, G);
     abcd_status s = check_launch(ctx, "radix_hist_kernel");
     if (s) return s;
     radix_rowscan_kernel<<<kRadixBins, ((G + 31) / 32) * 32, 0, ctx->stream>>>(ctx->ws.hist, G, totals);
     if ((s = check_launch(ctx, "radix_rowscan_kernel"))) return s;
-    radix_scatter_kernel<<<G, kRadixBins, 0, ctx->stream>>>(src, dst, last ? ids_out : nullptr,
-                                                            n_static, n_dev, cap, shift,
-                                                            ctx->ws.hist, totals, G);
-    if ((s = check_launch(ctx, "radix_scatter_kernel"))) return s;
-    u64* t = src; src = dst; dst = t;
+    if ((s = launch_scatter<T>(ctx, bits, G, src, dst, last ? ids_out : nullptr, id_mask, n_static,
+                               n_dev, cap, shift, totals)))
+      return s;
+    T* t = src; src = dst; dst = t;
   }
   if (result) *result = src;
   return ABCD_OK;
@@ -646,8 +760,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   }
   u64* by_depth = nullptr;
   const int Gd = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));   // depth sort
-  if ((s = radix_sort(ctx, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64, Gd, &by_depth,
-                      nullptr)))
+  if ((s = radix_sort<u64>(ctx, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64, Gd,
+                           &by_depth, nullptr, 0xffffffffu)))
     return s;
   const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
   count_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, ctx->ws.counts, ctx->ws.block_sums, Ge);
@@ -674,14 +788,28 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       if ((s = check_launch(ctx, "ranges_from_diff_kernel"))) return s;
     }
   }
-  emit_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, (const float2*)proj->uv,
-                                           (const float4*)proj->conic_opacity, ctx->ws.rects,
-                                           ctx->ws.counts, ctx->ws.block_sums, out->count, cap,
-                                           tiles_x, alpha_min, ctx->ws.pairs[0], Ge);
-  if ((s = check_launch(ctx, "emit_kernel"))) return s;
   int tile_bits = 1;
   while ((1LL << tile_bits) < n_tiles) ++tile_bits;
-  // K lives on the device: the tile passes take the largest grid; blocks past K exit at once
-  return radix_sort(ctx, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap, 32, 32 + tile_bits,
-                    kMaxRadixBlocks, nullptr, out->ids);
+  int id_bits = 1;
+  while ((1LL << id_bits) < n) ++id_bits;
+  // K lives on the device: the tile passes take the largest grid; blocks past K exit at once.
+  // (tile, id) pairs pack into 32 bits when they fit (half the bytes per pass), else 64.
+  if (tile_bits + id_bits <= 32) {
+    unsigned* pairs = reinterpret_cast<unsigned*>(ctx->ws.pairs[0]);
+    unsigned* pairs_b = reinterpret_cast<unsigned*>(ctx->ws.pairs[1]);
+    if ((s = emit_smem_attr<unsigned>(ctx))) return s;
+    emit_kernel<unsigned><<<Ge, kEmitThreads, kEmitSmem, ctx->stream>>>(
+        by_depth, n, (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects,
+        ctx->ws.counts, ctx->ws.block_sums, out->count, cap, tiles_x, alpha_min, id_bits, pairs, Ge);
+    if ((s = check_launch(ctx, "emit_kernel"))) return s;
+    return radix_sort<unsigned>(ctx, pairs, pairs_b, 0, out->count, cap, id_bits, id_bits + tile_bits,
+                                kMaxRadixBlocks, nullptr, out->ids, (1u << id_bits) - 1u);
+  }
+  if ((s = emit_smem_attr<u64>(ctx))) return s;
+  emit_kernel<u64><<<Ge, kEmitThreads, kEmitSmem, ctx->stream>>>(
+      by_depth, n, (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects,
+      ctx->ws.counts, ctx->ws.block_sums, out->count, cap, tiles_x, alpha_min, 32, ctx->ws.pairs[0], Ge);
+  if ((s = check_launch(ctx, "emit_kernel"))) return s;
+  return radix_sort<u64>(ctx, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap, 32,
+                         32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu);
 }

@@ -24,12 +24,24 @@ constexpr int RUN = 8;            // outputs per thread per window pass
 constexpr int IW = TW + 20, IH = TH + 20;    // inputs: tile + 10-pixel halo
 constexpr int MW = TW + 10, MH = TH + 10;    // windowed moments: tile + 5-pixel halo
 constexpr int kThreads = 512;
-// shared memory: x, y [IH][IW]; the five horizontal moment rows [5][IH][MW]; A, B, C
-// [3][MH][MW]; their horizontal windows [3][MH][TW] reuse the moment rows' space
-constexpr int kH5 = 5 * IH * MW;
-constexpr int kABC = 3 * MH * MW;
-constexpr int kSmemFloats = 2 * IH * IW + kH5 + kABC;
-static_assert(3 * MH * TW <= kH5, "windows of A, B, C fit in the moment space");
+constexpr int HSEG = (MW + RUN - 1) / RUN;   // column runs of the horizontal moment pass
+constexpr int VSEG = (MH + RUN - 1) / RUN;   // row runs of the vertical moment pass
+// Row pitches are odd (consecutive lanes take consecutive rows in the horizontal passes and
+// consecutive columns in the vertical ones: no bank conflicts) and wide or tall enough that a
+// run never reads past its array (the values read beyond the valid region only feed outputs
+// that are discarded).
+constexpr int IP = ((HSEG * RUN + 10) | 1);          // x, y row pitch (>= IW)
+constexpr int MP = (MW | 1);                         // moment / A, B, C row pitch (>= MW)
+constexpr int MROWS = VSEG * RUN + 10;               // rows of the moment rows (>= IH)
+constexpr int TP = (TW | 1);                         // pitch of the windows of A, B, C
+// shared memory: x, y [IH][IP]; the five horizontal moment rows [5][MROWS][MP]; A, B, C
+// [3][MH][MP]; their horizontal windows [3][MH][TP] reuse the moment rows' space
+constexpr int kH5 = 5 * MROWS * MP;
+constexpr int kABC = 3 * MH * MP;
+constexpr int kSmemFloats = 2 * IH * IP + kH5 + kABC;
+static_assert(IP >= IW && MP >= MW && MROWS >= IH, "padded pitches");
+static_assert(3 * MH * TP <= kH5, "windows of A, B, C fit in the moment space");
+static_assert((TW / RUN - 1) * RUN + RUN + 10 <= MP, "horizontal A, B, C runs stay in a row");
 
 __device__ __forceinline__ void load_weights(float* w) {
   float s = 0.f;
@@ -44,11 +56,11 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
             float lam, float* __restrict__ grad, float* partials, unsigned* ticket,
             float* loss_out) {
   extern __shared__ float sm[];
-  float* sX = sm;                     // [IH][IW]
-  float* sY = sX + IH * IW;           // [IH][IW]
-  float* h5 = sY + IH * IW;           // [5][IH][MW]
-  float* abc = h5 + kH5;              // [3][MH][MW]
-  float* h3 = h5;                     // [3][MH][TW] (moment rows are consumed by then)
+  float* sX = sm;                     // [IH][IP]
+  float* sY = sX + IH * IP;           // [IH][IP]
+  float* h5 = sY + IH * IP;           // [5][MROWS][MP]
+  float* abc = h5 + kH5;              // [3][MH][MP]
+  float* h3 = h5;                     // [3][MH][TP] (moment rows are consumed by then)
   __shared__ float red[2][kThreads / 32];
   float w[11];
   load_weights(w);
@@ -58,11 +70,11 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
   float l1 = 0.f, ssim = 0.f;
   for (int ch = 0; ch < 3; ++ch) {
     // ---- inputs with a 10-pixel halo, zero outside the image
-    for (int k = threadIdx.x; k < IH * IW; k += kThreads) {
-      const int r = k / IW, c = k - r * IW;
+    for (int k = threadIdx.x; k < IH * IP; k += kThreads) {
+      const int r = k / IP, c = k - r * IP;
       const int gy = oy - 10 + r, gx = ox - 10 + c;
       float xv = 0.f, yv = 0.f;
-      if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
+      if (c < IW && gx >= 0 && gx < W && gy >= 0 && gy < H) {
         const long long p = (long long)gy * W + gx;
         xv = xin[4 * p + ch];
         yv = yin[3 * p + ch];
@@ -72,15 +84,14 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
     }
     __syncthreads();
     // ---- horizontal windows of x, y, x^2, y^2, xy: RUN outputs per item from RUN+10 inputs
-    constexpr int HSEG = (MW + RUN - 1) / RUN;
     for (int it = threadIdx.x; it < IH * HSEG; it += kThreads) {
-      const int r = it / HSEG, c0 = (it - r * HSEG) * RUN;
+      const int r = it % IH, c0 = (it / IH) * RUN;   // consecutive lanes: consecutive rows
       float xs[RUN + 10], ys[RUN + 10], xx[RUN + 10], yy[RUN + 10], xy[RUN + 10];
 #pragma unroll
       for (int t = 0; t < RUN + 10; ++t) {
-        const int c = min(c0 + t, IW - 1);
-        xs[t] = sX[r * IW + c];
-        ys[t] = sY[r * IW + c];
+        const int c = c0 + t;
+        xs[t] = sX[r * IP + c];
+        ys[t] = sY[r * IP + c];
         xx[t] = xs[t] * xs[t];
         yy[t] = ys[t] * ys[t];
         xy[t] = xs[t] * ys[t];
@@ -94,15 +105,14 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
           a2 = fmaf(w[t], xx[o + t], a2); a3 = fmaf(w[t], yy[o + t], a3); a4 = fmaf(w[t], xy[o + t], a4);
         }
         if (c0 + o < MW) {
-          const int k = r * MW + c0 + o;
-          h5[k] = a0; h5[IH * MW + k] = a1; h5[2 * IH * MW + k] = a2;
-          h5[3 * IH * MW + k] = a3; h5[4 * IH * MW + k] = a4;
+          const int k = r * MP + c0 + o;
+          h5[k] = a0; h5[MROWS * MP + k] = a1; h5[2 * MROWS * MP + k] = a2;
+          h5[3 * MROWS * MP + k] = a3; h5[4 * MROWS * MP + k] = a4;
         }
       }
     }
     __syncthreads();
     // ---- vertical windows -> moments -> SSIM and its partials A, B, C (zero off-image)
-    constexpr int VSEG = (MH + RUN - 1) / RUN;
     for (int it = threadIdx.x; it < MW * VSEG; it += kThreads) {
       const int c = it % MW, r0 = (it / MW) * RUN;
       float m[5][RUN];
@@ -110,7 +120,7 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
       for (int q = 0; q < 5; ++q) {
         float col[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) col[t] = h5[q * IH * MW + min(r0 + t, IH - 1) * MW + c];
+        for (int t = 0; t < RUN + 10; ++t) col[t] = h5[q * MROWS * MP + (r0 + t) * MP + c];
 #pragma unroll
         for (int o = 0; o < RUN; ++o) {
           float a = 0.f;
@@ -139,26 +149,26 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
           Cc = dcxy;
           if (r >= 5 && r < 5 + TH && c >= 5 && c < 5 + TW) ssim += S;
         }
-        const int k = r * MW + c;
-        abc[k] = A; abc[MH * MW + k] = B; abc[2 * MH * MW + k] = Cc;
+        const int k = r * MP + c;
+        abc[k] = A; abc[MH * MP + k] = B; abc[2 * MH * MP + k] = Cc;
       }
     }
     __syncthreads();
     // ---- horizontal windows of A, B, C: [MH][TW]
     constexpr int HSEG3 = TW / RUN;
     for (int it = threadIdx.x; it < MH * HSEG3; it += kThreads) {
-      const int r = it / HSEG3, c0 = (it - r * HSEG3) * RUN;
+      const int r = it % MH, c0 = (it / MH) * RUN;   // consecutive lanes: consecutive rows
 #pragma unroll
       for (int q = 0; q < 3; ++q) {
         float v[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = abc[q * MH * MW + r * MW + c0 + t];
+        for (int t = 0; t < RUN + 10; ++t) v[t] = abc[q * MH * MP + r * MP + c0 + t];
 #pragma unroll
         for (int o = 0; o < RUN; ++o) {
           float a = 0.f;
 #pragma unroll
           for (int t = 0; t < 11; ++t) a = fmaf(w[t], v[o + t], a);
-          h3[q * MH * TW + r * TW + c0 + o] = a;
+          h3[q * MH * TP + r * TP + c0 + o] = a;
         }
       }
     }
@@ -172,7 +182,7 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
       for (int q = 0; q < 3; ++q) {
         float v[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = h3[q * MH * TW + (r0 + t) * TW + c];
+        for (int t = 0; t < RUN + 10; ++t) v[t] = h3[q * MH * TP + (r0 + t) * TP + c];
 #pragma unroll
         for (int o = 0; o < RUN; ++o) {
           float a = 0.f;
@@ -185,7 +195,7 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
       for (int o = 0; o < RUN; ++o) {
         const int gy = oy + r0 + o, gx = ox + c;
         if (gx >= W || gy >= H) continue;
-        const float xv = sX[(r0 + o + 10) * IW + c + 10], yv = sY[(r0 + o + 10) * IW + c + 10];
+        const float xv = sX[(r0 + o + 10) * IP + c + 10], yv = sY[(r0 + o + 10) * IP + c + 10];
         const float d = xv - yv;
         l1 += fabsf(d);
         const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
