@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/abcd.h"
 
 namespace abcd {
@@ -55,6 +57,35 @@ struct Workspace {
 
 constexpr int kRenderSubPerTile = 4;      // render CTAs (8x8 pixel blocks) per 16x16 tile
 
+// Programmatic dependent launch.  Every kernel of the library starts with pdl_prologue(): it
+// waits until the grid before it in the stream has completed and its writes are visible
+// (griddepcontrol.wait; immediate when the kernel was launched without the attribute), then
+// lets the next grid be launched (griddepcontrol.launch_dependents), whose CTAs wait the same
+// way before touching memory.  Launching and rasterising a kernel thus overlaps the tail of the
+// one before it instead of following it.  The next grid only starts once every CTA of this one
+// is resident, so it takes resources this grid no longer needs.
+__device__ __forceinline__ void pdl_prologue() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Launches kernel on stream with programmatic stream serialisation allowed.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // Mask of the lanes whose value equals this lane's, for values 0..256 (256 marks an unused
 // lane; it matches only other unused lanes).  Nine ballots: the cost does not depend on how
 // many distinct values the warp holds, unlike __match_any_sync's.
@@ -96,6 +127,7 @@ namespace abcd {
 
 abcd_status fail(abcd_ctx* ctx, abcd_status code, const char* fmt, ...);
 abcd_status check_launch(abcd_ctx* ctx, const char* what);
+abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched);
 bool has_workspace(const abcd_ctx* ctx);
 Cam make_cam(const abcd_camera* c, const abcd_render_opts* o);
 Opts make_opts(const abcd_render_opts* o);

@@ -29,6 +29,7 @@ struct AdamArgs {
 };
 
 __global__ void __launch_bounds__(256) adam_kernel(const __grid_constant__ AdamArgs a) {
+  pdl_prologue();
   const long long total = a.start[5];
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
@@ -90,6 +91,6 @@ extern "C" abcd_status abcd_adam_active(abcd_ctx* ctx, abcd_gaussians* theta,
   a.eps = eps;
   a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
   const long long blocks = std::min<long long>((a.start[5] + 255) / 256, (long long)ctx->num_sms * 16);
-  adam_kernel<<<(int)blocks, 256, 0, ctx->stream>>>(a);
-  return check_launch(ctx, "adam_kernel");
+  return check_launch(ctx, "adam_kernel",
+                      launch_pdl(adam_kernel, dim3((unsigned)blocks), dim3(256), 0, ctx->stream, a));
 }

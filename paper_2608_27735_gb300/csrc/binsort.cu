@@ -60,6 +60,7 @@ __device__ __forceinline__ int4 tile_rect(float2 m, int r, int tiles_x, int tile
 // rectangle of its square
 __global__ void keys_rects_kernel(const float* depth, const int* radius, const float2* uv, int n,
                                   int tiles_x, int tiles_y, u64* items, int4* rects) {
+  pdl_prologue();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   int4 q = make_int4(0, 0, 0, 0);
@@ -157,6 +158,7 @@ constexpr int kSmemDiffCells = 12288;      // 48 KB: tile grids up to ~1900x1500
 __global__ void __launch_bounds__(256)
 tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, int tiles_x,
                  int tiles_y, float alpha_min, unsigned* counts, int* diff) {
+  pdl_prologue();
   extern __shared__ int sdiff[];
   const int W1 = tiles_x + 1;
   const int cells = W1 * (tiles_y + 1);
@@ -231,6 +233,7 @@ template <typename T>
 __global__ void __launch_bounds__(256)
 radix_hist_kernel(const T* in, long long n_static, const long long* n_dev, long long cap,
                   int shift, unsigned mask, unsigned* hist, int G) {
+  pdl_prologue();
   __shared__ unsigned h[kRadixBins];
   for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) h[d] = 0;
   __syncthreads();
@@ -285,6 +288,7 @@ __device__ __forceinline__ unsigned long long block_exclusive_scan(unsigned long
 // digit); the row totals go to totals[d]
 __global__ void __launch_bounds__(1024) radix_rowscan_kernel(unsigned* hist, int G,
                                                             unsigned* totals) {
+  pdl_prologue();
   const int d = blockIdx.x;
   const unsigned v = (int)threadIdx.x < G ? hist[d * G + threadIdx.x] : 0u;
   unsigned long long tot = 0;
@@ -301,6 +305,7 @@ __global__ void __launch_bounds__(256)
 radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
                      const long long* n_dev, long long cap, int shift, const unsigned* hist,
                      const unsigned* totals, int G) {
+  pdl_prologue();
   constexpr int W = 8;
   constexpr unsigned BINS = 1u << BITS, MASK = BINS - 1;
   __shared__ unsigned cnt[W][BINS];
@@ -373,6 +378,7 @@ radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, l
 __global__ void __launch_bounds__(256)
 count_kernel(const u64* sorted, int n, const unsigned* counts, unsigned long long* block_sums,
              int G) {
+  pdl_prologue();
   long long lo, hi;
   block_range(n, G, &lo, &hi);
   unsigned long long s = 0;
@@ -392,6 +398,7 @@ count_kernel(const u64* sorted, int n, const unsigned* counts, unsigned long lon
 __global__ void __launch_bounds__(1024)
 scan_blocks_kernel(unsigned long long* block_sums, int G, long long* count, long long cap,
                    unsigned* status) {
+  pdl_prologue();
   const unsigned long long v = (int)threadIdx.x < G ? block_sums[threadIdx.x] : 0ull;
   unsigned long long total = 0;
   const unsigned long long ex = block_exclusive_scan(v, &total);
@@ -407,6 +414,7 @@ scan_blocks_kernel(unsigned long long* block_sums, int G, long long* count, long
 __global__ void __launch_bounds__(1024)
 ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* count, long long cap,
                         unsigned* ranges) {
+  pdl_prologue();
   const int W1 = tiles_x + 1;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   for (int y = wid; y < tiles_y; y += nw) {                        // prefix along each row
@@ -454,6 +462,7 @@ __device__ __forceinline__ unsigned count_bucket(unsigned c) {
 __global__ void __launch_bounds__(1024)
 ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, const long long* count,
                     long long cap, unsigned* ranges, unsigned* tile_order) {
+  pdl_prologue();
   extern __shared__ int sd[];              // [(tiles_x + 1) (tiles_y + 1)] cells, then [nt] keys
   __shared__ unsigned hist[kOrderBuckets];
   const int W1 = tiles_x + 1, cells = W1 * (tiles_y + 1), nt = tiles_x * tiles_y;
@@ -555,6 +564,7 @@ __global__ void __launch_bounds__(kEmitThreads)
 emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const int4* rects,
             const unsigned* counts, const unsigned long long* block_off, const long long* count,
             long long cap, int tiles_x, float alpha_min, int id_bits, T* pairs, int G) {
+  pdl_prologue();
   constexpr unsigned kBuf = kEmitBufBytes / sizeof(T);
   extern __shared__ __align__(16) unsigned char emit_smem[];
   if (*count > cap) return;
@@ -662,15 +672,17 @@ abcd_status launch_scatter(abcd_ctx* ctx, int bits, int G, const T* src, T* dst,
                            long long cap, int shift, const unsigned* totals) {
 #define ABCD_SCATTER(B)                                                                     \
   case B:                                                                                   \
-    radix_scatter_kernel<T, B><<<G, kRadixBins, 0, ctx->stream>>>(                          \
-        src, dst, ids, id_mask, n_static, n_dev, cap, shift, ctx->ws.hist, totals, G);      \
+    e = launch_pdl(radix_scatter_kernel<T, B>, dim3(G), dim3(kRadixBins), 0, ctx->stream,     \
+                   src, dst, ids, id_mask, n_static, n_dev, cap, shift,                     \
+                   (const unsigned*)ctx->ws.hist, totals, G);                               \
     break;
+  cudaError_t e = cudaSuccess;
   switch (bits) {
     ABCD_SCATTER(4) ABCD_SCATTER(5) ABCD_SCATTER(6) ABCD_SCATTER(7) ABCD_SCATTER(8)
     default: return fail(ctx, ABCD_ERR_INVALID_ARG, "radix digit of %d bits", bits);
   }
 #undef ABCD_SCATTER
-  return check_launch(ctx, "radix_scatter_kernel");
+  return check_launch(ctx, "radix_scatter_kernel", e);
 }
 
 // LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi), in the fewest passes of at
@@ -690,12 +702,15 @@ abcd_status radix_sort(abcd_ctx* ctx, T* a, T* b, long long n_static, const long
   for (int shift = bit_lo; shift < bit_hi; shift += width) {
     const int bits = std::min(width, bit_hi - shift) < 4 ? 4 : std::min(width, bit_hi - shift);
     const bool last = shift + width >= bit_hi;
-    radix_hist_kernel<T><<<G, 256, 0, ctx->stream>>>(src, n_static, n_dev, cap, shift,
-                                                     (1u << bits) - 1u, ctx->ws.hist, G);
-    abcd_status s = check_launch(ctx, "radix_hist_kernel");
+    abcd_status s = check_launch(
+        ctx, "radix_hist_kernel",
+        launch_pdl(radix_hist_kernel<T>, dim3(G), dim3(256), 0, ctx->stream, (const T*)src, n_static,
+                   n_dev, cap, shift, (1u << bits) - 1u, ctx->ws.hist, G));
     if (s) return s;
-    radix_rowscan_kernel<<<kRadixBins, ((G + 31) / 32) * 32, 0, ctx->stream>>>(ctx->ws.hist, G, totals);
-    if ((s = check_launch(ctx, "radix_rowscan_kernel"))) return s;
+    if ((s = check_launch(ctx, "radix_rowscan_kernel",
+                          launch_pdl(radix_rowscan_kernel, dim3(kRadixBins), dim3(((G + 31) / 32) * 32),
+                                     0, ctx->stream, ctx->ws.hist, G, totals))))
+      return s;
     if ((s = launch_scatter<T>(ctx, bits, G, src, dst, last ? ids_out : nullptr, id_mask, n_static,
                                n_dev, cap, shift, totals)))
       return s;
@@ -742,10 +757,12 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "diff memset: %s", cudaGetErrorString(e));
   abcd_status s;
   const float alpha_min = make_opts(opts).alpha_min;
-  keys_rects_kernel<<<(n + 255) / 256, 256, 0, ctx->stream>>>(
-      proj->depth, proj->radius, (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
-      ctx->ws.rects);
-  if ((s = check_launch(ctx, "keys_rects_kernel"))) return s;
+  if ((s = check_launch(ctx, "keys_rects_kernel",
+                        launch_pdl(keys_rects_kernel, dim3((n + 255) / 256), dim3(256), 0, ctx->stream,
+                                   (const float*)proj->depth, (const int*)proj->radius,
+                                   (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
+                                   ctx->ws.rects))))
+    return s;
   {
     const int cells = (tiles_x + 1) * (tiles_y + 1);
     const size_t smem = cells <= kSmemDiffCells ? sizeof(int) * cells : 0;
@@ -753,10 +770,12 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       const cudaError_t e2 = cudaFuncSetAttribute(tile_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile_rows smem: %s", cudaGetErrorString(e2));
     }
-    tile_rows_kernel<<<(n + 255) / 256, 256, smem, ctx->stream>>>(
-        (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects, n, tiles_x,
-        tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff);
-    if ((s = check_launch(ctx, "tile_rows_kernel"))) return s;
+    if ((s = check_launch(ctx, "tile_rows_kernel",
+                          launch_pdl(tile_rows_kernel, dim3((n + 255) / 256), dim3(256), smem,
+                                     ctx->stream, (const float2*)proj->uv,
+                                     (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
+                                     n, tiles_x, tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff))))
+      return s;
   }
   u64* by_depth = nullptr;
   const int Gd = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));   // depth sort
@@ -764,10 +783,15 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                            &by_depth, nullptr, 0xffffffffu)))
     return s;
   const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
-  count_kernel<<<Ge, 256, 0, ctx->stream>>>(by_depth, n, ctx->ws.counts, ctx->ws.block_sums, Ge);
-  if ((s = check_launch(ctx, "count_kernel"))) return s;
-  scan_blocks_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status);
-  if ((s = check_launch(ctx, "scan_blocks_kernel"))) return s;
+  if ((s = check_launch(ctx, "count_kernel",
+                        launch_pdl(count_kernel, dim3(Ge), dim3(256), 0, ctx->stream,
+                                   (const u64*)by_depth, n, (const unsigned*)ctx->ws.counts,
+                                   ctx->ws.block_sums, Ge))))
+    return s;
+  if ((s = check_launch(ctx, "scan_blocks_kernel",
+                        launch_pdl(scan_blocks_kernel, dim3(1), dim3(1024), 0, ctx->stream,
+                                   ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status))))
+    return s;
   {
     const int cells = (tiles_x + 1) * (tiles_y + 1);
     ctx->order_ranges = nullptr;
@@ -777,15 +801,20 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
         const cudaError_t e2 = cudaFuncSetAttribute(ranges_order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "ranges smem: %s", cudaGetErrorString(e2));
       }
-      ranges_order_kernel<<<1, 1024, smem, ctx->stream>>>(ctx->ws.diff, tiles_x, tiles_y, out->count,
-                                                          cap, out->ranges, ctx->ws.tile_order);
-      if ((s = check_launch(ctx, "ranges_order_kernel"))) return s;
+      if ((s = check_launch(ctx, "ranges_order_kernel",
+                            launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->stream,
+                                       (const int*)ctx->ws.diff, tiles_x, tiles_y,
+                                       (const long long*)out->count, cap, out->ranges,
+                                       ctx->ws.tile_order))))
+        return s;
       ctx->order_ranges = out->ranges;           // the order belongs to these ranges
       ctx->order_tiles = n_tiles;
     } else {
-      ranges_from_diff_kernel<<<1, 1024, 0, ctx->stream>>>(ctx->ws.diff, tiles_x, tiles_y, out->count,
-                                                          cap, out->ranges);
-      if ((s = check_launch(ctx, "ranges_from_diff_kernel"))) return s;
+      if ((s = check_launch(ctx, "ranges_from_diff_kernel",
+                            launch_pdl(ranges_from_diff_kernel, dim3(1), dim3(1024), 0, ctx->stream,
+                                       ctx->ws.diff, tiles_x, tiles_y, (const long long*)out->count,
+                                       cap, out->ranges))))
+        return s;
     }
   }
   int tile_bits = 1;
@@ -798,18 +827,28 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
     unsigned* pairs = reinterpret_cast<unsigned*>(ctx->ws.pairs[0]);
     unsigned* pairs_b = reinterpret_cast<unsigned*>(ctx->ws.pairs[1]);
     if ((s = emit_smem_attr<unsigned>(ctx))) return s;
-    emit_kernel<unsigned><<<Ge, kEmitThreads, kEmitSmem, ctx->stream>>>(
-        by_depth, n, (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects,
-        ctx->ws.counts, ctx->ws.block_sums, out->count, cap, tiles_x, alpha_min, id_bits, pairs, Ge);
-    if ((s = check_launch(ctx, "emit_kernel"))) return s;
+    if ((s = check_launch(ctx, "emit_kernel",
+                          launch_pdl(emit_kernel<unsigned>, dim3(Ge), dim3(kEmitThreads), kEmitSmem,
+                                     ctx->stream, (const u64*)by_depth, n, (const float2*)proj->uv,
+                                     (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
+                                     (const unsigned*)ctx->ws.counts,
+                                     (const unsigned long long*)ctx->ws.block_sums,
+                                     (const long long*)out->count, cap, tiles_x, alpha_min, id_bits,
+                                     pairs, Ge))))
+      return s;
     return radix_sort<unsigned>(ctx, pairs, pairs_b, 0, out->count, cap, id_bits, id_bits + tile_bits,
                                 kMaxRadixBlocks, nullptr, out->ids, (1u << id_bits) - 1u);
   }
   if ((s = emit_smem_attr<u64>(ctx))) return s;
-  emit_kernel<u64><<<Ge, kEmitThreads, kEmitSmem, ctx->stream>>>(
-      by_depth, n, (const float2*)proj->uv, (const float4*)proj->conic_opacity, ctx->ws.rects,
-      ctx->ws.counts, ctx->ws.block_sums, out->count, cap, tiles_x, alpha_min, 32, ctx->ws.pairs[0], Ge);
-  if ((s = check_launch(ctx, "emit_kernel"))) return s;
+  if ((s = check_launch(ctx, "emit_kernel",
+                        launch_pdl(emit_kernel<u64>, dim3(Ge), dim3(kEmitThreads), kEmitSmem,
+                                   ctx->stream, (const u64*)by_depth, n, (const float2*)proj->uv,
+                                   (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
+                                   (const unsigned*)ctx->ws.counts,
+                                   (const unsigned long long*)ctx->ws.block_sums,
+                                   (const long long*)out->count, cap, tiles_x, alpha_min, 32,
+                                   ctx->ws.pairs[0], Ge))))
+    return s;
   return radix_sort<u64>(ctx, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap, 32,
                          32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu);
 }

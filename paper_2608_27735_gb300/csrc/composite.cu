@@ -100,6 +100,7 @@ template <int PIX, bool F16>
 __global__ void __launch_bounds__(256)
 composite_kernel(const __grid_constant__ LayerTable lt, int nf, int nb, long long groups,
                  void* Fout, void* Bout, int out_f16) {
+  pdl_prologue();
   for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < groups;
        g += (long long)gridDim.x * blockDim.x) {
     float acc[4 * PIX];
@@ -155,12 +156,14 @@ extern "C" abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* la
   if (!F_out && !B_out) return ABCD_OK;
   const int grid = ctx->num_sms * 8;
   const bool pairs = al16 && (npix % 2 == 0);
-  if (layer_dtype == ABCD_F16) {
-    if (pairs) composite_kernel<2, true><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix / 2, F_out, B_out, out_dtype == ABCD_F16);
-    else composite_kernel<1, true><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix, F_out, B_out, out_dtype == ABCD_F16);
-  } else {
-    if (pairs) composite_kernel<2, false><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix / 2, F_out, B_out, out_dtype == ABCD_F16);
-    else composite_kernel<1, false><<<grid, 256, 0, ctx->stream>>>(lt, nf, nb, npix, F_out, B_out, out_dtype == ABCD_F16);
-  }
-  return check_launch(ctx, "composite_kernel");
+  const bool o16 = out_dtype == ABCD_F16;
+  const long long units = pairs ? npix / 2 : npix;
+  cudaError_t e;
+  if (layer_dtype == ABCD_F16)
+    e = pairs ? launch_pdl(composite_kernel<2, true>, dim3(grid), dim3(256), 0, ctx->stream, lt, nf, nb, units, F_out, B_out, o16)
+              : launch_pdl(composite_kernel<1, true>, dim3(grid), dim3(256), 0, ctx->stream, lt, nf, nb, units, F_out, B_out, o16);
+  else
+    e = pairs ? launch_pdl(composite_kernel<2, false>, dim3(grid), dim3(256), 0, ctx->stream, lt, nf, nb, units, F_out, B_out, o16)
+              : launch_pdl(composite_kernel<1, false>, dim3(grid), dim3(256), 0, ctx->stream, lt, nf, nb, units, F_out, B_out, o16);
+  return check_launch(ctx, "composite_kernel", e);
 }

@@ -27,6 +27,15 @@ abcd_status check_launch(abcd_ctx* ctx, const char* what) {
   return ABCD_OK;
 }
 
+abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched) {
+  if (launched != cudaSuccess) {
+    ctx->launches++;
+    (void)cudaGetLastError();
+    return fail(ctx, ABCD_ERR_CUDA, "%s: %s", what, cudaGetErrorString(launched));
+  }
+  return check_launch(ctx, what);
+}
+
 bool has_workspace(const abcd_ctx* ctx) { return ctx && ctx->ws_base != nullptr; }
 
 Opts make_opts(const abcd_render_opts* o) {

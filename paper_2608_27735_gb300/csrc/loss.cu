@@ -55,6 +55,7 @@ __global__ void __launch_bounds__(kThreads)
 loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W, int H,
             float lam, float* __restrict__ grad, float* partials, unsigned* ticket,
             float* loss_out) {
+  pdl_prologue();
   extern __shared__ float sm[];
   float* sX = sm;                     // [IH][IP]
   float* sY = sX + IH * IP;           // [IH][IP]
@@ -263,10 +264,10 @@ abcd_status loss_launch(abcd_ctx* ctx, const float* out_rgba, const float* gt_rg
   const size_t smem = sizeof(float) * kSmemFloats;
   cudaError_t e = cudaFuncSetAttribute(loss_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "loss smem attribute: %s", cudaGetErrorString(e));
-  loss_kernel<<<grid, kThreads, smem, ctx->stream>>>(out_rgba, gt_rgb, width, height, lambda_ssim,
-                                                    dL_dout, ctx->ws.loss_partials,
-                                                    ctx->ws.status + 1, loss_out);
-  return check_launch(ctx, "loss_kernel");
+  return check_launch(ctx, "loss_kernel",
+                      launch_pdl(loss_kernel, grid, dim3(kThreads), smem, ctx->stream, out_rgba, gt_rgb,
+                                 width, height, lambda_ssim, dL_dout, ctx->ws.loss_partials,
+                                 ctx->ws.status + 1, loss_out));
 }
 
 }  // namespace abcd
@@ -334,7 +335,8 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
   if (cudaFuncSetAttribute(loss_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
       cudaSuccess)
     return ABCD_ERR_CUDA;
-  loss_kernel<<<grid, kThreads, smem, stream>>>(out_rgba, gt_rgb, width, height, lambda_ssim,
-                                                dL_dout, partials, ticket, loss_out);
-  return cudaGetLastError() == cudaSuccess ? ABCD_OK : ABCD_ERR_CUDA;
+  const cudaError_t e = launch_pdl(loss_kernel, grid, dim3(kThreads), smem, stream, out_rgba,
+                                   gt_rgb, width, height, lambda_ssim, dL_dout, partials, ticket,
+                                   loss_out);
+  return e == cudaSuccess && cudaGetLastError() == cudaSuccess ? ABCD_OK : ABCD_ERR_CUDA;
 }

@@ -139,6 +139,7 @@ __global__ void __launch_bounds__(256)
 project_fwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, float2* uv,
                    float4* conic_op, float* rgb, float* depth, int* radius,
                    unsigned* tiles_touched) {
+  pdl_prologue();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const float tz = view_depth(cam, p.means[3 * i], p.means[3 * i + 1], p.means[3 * i + 2]);
@@ -206,6 +207,7 @@ struct Grads {
 __global__ void __launch_bounds__(128)
 project_bwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, const float* grad2d,
                    Grads out) {
+  pdl_prologue();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const int D = (deg + 1) * (deg + 1);
@@ -352,11 +354,12 @@ extern "C" abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta,
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_project: uv must be 8-byte and conic_opacity 16-byte aligned");
   if (theta->n == 0) return ABCD_OK;
   const int threads = 256, blocks = (theta->n + threads - 1) / threads;
-  project_fwd_kernel<<<blocks, threads, 0, ctx->stream>>>(
-      params_of(theta), theta->n, theta->sh_degree, make_cam(cam, opts), make_opts(opts), ctx->sh,
-      (float2*)out->uv, (float4*)out->conic_opacity, out->rgb, out->depth, out->radius,
-      out->tiles_touched);
-  return check_launch(ctx, "project_fwd_kernel");
+  return check_launch(ctx, "project_fwd_kernel",
+                      launch_pdl(project_fwd_kernel, dim3(blocks), dim3(threads), 0, ctx->stream,
+                                 params_of(theta), theta->n, theta->sh_degree, make_cam(cam, opts),
+                                 make_opts(opts), ctx->sh, (float2*)out->uv,
+                                 (float4*)out->conic_opacity, out->rgb, out->depth, out->radius,
+                                 out->tiles_touched));
 }
 
 extern "C" abcd_status abcd_project_backward(abcd_ctx* ctx, const abcd_gaussians* theta,
@@ -370,8 +373,10 @@ extern "C" abcd_status abcd_project_backward(abcd_ctx* ctx, const abcd_gaussians
   if (theta->n > 0 && !grad2d) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_project_backward: null grad2d");
   if (theta->n == 0) return ABCD_OK;
   const int threads = 128, blocks = (theta->n + threads - 1) / threads;
-  project_bwd_kernel<<<blocks, threads, 0, ctx->stream>>>(
-      params_of(theta), theta->n, theta->sh_degree, make_cam(cam, opts), make_opts(opts), ctx->sh,
-      grad2d, Grads{grads->means, grads->log_scales, grads->quats, grads->opacity_logits, grads->sh});
-  return check_launch(ctx, "project_bwd_kernel");
+  return check_launch(ctx, "project_bwd_kernel",
+                      launch_pdl(project_bwd_kernel, dim3(blocks), dim3(threads), 0, ctx->stream,
+                                 params_of(theta), theta->n, theta->sh_degree, make_cam(cam, opts),
+                                 make_opts(opts), ctx->sh, grad2d,
+                                 Grads{grads->means, grads->log_scales, grads->quats,
+                                       grads->opacity_logits, grads->sh}));
 }

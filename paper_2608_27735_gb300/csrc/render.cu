@@ -295,6 +295,7 @@ __device__ __forceinline__ void store_pixel(const FwdArgs& a, long long p, const
 }
 
 __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
+  pdl_prologue();
   __shared__ float2 s_uv[kBatch];
   __shared__ float4 s_co[kBatch];
   __shared__ float4 s_rgb[kBatch];
@@ -429,6 +430,7 @@ __device__ __forceinline__ float warp_sum32(float (&x)[32], int lane) {
 }
 
 __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
+  pdl_prologue();
   __shared__ float2 s_uv[kBatch + 2];
   __shared__ float4 s_co[kBatch + 2];
   __shared__ float4 s_rgb[kBatch + 2];
@@ -531,8 +533,8 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.refresh = (uint2*)refresh_f16;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
   a.tile_order = tile_order_for(ctx, tiles, n_tiles);
-  render_fwd_kernel<<<n_blocks, kSubThreads, 0, ctx->stream>>>(a);
-  return check_launch(ctx, "render_fwd_kernel");
+  return check_launch(ctx, "render_fwd_kernel",
+                      launch_pdl(render_fwd_kernel, dim3(n_blocks), dim3(kSubThreads), 0, ctx->stream, a));
 }
 
 extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* cam,
@@ -567,6 +569,6 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   a.grad2d = grad2d;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
   a.tile_order = tile_order_for(ctx, tiles, n_tiles);
-  render_bwd_kernel<<<n_blocks, kSubThreads, 0, ctx->stream>>>(a);
-  return check_launch(ctx, "render_bwd_kernel");
+  return check_launch(ctx, "render_bwd_kernel",
+                      launch_pdl(render_bwd_kernel, dim3(n_blocks), dim3(kSubThreads), 0, ctx->stream, a));
 }
