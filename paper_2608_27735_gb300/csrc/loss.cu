@@ -8,7 +8,8 @@
 // A = dS/dmu_x - 2 mu_x dS/dsigma_xx - mu_y dS/dsigma_xy, B = dS/dsigma_xx, C = dS/dsigma_xy,
 // and windows them again: dSSIM_sum/dx(q) = (w*A)(q) + 2 x(q) (w*B)(q) + y(q) (w*C)(q).
 // Every window pass is register-blocked: a thread produces 8 consecutive outputs from a
-// sliding run of 18 staged values (about 12 FMAs per shared-memory load).
+// sliding run of 18 staged values (about 12 FMAs per shared-memory load), and the windows of
+// x and y (of x^2 and y^2, of A and B) share packed two-lane FMAs.
 // The scalar is reduced deterministically: per-CTA partial sums, then the last CTA to finish
 // adds them in a fixed order (no waiting on other CTAs).
 #include <mutex>
@@ -23,25 +24,31 @@ constexpr int TH = 32;
 constexpr int RUN = 8;            // outputs per thread per window pass
 constexpr int IW = TW + 20, IH = TH + 20;    // inputs: tile + 10-pixel halo
 constexpr int MW = TW + 10, MH = TH + 10;    // windowed moments: tile + 5-pixel halo
-constexpr int kThreads = 512;
 constexpr int HSEG = (MW + RUN - 1) / RUN;   // column runs of the horizontal moment pass
 constexpr int VSEG = (MH + RUN - 1) / RUN;   // row runs of the vertical moment pass
+constexpr int kThreads = 544;                // 17 warps: one horizontal moment run per thread
+static_assert(IH * HSEG <= kThreads, "the horizontal moment pass is one round");
 // Row pitches are odd (consecutive lanes take consecutive rows in the horizontal passes and
-// consecutive columns in the vertical ones: no bank conflicts) and wide or tall enough that a
-// run never reads past its array (the values read beyond the valid region only feed outputs
-// that are discarded).
-constexpr int IP = ((HSEG * RUN + 10) | 1);          // x, y row pitch (>= IW)
+// consecutive columns in the vertical ones: no bank conflicts, also for the 8-byte pairs) and
+// wide or tall enough that a run never reads past its array (the values read beyond the valid
+// region only feed outputs that are discarded).
+constexpr int IP = ((HSEG * RUN + 10) | 1);          // x|y row pitch (>= IW)
 constexpr int MP = (MW | 1);                         // moment / A, B, C row pitch (>= MW)
 constexpr int MROWS = VSEG * RUN + 10;               // rows of the moment rows (>= IH)
 constexpr int TP = (TW | 1);                         // pitch of the windows of A, B, C
-// shared memory: x, y [IH][IP]; the five horizontal moment rows [5][MROWS][MP]; A, B, C
-// [3][MH][MP]; their horizontal windows [3][MH][TP] reuse the moment rows' space
-constexpr int kH5 = 5 * MROWS * MP;
+// Shared memory, in floats: (x, y) pairs [IH][IP]; the horizontal moment rows as pairs
+// (mu_x, mu_y), (s_xx, s_yy) [MROWS][MP] and s_xy [MROWS][MP]; (A, B) pairs and C [MH][MP];
+// their horizontal windows, (A, B) pairs and C [MH][TP], reuse the moment rows' space.  The
+// pairs go through the packed fp32 FMA (__ffma2_rn), two windows per instruction; each
+// component is rounded exactly as a scalar fmaf.
+constexpr int kXY = 2 * IH * IP;
+constexpr int kMom = 5 * MROWS * MP;
 constexpr int kABC = 3 * MH * MP;
-constexpr int kSmemFloats = 2 * IH * IP + kH5 + kABC;
+constexpr int kSmemFloats = kXY + kMom + kABC;
 static_assert(IP >= IW && MP >= MW && MROWS >= IH, "padded pitches");
-static_assert(3 * MH * TP <= kH5, "windows of A, B, C fit in the moment space");
+static_assert(3 * MH * TP <= kMom, "windows of A, B, C fit in the moment space");
 static_assert((TW / RUN - 1) * RUN + RUN + 10 <= MP, "horizontal A, B, C runs stay in a row");
+static_assert(kXY % 2 == 0 && (kXY + kMom) % 2 == 0, "pair arrays 8-byte aligned");
 
 __device__ __forceinline__ void load_weights(float* w) {
   float s = 0.f;
@@ -51,20 +58,51 @@ __device__ __forceinline__ void load_weights(float* w) {
   for (int t = 0; t < 11; ++t) w[t] /= s;
 }
 
+// RUN outputs of an 11-tap window from RUN + 10 staged pairs / values.
+__device__ __forceinline__ void window_pairs(const float2 (&v)[RUN + 10], const float2 (&w2)[11],
+                                             float2 (&out)[RUN]) {
+#pragma unroll
+  for (int o = 0; o < RUN; ++o) {
+    float2 a = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int t = 0; t < 11; ++t) a = __ffma2_rn(w2[t], v[o + t], a);
+    out[o] = a;
+  }
+}
+
+__device__ __forceinline__ void window_scalars(const float (&v)[RUN + 10], const float2 (&w2)[11],
+                                               float (&out)[RUN]) {
+#pragma unroll
+  for (int o = 0; o < RUN; ++o) {
+    float a = 0.f;
+#pragma unroll
+    for (int t = 0; t < 11; ++t) a = fmaf(w2[t].x, v[o + t], a);
+    out[o] = a;
+  }
+}
+
 __global__ void __launch_bounds__(kThreads)
 loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W, int H,
             float lam, float* __restrict__ grad, float* partials, unsigned* ticket,
             float* loss_out) {
   pdl_prologue();
-  extern __shared__ float sm[];
-  float* sX = sm;                     // [IH][IP]
-  float* sY = sX + IH * IP;           // [IH][IP]
-  float* h5 = sY + IH * IP;           // [5][MROWS][MP]
-  float* abc = h5 + kH5;              // [3][MH][MP]
-  float* h3 = h5;                     // [3][MH][TP] (moment rows are consumed by then)
+  extern __shared__ __align__(16) float sm[];
+  float2* sXY = reinterpret_cast<float2*>(sm);                        // [IH][IP]
+  float2* hM = reinterpret_cast<float2*>(sm + kXY);                   // [MROWS][MP]
+  float2* hS = hM + MROWS * MP;                                       // [MROWS][MP]
+  float* hC = reinterpret_cast<float*>(hS + MROWS * MP);              // [MROWS][MP]
+  float2* aAB = reinterpret_cast<float2*>(sm + kXY + kMom);           // [MH][MP]
+  float* aC = reinterpret_cast<float*>(aAB + MH * MP);                // [MH][MP]
+  float2* gAB = hM;                                                   // [MH][TP]
+  float* gC = reinterpret_cast<float*>(gAB + MH * TP);                // [MH][TP]
   __shared__ float red[2][kThreads / 32];
-  float w[11];
-  load_weights(w);
+  float2 w2[11];
+  {
+    float w[11];
+    load_weights(w);
+#pragma unroll
+    for (int t = 0; t < 11; ++t) w2[t] = make_float2(w[t], w[t]);
+  }
   const int ox = blockIdx.x * TW, oy = blockIdx.y * TH;
   const float inv = 1.f / (3.f * (float)W * (float)H);
   const float C1 = 0.01f * 0.01f, C2 = 0.03f * 0.03f;
@@ -80,55 +118,51 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
         xv = xin[4 * p + ch];
         yv = yin[3 * p + ch];
       }
-      sX[k] = xv;
-      sY[k] = yv;
+      sXY[k] = make_float2(xv, yv);
     }
     __syncthreads();
-    // ---- horizontal windows of x, y, x^2, y^2, xy: RUN outputs per item from RUN+10 inputs
+    // ---- horizontal windows of (x, y), (x^2, y^2) and xy: RUN outputs per run
     for (int it = threadIdx.x; it < IH * HSEG; it += kThreads) {
       const int r = it % IH, c0 = (it / IH) * RUN;   // consecutive lanes: consecutive rows
-      float xs[RUN + 10], ys[RUN + 10], xx[RUN + 10], yy[RUN + 10], xy[RUN + 10];
+      float2 v[RUN + 10], q[RUN + 10], o2[RUN];
 #pragma unroll
       for (int t = 0; t < RUN + 10; ++t) {
-        const int c = c0 + t;
-        xs[t] = sX[r * IP + c];
-        ys[t] = sY[r * IP + c];
-        xx[t] = xs[t] * xs[t];
-        yy[t] = ys[t] * ys[t];
-        xy[t] = xs[t] * ys[t];
+        v[t] = sXY[r * IP + c0 + t];
+        q[t] = __fmul2_rn(v[t], v[t]);
       }
+      window_pairs(v, w2, o2);
 #pragma unroll
-      for (int o = 0; o < RUN; ++o) {
-        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, a4 = 0.f;
+      for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hM[r * MP + c0 + o] = o2[o];
+      window_pairs(q, w2, o2);
 #pragma unroll
-        for (int t = 0; t < 11; ++t) {
-          a0 = fmaf(w[t], xs[o + t], a0); a1 = fmaf(w[t], ys[o + t], a1);
-          a2 = fmaf(w[t], xx[o + t], a2); a3 = fmaf(w[t], yy[o + t], a3); a4 = fmaf(w[t], xy[o + t], a4);
-        }
-        if (c0 + o < MW) {
-          const int k = r * MP + c0 + o;
-          h5[k] = a0; h5[MROWS * MP + k] = a1; h5[2 * MROWS * MP + k] = a2;
-          h5[3 * MROWS * MP + k] = a3; h5[4 * MROWS * MP + k] = a4;
-        }
-      }
+      for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hS[r * MP + c0 + o] = o2[o];
+      float p[RUN + 10], o1[RUN];
+#pragma unroll
+      for (int t = 0; t < RUN + 10; ++t) p[t] = v[t].x * v[t].y;
+      window_scalars(p, w2, o1);
+#pragma unroll
+      for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hC[r * MP + c0 + o] = o1[o];
     }
     __syncthreads();
     // ---- vertical windows -> moments -> SSIM and its partials A, B, C (zero off-image)
     for (int it = threadIdx.x; it < MW * VSEG; it += kThreads) {
       const int c = it % MW, r0 = (it / MW) * RUN;
-      float m[5][RUN];
+      float2 mm[RUN], ss[RUN];
+      float mc[RUN];
+      {
+        float2 col[RUN + 10];
 #pragma unroll
-      for (int q = 0; q < 5; ++q) {
+        for (int t = 0; t < RUN + 10; ++t) col[t] = hM[(r0 + t) * MP + c];
+        window_pairs(col, w2, mm);
+#pragma unroll
+        for (int t = 0; t < RUN + 10; ++t) col[t] = hS[(r0 + t) * MP + c];
+        window_pairs(col, w2, ss);
+      }
+      {
         float col[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) col[t] = h5[q * MROWS * MP + (r0 + t) * MP + c];
-#pragma unroll
-        for (int o = 0; o < RUN; ++o) {
-          float a = 0.f;
-#pragma unroll
-          for (int t = 0; t < 11; ++t) a = fmaf(w[t], col[o + t], a);
-          m[q][o] = a;
-        }
+        for (int t = 0; t < RUN + 10; ++t) col[t] = hC[(r0 + t) * MP + c];
+        window_scalars(col, w2, mc);
       }
 #pragma unroll
       for (int o = 0; o < RUN; ++o) {
@@ -137,8 +171,8 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
         const int gy = oy - 5 + r, gx = ox - 5 + c;
         float A = 0.f, B = 0.f, Cc = 0.f;
         if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
-          const float mx = m[0][o], my = m[1][o];
-          const float vx = m[2][o] - mx * mx, vy = m[3][o] - my * my, cxy = m[4][o] - mx * my;
+          const float mx = mm[o].x, my = mm[o].y;
+          const float vx = ss[o].x - mx * mx, vy = ss[o].y - my * my, cxy = mc[o] - mx * my;
           const float N1 = 2.f * mx * my + C1, N2 = 2.f * cxy + C2;
           const float D1 = mx * mx + my * my + C1, D2 = vx + vy + C2;
           const float iD = 1.f / (D1 * D2);
@@ -150,27 +184,30 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
           Cc = dcxy;
           if (r >= 5 && r < 5 + TH && c >= 5 && c < 5 + TW) ssim += S;
         }
-        const int k = r * MP + c;
-        abc[k] = A; abc[MH * MP + k] = B; abc[2 * MH * MP + k] = Cc;
+        aAB[r * MP + c] = make_float2(A, B);
+        aC[r * MP + c] = Cc;
       }
     }
     __syncthreads();
-    // ---- horizontal windows of A, B, C: [MH][TW]
+    // ---- horizontal windows of (A, B) and C: [MH][TW]
     constexpr int HSEG3 = TW / RUN;
     for (int it = threadIdx.x; it < MH * HSEG3; it += kThreads) {
       const int r = it % MH, c0 = (it / MH) * RUN;   // consecutive lanes: consecutive rows
+      {
+        float2 v[RUN + 10], o2[RUN];
 #pragma unroll
-      for (int q = 0; q < 3; ++q) {
-        float v[RUN + 10];
+        for (int t = 0; t < RUN + 10; ++t) v[t] = aAB[r * MP + c0 + t];
+        window_pairs(v, w2, o2);
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = abc[q * MH * MP + r * MP + c0 + t];
+        for (int o = 0; o < RUN; ++o) gAB[r * TP + c0 + o] = o2[o];
+      }
+      {
+        float v[RUN + 10], o1[RUN];
 #pragma unroll
-        for (int o = 0; o < RUN; ++o) {
-          float a = 0.f;
+        for (int t = 0; t < RUN + 10; ++t) v[t] = aC[r * MP + c0 + t];
+        window_scalars(v, w2, o1);
 #pragma unroll
-          for (int t = 0; t < 11; ++t) a = fmaf(w[t], v[o + t], a);
-          h3[q * MH * TP + r * TP + c0 + o] = a;
-        }
+        for (int o = 0; o < RUN; ++o) gC[r * TP + c0 + o] = o1[o];
       }
     }
     __syncthreads();
@@ -178,29 +215,30 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
     constexpr int VSEG3 = TH / RUN;
     for (int it = threadIdx.x; it < TW * VSEG3; it += kThreads) {
       const int c = it % TW, r0 = (it / TW) * RUN;
-      float g[3][RUN];
+      float2 gab[RUN];
+      float gc[RUN];
+      {
+        float2 v[RUN + 10];
 #pragma unroll
-      for (int q = 0; q < 3; ++q) {
+        for (int t = 0; t < RUN + 10; ++t) v[t] = gAB[(r0 + t) * TP + c];
+        window_pairs(v, w2, gab);
+      }
+      {
         float v[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = h3[q * MH * TP + (r0 + t) * TP + c];
-#pragma unroll
-        for (int o = 0; o < RUN; ++o) {
-          float a = 0.f;
-#pragma unroll
-          for (int t = 0; t < 11; ++t) a = fmaf(w[t], v[o + t], a);
-          g[q][o] = a;
-        }
+        for (int t = 0; t < RUN + 10; ++t) v[t] = gC[(r0 + t) * TP + c];
+        window_scalars(v, w2, gc);
       }
 #pragma unroll
       for (int o = 0; o < RUN; ++o) {
         const int gy = oy + r0 + o, gx = ox + c;
         if (gx >= W || gy >= H) continue;
-        const float xv = sX[(r0 + o + 10) * IP + c + 10], yv = sY[(r0 + o + 10) * IP + c + 10];
+        const float2 xy = sXY[(r0 + o + 10) * IP + c + 10];
+        const float xv = xy.x, yv = xy.y;
         const float d = xv - yv;
         l1 += fabsf(d);
         const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
-        const float dS = g[0][o] + 2.f * xv * g[1][o] + yv * g[2][o];
+        const float dS = gab[o].x + 2.f * xv * gab[o].y + yv * gc[o];
         if (grad) grad[3 * ((long long)gy * W + gx) + ch] = ((1.f - lam) * sgn - lam * dS) * inv;
       }
     }
@@ -233,20 +271,18 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
     s0 += (double)__ldcg(&partials[2 * k]);
     s1 += (double)__ldcg(&partials[2 * k + 1]);
   }
-  __shared__ double dred[2][kThreads];
-  dred[0][threadIdx.x] = s0;
-  dred[1][threadIdx.x] = s1;
-  __syncthreads();
-  for (int st = kThreads / 2; st > 0; st >>= 1) {
-    if ((int)threadIdx.x < st) {
-      dred[0][threadIdx.x] += dred[0][threadIdx.x + st];
-      dred[1][threadIdx.x] += dred[1][threadIdx.x + st];
-    }
-    __syncthreads();
+  for (int o = 16; o > 0; o >>= 1) {
+    s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, o);
   }
+  __shared__ double dred[2][kThreads / 32];
+  if ((threadIdx.x & 31) == 0) { dred[0][threadIdx.x >> 5] = s0; dred[1][threadIdx.x >> 5] = s1; }
+  __syncthreads();
   if (threadIdx.x == 0) {
+    double t0 = 0.0, t1 = 0.0;
+    for (int k = 0; k < kThreads / 32; ++k) { t0 += dred[0][k]; t1 += dred[1][k]; }
     const double n = 3.0 * (double)W * (double)H;
-    if (loss_out) *loss_out = (float)((1.0 - lam) * dred[0][0] / n + lam * (1.0 - dred[1][0] / n));
+    if (loss_out) *loss_out = (float)((1.0 - lam) * t0 / n + lam * (1.0 - t1 / n));
     *ticket = 0u;
   }
 }
