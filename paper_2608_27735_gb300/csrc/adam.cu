@@ -2,8 +2,9 @@
 // blocks are never touched).  torch semantics with bias correction, dense over every
 // parameter of the block: m = b1 m + (1 - b1) g, v = b2 v + (1 - b2) g^2,
 // theta -= (lr / (1 - b1^t)) m / (sqrt(v) / sqrt(1 - b2^t) + eps).
-// HBM-bound: 4 reads and 3 writes of 4 bytes per parameter; one grid-stride pass over the
-// five parameter arrays (the SH array carries two learning rates, degree 0 and the rest).
+// HBM-bound: 4 reads and 3 writes of 4 bytes per parameter; one grid-stride pass over groups of
+// four elements of the five parameter arrays (16-byte accesses; the SH array carries two
+// learning rates, degree 0 and the rest).
 #include <cmath>
 
 #include "abcd_internal.cuh"
@@ -16,35 +17,72 @@ struct Seg {
   const float* g;
   float* m;
   float* v;
-  long long n;
-  int period;      // SH: 3 * D (degree-0 entries are the first 3 of each period); else 0
-  float step_lr;   // lr / (1 - b1^t)
-  float step_lr_rest;
+  unsigned n;          // elements
+  unsigned period;     // SH: 3 * D (degree-0 entries are the first 3 of each period); else 0
+  float step_lr;       // lr / (1 - b1^t)
+  float step_lr_rest;  // the SH coefficients of degree >= 1
+  int vec;             // all four pointers 16-byte aligned: float4 groups
 };
 
 struct AdamArgs {
   Seg s[5];
-  long long start[6];
+  unsigned gstart[6];  // first group of each array (groups of 4 elements)
   float b1, b2, eps, inv_sqrt_bc2;
 };
 
+__device__ __forceinline__ float adam_one(float& th, float g, float& m, float& v, float lr,
+                                          const AdamArgs& a) {
+  m = a.b1 * m + (1.f - a.b1) * g;
+  v = a.b2 * v + (1.f - a.b2) * g * g;
+  th -= lr * m / (sqrtf(v) * a.inv_sqrt_bc2 + a.eps);
+  return th;
+}
+
+// One thread per group of four consecutive elements of one array (float4 loads and stores when
+// the array allows, else scalar), grid-stride over the groups of the five arrays.
 __global__ void __launch_bounds__(256) adam_kernel(const __grid_constant__ AdamArgs a) {
   pdl_prologue();
-  const long long total = a.start[5];
-  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
-       e += (long long)gridDim.x * blockDim.x) {
+  const unsigned total = a.gstart[5];
+  for (unsigned q = blockIdx.x * blockDim.x + threadIdx.x; q < total; q += gridDim.x * blockDim.x) {
     int k = 0;
 #pragma unroll
-    for (int j = 1; j < 5; ++j) k += (e >= a.start[j]) ? 1 : 0;
+    for (int j = 1; j < 5; ++j) k += (q >= a.gstart[j]) ? 1 : 0;
     const Seg& s = a.s[k];
-    const long long i = e - a.start[k];
-    const float g = s.g[i];
-    const float m = a.b1 * s.m[i] + (1.f - a.b1) * g;
-    const float v = a.b2 * s.v[i] + (1.f - a.b2) * g * g;
-    s.m[i] = m;
-    s.v[i] = v;
-    const float lr = (s.period > 0 && (i % s.period) >= 3) ? s.step_lr_rest : s.step_lr;
-    s.th[i] -= lr * m / (sqrtf(v) * a.inv_sqrt_bc2 + a.eps);
+    const unsigned i0 = 4u * (q - a.gstart[k]);
+    float lr[4];
+    {
+      unsigned r = s.period ? i0 % s.period : 0u;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        lr[c] = (s.period && r >= 3u) ? s.step_lr_rest : s.step_lr;
+        if (s.period && ++r == s.period) r = 0u;
+      }
+    }
+    if (s.vec && i0 + 4 <= s.n) {
+      float4 th = *reinterpret_cast<const float4*>(s.th + i0);
+      const float4 g = *reinterpret_cast<const float4*>(s.g + i0);
+      float4 m = *reinterpret_cast<const float4*>(s.m + i0);
+      float4 v = *reinterpret_cast<const float4*>(s.v + i0);
+      adam_one(th.x, g.x, m.x, v.x, lr[0], a);
+      adam_one(th.y, g.y, m.y, v.y, lr[1], a);
+      adam_one(th.z, g.z, m.z, v.z, lr[2], a);
+      adam_one(th.w, g.w, m.w, v.w, lr[3], a);
+      *reinterpret_cast<float4*>(s.m + i0) = m;
+      *reinterpret_cast<float4*>(s.v + i0) = v;
+      *reinterpret_cast<float4*>(s.th + i0) = th;
+    } else {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const unsigned i = i0 + c;
+        if (i < s.n) {
+          float th = s.th[i], m = s.m[i], v = s.v[i];
+          adam_one(th, s.g[i], m, v, lr[c], a);
+          s.m[i] = m;
+          s.v[i] = v;
+          s.th[i] = th;
+        }
+      }
+    }
   }
 }
 
@@ -80,17 +118,22 @@ extern "C" abcd_status abcd_adam_active(abcd_ctx* ctx, abcd_gaussians* theta,
   float* mm[5] = {m->means, m->log_scales, m->quats, m->opacity_logits, m->sh};
   float* vv[5] = {v->means, v->log_scales, v->quats, v->opacity_logits, v->sh};
   const long long len[5] = {3 * n, 3 * n, 4 * n, n, 3LL * D * n};
-  a.start[0] = 0;
+  long long groups = 0;
+  for (int k = 0; k < 5; ++k) groups += (len[k] + 3) / 4;
+  if (len[4] >= (1LL << 32) || groups >= (1LL << 32))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_adam_active: too many parameters");
+  a.gstart[0] = 0;
   for (int k = 0; k < 5; ++k) {
-    a.s[k] = Seg{th[k], gg[k], mm[k], vv[k], len[k], k == 4 ? 3 * D : 0,
-                 (float)(lr[k] / bc1), (float)((k == 4 ? lr[5] : lr[k]) / bc1)};
-    a.start[k + 1] = a.start[k] + len[k];
+    const bool vec = (((uintptr_t)th[k] | (uintptr_t)gg[k] | (uintptr_t)mm[k] | (uintptr_t)vv[k]) & 15) == 0;
+    a.s[k] = Seg{th[k], gg[k], mm[k], vv[k], (unsigned)len[k], k == 4 ? (unsigned)(3 * D) : 0u,
+                 (float)(lr[k] / bc1), (float)((k == 4 ? lr[5] : lr[k]) / bc1), vec ? 1 : 0};
+    a.gstart[k + 1] = a.gstart[k] + (unsigned)((len[k] + 3) / 4);
   }
   a.b1 = beta1;
   a.b2 = beta2;
   a.eps = eps;
   a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
-  const long long blocks = std::min<long long>((a.start[5] + 255) / 256, (long long)ctx->num_sms * 16);
+  const long long blocks = std::min<long long>((a.gstart[5] + 255) / 256, (long long)ctx->num_sms * 16);
   return check_launch(ctx, "adam_kernel",
                       launch_pdl(adam_kernel, dim3((unsigned)blocks), dim3(256), 0, ctx->stream, a));
 }

@@ -135,12 +135,51 @@ __device__ __forceinline__ void geometry(const Cam& cam, const Opts& op, const P
   G.det = (cx * cx + cy * cy + cz * cz) + op.dilation * (a0 + c0) + op.dilation * op.dilation;
 }
 
-__global__ void __launch_bounds__(256)
-project_fwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, float2* uv,
+// SH coefficients of a warp's 32 consecutive Gaussians form one contiguous block of 32 x 3D
+// floats ([n][D][3] layout); it goes through shared memory (row pitch 3D + 1, so a lane's row
+// reads are conflict-free) so that the global reads and writes are coalesced.
+template <int DEG>
+struct ShLayout {
+  static constexpr int D = (DEG + 1) * (DEG + 1);
+  static constexpr int N = 3 * D;        // floats per Gaussian
+  static constexpr int P = N + 1;        // shared-memory row pitch
+};
+
+template <int DEG>
+__device__ __forceinline__ void sh_to_shared(const float* sh, int n, int first, float* buf) {
+  constexpr int N = ShLayout<DEG>::N, P = ShLayout<DEG>::P;
+  const int lane = threadIdx.x & 31;
+  const int cnt = min(32, n - first);
+  const float* src = sh + (size_t)first * N;
+  for (int j = lane; j < cnt * N; j += 32) buf[(j / N) * P + (j % N)] = src[j];
+  __syncwarp();
+}
+
+template <int DEG>
+__device__ __forceinline__ void sh_from_shared(float* sh, int n, int first, const float* buf) {
+  constexpr int N = ShLayout<DEG>::N, P = ShLayout<DEG>::P;
+  const int lane = threadIdx.x & 31;
+  const int cnt = min(32, n - first);
+  float* dst = sh + (size_t)first * N;
+  __syncwarp();
+  for (int j = lane; j < cnt * N; j += 32) dst[j] = buf[(j / N) * P + (j % N)];
+}
+
+constexpr int kProjThreads = 128;
+
+template <int DEG>
+__global__ void __launch_bounds__(kProjThreads)
+project_fwd_kernel(Params p, int n, Cam cam, Opts op, SHConst K, float2* uv,
                    float4* conic_op, float* rgb, float* depth, int* radius,
                    unsigned* tiles_touched) {
   pdl_prologue();
+  constexpr int D = ShLayout<DEG>::D, P = ShLayout<DEG>::P;
+  __shared__ float s_sh[kProjThreads / 32][32 * P];
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31, first = i - lane;
+  if (first >= n) return;                                  // whole warp
+  float* buf = s_sh[threadIdx.x >> 5];
+  sh_to_shared<DEG>(p.sh, n, first, buf);
   if (i >= n) return;
   const float tz = view_depth(cam, p.means[3 * i], p.means[3 * i + 1], p.means[3 * i + 2]);
   depth[i] = tz;
@@ -177,11 +216,12 @@ project_fwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, float2
       const float dz = p.means[3 * i + 2] - cam.campos[2];
       const float il = 1.f / sqrtf(dx * dx + dy * dy + dz * dz);
       float Y[16];
-      sh_eval(K, deg, dx * il, dy * il, dz * il, Y, nullptr);
-      const int D = (deg + 1) * (deg + 1);
-      const float* sh = p.sh + (size_t)i * D * 3;
+      sh_eval(K, DEG, dx * il, dy * il, dz * il, Y, nullptr);
+      const float* sh = buf + lane * P;
+#pragma unroll
       for (int ch = 0; ch < 3; ++ch) {
         float acc = 0.5f;
+#pragma unroll
         for (int k = 0; k < D; ++k) acc += Y[k] * sh[3 * k + ch];
         col[ch] = fmaxf(acc, 0.f);
       }
@@ -204,25 +244,26 @@ struct Grads {
   float* sh;
 };
 
-__global__ void __launch_bounds__(128)
-project_bwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, const float* grad2d,
-                   Grads out) {
-  pdl_prologue();
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+template <int DEG>
+__device__ __forceinline__ void project_bwd_one(const Params& p, int n, int i, const Cam& cam,
+                                                const Opts& op, const SHConst& K,
+                                                const float* grad2d, const Grads& out,
+                                                float* shrow) {
+  constexpr int D = ShLayout<DEG>::D;
   if (i >= n) return;
-  const int D = (deg + 1) * (deg + 1);
   const float* g9 = grad2d + 9 * (size_t)i;
   float gin[9];
   bool any = false;
+#pragma unroll
   for (int k = 0; k < 9; ++k) { gin[k] = g9[k]; any |= gin[k] != 0.f; }
   const float mx = p.means[3 * i], my = p.means[3 * i + 1], mz = p.means[3 * i + 2];
   const float tz = view_depth(cam, mx, my, mz);
-  float* gsh = out.sh + (size_t)i * D * 3;
   if (!any || !(tz > op.near_z)) {   // no contribution: every gradient is 0
     for (int k = 0; k < 3; ++k) { out.means[3 * i + k] = 0.f; out.log_scales[3 * i + k] = 0.f; }
     for (int k = 0; k < 4; ++k) out.quats[4 * i + k] = 0.f;
     out.logits[i] = 0.f;
-    for (int k = 0; k < 3 * D; ++k) gsh[k] = 0.f;
+#pragma unroll
+    for (int k = 0; k < 3 * D; ++k) shrow[k] = 0.f;
     return;
   }
   Geo G;
@@ -238,16 +279,18 @@ project_bwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, const 
     const float il = 1.f / sqrtf(dx * dx + dy * dy + dz * dz);
     const float d[3] = {dx * il, dy * il, dz * il};
     float Y[16], dY[16][3];
-    sh_eval(K, deg, d[0], d[1], d[2], Y, dY);
-    const float* sh = p.sh + (size_t)i * D * 3;
+    sh_eval(K, DEG, d[0], d[1], d[2], Y, dY);
     float gdir[3] = {0.f, 0.f, 0.f};
+#pragma unroll
     for (int ch = 0; ch < 3; ++ch) {
       float raw = 0.5f;
-      for (int k = 0; k < D; ++k) raw += Y[k] * sh[3 * k + ch];
+#pragma unroll
+      for (int k = 0; k < D; ++k) raw += Y[k] * shrow[3 * k + ch];
       const float gc = raw < 0.f ? 0.f : gin[6 + ch];
+#pragma unroll
       for (int k = 0; k < D; ++k) {
-        gsh[3 * k + ch] = Y[k] * gc;
-        const float s = sh[3 * k + ch] * gc;
+        const float s = shrow[3 * k + ch] * gc;
+        shrow[3 * k + ch] = Y[k] * gc;             // the coefficient's gradient, in place
         gdir[0] += s * dY[k][0]; gdir[1] += s * dY[k][1]; gdir[2] += s * dY[k][2];
       }
     }
@@ -321,6 +364,23 @@ project_bwd_kernel(Params p, int n, int deg, Cam cam, Opts op, SHConst K, const 
     out.means[3 * i + k] = gmu[k] + cam.R[k] * gtx + cam.R[3 + k] * gty + cam.R[6 + k] * gtz;
 }
 
+template <int DEG>
+__global__ void __launch_bounds__(kProjThreads)
+project_bwd_kernel(Params p, int n, Cam cam, Opts op, SHConst K, const float* grad2d,
+                   Grads out) {
+  pdl_prologue();
+  constexpr int P = ShLayout<DEG>::P;
+  __shared__ float s_sh[kProjThreads / 32][32 * P];
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31, first = i - lane;
+  if (first >= n) return;                                  // whole warp
+  float* buf = s_sh[threadIdx.x >> 5];
+  sh_to_shared<DEG>(p.sh, n, first, buf);
+  // every lane's sh row is replaced by its gradient in place, then written out together
+  project_bwd_one<DEG>(p, n, i, cam, op, K, grad2d, out, buf + lane * P);
+  sh_from_shared<DEG>(out.sh, n, first, buf);
+}
+
 Params params_of(const abcd_gaussians* g) {
   return Params{g->means, g->log_scales, g->quats, g->opacity_logits, g->sh};
 }
@@ -353,13 +413,15 @@ extern "C" abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta,
   if (((uintptr_t)out->uv & 7) || ((uintptr_t)out->conic_opacity & 15))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_project: uv must be 8-byte and conic_opacity 16-byte aligned");
   if (theta->n == 0) return ABCD_OK;
-  const int threads = 256, blocks = (theta->n + threads - 1) / threads;
+  const int blocks = (theta->n + kProjThreads - 1) / kProjThreads;
+  void (*kern)(Params, int, Cam, Opts, SHConst, float2*, float4*, float*, float*, int*, unsigned*) =
+      theta->sh_degree == 0 ? project_fwd_kernel<0> : theta->sh_degree == 1 ? project_fwd_kernel<1>
+      : theta->sh_degree == 2 ? project_fwd_kernel<2> : project_fwd_kernel<3>;
   return check_launch(ctx, "project_fwd_kernel",
-                      launch_pdl(project_fwd_kernel, dim3(blocks), dim3(threads), 0, ctx->stream,
-                                 params_of(theta), theta->n, theta->sh_degree, make_cam(cam, opts),
-                                 make_opts(opts), ctx->sh, (float2*)out->uv,
-                                 (float4*)out->conic_opacity, out->rgb, out->depth, out->radius,
-                                 out->tiles_touched));
+                      launch_pdl(kern, dim3(blocks), dim3(kProjThreads), 0, ctx->stream,
+                                 params_of(theta), theta->n, make_cam(cam, opts), make_opts(opts),
+                                 ctx->sh, (float2*)out->uv, (float4*)out->conic_opacity, out->rgb,
+                                 out->depth, out->radius, out->tiles_touched));
 }
 
 extern "C" abcd_status abcd_project_backward(abcd_ctx* ctx, const abcd_gaussians* theta,
@@ -372,11 +434,14 @@ extern "C" abcd_status abcd_project_backward(abcd_ctx* ctx, const abcd_gaussians
   if (!camera_ok(cam)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_project_backward: bad camera");
   if (theta->n > 0 && !grad2d) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_project_backward: null grad2d");
   if (theta->n == 0) return ABCD_OK;
-  const int threads = 128, blocks = (theta->n + threads - 1) / threads;
+  const int blocks = (theta->n + kProjThreads - 1) / kProjThreads;
+  void (*kern)(Params, int, Cam, Opts, SHConst, const float*, Grads) =
+      theta->sh_degree == 0 ? project_bwd_kernel<0> : theta->sh_degree == 1 ? project_bwd_kernel<1>
+      : theta->sh_degree == 2 ? project_bwd_kernel<2> : project_bwd_kernel<3>;
   return check_launch(ctx, "project_bwd_kernel",
-                      launch_pdl(project_bwd_kernel, dim3(blocks), dim3(threads), 0, ctx->stream,
-                                 params_of(theta), theta->n, theta->sh_degree, make_cam(cam, opts),
-                                 make_opts(opts), ctx->sh, grad2d,
+                      launch_pdl(kern, dim3(blocks), dim3(kProjThreads), 0, ctx->stream,
+                                 params_of(theta), theta->n, make_cam(cam, opts), make_opts(opts),
+                                 ctx->sh, grad2d,
                                  Grads{grads->means, grads->log_scales, grads->quats,
                                        grads->opacity_logits, grads->sh}));
 }
