@@ -108,6 +108,8 @@ inline long long max_order_tiles(long long max_pixels) { return max_pixels / 256
 struct abcd_ctx {
   int device = 0;
   cudaStream_t stream = nullptr;
+  cudaStream_t side = nullptr;          // forked work inside one call, joined before it returns
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   int num_sms = 0;
   int radix_blocks = 0;
   char* ws_base = nullptr;

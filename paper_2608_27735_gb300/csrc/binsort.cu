@@ -667,12 +667,13 @@ abcd_status emit_smem_attr(abcd_ctx* ctx) {
 // LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi); returns the buffer holding
 // the result, or writes the bits id_mask of the sorted items to ids_out on the last pass.
 template <typename T>
-abcd_status launch_scatter(abcd_ctx* ctx, int bits, int G, const T* src, T* dst, unsigned* ids,
-                           unsigned id_mask, long long n_static, const long long* n_dev,
-                           long long cap, int shift, const unsigned* totals) {
+abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, int G, const T* src, T* dst,
+                           unsigned* ids, unsigned id_mask, long long n_static,
+                           const long long* n_dev, long long cap, int shift,
+                           const unsigned* totals) {
 #define ABCD_SCATTER(B)                                                                     \
   case B:                                                                                   \
-    e = launch_pdl(radix_scatter_kernel<T, B>, dim3(G), dim3(kRadixBins), 0, ctx->stream,     \
+    e = launch_pdl(radix_scatter_kernel<T, B>, dim3(G), dim3(kRadixBins), 0, st,              \
                    src, dst, ids, id_mask, n_static, n_dev, cap, shift,                     \
                    (const unsigned*)ctx->ws.hist, totals, G);                               \
     break;
@@ -690,9 +691,9 @@ abcd_status launch_scatter(abcd_ctx* ctx, int bits, int G, const T* src, T* dst,
 // the buffer holding the result, or writes the bits id_mask of the sorted items to ids_out on
 // the last pass.
 template <typename T>
-abcd_status radix_sort(abcd_ctx* ctx, T* a, T* b, long long n_static, const long long* n_dev,
-                       long long cap, int bit_lo, int bit_hi, int G, T** result,
-                       unsigned* ids_out, unsigned id_mask) {
+abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_static,
+                       const long long* n_dev, long long cap, int bit_lo, int bit_hi, int G,
+                       T** result, unsigned* ids_out, unsigned id_mask) {
   unsigned* totals = ctx->ws.hist + kRadixBins * G;
   T* src = a;
   T* dst = b;
@@ -704,14 +705,14 @@ abcd_status radix_sort(abcd_ctx* ctx, T* a, T* b, long long n_static, const long
     const bool last = shift + width >= bit_hi;
     abcd_status s = check_launch(
         ctx, "radix_hist_kernel",
-        launch_pdl(radix_hist_kernel<T>, dim3(G), dim3(256), 0, ctx->stream, (const T*)src, n_static,
+        launch_pdl(radix_hist_kernel<T>, dim3(G), dim3(256), 0, st, (const T*)src, n_static,
                    n_dev, cap, shift, (1u << bits) - 1u, ctx->ws.hist, G));
     if (s) return s;
     if ((s = check_launch(ctx, "radix_rowscan_kernel",
                           launch_pdl(radix_rowscan_kernel, dim3(kRadixBins), dim3(((G + 31) / 32) * 32),
-                                     0, ctx->stream, ctx->ws.hist, G, totals))))
+                                     0, st, ctx->ws.hist, G, totals))))
       return s;
-    if ((s = launch_scatter<T>(ctx, bits, G, src, dst, last ? ids_out : nullptr, id_mask, n_static,
+    if ((s = launch_scatter<T>(ctx, st, bits, G, src, dst, last ? ids_out : nullptr, id_mask, n_static,
                                n_dev, cap, shift, totals)))
       return s;
     T* t = src; src = dst; dst = t;
@@ -763,6 +764,17 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
                                    ctx->ws.rects))))
     return s;
+  // the depth sort only needs the keys: it runs on the side stream while tile_rows runs here
+  e = cudaEventRecord(ctx->ev_fork, ctx->stream);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->side, ctx->ev_fork, 0);
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort fork: %s", cudaGetErrorString(e));
+  u64* by_depth = nullptr;
+  const int Gd = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));   // depth sort
+  if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64,
+                           Gd, &by_depth, nullptr, 0xffffffffu)))
+    return s;
+  e = cudaEventRecord(ctx->ev_join, ctx->side);
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
   {
     const int cells = (tiles_x + 1) * (tiles_y + 1);
     const size_t smem = cells <= kSmemDiffCells ? sizeof(int) * cells : 0;
@@ -777,11 +789,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                      n, tiles_x, tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff))))
       return s;
   }
-  u64* by_depth = nullptr;
-  const int Gd = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));   // depth sort
-  if ((s = radix_sort<u64>(ctx, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64, Gd,
-                           &by_depth, nullptr, 0xffffffffu)))
-    return s;
+  e = cudaStreamWaitEvent(ctx->stream, ctx->ev_join, 0);
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
   const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
   if ((s = check_launch(ctx, "count_kernel",
                         launch_pdl(count_kernel, dim3(Ge), dim3(256), 0, ctx->stream,
@@ -836,8 +845,9 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                      (const long long*)out->count, cap, tiles_x, alpha_min, id_bits,
                                      pairs, Ge))))
       return s;
-    return radix_sort<unsigned>(ctx, pairs, pairs_b, 0, out->count, cap, id_bits, id_bits + tile_bits,
-                                kMaxRadixBlocks, nullptr, out->ids, (1u << id_bits) - 1u);
+    return radix_sort<unsigned>(ctx, ctx->stream, pairs, pairs_b, 0, out->count, cap, id_bits,
+                                id_bits + tile_bits, kMaxRadixBlocks, nullptr, out->ids,
+                                (1u << id_bits) - 1u);
   }
   if ((s = emit_smem_attr<u64>(ctx))) return s;
   if ((s = check_launch(ctx, "emit_kernel",
@@ -849,6 +859,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    (const long long*)out->count, cap, tiles_x, alpha_min, 32,
                                    ctx->ws.pairs[0], Ge))))
     return s;
-  return radix_sort<u64>(ctx, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap, 32,
-                         32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu);
+  return radix_sort<u64>(ctx, ctx->stream, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap,
+                         32, 32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu);
 }

@@ -103,9 +103,13 @@ abcd_status abcd_create(abcd_ctx** out, int device, void* stream) {
   cudaGetDevice(&prev);
   cudaError_t e = cudaSetDevice(device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device);
+  // side stream for work that runs beside the main stream inside one call (fork / join)
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&ctx->side, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming);
   cudaSetDevice(prev);
   if (e != cudaSuccess) {
-    delete ctx;
+    abcd_destroy(ctx);
     return ABCD_ERR_CUDA;
   }
   ctx->radix_blocks = std::min(kMaxRadixBlocks, 2 * ctx->num_sms);
@@ -115,6 +119,10 @@ abcd_status abcd_create(abcd_ctx** out, int device, void* stream) {
 }
 
 abcd_status abcd_destroy(abcd_ctx* ctx) {
+  if (!ctx) return ABCD_OK;
+  if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
+  if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
+  if (ctx->side) cudaStreamDestroy(ctx->side);
   delete ctx;
   return ABCD_OK;
 }
