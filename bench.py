@@ -38,7 +38,7 @@ METRIC = "ABCD active-block steps/s @1237x822, 100k Gaussians; % of roofline"
 UNIT = "steps/s"
 ACTIVE_CELL = (1, 1, 0)
 LR = [1.6e-4 * 15.0, 5e-3, 1e-3, 0.025, 2.5e-3, 2.5e-3 / 20]   # means lr scaled by the scene extent
-REFRESH_STREAMS = 4         # concurrent cache-refresh pipelines (contexts with their own streams)
+REFRESH_STREAMS = 8         # concurrent cache-refresh pipelines (contexts with their own streams)
 FWD_FLOP_PER_PAIR = 25      # per (pixel, list entry) walked: offset, sigma, alpha, tests, blend
 BWD_FLOP_PER_PAIR = 68      # recompute + d alpha + colour, opacity, mean and conic terms
 LOSS_FLOP_PER_PX = 1000     # five 11-tap windows twice (separable), SSIM terms, 3 channels

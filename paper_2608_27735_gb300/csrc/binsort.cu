@@ -412,8 +412,7 @@ scan_blocks_kernel(unsigned long long* block_sums, int G, long long* count, long
 // ---- tile ranges from the per-row difference array: prefix sums along each row -> per-tile
 // counts -> exclusive scan (one block).  Empty ranges when K overflowed the capacity.
 __global__ void __launch_bounds__(1024)
-ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* count, long long cap,
-                        unsigned* ranges) {
+ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, long long cap, unsigned* ranges) {
   pdl_prologue();
   const int W1 = tiles_x + 1;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
@@ -431,13 +430,14 @@ ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, const long long* co
     }
   }
   __syncthreads();
-  const bool ok = *count <= cap;
   const int nt = tiles_x * tiles_y;
   const int per = (nt + blockDim.x - 1) / blockDim.x;
   const int lo = min(nt, (int)threadIdx.x * per), hi = min(nt, lo + per);
   unsigned long long s = 0;
   for (int t = lo; t < hi; ++t) s += (unsigned)diff[(t / tiles_x) * W1 + (t % tiles_x)];
-  unsigned long long run = block_exclusive_scan(s, nullptr);
+  unsigned long long total = 0;
+  unsigned long long run = block_exclusive_scan(s, &total);
+  const bool ok = (long long)total <= cap;          // K: the same total the count scan finds
   for (int t = lo; t < hi; ++t) {
     const unsigned c = (unsigned)diff[(t / tiles_x) * W1 + (t % tiles_x)];
     ranges[2 * t] = ok ? (unsigned)run : 0u;
@@ -460,8 +460,8 @@ __device__ __forceinline__ unsigned count_bucket(unsigned c) {
 }
 
 __global__ void __launch_bounds__(1024)
-ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, const long long* count,
-                    long long cap, unsigned* ranges, unsigned* tile_order) {
+ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, long long cap, unsigned* ranges,
+                    unsigned* tile_order) {
   pdl_prologue();
   extern __shared__ int sd[];              // [(tiles_x + 1) (tiles_y + 1)] cells, then [nt] keys
   __shared__ unsigned hist[kOrderBuckets];
@@ -499,12 +499,13 @@ ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, const long long* 
     }
   }
   __syncthreads();
-  const bool ok = *count <= cap;
   const int per = (nt + blockDim.x - 1) / blockDim.x;
   const int lo = min(nt, (int)threadIdx.x * per), hi = min(nt, lo + per);
   unsigned long long s = 0;
   for (int t = lo; t < hi; ++t) s += (unsigned)sd[(t / tiles_x) * W1 + (t % tiles_x)];
-  unsigned long long run = block_exclusive_scan(s, nullptr);
+  unsigned long long total = 0;
+  unsigned long long run = block_exclusive_scan(s, &total);
+  const bool ok = (long long)total <= cap;          // K: the same total the count scan finds
   for (int t = lo; t < hi; ++t) {
     const unsigned c = (unsigned)sd[(t / tiles_x) * W1 + (t % tiles_x)];
     ranges[2 * t] = ok ? (unsigned)run : 0u;
@@ -764,15 +765,18 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
                                    ctx->ws.rects))))
     return s;
-  // the depth sort only needs the keys: it runs on the side stream while tile_rows runs here
+  // the depth sort only needs the keys: it runs on the side stream while the tile rows and
+  // ranges are made here
   e = cudaEventRecord(ctx->ev_fork, ctx->stream);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->side, ctx->ev_fork, 0);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort fork: %s", cudaGetErrorString(e));
   u64* by_depth = nullptr;
-  const int Gd = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));   // depth sort
-  if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32, 64,
-                           Gd, &by_depth, nullptr, 0xffffffffu)))
-    return s;
+  {
+    const int G = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));
+    if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32,
+                             64, G, &by_depth, nullptr, 0xffffffffu)))
+      return s;
+  }
   e = cudaEventRecord(ctx->ev_join, ctx->side);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
   {
@@ -789,6 +793,29 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                      n, tiles_x, tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff))))
       return s;
   }
+  {
+    const int cells = (tiles_x + 1) * (tiles_y + 1);
+    ctx->order_ranges = nullptr;
+    if (cells <= kSmemDiffCells && n_tiles <= ctx->ws.max_tiles) {
+      const size_t smem = sizeof(int) * cells + (size_t)n_tiles;
+      if (smem > 48 * 1024) {
+        const cudaError_t e2 = cudaFuncSetAttribute(ranges_order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "ranges smem: %s", cudaGetErrorString(e2));
+      }
+      if ((s = check_launch(ctx, "ranges_order_kernel",
+                            launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->stream,
+                                       (const int*)ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges,
+                                       ctx->ws.tile_order))))
+        return s;
+      ctx->order_ranges = out->ranges;           // the order belongs to these ranges
+      ctx->order_tiles = n_tiles;
+    } else {
+      if ((s = check_launch(ctx, "ranges_from_diff_kernel",
+                            launch_pdl(ranges_from_diff_kernel, dim3(1), dim3(1024), 0, ctx->stream,
+                                       ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges))))
+        return s;
+    }
+  }
   e = cudaStreamWaitEvent(ctx->stream, ctx->ev_join, 0);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
   const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
@@ -801,31 +828,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                         launch_pdl(scan_blocks_kernel, dim3(1), dim3(1024), 0, ctx->stream,
                                    ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status))))
     return s;
-  {
-    const int cells = (tiles_x + 1) * (tiles_y + 1);
-    ctx->order_ranges = nullptr;
-    if (cells <= kSmemDiffCells && n_tiles <= ctx->ws.max_tiles) {
-      const size_t smem = sizeof(int) * cells + (size_t)n_tiles;
-      if (smem > 48 * 1024) {
-        const cudaError_t e2 = cudaFuncSetAttribute(ranges_order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "ranges smem: %s", cudaGetErrorString(e2));
-      }
-      if ((s = check_launch(ctx, "ranges_order_kernel",
-                            launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->stream,
-                                       (const int*)ctx->ws.diff, tiles_x, tiles_y,
-                                       (const long long*)out->count, cap, out->ranges,
-                                       ctx->ws.tile_order))))
-        return s;
-      ctx->order_ranges = out->ranges;           // the order belongs to these ranges
-      ctx->order_tiles = n_tiles;
-    } else {
-      if ((s = check_launch(ctx, "ranges_from_diff_kernel",
-                            launch_pdl(ranges_from_diff_kernel, dim3(1), dim3(1024), 0, ctx->stream,
-                                       ctx->ws.diff, tiles_x, tiles_y, (const long long*)out->count,
-                                       cap, out->ranges))))
-        return s;
-    }
-  }
   int tile_bits = 1;
   while ((1LL << tile_bits) < n_tiles) ++tile_bits;
   int id_bits = 1;
