@@ -10,20 +10,25 @@
 //
 // How (GB300 design, different from sorting 64-bit (tile | depth) keys):
 //   1. per Gaussian: its tile rectangle (kept in the workspace) and a sort key (fp32 depth
-//      bits, all ones when culled); then, one warp per Gaussian, one lane per tile row: the
-//      contiguous run of kept tiles in that row (the kept set is convex), the Gaussian's pair
-//      count, and +-1 at the run's ends in a per-row difference array over the tile grid;
-//   2. stable LSD radix sort of the n Gaussians by the 32 depth bits;
-//   3. exclusive scan of the pair counts in that order: K = total pairs; the row prefix sums
-//      of the difference array give every tile's pair count, hence its range, and the tiles
-//      sorted by decreasing count (the order the render kernels launch them in);
-//   4. emission of (tile << 32 | id) items in depth order (the runs are recomputed with the
-//      same round-to-nearest arithmetic, so they match step 1 bit for bit);
-//   5. stable LSD radix sort of the K items on the tile bits only (ceil(log2 n_tiles) <= 16
-//      bits, 8 per pass), which keeps depth order inside each tile; the last pass writes ids.
+//      bits, all ones when culled); then, one thread per Gaussian: the contiguous run of kept
+//      tiles in each of its tile rows (the kept set is convex), its pair count, and +-1 at the
+//      run's ends in a per-row difference array over the tile grid (block-local first);
+//   2. stable LSD radix sort of the n Gaussians by the 32 depth bits, on the context's side
+//      stream, while the main stream makes the row runs and then, in one block, the tile
+//      ranges (row prefix sums of the difference array, an exclusive scan, K) and the tiles
+//      ordered by decreasing pair count (the order the render kernels launch them in);
+//   3. exclusive scan of the pair counts in depth order: every Gaussian's output offset;
+//   4. emission of (tile << id_bits | id) items in depth order, 32-bit when tile and id bits
+//      fit (else 64-bit); the runs are recomputed with the same round-to-nearest arithmetic,
+//      so they match step 1 bit for bit; each warp's contiguous output is built in shared
+//      memory and written out coalesced;
+//   5. stable LSD radix sort of the K items on the tile bits only, in passes of equal width,
+//      which keeps depth order inside each tile; the last pass writes ids.
 // Radix passes are reduce-then-scan (per-block digit counts, per-digit row scans, stable
-// scatter ranked with ballots): no inter-block waits, so nothing can spin.  Counts that live on the device (K)
-// are read by the kernels themselves; grids are fixed, so the step has no host sync.
+// scatter): no inter-block waits, so nothing can spin.  Lanes of equal digit are ranked with
+// ballots on the low, scattered digits and with __match_any_sync on the high, grouped ones.
+// Counts that live on the device (K) are read by the kernels themselves; grids are fixed, so
+// the step has no host sync.
 #include <algorithm>
 
 #include "abcd_internal.cuh"
@@ -300,7 +305,17 @@ __global__ void __launch_bounds__(1024) radix_rowscan_kernel(unsigned* hist, int
 // ---- radix pass, step 3: stable scatter of BITS-bit digits.  Each warp owns a contiguous
 // slice of the block's range; lanes of equal digit are ranked with match_digit, once per item
 // (the masks are kept for the scatter when the slice is one round of loads).
-template <typename T, int BITS>
+// Lanes of the warp holding the same digit: one ballot per bit (a cost independent of how many
+// distinct digits the warp holds: the right choice for the low, scattered digits) or
+// __match_any_sync (fast when a warp holds few distinct digits: the high digits of depth keys and
+// of tile indices, whose items arrive nearly grouped).
+template <int BITS, bool MATCH>
+__device__ __forceinline__ unsigned rank_peers(unsigned d, bool valid) {
+  if (MATCH) return __match_any_sync(0xffffffffu, d);
+  return match_digit<BITS>(d, __ballot_sync(0xffffffffu, valid));
+}
+
+template <typename T, int BITS, bool MATCH>
 __global__ void __launch_bounds__(256)
 radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
                      const long long* n_dev, long long cap, int shift, const unsigned* hist,
@@ -339,7 +354,7 @@ radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, l
     for (int j = 0; j < U; ++j) {
       if (b0 + 32 * j >= wh) break;                // warp-uniform
       const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, wh, shift, MASK);
-      const unsigned peers = match_digit<BITS>(d, __ballot_sync(0xffffffffu, d < 0x100u));
+      const unsigned peers = rank_peers<BITS, MATCH>(d, d < 0x100u);
       pm[j] = peers;
       if (d < 0x100u && (peers & lt) == 0) cnt[w][d] += __popc(peers);
       __syncwarp();
@@ -360,7 +375,7 @@ radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, l
       const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, wh, shift, MASK);
       const bool valid = d < 0x100u;
       const unsigned peers =
-          rounds > 1 ? match_digit<BITS>(d, __ballot_sync(0xffffffffu, valid)) : pm[j];
+          rounds > 1 ? rank_peers<BITS, MATCH>(d, valid) : pm[j];
       unsigned pos = 0;
       if (valid) pos = cnt[w][d] + __popc(peers & lt);
       __syncwarp();
@@ -665,18 +680,20 @@ abcd_status emit_smem_attr(abcd_ctx* ctx) {
   return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "emit smem: %s", cudaGetErrorString(e));
 }
 
-// LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi); returns the buffer holding
-// the result, or writes the bits id_mask of the sorted items to ids_out on the last pass.
+// Launches the scatter of one radix pass for a digit of `bits` bits (4..8).
 template <typename T>
-abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, int G, const T* src, T* dst,
-                           unsigned* ids, unsigned id_mask, long long n_static,
-                           const long long* n_dev, long long cap, int shift,
+abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, bool match, int G,
+                           const T* src, T* dst, unsigned* ids, unsigned id_mask,
+                           long long n_static, const long long* n_dev, long long cap, int shift,
                            const unsigned* totals) {
 #define ABCD_SCATTER(B)                                                                     \
   case B:                                                                                   \
-    e = launch_pdl(radix_scatter_kernel<T, B>, dim3(G), dim3(kRadixBins), 0, st,              \
-                   src, dst, ids, id_mask, n_static, n_dev, cap, shift,                     \
-                   (const unsigned*)ctx->ws.hist, totals, G);                               \
+    e = match ? launch_pdl(radix_scatter_kernel<T, B, true>, dim3(G), dim3(kRadixBins), 0, st, \
+                           src, dst, ids, id_mask, n_static, n_dev, cap, shift,             \
+                           (const unsigned*)ctx->ws.hist, totals, G)                        \
+              : launch_pdl(radix_scatter_kernel<T, B, false>, dim3(G), dim3(kRadixBins), 0, st, \
+                           src, dst, ids, id_mask, n_static, n_dev, cap, shift,             \
+                           (const unsigned*)ctx->ws.hist, totals, G);                       \
     break;
   cudaError_t e = cudaSuccess;
   switch (bits) {
@@ -687,6 +704,11 @@ abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, int G, cons
   return check_launch(ctx, "radix_scatter_kernel", e);
 }
 
+// First pass ranked with __match_any_sync (earlier passes use ballots): the depth keys' two
+// high bytes and the tile index's high bits come nearly grouped.
+constexpr int kDepthMatchFrom = 2;
+constexpr int kTileMatchFrom = 1;
+
 // LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi), in the fewest passes of at
 // most 8 bits, of equal width (fewer bits per pass: fewer ballots per ranked item); returns
 // the buffer holding the result, or writes the bits id_mask of the sorted items to ids_out on
@@ -694,14 +716,14 @@ abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, int G, cons
 template <typename T>
 abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_static,
                        const long long* n_dev, long long cap, int bit_lo, int bit_hi, int G,
-                       T** result, unsigned* ids_out, unsigned id_mask) {
+                       T** result, unsigned* ids_out, unsigned id_mask, int match_from) {
   unsigned* totals = ctx->ws.hist + kRadixBins * G;
   T* src = a;
   T* dst = b;
   const int nbits = bit_hi - bit_lo;
   const int passes = (nbits + kRadixBits - 1) / kRadixBits;
   const int width = std::max(4, (nbits + passes - 1) / passes);
-  for (int shift = bit_lo; shift < bit_hi; shift += width) {
+  for (int shift = bit_lo, pass = 0; shift < bit_hi; shift += width, ++pass) {
     const int bits = std::min(width, bit_hi - shift) < 4 ? 4 : std::min(width, bit_hi - shift);
     const bool last = shift + width >= bit_hi;
     abcd_status s = check_launch(
@@ -713,8 +735,9 @@ abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_s
                           launch_pdl(radix_rowscan_kernel, dim3(kRadixBins), dim3(((G + 31) / 32) * 32),
                                      0, st, ctx->ws.hist, G, totals))))
       return s;
-    if ((s = launch_scatter<T>(ctx, st, bits, G, src, dst, last ? ids_out : nullptr, id_mask, n_static,
-                               n_dev, cap, shift, totals)))
+    if ((s = launch_scatter<T>(ctx, st, bits, pass >= match_from, G, src, dst,
+                               last ? ids_out : nullptr, id_mask, n_static, n_dev, cap, shift,
+                               totals)))
       return s;
     T* t = src; src = dst; dst = t;
   }
@@ -774,7 +797,7 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   {
     const int G = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));
     if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32,
-                             64, G, &by_depth, nullptr, 0xffffffffu)))
+                             64, G, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom)))
       return s;
   }
   e = cudaEventRecord(ctx->ev_join, ctx->side);
@@ -849,7 +872,7 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       return s;
     return radix_sort<unsigned>(ctx, ctx->stream, pairs, pairs_b, 0, out->count, cap, id_bits,
                                 id_bits + tile_bits, kMaxRadixBlocks, nullptr, out->ids,
-                                (1u << id_bits) - 1u);
+                                (1u << id_bits) - 1u, kTileMatchFrom);
   }
   if ((s = emit_smem_attr<u64>(ctx))) return s;
   if ((s = check_launch(ctx, "emit_kernel",
@@ -862,5 +885,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    ctx->ws.pairs[0], Ge))))
     return s;
   return radix_sort<u64>(ctx, ctx->stream, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap,
-                         32, 32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu);
+                         32, 32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu,
+                         kTileMatchFrom);
 }
