@@ -352,32 +352,37 @@ struct BwdArgs {
   const unsigned* tile_order;   // tiles, longest list first (nullptr: launch order)
 };
 
-// Backward state of one pixel.
+// Backward state of one pixel.  With G = dL/dA.rgb and G_a = dL/dA.a, the derivative of the
+// loss w.r.t. an entry's alpha is
+//   sum_ch G_ch (T col_ch - (A_ch - C_ch) / (1 - alpha)) + G_a T_final / (1 - alpha)
+//   = T (G . col) - (K - G . C) / (1 - alpha),   K = G . A - G_a T_final,
+// C the colour accumulated up to and including the entry: only the scalar G . C is replayed.
 struct PixB {
-  float T, c0, c1, c2;          // transmittance and colour replayed up to the current entry
-  float A0, A1, A2, Tf;         // the forward's final active colour and transmittance
-  float Gr, Gg, Gb, Ga;         // dL/dA.rgb and dL/dA.a
+  float T, Gc;                  // transmittance and G . C replayed up to the current entry
+  float Gr, Gg, Gb, K;          // dL/dA.rgb; G . A - G_a T_final
   unsigned last;                // replay only list positions below this
 };
 
 __device__ __forceinline__ void load_pixel_grad(const BwdArgs& a, long long p, int n, PixB& q) {
   q.last = min(a.n_last[p], (unsigned)n);
   const float4 at = a.state_at[p];
-  q.A0 = at.x; q.A1 = at.y; q.A2 = at.z; q.Tf = at.w;
   const float g0 = a.dl_dout[3 * p], g1 = a.dl_dout[3 * p + 1], g2 = a.dl_dout[3 * p + 2];
   const float4 Fv = a.F ? load_px(a.F, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
   const float4 Bv = a.B ? load_px(a.B, a.fb_dtype, p) : make_float4(0.f, 0.f, 0.f, 0.f);
   const float kf = 1.f - Fv.w;
   q.Gr = kf * g0; q.Gg = kf * g1; q.Gb = kf * g2;
   // d final / d A.a = -(1 - F.a) (B.rgb + (1 - B.a) bg)
-  q.Ga = -kf * (g0 * (Bv.x + (1.f - Bv.w) * a.bg[0]) + g1 * (Bv.y + (1.f - Bv.w) * a.bg[1]) +
-                g2 * (Bv.z + (1.f - Bv.w) * a.bg[2]));
+  const float Ga = -kf * (g0 * (Bv.x + (1.f - Bv.w) * a.bg[0]) + g1 * (Bv.y + (1.f - Bv.w) * a.bg[1]) +
+                          g2 * (Bv.z + (1.f - Bv.w) * a.bg[2]));
+  q.K = q.Gr * at.x + q.Gg * at.y + q.Gb * at.z - Ga * at.w;
 }
 
 // Backward of one pixel for one list entry (selects, no branches): when the entry contributed
 // to the pixel (live: a position below the pixel's last contributor; sigma >= 0; alpha >=
-// alpha_min) adds d(u, v, a, b, c, opacity, r, g, b) into v and advances the replayed
-// transmittance and colour exactly as the forward did.  Returns whether it contributed.
+// alpha_min) adds to v the opacity and colour gradients (v[5..8]) and the moments of d =
+// pixel - uv weighted by dL/dsigma, (sum w dx, w dy, w dx^2, w dx dy, w dy^2) in v[0..4] (the
+// conic and mean gradients follow from them once per entry), and advances the replayed
+// transmittance exactly as the forward did.  Returns whether the entry contributed.
 __device__ __forceinline__ bool pixel_backward(PixB& p, float4 s, float4 col, float sg, float dx,
                                                float dy, bool live, const Opts& op, float* v) {
   const float G = ex2_approx(-sg);
@@ -385,48 +390,47 @@ __device__ __forceinline__ bool pixel_backward(PixB& p, float4 s, float4 col, fl
   const float alpha = fminf(op.alpha_max, raw);
   const bool ok = live && sg >= 0.f && alpha >= op.alpha_min;
   const float w = __fmul_rn(alpha, p.T);
-  const float c0 = __fmaf_rn(w, col.x, p.c0);
-  const float c1 = __fmaf_rn(w, col.y, p.c1);
-  const float c2 = __fmaf_rn(w, col.z, p.c2);
+  const float gcol = p.Gr * col.x + p.Gg * col.y + p.Gb * col.z;
+  const float gc = fmaf(w, gcol, p.Gc);               // G . C including this entry
   const float ioma = __fdividef(1.f, 1.f - alpha);   // gradient scale only
-  // colour accumulated behind this Gaussian = A - (sum up to and including it)
-  const float dalpha = p.Gr * (p.T * col.x - (p.A0 - c0) * ioma) +
-                       p.Gg * (p.T * col.y - (p.A1 - c1) * ioma) +
-                       p.Gb * (p.T * col.z - (p.A2 - c2) * ioma) + p.Ga * p.Tf * ioma;
+  const float dalpha = p.T * gcol - (p.K - gc) * ioma;
   const bool grad_a = ok && raw <= op.alpha_max;      // derivative of min() is 0 once clamped
   const float wk = ok ? w : 0.f;
   const float dop = grad_a ? dalpha * G : 0.f;        // d alpha / d opacity = exp(-sigma)
   const float dsig = grad_a ? -dalpha * raw : 0.f;    // d alpha / d sigma = -alpha
-  v[6] += p.Gr * wk; v[7] += p.Gg * wk; v[8] += p.Gb * wk;
+  v[6] = fmaf(p.Gr, wk, v[6]); v[7] = fmaf(p.Gg, wk, v[7]); v[8] = fmaf(p.Gb, wk, v[8]);
   v[5] += dop;
-  const float ca = 2.f * kLn2 * s.x, cb = kLn2 * s.y, cc = 2.f * kLn2 * s.z;
-  v[0] -= dsig * (ca * dx + cb * dy);                 // d = pixel - uv
-  v[1] -= dsig * (cb * dx + cc * dy);
-  v[2] += 0.5f * dsig * dx * dx;
-  v[3] += dsig * dx * dy;
-  v[4] += 0.5f * dsig * dy * dy;
-  p.c0 = ok ? c0 : p.c0;
-  p.c1 = ok ? c1 : p.c1;
-  p.c2 = ok ? c2 : p.c2;
+  const float t = dsig * dx, u = dsig * dy;
+  v[0] += t;
+  v[1] += u;
+  v[2] = fmaf(t, dx, v[2]);
+  v[3] = fmaf(t, dy, v[3]);
+  v[4] = fmaf(u, dy, v[4]);
+  p.Gc = ok ? gc : p.Gc;
   p.T = ok ? __fmul_rn(p.T, __fsub_rn(1.f, alpha)) : p.T;
   return ok;
 }
 
-// Warp transpose reduction of 32 per-lane values: at each level a lane keeps half of its
-// values and adds the partner's matching half (31 shuffles in 5 dependent levels); lane l
-// returns the warp-wide sum of x[l].
-__device__ __forceinline__ float warp_sum32(float (&x)[32], int lane) {
+// Warp sum of 27 per-lane values through shared memory: each lane writes its row, lane l < 27
+// reads column l (32 values, 8 float4 loads; pitch 36 keeps stores and loads conflict-free)
+// and returns its sum.
+constexpr int kRedPitch = 36;
+
+__device__ __forceinline__ float warp_sum27(const float (&x)[27], float* red, int lane) {
 #pragma unroll
-  for (int w = 16; w >= 1; w >>= 1) {
-    const bool up = (lane & w) != 0;
+  for (int k = 0; k < 27; ++k) red[k * kRedPitch + lane] = x[k];
+  __syncwarp();
+  float r = 0.f;
+  if (lane < 27) {
+    const float4* col = reinterpret_cast<const float4*>(red + lane * kRedPitch);
 #pragma unroll
-    for (int k = 0; k < w; ++k) {
-      const float send = up ? x[k] : x[k + w];
-      const float keep = up ? x[k + w] : x[k];
-      x[k] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+    for (int q = 0; q < 8; ++q) {
+      const float4 a = col[q];
+      r += (a.x + a.y) + (a.z + a.w);
     }
   }
-  return x[0];
+  __syncwarp();
+  return r;
 }
 
 __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
@@ -435,6 +439,7 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
   __shared__ float4 s_co[kBatch + 2];
   __shared__ float4 s_rgb[kBatch + 2];
   __shared__ unsigned s_id[kBatch + 2];
+  __shared__ __align__(16) float s_red[27 * kRedPitch];
   const int blk = block_index(a.tile_order);
   const Block bk = block_of(a.cam, blk);
   const int lane = threadIdx.x & 31;
@@ -452,12 +457,12 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
     __syncwarp();
     const int cnt = stage_fill<true>(a.ids, rg.x, span, next, a.uv, a.co, a.rgb, bx0, by0,
                                      a.op.alpha_min, s_uv, s_co, s_rgb, s_id);
-    // three entries per iteration, their 27 gradient components summed over the warp in one
-    // transpose reduction (slots up to j + 2 <= kBatch + 1 exist; unused past cnt)
+    // three entries per iteration, their 27 components summed over the warp at once (slots up
+    // to j + 2 <= kBatch + 1 exist; unused past cnt)
     for (int j = 0; j < cnt; j += 3) {
-      float x[32];
+      float x[27];
 #pragma unroll
-      for (int k = 0; k < 32; ++k) x[k] = 0.f;
+      for (int k = 0; k < 27; ++k) x[k] = 0.f;
       unsigned who[3];
 #pragma unroll
       for (int i = 0; i < 3; ++i) {
@@ -471,10 +476,25 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
         who[i] = __ballot_sync(0xffffffffu, c0 || c1);
       }
       if ((who[0] | who[1] | who[2]) == 0) continue;
-      const float r = warp_sum32(x, lane);
-      const int ei = lane / 9, comp = lane - 9 * ei;
+      const float r = warp_sum27(x, s_red, lane);
+      const int ei = min(lane / 9, 2), comp = lane - 9 * ei;
+      // mean and conic gradients from the weighted moments of entry ei:
+      // d/du = -(ca Sx + cb Sy), d/dv = -(cb Sx + cc Sy), d/da = Sxx / 2, d/db = Sxy,
+      // d/dc = Syy / 2, with (ca, cb, cc) = ln 2 (2 a', b', 2 c') of the scaled conic
+      const float sx = __shfl_sync(0xffffffffu, r, 9 * ei);
+      const float sy = __shfl_sync(0xffffffffu, r, 9 * ei + 1);
       const unsigned wi = ei == 0 ? who[0] : (ei == 1 ? who[1] : who[2]);
-      if (lane < 27 && wi != 0) atomicAdd(a.grad2d + 9 * (size_t)s_id[j + ei] + comp, r);
+      if (lane < 27 && wi != 0) {
+        float g = r;
+        if (comp <= 1) {
+          const float4 sc = s_co[j + ei];
+          const float ca = 2.f * kLn2 * sc.x, cb = kLn2 * sc.y, cc = 2.f * kLn2 * sc.z;
+          g = comp == 0 ? -(ca * sx + cb * sy) : -(cb * sx + cc * sy);
+        } else if (comp == 2 || comp == 4) {
+          g = 0.5f * r;
+        }
+        atomicAdd(a.grad2d + 9 * (size_t)s_id[j + ei] + comp, g);
+      }
     }
   }
 }
