@@ -53,6 +53,14 @@ struct Workspace {
   float* loss_partials;             // [kMaxLossBlocks][2]
   unsigned* tile_order;             // [max_tiles] tiles by decreasing list length (bin_sort)
   long long max_tiles;
+  // render checkpoints: the forward saves each pixel's (colour, T) where a block's walk crosses
+  // a multiple of kCkChunk list positions, and lists the chunks after the first as work items
+  // (block, start, end) that the backward replays in parallel CTAs
+  float4* ckpt;                     // [ck_cap][64]
+  uint4* ck_items;                  // [ck_cap]
+  unsigned* ck_count;               // items allocated by the last forward with a state
+  unsigned* ck_first;               // [4 max_tiles] end of each block's first chunk, or ~0
+  int ck_cap;
 };
 
 constexpr int kRenderSubPerTile = 4;      // render CTAs (8x8 pixel blocks) per 16x16 tile
@@ -119,6 +127,9 @@ struct abcd_ctx {
   long long max_pixels = 0;
   abcd::Workspace ws{};
   const void* order_ranges = nullptr;   // tile ranges the order in ws.tile_order belongs to
+  const void* ck_state = nullptr;       // forward state the render checkpoints belong to
+  const void* ck_ranges = nullptr;      // and the tile ranges and block count they were made for
+  long long ck_blocks = 0;
   long long order_tiles = 0;
   abcd::SHConst sh{};
   long long launches = 0;

@@ -154,6 +154,11 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.loss_partials = (float*)take(4ull * 2 * kMaxLossBlocks);
   w.max_tiles = max_order_tiles(max_pixels);
   w.tile_order = (unsigned*)take(4ull * (size_t)w.max_tiles);
+  w.ck_cap = (int)std::max<long long>(1024, max_pixels / 128);
+  w.ckpt = (float4*)take(16ull * 64 * (size_t)w.ck_cap);
+  w.ck_items = (uint4*)take(16ull * (size_t)w.ck_cap);
+  w.ck_count = (unsigned*)take(256);
+  w.ck_first = (unsigned*)take(4ull * 4 * (size_t)w.max_tiles);
   if (ws) *ws = w;
   return off;
 }

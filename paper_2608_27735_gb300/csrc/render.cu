@@ -41,6 +41,9 @@ static_assert(kSubPerTile == kRenderSubPerTile, "tile order expands to kRenderSu
 constexpr int kRounds = 2;                       // list entries per lane per staging group
 constexpr int kGroup = kSubThreads * kRounds;    // 64 entries loaded together
 constexpr int kBatch = 2 * kGroup;               // staged survivors per batch (at most)
+constexpr int kCkChunk = 256;                    // list positions per backward chunk
+constexpr int kItemCtasPerSm = 8;                // backward CTAs that replay listed chunks
+static_assert(kCkChunk % kGroup == 0, "checkpoints fall on staging group boundaries");
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -166,11 +169,13 @@ __device__ __forceinline__ int stage_fill(const unsigned* ids, unsigned start, i
 
 // Render CTA b handles the 8x8 block tile_order[b / 4] * 4 + b % 4 (tile_order: a permutation
 // of the tiles, longest list first), or block b.
-__device__ __forceinline__ int block_index(const unsigned* tile_order) {
-  const int b = (int)blockIdx.x;
+__device__ __forceinline__ int block_index(const unsigned* tile_order, int b) {
   if (tile_order) return (int)tile_order[b / kSubPerTile] * kSubPerTile + b % kSubPerTile;
   return b;
 }
+
+// Index, within its 8x8 block, of the lane's first pixel (the second is 4 further).
+__device__ __forceinline__ int block_pixel(int lane) { return (lane >> 2) * kSub + (lane & 3); }
 
 // The CTA's 8x8 pixel block and the lane's two pixels (qx0, py), (qx1 = qx0 + 4, py).
 struct Block {
@@ -211,6 +216,11 @@ struct FwdArgs {
   unsigned* n_last;
   uint2* refresh;      // fp16 x4 per pixel
   const unsigned* tile_order;   // tiles, longest list first (nullptr: launch order)
+  float4* ckpt;                 // render checkpoints (nullptr: none), see the workspace
+  uint4* ck_items;
+  unsigned* ck_count;
+  unsigned* ck_first;
+  int ck_cap;
 };
 
 // Blend state of one pixel.
@@ -299,8 +309,9 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
   __shared__ float2 s_uv[kBatch];
   __shared__ float4 s_co[kBatch];
   __shared__ float4 s_rgb[kBatch];
-  const int blk = block_index(a.tile_order);
+  const int blk = block_index(a.tile_order, (int)blockIdx.x);
   const Block bk = block_of(a.cam, blk);
+  const int lane = threadIdx.x & 31;
   const uint2 rg = a.ranges[bk.tile];
   const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
   const float fx0 = (float)bk.qx0 + 0.5f, fx1 = (float)bk.qx1 + 0.5f, fy = (float)bk.py + 0.5f;
@@ -308,10 +319,15 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
   PixF p0 = {1.f, 0.f, 0.f, 0.f, 0u, !bk.in0};
   PixF p1 = {1.f, 0.f, 0.f, 0.f, 0u, !bk.in1};
   int next = 0;
+  bool ck_on = a.ckpt != nullptr;          // warp-uniform
+  int n_items = 0;
+  unsigned my_slot = 0u;                   // lane k: the slot of this block's item k
   while (next < n) {
     if (__all_sync(0xffffffffu, p0.done && p1.done)) break;
     __syncwarp();
-    const int cnt = stage_fill<false>(a.ids, rg.x, n, next, a.uv, a.co, a.rgb, bx0, by0,
+    // with checkpoints, a batch ends at the next multiple of kCkChunk
+    const int lim = ck_on ? min(n, (next / kCkChunk + 1) * kCkChunk) : n;
+    const int cnt = stage_fill<false>(a.ids, rg.x, lim, next, a.uv, a.co, a.rgb, bx0, by0,
                                       a.op.alpha_min, s_uv, s_co, s_rgb, nullptr);
     // two entries per iteration (slot j + 1 <= kBatch - 1 exists; unused when j + 1 == cnt)
     for (int j = 0; j < cnt; j += 2) {
@@ -327,6 +343,29 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
       blend(p0, a10, k10 && v1, e1.col, a.op);
       blend(p1, a11, k11 && v1, e1.col, a.op);
       if ((j & 30) == 30 && __all_sync(0xffffffffu, p0.done && p1.done)) break;
+    }
+    if (ck_on && next == lim && lim < n && !__all_sync(0xffffffffu, p0.done && p1.done)) {
+      // the state after every position below lim, for the backward's chunk starting there
+      unsigned slot = 0u;
+      if (lane == 0) slot = atomicAdd(a.ck_count, 1u);
+      slot = __shfl_sync(0xffffffffu, slot, 0);
+      if (slot < (unsigned)a.ck_cap) {
+        float4* ck = a.ckpt + (size_t)slot * (kSub * kSub);
+        const int k0 = block_pixel(lane);
+        ck[k0] = make_float4(p0.c0, p0.c1, p0.c2, p0.T);
+        ck[k0 + 4] = make_float4(p1.c0, p1.c1, p1.c2, p1.T);
+        if (lane == n_items) my_slot = slot;
+        ++n_items;
+      }
+      // past 32 items or a full buffer the last item listed runs to the end of the walk
+      ck_on = slot < (unsigned)a.ck_cap && n_items < 32;
+    }
+  }
+  if (a.ckpt) {
+    if (lane == 0) a.ck_first[blk] = n_items > 0 ? (unsigned)kCkChunk : 0xffffffffu;
+    if (lane < n_items) {
+      const unsigned start = (unsigned)((lane + 1) * kCkChunk);
+      a.ck_items[my_slot] = make_uint4((unsigned)blk, start, lane == n_items - 1 ? 0xffffffffu : start + kCkChunk, 0u);
     }
   }
   if (bk.in0) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx0, p0);
@@ -350,6 +389,12 @@ struct BwdArgs {
   const float* dl_dout;
   float* grad2d;
   const unsigned* tile_order;   // tiles, longest list first (nullptr: launch order)
+  const float4* ckpt;           // the forward's checkpoints (nullptr: every block walks whole)
+  const uint4* ck_items;
+  const unsigned* ck_count;
+  const unsigned* ck_first;
+  int ck_cap;
+  int n_item_ctas;              // the first CTAs of the launch replay the listed chunks
 };
 
 // Backward state of one pixel.  With G = dL/dA.rgb and G_a = dL/dA.a, the derivative of the
@@ -433,14 +478,11 @@ __device__ __forceinline__ float warp_sum27(const float (&x)[27], float* red, in
   return r;
 }
 
-__global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
-  pdl_prologue();
-  __shared__ float2 s_uv[kBatch + 2];
-  __shared__ float4 s_co[kBatch + 2];
-  __shared__ float4 s_rgb[kBatch + 2];
-  __shared__ unsigned s_id[kBatch + 2];
-  __shared__ __align__(16) float s_red[27 * kRedPitch];
-  const int blk = block_index(a.tile_order);
+// Backward of list positions [start, end) of block blk (clipped to the block's walk), from the
+// forward's checkpoint `ck` when start > 0.
+__device__ __forceinline__ void bwd_chunk(const BwdArgs& a, int blk, int start, unsigned end,
+                                          const float4* ck, float2* s_uv, float4* s_co,
+                                          float4* s_rgb, unsigned* s_id, float* s_red) {
   const Block bk = block_of(a.cam, blk);
   const int lane = threadIdx.x & 31;
   const uint2 rg = a.ranges[bk.tile];
@@ -451,8 +493,14 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
   p0.T = p1.T = 1.f;
   if (bk.in0) load_pixel_grad(a, (long long)bk.py * a.cam.width + bk.qx0, n, p0);
   if (bk.in1) load_pixel_grad(a, (long long)bk.py * a.cam.width + bk.qx1, n, p1);
-  const int span = (int)__reduce_max_sync(0xffffffffu, max(p0.last, p1.last));
-  int next = 0;
+  if (ck) {
+    const int k0 = block_pixel(lane);
+    const float4 c0 = ck[k0], c1 = ck[k0 + 4];
+    p0.T = c0.w; p0.Gc = p0.Gr * c0.x + p0.Gg * c0.y + p0.Gb * c0.z;
+    p1.T = c1.w; p1.Gc = p1.Gr * c1.x + p1.Gg * c1.y + p1.Gb * c1.z;
+  }
+  const int span = (int)min((unsigned)__reduce_max_sync(0xffffffffu, max(p0.last, p1.last)), end);
+  int next = start;
   while (next < span) {
     __syncwarp();
     const int cnt = stage_fill<true>(a.ids, rg.x, span, next, a.uv, a.co, a.rgb, bx0, by0,
@@ -499,10 +547,45 @@ __global__ void __launch_bounds__(kSubThreads) render_bwd_kernel(BwdArgs a) {
   }
 }
 
+__global__ void __launch_bounds__(kSubThreads, 24) render_bwd_kernel(BwdArgs a) {
+  pdl_prologue();
+  __shared__ float2 s_uv[kBatch + 2];
+  __shared__ float4 s_co[kBatch + 2];
+  __shared__ float4 s_rgb[kBatch + 2];
+  __shared__ unsigned s_id[kBatch + 2];
+  __shared__ __align__(16) float s_red[27 * kRedPitch];
+  // the first n_item_ctas CTAs replay the listed chunks after the first of the long walks, the
+  // others each a block's walk up to its first checkpoint
+  const int b = (int)blockIdx.x;
+  const bool item_cta = b < a.n_item_ctas;
+  const unsigned items = item_cta ? min(*a.ck_count, (unsigned)a.ck_cap) : 0u;
+  for (unsigned i = b; !item_cta || i < items; i += a.n_item_ctas) {
+    int blk, start = 0;
+    unsigned end = 0xffffffffu;
+    const float4* ck = nullptr;
+    if (item_cta) {
+      const uint4 it = a.ck_items[i];
+      blk = (int)it.x; start = (int)it.y; end = it.z;
+      ck = a.ckpt + (size_t)i * (kSub * kSub);
+    } else {
+      blk = block_index(a.tile_order, b - a.n_item_ctas);
+      if (a.ckpt) end = a.ck_first[blk];
+    }
+    __syncwarp();
+    bwd_chunk(a, blk, start, end, ck, s_uv, s_co, s_rgb, s_id, s_red);
+    if (!item_cta) break;
+  }
+}
+
 // The tile order bin_sort left in the workspace, if it was made for these ranges.
 const unsigned* tile_order_for(const abcd_ctx* ctx, const abcd_tiles* tiles, long long n_tiles) {
   return (has_workspace(ctx) && ctx->order_ranges == tiles->ranges && ctx->order_tiles == n_tiles)
              ? ctx->ws.tile_order : nullptr;
+}
+
+// Checkpoints need the workspace and room for a first-chunk end per block.
+bool ckpt_ok(const abcd_ctx* ctx, long long n_blocks) {
+  return has_workspace(ctx) && ctx->ws.ckpt && n_blocks <= kSubPerTile * ctx->ws.max_tiles;
 }
 
 bool fb_ok(const void* F, const void* B, int dtype) {
@@ -553,6 +636,19 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.refresh = (uint2*)refresh_f16;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
   a.tile_order = tile_order_for(ctx, tiles, n_tiles);
+  a.ckpt = nullptr; a.ck_items = nullptr; a.ck_count = nullptr; a.ck_first = nullptr;
+  a.ck_cap = 0;
+  if (state && ckpt_ok(ctx, n_blocks)) {
+    const cudaError_t e = cudaMemsetAsync(ctx->ws.ck_count, 0, sizeof(unsigned), ctx->stream);
+    if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "checkpoint count memset: %s", cudaGetErrorString(e));
+    a.ckpt = ctx->ws.ckpt; a.ck_items = ctx->ws.ck_items; a.ck_count = ctx->ws.ck_count;
+    a.ck_first = ctx->ws.ck_first; a.ck_cap = ctx->ws.ck_cap;
+    ctx->ck_state = state->A_T;
+    ctx->ck_blocks = n_blocks;
+    ctx->ck_ranges = tiles->ranges;
+  } else if (state && ctx->ck_state == state->A_T) {
+    ctx->ck_state = nullptr;               // this state's checkpoints are gone
+  }
   return check_launch(ctx, "render_fwd_kernel",
                       launch_pdl(render_fwd_kernel, dim3(n_blocks), dim3(kSubThreads), 0, ctx->stream, a));
 }
@@ -589,6 +685,15 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   a.grad2d = grad2d;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
   a.tile_order = tile_order_for(ctx, tiles, n_tiles);
+  a.ckpt = nullptr; a.ck_items = nullptr; a.ck_count = nullptr; a.ck_first = nullptr;
+  a.ck_cap = 0; a.n_item_ctas = 0;
+  if (ckpt_ok(ctx, n_blocks) && ctx->ck_state == state->A_T && ctx->ck_blocks == n_blocks &&
+      ctx->ck_ranges == tiles->ranges) {
+    a.ckpt = ctx->ws.ckpt; a.ck_items = ctx->ws.ck_items; a.ck_count = ctx->ws.ck_count;
+    a.ck_first = ctx->ws.ck_first; a.ck_cap = ctx->ws.ck_cap;
+    a.n_item_ctas = std::min(ctx->ws.ck_cap, kItemCtasPerSm * ctx->num_sms);
+  }
   return check_launch(ctx, "render_bwd_kernel",
-                      launch_pdl(render_bwd_kernel, dim3(n_blocks), dim3(kSubThreads), 0, ctx->stream, a));
+                      launch_pdl(render_bwd_kernel, dim3(a.n_item_ctas + n_blocks), dim3(kSubThreads),
+                                 0, ctx->stream, a));
 }

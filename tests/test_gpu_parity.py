@@ -229,17 +229,14 @@ def test_refresh_fp16_matches_oracle(ctx, tiny):
     assert np.all(got[exact] == ref.astype(np.float16)[exact])
 
 
-@pytest.mark.parametrize("cam_idx", [0, 2])
-def test_render_backward_matches_oracle(ctx, tiny, cam_idx):
-    case = Case(tiny, cam_idx, fb=True)
-    bg = (0.1, 0.2, 0.3)
-    r = run_forward(ctx, case, bg=bg)
+def check_backward(ctx, case, r, bg, seed, state=None):
+    """Render backward of a forward result `r` against the oracle's, for a seeded dL/dA."""
     H, W = case.cam.height, case.cam.width
-    rng = np.random.default_rng(100 + cam_idx)
+    rng = np.random.default_rng(seed)
     G = (rng.normal(size=(H, W, 3)) / (3.0 * H * W)).astype(np.float32)
     grad2d = torch.empty(case.g.n, 9, device="cuda")
     ab.abcd_render_backward(ctx, r["cam"], None, r["proj"], r["tiles"], r["F"], r["B"], r["fbd"],
-                            bg, r["state"], torch.from_numpy(G).cuda(), case.g.n, grad2d)
+                            bg, state or r["state"], torch.from_numpy(G).cuda(), case.g.n, grad2d)
     ctx.sync()
     ref = oracle.backward(case.sp, case.off, case.ids, W, H, G.astype(np.float64), F=case.F64(),
                           B=case.B64(), bg=bg)
@@ -251,6 +248,68 @@ def test_render_backward_matches_oracle(ctx, tiny, cam_idx):
     scale = np.abs(ref).max(0, keepdims=True)
     par.assert_grad_close(grad2d.cpu().numpy(), ref, lo, hi, rtol=1e-3, atol=1e-5 * scale,
                           what="grad2d")
+    return R
+
+
+@pytest.mark.parametrize("cam_idx", [0, 2])
+def test_render_backward_matches_oracle(ctx, tiny, cam_idx):
+    case = Case(tiny, cam_idx, fb=True)
+    bg = (0.1, 0.2, 0.3)
+    r = run_forward(ctx, case, bg=bg)
+    check_backward(ctx, case, r, bg, 100 + cam_idx)
+
+
+def faint_scene(n, width, height, seed=93):
+    """One cell of n faint Gaussians (opacity logits N(-5, 0.3^2)): tile lists of thousands of
+    entries that the pixels stay open through, so the backward splits them into many chunks."""
+    s = sg.grid_scene((1, 1, 1), 5.0, n, 0, seed=seed)
+    s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), width, height,
+                                seed=seed, height_jitter=1.0)
+    g = s.gaussians
+    g.opacity_logits[:] = (-5.0 + 0.3 * np.random.default_rng(seed).normal(size=g.n)).astype(np.float32)
+    return s
+
+
+@pytest.fixture(scope="module")
+def faint():
+    return faint_scene(60_000, 64, 48)
+
+
+def test_render_backward_long_walks(ctx, faint):
+    """Walks of up to ~13,500 list positions: past the 32 chunks a block can list, so its last
+    listed chunk runs to the end of the walk."""
+    case = Case(faint, 0, fb=False)
+    assert np.diff(case.off).max() > 33 * 256
+    r = run_forward(ctx, case)
+    R = oracle.render(case.sp, case.off, case.ids, case.cam.width, case.cam.height)
+    par.compare_render(r["out"].cpu().numpy(), r["state"].A_T.cpu().numpy()[..., 3], R, case.sp,
+                       case.off, case.ids, case.P, case.opt, case.cam)
+    assert R["n_used"].max() > 33 * 256
+    check_backward(ctx, case, r, None, 7)
+    # a second backward of the same forward reuses its checkpoints
+    check_backward(ctx, case, r, None, 8)
+
+
+def test_render_backward_checkpoint_buffer_full():
+    """A context sized for a 96x64 image holds 1,024 chunk checkpoints, fewer than the faint
+    scene's long walks ask for: blocks that find the buffer full walk on to their end."""
+    c = ab.Context(0)
+    c.reserve(60_000, 1_000_000, 96 * 64)
+    case = Case(faint_scene(60_000, 96, 64), 0, fb=False)
+    r = run_forward(c, case)
+    n_chunks = sum(max(0, (int(n) - 1) // 256) for n in np.diff(case.off)) * 4
+    assert n_chunks > 1024
+    check_backward(c, case, r, None, 9)
+
+
+def test_render_backward_after_other_forward(ctx, tiny):
+    """A forward into another state replaces the checkpoints; the backward of the first state
+    then walks each block whole and still matches."""
+    case = Case(tiny, 1, fb=True)
+    bg = (0.3, 0.3, 0.3)
+    r = run_forward(ctx, case, bg=bg)
+    run_forward(ctx, Case(tiny, 3, fb=False))
+    check_backward(ctx, case, r, bg, 11)
 
 
 def test_project_backward_matches_oracle(ctx, ragged):
