@@ -259,6 +259,9 @@ def test_render_backward_matches_oracle(ctx, tiny, cam_idx):
     check_backward(ctx, case, r, bg, 100 + cam_idx)
 
 
+CK_CHUNK = 128   # list positions between the render checkpoints
+
+
 def faint_scene(n, width, height, seed=93):
     """One cell of n faint Gaussians (opacity logits N(-5, 0.3^2)): tile lists of thousands of
     entries that the pixels stay open through, so the backward splits them into many chunks."""
@@ -279,12 +282,12 @@ def test_render_backward_long_walks(ctx, faint):
     """Walks of up to ~13,500 list positions: past the 32 chunks a block can list, so its last
     listed chunk runs to the end of the walk."""
     case = Case(faint, 0, fb=False)
-    assert np.diff(case.off).max() > 33 * 256
+    assert np.diff(case.off).max() > 33 * CK_CHUNK
     r = run_forward(ctx, case)
     R = oracle.render(case.sp, case.off, case.ids, case.cam.width, case.cam.height)
     par.compare_render(r["out"].cpu().numpy(), r["state"].A_T.cpu().numpy()[..., 3], R, case.sp,
                        case.off, case.ids, case.P, case.opt, case.cam)
-    assert R["n_used"].max() > 33 * 256
+    assert R["n_used"].max() > 33 * CK_CHUNK
     check_backward(ctx, case, r, None, 7)
     # a second backward of the same forward reuses its checkpoints
     check_backward(ctx, case, r, None, 8)
@@ -297,7 +300,7 @@ def test_render_backward_checkpoint_buffer_full():
     c.reserve(60_000, 1_000_000, 96 * 64)
     case = Case(faint_scene(60_000, 96, 64), 0, fb=False)
     r = run_forward(c, case)
-    n_chunks = sum(max(0, (int(n) - 1) // 256) for n in np.diff(case.off)) * 4
+    n_chunks = sum(max(0, (int(n) - 1) // CK_CHUNK) for n in np.diff(case.off)) * 4
     assert n_chunks > 1024
     check_backward(c, case, r, None, 9)
 
