@@ -213,10 +213,10 @@ abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* layers, int L
  * (its own pool or arena, with raw cudaMalloc forbidden), or a caller that must not allocate
  * between set-up and a latency-critical loop.  The paper has no counterpart; it exists only
  * for those callers.  Same arguments and results as abcd_loss, with an explicit stream.
- * Its scratch (per-CTA partial sums and a completion counter, about 128 KB) is a static
+ * Its scratch (per-CTA partial sums and a completion counter, about 512 KB) is a static
  * device array of this library, held by every GPU that loads the library until the process
- * exits; images may have at most 16384 CTAs of 64x32 pixels (e.g. 8192 x 4096), larger ones
- * return ABCD_ERR_WORKSPACE.  The first call on a device looks up the array's address (with
+ * exits; images may have at most 65536 CTAs, one per channel of a 64x28-pixel tile (e.g.
+ * 8192 x 4096), larger ones return ABCD_ERR_WORKSPACE.  The first call on a device looks up the array's address (with
  * that device current), so make it before any stream capture.  All calls on a device share
  * the array: calls whose kernels overlap on the GPU race and give wrong losses, so order them
  * (one stream, or events).  The counter is cleared at the start of every call.  Returns

@@ -2,16 +2,18 @@
 // and dL/dx, fused in one kernel (each step of Section 2 scores the composited image against
 // the target; the L1 + D-SSIM form is that of 3D Gaussian Splatting).
 //
-// SSIM uses an 11x11 Gaussian window (sigma 1.5) with zero padding.  Per output tile of 64x32
-// pixels and per channel, a CTA stages x, y over the tile plus a 10-pixel halo, computes the
-// five windowed moments (separably) on the tile plus a 5-pixel halo, the per-pixel partials
-// A = dS/dmu_x - 2 mu_x dS/dsigma_xx - mu_y dS/dsigma_xy, B = dS/dsigma_xx, C = dS/dsigma_xy,
-// and windows them again: dSSIM_sum/dx(q) = (w*A)(q) + 2 x(q) (w*B)(q) + y(q) (w*C)(q).
-// Every window pass is register-blocked: a thread produces 8 consecutive outputs from a
-// sliding run of 18 staged values (about 12 FMAs per shared-memory load), and the windows of
-// x and y (of x^2 and y^2, of A and B) share packed two-lane FMAs.
+// SSIM uses an 11x11 Gaussian window (sigma 1.5) with zero padding.  A CTA takes one channel
+// of an output tile of 64x28 pixels: it stages x, y over the tile plus a 10-pixel halo,
+// computes the five windowed moments (separably) on the tile plus a 5-pixel halo, the
+// per-pixel partials A = dS/dmu_x - 2 mu_x dS/dsigma_xx - mu_y dS/dsigma_xy, B = dS/dsigma_xx,
+// C = dS/dsigma_xy, and windows them again: dSSIM_sum/dx(q) = (w*A)(q) + 2 x(q) (w*B)(q) +
+// y(q) (w*C)(q).  Every window pass is register-blocked: a thread produces 8 consecutive
+// outputs from a sliding run of 18 staged values, and the windows of x and y (of x^2 and
+// y^2, of A and B) share packed two-lane FMAs.  Shared memory (about 105 KB) and registers
+// (at most 64) are sized for two CTAs per SM, so one CTA's barriers overlap the other's work.
 // The scalar is reduced deterministically: per-CTA partial sums, then the last CTA to finish
 // adds them in a fixed order (no waiting on other CTAs).
+#include <cmath>
 #include <mutex>
 
 #include "abcd_internal.cuh"
@@ -20,229 +22,222 @@ namespace abcd {
 namespace {
 
 constexpr int TW = 64;            // output tile (pixels)
-constexpr int TH = 32;
+constexpr int TH = 28;
 constexpr int RUN = 8;            // outputs per thread per window pass
 constexpr int IW = TW + 20, IH = TH + 20;    // inputs: tile + 10-pixel halo
 constexpr int MW = TW + 10, MH = TH + 10;    // windowed moments: tile + 5-pixel halo
 constexpr int HSEG = (MW + RUN - 1) / RUN;   // column runs of the horizontal moment pass
 constexpr int VSEG = (MH + RUN - 1) / RUN;   // row runs of the vertical moment pass
-constexpr int kThreads = 544;                // 17 warps: one horizontal moment run per thread
+constexpr int HSEG3 = TW / RUN;              // column runs of the horizontal A, B, C pass
+constexpr int VSEG3 = (TH + RUN - 1) / RUN;  // row runs of the vertical A, B, C pass
+constexpr int kThreads = 480;                // 15 warps: one horizontal moment run per thread
 static_assert(IH * HSEG <= kThreads, "the horizontal moment pass is one round");
+static_assert(TW % RUN == 0 && MH >= RUN && TH >= RUN, "run tiling");
 // Row pitches are odd (consecutive lanes take consecutive rows in the horizontal passes and
 // consecutive columns in the vertical ones: no bank conflicts, also for the 8-byte pairs) and
-// wide or tall enough that a run never reads past its array (the values read beyond the valid
-// region only feed outputs that are discarded).
+// wide enough that a horizontal run never reads past its row (values read beyond the valid
+// region only feed outputs that are discarded).  A vertical pass's last run starts early
+// enough to stay inside its rows and skips the outputs the run before it made.
 constexpr int IP = ((HSEG * RUN + 10) | 1);          // x|y row pitch (>= IW)
 constexpr int MP = (MW | 1);                         // moment / A, B, C row pitch (>= MW)
-constexpr int MROWS = VSEG * RUN + 10;               // rows of the moment rows (>= IH)
 constexpr int TP = (TW | 1);                         // pitch of the windows of A, B, C
-// Shared memory, in floats: (x, y) pairs [IH][IP]; the horizontal moment rows as pairs
-// (mu_x, mu_y), (s_xx, s_yy) [MROWS][MP] and s_xy [MROWS][MP]; (A, B) pairs and C [MH][MP];
-// their horizontal windows, (A, B) pairs and C [MH][TP], reuse the moment rows' space.  The
-// pairs go through the packed fp32 FMA (__ffma2_rn), two windows per instruction; each
-// component is rounded exactly as a scalar fmaf.
-constexpr int kXY = 2 * IH * IP;
-constexpr int kMom = 5 * MROWS * MP;
-constexpr int kABC = 3 * MH * MP;
-constexpr int kSmemFloats = kXY + kMom + kABC;
-static_assert(IP >= IW && MP >= MW && MROWS >= IH, "padded pitches");
-static_assert(3 * MH * TP <= kMom, "windows of A, B, C fit in the moment space");
-static_assert((TW / RUN - 1) * RUN + RUN + 10 <= MP, "horizontal A, B, C runs stay in a row");
-static_assert(kXY % 2 == 0 && (kXY + kMom) % 2 == 0, "pair arrays 8-byte aligned");
+// Shared memory, in floats, two regions:
+//   R0: (x, y) pairs [IH][IP]; later (A, B) pairs and C [MH][MP]
+//   R1: horizontal moment rows (mu_x, mu_y), (s_xx, s_yy) pairs and s_xy [IH][MP]; later the
+//       horizontal windows of A, B, C: (A, B) pairs and C [MH][TP]
+// The pairs go through the packed fp32 FMA (__ffma2_rn), two windows per instruction; each
+// component is rounded exactly as a scalar fmaf.  The gradient pass reads x and y back from
+// global memory (L2): R0 holds A, B, C by then.
+constexpr int kR0 = 2 * IH * IP;
+constexpr int kR1 = 5 * IH * MP;
+constexpr int kSmemFloats = kR0 + kR1;
+static_assert(IP >= IW && MP >= MW, "padded pitches");
+static_assert(3 * MH * MP <= kR0, "A, B, C fit in the input region");
+static_assert(3 * MH * TP <= kR1, "windows of A, B, C fit in the moment region");
+static_assert((HSEG3 - 1) * RUN + RUN + 10 <= MP, "horizontal A, B, C runs stay in a row");
+static_assert(kR0 % 2 == 0 && (2 * MH * MP) % 2 == 0 && (2 * IH * MP) % 2 == 0, "pairs 8-byte aligned");
+static_assert(sizeof(float) * kSmemFloats <= 110 * 1024, "two CTAs per SM");
 
-__device__ __forceinline__ void load_weights(float* w) {
-  float s = 0.f;
-#pragma unroll
-  for (int t = 0; t < 11; ++t) { const float d = (float)t - 5.f; w[t] = expf(-d * d / (2.f * 1.5f * 1.5f)); s += w[t]; }
-#pragma unroll
-  for (int t = 0; t < 11; ++t) w[t] /= s;
-}
+struct Window {
+  float w[11];      // normalised 11-tap Gaussian, sigma 1.5
+};
 
 // RUN outputs of an 11-tap window from RUN + 10 staged pairs / values.
-__device__ __forceinline__ void window_pairs(const float2 (&v)[RUN + 10], const float2 (&w2)[11],
+__device__ __forceinline__ void window_pairs(const float2 (&v)[RUN + 10], const Window& win,
                                              float2 (&out)[RUN]) {
 #pragma unroll
   for (int o = 0; o < RUN; ++o) {
     float2 a = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int t = 0; t < 11; ++t) a = __ffma2_rn(w2[t], v[o + t], a);
+    for (int t = 0; t < 11; ++t) a = __ffma2_rn(make_float2(win.w[t], win.w[t]), v[o + t], a);
     out[o] = a;
   }
 }
 
-__device__ __forceinline__ void window_scalars(const float (&v)[RUN + 10], const float2 (&w2)[11],
+__device__ __forceinline__ void window_scalars(const float (&v)[RUN + 10], const Window& win,
                                                float (&out)[RUN]) {
 #pragma unroll
   for (int o = 0; o < RUN; ++o) {
     float a = 0.f;
 #pragma unroll
-    for (int t = 0; t < 11; ++t) a = fmaf(w2[t].x, v[o + t], a);
+    for (int t = 0; t < 11; ++t) a = fmaf(win.w[t], v[o + t], a);
     out[o] = a;
   }
 }
 
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 2)
 loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W, int H,
-            float lam, float* __restrict__ grad, float* partials, unsigned* ticket,
-            float* loss_out) {
+            float lam, const Window win, float* __restrict__ grad, float* partials,
+            unsigned* ticket, float* loss_out) {
   pdl_prologue();
   extern __shared__ __align__(16) float sm[];
   float2* sXY = reinterpret_cast<float2*>(sm);                        // [IH][IP]
-  float2* hM = reinterpret_cast<float2*>(sm + kXY);                   // [MROWS][MP]
-  float2* hS = hM + MROWS * MP;                                       // [MROWS][MP]
-  float* hC = reinterpret_cast<float*>(hS + MROWS * MP);              // [MROWS][MP]
-  float2* aAB = reinterpret_cast<float2*>(sm + kXY + kMom);           // [MH][MP]
+  float2* aAB = reinterpret_cast<float2*>(sm);                        // [MH][MP]
   float* aC = reinterpret_cast<float*>(aAB + MH * MP);                // [MH][MP]
+  float2* hM = reinterpret_cast<float2*>(sm + kR0);                   // [IH][MP]
+  float2* hS = hM + IH * MP;                                          // [IH][MP]
+  float* hC = reinterpret_cast<float*>(hS + IH * MP);                 // [IH][MP]
   float2* gAB = hM;                                                   // [MH][TP]
   float* gC = reinterpret_cast<float*>(gAB + MH * TP);                // [MH][TP]
   __shared__ float red[2][kThreads / 32];
-  float2 w2[11];
-  {
-    float w[11];
-    load_weights(w);
-#pragma unroll
-    for (int t = 0; t < 11; ++t) w2[t] = make_float2(w[t], w[t]);
-  }
-  const int ox = blockIdx.x * TW, oy = blockIdx.y * TH;
+  const int ox = blockIdx.x * TW, oy = blockIdx.y * TH, ch = blockIdx.z;
   const float inv = 1.f / (3.f * (float)W * (float)H);
   const float C1 = 0.01f * 0.01f, C2 = 0.03f * 0.03f;
   float l1 = 0.f, ssim = 0.f;
-  for (int ch = 0; ch < 3; ++ch) {
-    // ---- inputs with a 10-pixel halo, zero outside the image
-    for (int k = threadIdx.x; k < IH * IP; k += kThreads) {
-      const int r = k / IP, c = k - r * IP;
-      const int gy = oy - 10 + r, gx = ox - 10 + c;
-      float xv = 0.f, yv = 0.f;
-      if (c < IW && gx >= 0 && gx < W && gy >= 0 && gy < H) {
-        const long long p = (long long)gy * W + gx;
-        xv = xin[4 * p + ch];
-        yv = yin[3 * p + ch];
-      }
-      sXY[k] = make_float2(xv, yv);
+  // ---- inputs with a 10-pixel halo, zero outside the image
+  for (int k = threadIdx.x; k < IH * IP; k += kThreads) {
+    const int r = k / IP, c = k - r * IP;
+    const int gy = oy - 10 + r, gx = ox - 10 + c;
+    float xv = 0.f, yv = 0.f;
+    if (c < IW && gx >= 0 && gx < W && gy >= 0 && gy < H) {
+      const long long p = (long long)gy * W + gx;
+      xv = __ldg(xin + 4 * p + ch);
+      yv = __ldg(yin + 3 * p + ch);
     }
-    __syncthreads();
-    // ---- horizontal windows of (x, y), (x^2, y^2) and xy: RUN outputs per run
-    for (int it = threadIdx.x; it < IH * HSEG; it += kThreads) {
-      const int r = it % IH, c0 = (it / IH) * RUN;   // consecutive lanes: consecutive rows
-      float2 v[RUN + 10], q[RUN + 10], o2[RUN];
+    sXY[k] = make_float2(xv, yv);
+  }
+  __syncthreads();
+  // ---- horizontal windows of (x, y), (x^2, y^2) and xy: RUN outputs per run
+  for (int it = threadIdx.x; it < IH * HSEG; it += kThreads) {
+    const int r = it % IH, c0 = (it / IH) * RUN;   // consecutive lanes: consecutive rows
+    float2 v[RUN + 10], o2[RUN];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) {
-        v[t] = sXY[r * IP + c0 + t];
-        q[t] = __fmul2_rn(v[t], v[t]);
-      }
-      window_pairs(v, w2, o2);
+    for (int t = 0; t < RUN + 10; ++t) v[t] = sXY[r * IP + c0 + t];
+    window_pairs(v, win, o2);
 #pragma unroll
-      for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hM[r * MP + c0 + o] = o2[o];
-      window_pairs(q, w2, o2);
+    for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hM[r * MP + c0 + o] = o2[o];
+    float p[RUN + 10], o1[RUN];
 #pragma unroll
-      for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hS[r * MP + c0 + o] = o2[o];
-      float p[RUN + 10], o1[RUN];
-#pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) p[t] = v[t].x * v[t].y;
-      window_scalars(p, w2, o1);
-#pragma unroll
-      for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hC[r * MP + c0 + o] = o1[o];
+    for (int t = 0; t < RUN + 10; ++t) {
+      p[t] = v[t].x * v[t].y;
+      v[t] = __fmul2_rn(v[t], v[t]);
     }
-    __syncthreads();
-    // ---- vertical windows -> moments -> SSIM and its partials A, B, C (zero off-image)
-    for (int it = threadIdx.x; it < MW * VSEG; it += kThreads) {
-      const int c = it % MW, r0 = (it / MW) * RUN;
-      float2 mm[RUN], ss[RUN];
-      float mc[RUN];
-      {
-        float2 col[RUN + 10];
+    window_pairs(v, win, o2);
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) col[t] = hM[(r0 + t) * MP + c];
-        window_pairs(col, w2, mm);
+    for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hS[r * MP + c0 + o] = o2[o];
+    window_scalars(p, win, o1);
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) col[t] = hS[(r0 + t) * MP + c];
-        window_pairs(col, w2, ss);
-      }
-      {
-        float col[RUN + 10];
+    for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hC[r * MP + c0 + o] = o1[o];
+  }
+  __syncthreads();
+  // ---- vertical windows -> moments -> SSIM and its partials A, B, C (zero off-image)
+  for (int it = threadIdx.x; it < MW * VSEG; it += kThreads) {
+    const int c = it % MW, k0 = (it / MW) * RUN;
+    const int r0 = min(k0, MH - RUN);              // the last run starts early ...
+    const int o0 = k0 - r0;                        // ... and skips what the run before made
+    float2 mm[RUN], ss[RUN];
+    float mc[RUN];
+    {
+      float2 col[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) col[t] = hC[(r0 + t) * MP + c];
-        window_scalars(col, w2, mc);
-      }
+      for (int t = 0; t < RUN + 10; ++t) col[t] = hM[(r0 + t) * MP + c];
+      window_pairs(col, win, mm);
 #pragma unroll
-      for (int o = 0; o < RUN; ++o) {
-        const int r = r0 + o;
-        if (r >= MH) continue;
-        const int gy = oy - 5 + r, gx = ox - 5 + c;
-        float A = 0.f, B = 0.f, Cc = 0.f;
-        if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
-          const float mx = mm[o].x, my = mm[o].y;
-          const float vx = ss[o].x - mx * mx, vy = ss[o].y - my * my, cxy = mc[o] - mx * my;
-          const float N1 = 2.f * mx * my + C1, N2 = 2.f * cxy + C2;
-          const float D1 = mx * mx + my * my + C1, D2 = vx + vy + C2;
-          const float iD = 1.f / (D1 * D2);
-          const float S = N1 * N2 * iD;
-          const float dvx = -S / D2;
-          const float dcxy = 2.f * N1 * iD;
-          A = (2.f * my * N2 - S * 2.f * mx * D2) * iD - 2.f * mx * dvx - my * dcxy;
-          B = dvx;
-          Cc = dcxy;
-          if (r >= 5 && r < 5 + TH && c >= 5 && c < 5 + TW) ssim += S;
-        }
-        aAB[r * MP + c] = make_float2(A, B);
-        aC[r * MP + c] = Cc;
-      }
+      for (int t = 0; t < RUN + 10; ++t) col[t] = hS[(r0 + t) * MP + c];
+      window_pairs(col, win, ss);
     }
-    __syncthreads();
-    // ---- horizontal windows of (A, B) and C: [MH][TW]
-    constexpr int HSEG3 = TW / RUN;
-    for (int it = threadIdx.x; it < MH * HSEG3; it += kThreads) {
-      const int r = it % MH, c0 = (it / MH) * RUN;   // consecutive lanes: consecutive rows
-      {
-        float2 v[RUN + 10], o2[RUN];
+    {
+      float col[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = aAB[r * MP + c0 + t];
-        window_pairs(v, w2, o2);
-#pragma unroll
-        for (int o = 0; o < RUN; ++o) gAB[r * TP + c0 + o] = o2[o];
-      }
-      {
-        float v[RUN + 10], o1[RUN];
-#pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = aC[r * MP + c0 + t];
-        window_scalars(v, w2, o1);
-#pragma unroll
-        for (int o = 0; o < RUN; ++o) gC[r * TP + c0 + o] = o1[o];
-      }
+      for (int t = 0; t < RUN + 10; ++t) col[t] = hC[(r0 + t) * MP + c];
+      window_scalars(col, win, mc);
     }
-    __syncthreads();
-    // ---- vertical windows and the gradient on the output tile
-    constexpr int VSEG3 = TH / RUN;
-    for (int it = threadIdx.x; it < TW * VSEG3; it += kThreads) {
-      const int c = it % TW, r0 = (it / TW) * RUN;
-      float2 gab[RUN];
-      float gc[RUN];
-      {
-        float2 v[RUN + 10];
 #pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = gAB[(r0 + t) * TP + c];
-        window_pairs(v, w2, gab);
+    for (int o = 0; o < RUN; ++o) {
+      if (o < o0) continue;
+      const int r = r0 + o;
+      const int gy = oy - 5 + r, gx = ox - 5 + c;
+      float A = 0.f, B = 0.f, Cc = 0.f;
+      if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
+        const float mx = mm[o].x, my = mm[o].y;
+        const float vx = ss[o].x - mx * mx, vy = ss[o].y - my * my, cxy = mc[o] - mx * my;
+        const float N1 = 2.f * mx * my + C1, N2 = 2.f * cxy + C2;
+        const float D1 = mx * mx + my * my + C1, D2 = vx + vy + C2;
+        const float iD = 1.f / (D1 * D2);
+        const float S = N1 * N2 * iD;
+        const float dvx = -S / D2;
+        const float dcxy = 2.f * N1 * iD;
+        A = (2.f * my * N2 - S * 2.f * mx * D2) * iD - 2.f * mx * dvx - my * dcxy;
+        B = dvx;
+        Cc = dcxy;
+        if (r >= 5 && r < 5 + TH && c >= 5 && c < 5 + TW) ssim += S;
       }
-      {
-        float v[RUN + 10];
-#pragma unroll
-        for (int t = 0; t < RUN + 10; ++t) v[t] = gC[(r0 + t) * TP + c];
-        window_scalars(v, w2, gc);
-      }
-#pragma unroll
-      for (int o = 0; o < RUN; ++o) {
-        const int gy = oy + r0 + o, gx = ox + c;
-        if (gx >= W || gy >= H) continue;
-        const float2 xy = sXY[(r0 + o + 10) * IP + c + 10];
-        const float xv = xy.x, yv = xy.y;
-        const float d = xv - yv;
-        l1 += fabsf(d);
-        const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
-        const float dS = gab[o].x + 2.f * xv * gab[o].y + yv * gc[o];
-        if (grad) grad[3 * ((long long)gy * W + gx) + ch] = ((1.f - lam) * sgn - lam * dS) * inv;
-      }
+      aAB[r * MP + c] = make_float2(A, B);
+      aC[r * MP + c] = Cc;
     }
-    __syncthreads();
+  }
+  __syncthreads();
+  // ---- horizontal windows of (A, B) and C: [MH][TW]
+  for (int it = threadIdx.x; it < MH * HSEG3; it += kThreads) {
+    const int r = it % MH, c0 = (it / MH) * RUN;   // consecutive lanes: consecutive rows
+    {
+      float2 v[RUN + 10], o2[RUN];
+#pragma unroll
+      for (int t = 0; t < RUN + 10; ++t) v[t] = aAB[r * MP + c0 + t];
+      window_pairs(v, win, o2);
+#pragma unroll
+      for (int o = 0; o < RUN; ++o) gAB[r * TP + c0 + o] = o2[o];
+    }
+    {
+      float v[RUN + 10], o1[RUN];
+#pragma unroll
+      for (int t = 0; t < RUN + 10; ++t) v[t] = aC[r * MP + c0 + t];
+      window_scalars(v, win, o1);
+#pragma unroll
+      for (int o = 0; o < RUN; ++o) gC[r * TP + c0 + o] = o1[o];
+    }
+  }
+  __syncthreads();
+  // ---- vertical windows and the gradient on the output tile
+  for (int it = threadIdx.x; it < TW * VSEG3; it += kThreads) {
+    const int c = it % TW, k0 = (it / TW) * RUN;
+    const int r0 = min(k0, TH - RUN), o0 = k0 - r0;
+    float2 gab[RUN];
+    float gc[RUN];
+    {
+      float2 v[RUN + 10];
+#pragma unroll
+      for (int t = 0; t < RUN + 10; ++t) v[t] = gAB[(r0 + t) * TP + c];
+      window_pairs(v, win, gab);
+    }
+    {
+      float v[RUN + 10];
+#pragma unroll
+      for (int t = 0; t < RUN + 10; ++t) v[t] = gC[(r0 + t) * TP + c];
+      window_scalars(v, win, gc);
+    }
+#pragma unroll
+    for (int o = 0; o < RUN; ++o) {
+      const int gy = oy + r0 + o, gx = ox + c;
+      if (o < o0 || gx >= W || gy >= H) continue;
+      const long long q = (long long)gy * W + gx;
+      const float xv = __ldg(xin + 4 * q + ch), yv = __ldg(yin + 3 * q + ch);
+      const float d = xv - yv;
+      l1 += fabsf(d);
+      const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
+      const float dS = gab[o].x + 2.f * xv * gab[o].y + yv * gc[o];
+      if (grad) grad[3 * q + ch] = ((1.f - lam) * sgn - lam * dS) * inv;
+    }
   }
   // block partial sums -> last block finishes the scalar
   for (int o = 16; o > 0; o >>= 1) {
@@ -251,8 +246,8 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
   }
   if ((threadIdx.x & 31) == 0) { red[0][threadIdx.x >> 5] = l1; red[1][threadIdx.x >> 5] = ssim; }
   __syncthreads();
-  const int nb = gridDim.x * gridDim.y;
-  const int b = blockIdx.y * gridDim.x + blockIdx.x;
+  const int nb = gridDim.x * gridDim.y * gridDim.z;
+  const int b = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
   __shared__ bool is_last;
   if (threadIdx.x == 0) {
     float s0 = 0.f, s1 = 0.f;
@@ -287,6 +282,19 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
   }
 }
 
+// The SSIM window, computed in double and rounded once per tap.
+Window ssim_window() {
+  Window win;
+  double w[11], s = 0.0;
+  for (int t = 0; t < 11; ++t) { const double d = t - 5.0; w[t] = std::exp(-d * d / 4.5); s += w[t]; }
+  for (int t = 0; t < 11; ++t) win.w[t] = (float)(w[t] / s);
+  return win;
+}
+
+dim3 loss_grid(int width, int height) {
+  return dim3((width + TW - 1) / TW, (height + TH - 1) / TH, 3);
+}
+
 }  // namespace
 
 abcd_status loss_launch(abcd_ctx* ctx, const float* out_rgba, const float* gt_rgb, int width,
@@ -294,15 +302,15 @@ abcd_status loss_launch(abcd_ctx* ctx, const float* out_rgba, const float* gt_rg
   if (!has_workspace(ctx)) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_loss: no workspace");
   if (!out_rgba || !gt_rgb || width <= 0 || height <= 0 || !(lambda_ssim >= 0.f && lambda_ssim <= 1.f))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_loss: bad arguments");
-  const dim3 grid((width + TW - 1) / TW, (height + TH - 1) / TH);
-  if ((long long)grid.x * grid.y > kMaxLossBlocks)
+  const dim3 grid = loss_grid(width, height);
+  if ((long long)grid.x * grid.y * grid.z > kMaxLossBlocks)
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_loss: image too large (%d x %d)", width, height);
   const size_t smem = sizeof(float) * kSmemFloats;
   cudaError_t e = cudaFuncSetAttribute(loss_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "loss smem attribute: %s", cudaGetErrorString(e));
   return check_launch(ctx, "loss_kernel",
                       launch_pdl(loss_kernel, grid, dim3(kThreads), smem, ctx->stream, out_rgba, gt_rgb,
-                                 width, height, lambda_ssim, dL_dout, ctx->ws.loss_partials,
+                                 width, height, lambda_ssim, ssim_window(), dL_dout, ctx->ws.loss_partials,
                                  ctx->ws.status + 1, loss_out));
 }
 
@@ -322,7 +330,7 @@ extern "C" abcd_status abcd_loss(abcd_ctx* ctx, const float* out_rgba, const flo
 namespace abcd {
 namespace {
 
-constexpr int kStaticLossMaxBlocks = 16384;            // 64x32-pixel CTAs: up to 8192 x 4096
+constexpr int kStaticLossMaxBlocks = 65536;            // CTAs (64x28 pixels, one channel): 8192 x 4096
 constexpr int kStaticLossWords = 2 * kStaticLossMaxBlocks + 64;   // partial sums, then the ticket
 
 // Device scratch shared by every abcd_loss_static call on a device (held until exit).
@@ -355,8 +363,8 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
   if (!out_rgba || !gt_rgb || width <= 0 || height <= 0 ||
       !(lambda_ssim >= 0.f && lambda_ssim <= 1.f))
     return ABCD_ERR_INVALID_ARG;
-  const dim3 grid((width + TW - 1) / TW, (height + TH - 1) / TH);
-  if ((long long)grid.x * grid.y > kStaticLossMaxBlocks) return ABCD_ERR_WORKSPACE;
+  const dim3 grid = loss_grid(width, height);
+  if ((long long)grid.x * grid.y * grid.z > kStaticLossMaxBlocks) return ABCD_ERR_WORKSPACE;
   int device = 0;
   if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices)
     return ABCD_ERR_CUDA;
@@ -372,7 +380,7 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
       cudaSuccess)
     return ABCD_ERR_CUDA;
   const cudaError_t e = launch_pdl(loss_kernel, grid, dim3(kThreads), smem, stream, out_rgba,
-                                   gt_rgb, width, height, lambda_ssim, dL_dout, partials, ticket,
-                                   loss_out);
+                                   gt_rgb, width, height, lambda_ssim, ssim_window(), dL_dout,
+                                   partials, ticket, loss_out);
   return e == cudaSuccess && cudaGetLastError() == cudaSuccess ? ABCD_OK : ABCD_ERR_CUDA;
 }
