@@ -42,7 +42,10 @@ struct Workspace {
   unsigned* status;                 // [0] status word, [1] loss ticket
   unsigned long long* dsort[2];     // depth sort items [max_g]
   unsigned long long* pairs[2];     // (tile << 32 | id) items [max_pairs]
-  unsigned* hist;                   // [kRadixBins][kMaxRadixBlocks], then [kRadixBins] totals
+  unsigned* os_gh;                  // [2 sorts][4 passes][kRadixBins] digit counts
+  unsigned* os_ctr;                 // [2 sorts][2] tile and finished-CTA counters of a pass
+  unsigned long long* os_state;     // [os_tiles][kRadixBins] look-back words
+  long long os_tiles;
   int4* rects;                      // [max_g] tile rectangle per Gaussian
   unsigned* counts;                 // [max_g] listed tiles per Gaussian
   int* diff;                        // 2-D difference array over the tile grid
@@ -133,6 +136,7 @@ struct abcd_ctx {
   long long order_tiles = 0;
   abcd::SHConst sh{};
   long long launches = 0;
+  unsigned os_epoch = 0;                // last look-back epoch handed to a sort pass
   char err[512] = {0};
 };
 

@@ -24,9 +24,11 @@
 //      memory and written out coalesced;
 //   5. stable LSD radix sort of the K items on the tile bits only, in passes of equal width,
 //      which keeps depth order inside each tile; the last pass writes ids.
-// Radix passes are reduce-then-scan (per-block digit counts, per-digit row scans, stable
-// scatter): no inter-block waits, so nothing can spin.  Lanes of equal digit are ranked with
-// ballots on the low, scattered digits and with __match_any_sync on the high, grouped ones.
+// Radix sorts are one-sweep: one kernel counts the digits of all passes, then each pass is a
+// single kernel whose CTAs take tiles of items in order and find the offsets of their digits
+// by decoupled look-back over the tiles before theirs (bounded waits on CTAs that are already
+// running).  Lanes of equal digit are ranked with ballots on the low, scattered digits and
+// with __match_any_sync on the high, grouped ones.
 // Counts that live on the device (K) are read by the kernels themselves; grids are fixed, so
 // the step has no host sync.
 #include <algorithm>
@@ -64,8 +66,11 @@ __device__ __forceinline__ int4 tile_rect(float2 m, int r, int tiles_x, int tile
 // ---- per Gaussian: depth key (bits(depth) << 32 | id, all ones when culled) and the tile
 // rectangle of its square
 __global__ void keys_rects_kernel(const float* depth, const int* radius, const float2* uv, int n,
-                                  int tiles_x, int tiles_y, u64* items, int4* rects) {
+                                  int tiles_x, int tiles_y, u64* items, int4* rects,
+                                  unsigned* gh_zero, int gh_words) {
   pdl_prologue();
+  if (blockIdx.x == 0)                    // the radix sorts' digit counts start from zero
+    for (int k = threadIdx.x; k < gh_words; k += blockDim.x) gh_zero[k] = 0u;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   int4 q = make_int4(0, 0, 0, 0);
@@ -199,14 +204,12 @@ tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, i
   }
 }
 
-// Items per thread (hist) or per lane (scatter) loaded at once.
-constexpr int kRadixLoads = 8;
-
-template <typename T>
+// Items j = 0..U-1 of a warp's run: in[b0 + 32 j + lane] below wh (zero past it).
+template <typename T, int U>
 __device__ __forceinline__ void load_items(const T* in, long long b0, long long wh, int lane,
-                                           T (&xs)[kRadixLoads]) {
+                                           T (&xs)[U]) {
 #pragma unroll
-  for (int j = 0; j < kRadixLoads; ++j) {
+  for (int j = 0; j < U; ++j) {
     const long long i = b0 + 32 * j + lane;
     xs[j] = i < wh ? in[i] : (T)0;
   }
@@ -233,35 +236,7 @@ __device__ __forceinline__ unsigned match_digit(unsigned d, unsigned valid_mask)
   return peers;
 }
 
-// ---- radix pass, step 1: per-block digit counts hist[d * G + b]
-template <typename T>
-__global__ void __launch_bounds__(256)
-radix_hist_kernel(const T* in, long long n_static, const long long* n_dev, long long cap,
-                  int shift, unsigned mask, unsigned* hist, int G) {
-  pdl_prologue();
-  __shared__ unsigned h[kRadixBins];
-  for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) h[d] = 0;
-  __syncthreads();
-  const long long n = dev_count(n_static, n_dev, cap);
-  long long lo, hi;
-  block_range(n, G, &lo, &hi);
-  constexpr int U = kRadixLoads;
-  for (long long b0 = lo; b0 < hi; b0 += (long long)blockDim.x * U) {
-    unsigned d[U];
-#pragma unroll
-    for (int j = 0; j < U; ++j) {
-      const long long i = b0 + (long long)j * blockDim.x + threadIdx.x;
-      d[j] = i < hi ? ((unsigned)(in[i] >> shift) & mask) : 0x100u;
-    }
-#pragma unroll
-    for (int j = 0; j < U; ++j)
-      if (d[j] < 0x100u) atomicAdd(&h[d[j]], 1u);
-  }
-  __syncthreads();
-  for (int d = threadIdx.x; d < kRadixBins; d += blockDim.x) hist[d * G + blockIdx.x] = h[d];
-}
-
-// Exclusive scan of a block of per-thread sums (1024 threads).
+// Exclusive scan of a block of per-thread sums (any multiple of 32 threads up to 1024).
 __device__ __forceinline__ unsigned long long block_exclusive_scan(unsigned long long v,
                                                                    unsigned long long* total) {
   __shared__ unsigned long long warp_sums[32];
@@ -289,22 +264,6 @@ __device__ __forceinline__ unsigned long long block_exclusive_scan(unsigned long
   return before;
 }
 
-// ---- radix pass, step 2: exclusive scan of each digit's row hist[d][0..G) (one block per
-// digit); the row totals go to totals[d]
-__global__ void __launch_bounds__(1024) radix_rowscan_kernel(unsigned* hist, int G,
-                                                            unsigned* totals) {
-  pdl_prologue();
-  const int d = blockIdx.x;
-  const unsigned v = (int)threadIdx.x < G ? hist[d * G + threadIdx.x] : 0u;
-  unsigned long long tot = 0;
-  const unsigned long long ex = block_exclusive_scan(v, &tot);
-  if ((int)threadIdx.x < G) hist[d * G + threadIdx.x] = (unsigned)ex;
-  if (threadIdx.x == 0) totals[d] = (unsigned)tot;
-}
-
-// ---- radix pass, step 3: stable scatter of BITS-bit digits.  Each warp owns a contiguous
-// slice of the block's range; lanes of equal digit are ranked with match_digit, once per item
-// (the masks are kept for the scatter when the slice is one round of loads).
 // Lanes of the warp holding the same digit: one ballot per bit (a cost independent of how many
 // distinct digits the warp holds: the right choice for the low, scattered digits) or
 // __match_any_sync (fast when a warp holds few distinct digits: the high digits of depth keys and
@@ -315,77 +274,236 @@ __device__ __forceinline__ unsigned rank_peers(unsigned d, bool valid) {
   return match_digit<BITS>(d, __ballot_sync(0xffffffffu, valid));
 }
 
-template <typename T, int BITS, bool MATCH>
-__global__ void __launch_bounds__(256)
-radix_scatter_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
-                     const long long* n_dev, long long cap, int shift, const unsigned* hist,
-                     const unsigned* totals, int G) {
-  pdl_prologue();
-  constexpr int W = 8;
-  constexpr unsigned BINS = 1u << BITS, MASK = BINS - 1;
-  __shared__ unsigned cnt[W][BINS];
-  __shared__ unsigned base[kRadixBins];
-  {
-    // digit bases: exclusive scan of the digit totals (kRadixBins == blockDim.x; the totals of
-    // digits >= BINS are zero)
-    const unsigned t = totals[threadIdx.x];
-    unsigned long long tot = 0;
-    base[threadIdx.x] = (unsigned)block_exclusive_scan(t, &tot);
+// ---- one-sweep radix sort (decoupled look-back)
+// A sort of n items on bits [bit_lo, bit_hi) runs in passes of equal width.  One kernel counts
+// the digits of every pass at once; then each pass is a single kernel: CTAs claim tiles of
+// kOsWarps x 32 x U consecutive items in order (a global counter), rank each item among the
+// tile's items of equal digit (stable), publish the tile's per-digit counts, and add up the
+// counts of the tiles before theirs by looking back until a tile whose inclusive prefix is
+// published.  Item position = digit base + prefix of earlier tiles + rank in the tile.
+// A tile only waits for tiles claimed before it, whose CTAs are running, so the waits end;
+// each is bounded all the same (on expiry the status word gets ABCD_ERR_TIMEOUT and the pass
+// goes on with a wrong prefix instead of hanging).
+struct SortPasses {
+  int n;                 // passes (at most kMaxSortPasses)
+  int shift[4];          // low bit of each pass's digit
+  int bits[4];           // digit width of each pass (4..8)
+};
+// Passes of equal width (at least 4 bits) covering bits [bit_lo, bit_hi).
+__host__ __device__ inline SortPasses make_passes(int bit_lo, int bit_hi) {
+  SortPasses sp{};
+  const int nbits = bit_hi - bit_lo;
+  sp.n = (nbits + kRadixBits - 1) / kRadixBits;
+  const int width = (nbits + sp.n - 1) / sp.n > 4 ? (nbits + sp.n - 1) / sp.n : 4;
+  for (int p = 0; p < sp.n && p < 4; ++p) {
+    sp.shift[p] = bit_lo + p * width;
+    const int left = bit_hi - sp.shift[p];
+    sp.bits[p] = left < width ? (left < 4 ? 4 : left) : width;
   }
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  for (int k = threadIdx.x; k < W * (int)BINS; k += blockDim.x) (&cnt[0][0])[k] = 0;
+  return sp;
+}
+
+// Adds the digit counts of one tile's c items ((tile << bit_lo | id) items of a sort whose
+// passes `tp` are relative to the tile bits) to h.
+__device__ __forceinline__ void tile_digit_counts(unsigned t, unsigned c, const SortPasses& tp,
+                                                  unsigned (*h)[kRadixBins]) {
+  if (c == 0) return;
+  for (int p = 0; p < tp.n; ++p)
+    atomicAdd(&h[p][(t >> tp.shift[p]) & ((1u << tp.bits[p]) - 1u)], c);
+}
+
+constexpr int kOsWarps = 8;
+constexpr int kOsThreads = 32 * kOsWarps;
+constexpr unsigned kOsSpinLimit = 1u << 20;
+
+// Look-back state word: epoch (30 bits) | flag (2 bits: 1 aggregate, 2 inclusive) | count.
+// The epoch changes with every pass launch, so words left by earlier passes read as "not
+// published" and the array needs no clearing.
+__device__ __forceinline__ u64 os_word(unsigned epoch, unsigned flag, unsigned count) {
+  return ((u64)epoch << 34) | ((u64)flag << 32) | count;
+}
+
+__device__ __forceinline__ void os_publish(u64* p, u64 v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ u64 os_peek(const u64* p) {
+  u64 v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Digit counts of every pass: gh[p * kRadixBins + d] += count (gh zeroed by keys_rects).
+template <typename T>
+__global__ void __launch_bounds__(256)
+sort_digits_kernel(const T* in, long long n_static, const long long* n_dev, long long cap,
+                   SortPasses sp, int match_from, unsigned* gh) {
+  pdl_prologue();
+  __shared__ unsigned h[4][kRadixBins];
+  for (int k = threadIdx.x; k < 4 * kRadixBins; k += blockDim.x) (&h[0][0])[k] = 0;
   __syncthreads();
   const long long n = dev_count(n_static, n_dev, cap);
-  long long lo, hi;
-  block_range(n, G, &lo, &hi);
-  const long long wchunk = (hi - lo + W - 1) / W;
-  const long long wl = min(hi, lo + w * wchunk), wh = min(hi, wl + wchunk);
+  const int lane = threadIdx.x & 31;
   const unsigned lt = (1u << lane) - 1u;
-  constexpr int U = kRadixLoads;
-  // the warp's slice in rounds of 32 U items, all loaded at once; with one round (the usual
-  // case) the items and their peer masks stay in registers for the scatter
-  const int rounds = (int)((wh - wl + 32 * U - 1) / (32 * U));
-  T xs[U];
-  unsigned pm[U];
-  for (int r = 0; r < rounds; ++r) {
-    const long long b0 = wl + (long long)r * 32 * U;
-    load_items(in, b0, wh, lane, xs);
-#pragma unroll
-    for (int j = 0; j < U; ++j) {
-      if (b0 + 32 * j >= wh) break;                // warp-uniform
-      const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, wh, shift, MASK);
-      const unsigned peers = rank_peers<BITS, MATCH>(d, d < 0x100u);
-      pm[j] = peers;
-      if (d < 0x100u && (peers & lt) == 0) cnt[w][d] += __popc(peers);
-      __syncwarp();
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  // the loop runs while any lane of the warp has an item (the ranking is warp-collective)
+  for (long long b = (long long)blockIdx.x * blockDim.x + (threadIdx.x & ~31); b < n; b += stride) {
+    const long long i = b + lane;
+    const bool valid = i < n;
+    const T x = valid ? in[i] : (T)0;
+    for (int p = 0; p < sp.n; ++p) {
+      const unsigned d = valid ? (unsigned)(x >> sp.shift[p]) & ((1u << sp.bits[p]) - 1u) : 0x100u;
+      const unsigned peers = p >= match_from ? __match_any_sync(0xffffffffu, d) : match_byte(d);
+      if (valid && (peers & lt) == 0) atomicAdd(&h[p][d], __popc(peers));
     }
   }
   __syncthreads();
-  for (int d = threadIdx.x; d < (int)BINS; d += blockDim.x) {
-    unsigned run = base[d] + hist[d * G + blockIdx.x];
-    for (int k = 0; k < W; ++k) { const unsigned c = cnt[k][d]; cnt[k][d] = run; run += c; }
+  for (int k = threadIdx.x; k < sp.n * kRadixBins; k += blockDim.x) {
+    const unsigned c = (&h[0][0])[k];
+    if (c) atomicAdd(gh + k, c);
   }
-  __syncthreads();
-  for (int r = 0; r < rounds; ++r) {
-    const long long b0 = wl + (long long)r * 32 * U;
-    if (rounds > 1) load_items(in, b0, wh, lane, xs);
+}
+
+// One pass: stable scatter of the items of [0, n) by the BITS-bit digit at `shift`.  gh holds
+// this pass's digit counts; ctr[0] hands out tiles and ctr[1] counts finished CTAs (the last
+// one clears both); state holds kRadixBins words per tile.  On the last pass out_ids (when not
+// null) receives the bits id_mask of each item instead of the item.
+template <typename T, int BITS, bool MATCH>
+__global__ void __launch_bounds__(kOsThreads, 2)
+onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
+                const long long* n_dev, long long cap, int shift, const unsigned* gh, u64* state,
+                unsigned* ctr, unsigned epoch, unsigned* status) {
+  pdl_prologue();
+  constexpr unsigned BINS = 1u << BITS, MASK = BINS - 1;
+  constexpr int U = 64 / (int)sizeof(T);          // items per lane: 64 bytes in flight
+  constexpr int TILE = kOsThreads * U;
+  __shared__ unsigned cnt[kOsWarps][BINS];
+  __shared__ unsigned s_base[BINS];
+  __shared__ unsigned s_off[BINS];
+  __shared__ unsigned s_run[BINS];
+  __shared__ unsigned s_loc[BINS];                // start of each digit inside the tile
+  __shared__ T s_items[TILE];                     // the tile's items in digit order
+  __shared__ unsigned s_tile;
+  {
+    const unsigned v = threadIdx.x < BINS ? gh[threadIdx.x] : 0u;
+    const unsigned long long ex = block_exclusive_scan(v, nullptr);
+    if (threadIdx.x < BINS) s_base[threadIdx.x] = (unsigned)ex;
+  }
+  const long long n = dev_count(n_static, n_dev, cap);
+  const long long n_tiles = (n + TILE - 1) / TILE;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const unsigned lt = (1u << lane) - 1u;
+  for (;;) {
+    if (threadIdx.x == 0) s_tile = atomicAdd(ctr, 1u);
+    for (int k = threadIdx.x; k < kOsWarps * (int)BINS; k += kOsThreads) (&cnt[0][0])[k] = 0;
+    __syncthreads();
+    const long long t = s_tile;
+    if (t >= n_tiles) break;                         // block-uniform
+    const long long b0 = t * TILE + (long long)w * 32 * U;
+    T xs[U];
+    unsigned rk[U];
+    load_items(in, b0, n, lane, xs);
 #pragma unroll
     for (int j = 0; j < U; ++j) {
-      if (b0 + 32 * j >= wh) break;                // warp-uniform
-      const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, wh, shift, MASK);
+      const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, n, shift, MASK);
       const bool valid = d < 0x100u;
-      const unsigned peers =
-          rounds > 1 ? rank_peers<BITS, MATCH>(d, valid) : pm[j];
-      unsigned pos = 0;
-      if (valid) pos = cnt[w][d] + __popc(peers & lt);
+      const unsigned peers = rank_peers<BITS, MATCH>(d, valid);
+      rk[j] = valid ? cnt[w][d] + __popc(peers & lt) : 0u;
       __syncwarp();
-      if (valid) {
-        if (out_ids) out_ids[pos] = (unsigned)xs[j] & id_mask;
-        else out[pos] = xs[j];
-        if ((peers & lt) == 0) cnt[w][d] += __popc(peers);
-      }
+      if (valid && (peers & lt) == 0) cnt[w][d] += __popc(peers);
       __syncwarp();
     }
+    __syncthreads();
+    if (threadIdx.x < BINS) {
+      // warp bases per digit (exclusive over warps) and the tile's count: published at once
+      const unsigned d = threadIdx.x;
+      unsigned run = 0;
+#pragma unroll
+      for (int k = 0; k < kOsWarps; ++k) { const unsigned c = cnt[k][d]; cnt[k][d] = run; run += c; }
+      s_run[d] = run;
+      os_publish(state + (size_t)t * kRadixBins + d, os_word(epoch, t == 0 ? 2u : 1u, run));
+    }
+    __syncthreads();
+    {
+      // look-back: R threads per digit read 8 tiles each, nearest first, per round
+      constexpr int R = kOsThreads / (int)BINS;
+      constexpr int LB = 4;
+      const unsigned d = threadIdx.x / R;
+      const int q = threadIdx.x % R;
+      const unsigned gmask = R == 32 ? 0xffffffffu : (((1u << R) - 1u) << (lane & ~(R - 1)));
+      const int g0 = lane & ~(R - 1);
+      unsigned prefix = 0;
+      long long k0 = t - 1;                          // nearest tile not summed yet
+      unsigned spins = 0;
+      while (t > 0) {
+        u64 v[LB];
+#pragma unroll
+        for (int j = 0; j < LB; ++j) {
+          const long long k = k0 - (long long)LB * q - j;
+          v[j] = k >= 0 ? os_peek(state + (size_t)k * kRadixBins + d) : os_word(epoch, 2u, 0u);
+        }
+        unsigned sum = 0, used = LB;
+        int kind = 0;                                // 0: all aggregates, 1: inclusive, 2: blocked
+#pragma unroll
+        for (int j = 0; j < LB; ++j) {
+          if (kind != 0) continue;
+          const unsigned flag = (unsigned)(v[j] >> 32) & 3u;
+          if ((unsigned)(v[j] >> 34) != epoch || flag == 0u) { kind = 2; used = j; continue; }
+          sum += (unsigned)v[j];
+          if (flag == 2u) { kind = 1; used = j + 1; }
+        }
+        // combine the R windows in order (every thread of the group decides alike)
+        unsigned add = 0;
+        long long consumed = 0;
+        int res = 0;
+        for (int qq = 0; qq < R; ++qq) {
+          const unsigned sq = __shfl_sync(gmask, sum, g0 + qq);
+          const int kq = __shfl_sync(gmask, kind, g0 + qq);
+          const unsigned uq = __shfl_sync(gmask, used, g0 + qq);
+          if (res == 0) { add += sq; consumed += uq; res = kq; }
+        }
+        prefix += add;
+        k0 -= consumed;
+        if (res == 1) break;
+        if (res == 2) {
+          if (++spins > kOsSpinLimit) { if (q == 0) atomicOr(status, kStatusTimeout); break; }
+          __nanosleep(32);
+        }
+      }
+      if (q == 0) {
+        if (t > 0) os_publish(state + (size_t)t * kRadixBins + d, os_word(epoch, 2u, prefix + s_run[d]));
+        s_off[d] = s_base[d] + prefix;
+      }
+    }
+    {
+      // the tile's items in digit order in shared memory, then written out in that order:
+      // consecutive threads store consecutive addresses of a digit's run
+      const unsigned v = threadIdx.x < BINS ? s_run[threadIdx.x] : 0u;
+      const unsigned long long ex = block_exclusive_scan(v, nullptr);
+      if (threadIdx.x < BINS) s_loc[threadIdx.x] = (unsigned)ex;
+      __syncthreads();
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, n, shift, MASK);
+      if (d < 0x100u) s_items[s_loc[d] + cnt[w][d] + rk[j]] = xs[j];
+    }
+    __syncthreads();
+    const int in_tile = (int)min((long long)TILE, n - t * TILE);
+    for (int i = threadIdx.x; i < in_tile; i += kOsThreads) {
+      const T x = s_items[i];
+      const unsigned d = (unsigned)(x >> shift) & MASK;
+      const unsigned long long pos = (unsigned long long)s_off[d] + (unsigned)(i - (int)s_loc[d]);
+      if (pos < (unsigned long long)n) {             // always, unless a wait expired
+        if (out_ids) out_ids[pos] = (unsigned)x & id_mask;
+        else out[pos] = x;
+      }
+    }
+    __syncthreads();                                 // before the next tile reuses cnt, s_off
+  }
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(ctr + 1, 1u) == gridDim.x - 1) { ctr[0] = 0u; ctr[1] = 0u; }
   }
 }
 
@@ -427,8 +545,11 @@ scan_blocks_kernel(unsigned long long* block_sums, int G, long long* count, long
 // ---- tile ranges from the per-row difference array: prefix sums along each row -> per-tile
 // counts -> exclusive scan (one block).  Empty ranges when K overflowed the capacity.
 __global__ void __launch_bounds__(1024)
-ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, long long cap, unsigned* ranges) {
+ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, long long cap, unsigned* ranges,
+                        SortPasses tp, unsigned* gh) {
   pdl_prologue();
+  __shared__ unsigned dh[4][kRadixBins];
+  for (int k = threadIdx.x; k < 4 * kRadixBins; k += blockDim.x) (&dh[0][0])[k] = 0u;
   const int W1 = tiles_x + 1;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   for (int y = wid; y < tiles_y; y += nw) {                        // prefix along each row
@@ -457,8 +578,11 @@ ranges_from_diff_kernel(int* diff, int tiles_x, int tiles_y, long long cap, unsi
     const unsigned c = (unsigned)diff[(t / tiles_x) * W1 + (t % tiles_x)];
     ranges[2 * t] = ok ? (unsigned)run : 0u;
     ranges[2 * t + 1] = ok ? (unsigned)(run + c) : 0u;
+    tile_digit_counts((unsigned)t, c, tp, dh);
     run += c;
   }
+  __syncthreads();
+  for (int k = threadIdx.x; k < tp.n * kRadixBins; k += blockDim.x) gh[k] = (&dh[0][0])[k];
 }
 
 // ---- the same, with the difference array staged in shared memory (one load round trip
@@ -476,10 +600,12 @@ __device__ __forceinline__ unsigned count_bucket(unsigned c) {
 
 __global__ void __launch_bounds__(1024)
 ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, long long cap, unsigned* ranges,
-                    unsigned* tile_order) {
+                    unsigned* tile_order, SortPasses tp, unsigned* gh) {
   pdl_prologue();
   extern __shared__ int sd[];              // [(tiles_x + 1) (tiles_y + 1)] cells, then [nt] keys
   __shared__ unsigned hist[kOrderBuckets];
+  __shared__ unsigned dh[4][kRadixBins];   // digit counts of the tile sort's passes
+  for (int k = threadIdx.x; k < 4 * kRadixBins; k += blockDim.x) (&dh[0][0])[k] = 0u;
   const int W1 = tiles_x + 1, cells = W1 * (tiles_y + 1), nt = tiles_x * tiles_y;
   unsigned char* skey = reinterpret_cast<unsigned char*>(sd + cells);
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
@@ -526,9 +652,11 @@ ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, long long cap, un
     ranges[2 * t] = ok ? (unsigned)run : 0u;
     ranges[2 * t + 1] = ok ? (unsigned)(run + c) : 0u;
     skey[t] = (unsigned char)count_bucket(ok ? c : 0u);
+    tile_digit_counts((unsigned)t, c, tp, dh);
     run += c;
   }
   __syncthreads();
+  for (int k = threadIdx.x; k < tp.n * kRadixBins; k += blockDim.x) gh[k] = (&dh[0][0])[k];
   for (int i0 = 0; i0 < nt; i0 += blockDim.x) {
     const int i = i0 + threadIdx.x;
     const unsigned key = i < nt ? skey[i] : (unsigned)kOrderBuckets;
@@ -680,28 +808,29 @@ abcd_status emit_smem_attr(abcd_ctx* ctx) {
   return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "emit smem: %s", cudaGetErrorString(e));
 }
 
-// Launches the scatter of one radix pass for a digit of `bits` bits (4..8).
+// Launches one pass for a digit of `bits` bits (4..8).
 template <typename T>
-abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, bool match, int G,
-                           const T* src, T* dst, unsigned* ids, unsigned id_mask,
-                           long long n_static, const long long* n_dev, long long cap, int shift,
-                           const unsigned* totals) {
-#define ABCD_SCATTER(B)                                                                     \
-  case B:                                                                                   \
-    e = match ? launch_pdl(radix_scatter_kernel<T, B, true>, dim3(G), dim3(kRadixBins), 0, st, \
-                           src, dst, ids, id_mask, n_static, n_dev, cap, shift,             \
-                           (const unsigned*)ctx->ws.hist, totals, G)                        \
-              : launch_pdl(radix_scatter_kernel<T, B, false>, dim3(G), dim3(kRadixBins), 0, st, \
-                           src, dst, ids, id_mask, n_static, n_dev, cap, shift,             \
-                           (const unsigned*)ctx->ws.hist, totals, G);                       \
+abcd_status launch_onesweep(abcd_ctx* ctx, cudaStream_t st, int bits, bool match, int G,
+                            const T* src, T* dst, unsigned* ids, unsigned id_mask,
+                            long long n_static, const long long* n_dev, long long cap, int shift,
+                            const unsigned* gh, unsigned* ctr) {
+  const unsigned epoch = ++ctx->os_epoch;
+#define ABCD_PASS(B)                                                                              \
+  case B:                                                                                         \
+    e = match ? launch_pdl(onesweep_kernel<T, B, true>, dim3(G), dim3(kOsThreads), 0, st, src, dst, \
+                           ids, id_mask, n_static, n_dev, cap, shift, gh, ctx->ws.os_state, ctr,   \
+                           epoch, ctx->ws.status)                                                  \
+              : launch_pdl(onesweep_kernel<T, B, false>, dim3(G), dim3(kOsThreads), 0, st, src,    \
+                           dst, ids, id_mask, n_static, n_dev, cap, shift, gh, ctx->ws.os_state,   \
+                           ctr, epoch, ctx->ws.status);                                            \
     break;
   cudaError_t e = cudaSuccess;
   switch (bits) {
-    ABCD_SCATTER(4) ABCD_SCATTER(5) ABCD_SCATTER(6) ABCD_SCATTER(7) ABCD_SCATTER(8)
+    ABCD_PASS(4) ABCD_PASS(5) ABCD_PASS(6) ABCD_PASS(7) ABCD_PASS(8)
     default: return fail(ctx, ABCD_ERR_INVALID_ARG, "radix digit of %d bits", bits);
   }
-#undef ABCD_SCATTER
-  return check_launch(ctx, "radix_scatter_kernel", e);
+#undef ABCD_PASS
+  return check_launch(ctx, "onesweep_kernel", e);
 }
 
 // First pass ranked with __match_any_sync (earlier passes use ballots): the depth keys' two
@@ -709,35 +838,38 @@ abcd_status launch_scatter(abcd_ctx* ctx, cudaStream_t st, int bits, bool match,
 constexpr int kDepthMatchFrom = 2;
 constexpr int kTileMatchFrom = 1;
 
-// LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi), in the fewest passes of at
-// most 8 bits, of equal width (fewer bits per pass: fewer ballots per ranked item); returns
-// the buffer holding the result, or writes the bits id_mask of the sorted items to ids_out on
-// the last pass.
+// Stable LSD radix sort of 32- or 64-bit items on bits [bit_lo, bit_hi), in the fewest
+// one-sweep passes of at most 8 bits, of equal width (fewer bits per pass: fewer ballots per
+// ranked item); returns the buffer holding the result, or writes the bits id_mask of the
+// sorted items to ids_out on the last pass.  `slot` (0: depth sort, 1: tile sort) selects the
+// digit counts and tile counters.  n_max bounds the item count (it sizes the grid).
 template <typename T>
 abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_static,
-                       const long long* n_dev, long long cap, int bit_lo, int bit_hi, int G,
-                       T** result, unsigned* ids_out, unsigned id_mask, int match_from) {
-  unsigned* totals = ctx->ws.hist + kRadixBins * G;
+                       const long long* n_dev, long long cap, long long n_max, int bit_lo,
+                       int bit_hi, int slot, bool counted, T** result, unsigned* ids_out,
+                       unsigned id_mask, int match_from) {
+  const SortPasses sp = make_passes(bit_lo, bit_hi);
+  if (sp.n < 1 || sp.n > 4) return fail(ctx, ABCD_ERR_INVALID_ARG, "radix sort of %d bits", bit_hi - bit_lo);
+  unsigned* gh = ctx->ws.os_gh + (size_t)slot * 4 * kRadixBins;
+  unsigned* ctr = ctx->ws.os_ctr + 2 * slot;
+  const long long tile = (long long)kOsThreads * (64 / (int)sizeof(T));
+  const long long tiles = (n_max + tile - 1) / tile;
+  if (tiles > ctx->ws.os_tiles) return fail(ctx, ABCD_ERR_WORKSPACE, "radix sort: %lld tiles exceed the workspace", tiles);
+  const int G = (int)std::max<long long>(1, std::min<long long>(tiles, 4LL * ctx->num_sms));
+  const int Gd = (int)std::max<long long>(1, std::min<long long>((n_max + 255) / 256, 2LL * ctx->num_sms));
+  abcd_status s = ABCD_OK;
+  if (!counted &&                              // the tile sort's counts come with the ranges
+      (s = check_launch(ctx, "sort_digits_kernel",
+                        launch_pdl(sort_digits_kernel<T>, dim3(Gd), dim3(256), 0, st, (const T*)a,
+                                   n_static, n_dev, cap, sp, match_from, gh))))
+    return s;
   T* src = a;
   T* dst = b;
-  const int nbits = bit_hi - bit_lo;
-  const int passes = (nbits + kRadixBits - 1) / kRadixBits;
-  const int width = std::max(4, (nbits + passes - 1) / passes);
-  for (int shift = bit_lo, pass = 0; shift < bit_hi; shift += width, ++pass) {
-    const int bits = std::min(width, bit_hi - shift) < 4 ? 4 : std::min(width, bit_hi - shift);
-    const bool last = shift + width >= bit_hi;
-    abcd_status s = check_launch(
-        ctx, "radix_hist_kernel",
-        launch_pdl(radix_hist_kernel<T>, dim3(G), dim3(256), 0, st, (const T*)src, n_static,
-                   n_dev, cap, shift, (1u << bits) - 1u, ctx->ws.hist, G));
-    if (s) return s;
-    if ((s = check_launch(ctx, "radix_rowscan_kernel",
-                          launch_pdl(radix_rowscan_kernel, dim3(kRadixBins), dim3(((G + 31) / 32) * 32),
-                                     0, st, ctx->ws.hist, G, totals))))
-      return s;
-    if ((s = launch_scatter<T>(ctx, st, bits, pass >= match_from, G, src, dst,
-                               last ? ids_out : nullptr, id_mask, n_static, n_dev, cap, shift,
-                               totals)))
+  for (int p = 0; p < sp.n; ++p) {
+    const bool last = p == sp.n - 1;
+    if ((s = launch_onesweep<T>(ctx, st, sp.bits[p], p >= match_from, G, src, dst,
+                                last ? ids_out : nullptr, id_mask, n_static, n_dev, cap,
+                                sp.shift[p], gh + p * kRadixBins, ctr)))
       return s;
     T* t = src; src = dst; dst = t;
   }
@@ -775,6 +907,11 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
     e = cudaMemsetAsync(out->count, 0, sizeof(long long), ctx->stream);
     return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "count memset: %s", cudaGetErrorString(e));
   }
+  if (ctx->os_epoch > (1u << 30) - 64) {     // look-back epochs wrap: clear the old words
+    e = cudaMemsetAsync(ctx->ws.os_state, 0, 8ull * kRadixBins * (size_t)ctx->ws.os_tiles, ctx->stream);
+    if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "sort state memset: %s", cudaGetErrorString(e));
+    ctx->os_epoch = 0;
+  }
   const size_t diff_bytes = sizeof(int) * (size_t)(tiles_x + 1) * (tiles_y + 1);
   if (diff_bytes > ctx->ws.diff_bytes)
     return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_bin_sort: tile grid exceeds the workspace");
@@ -782,11 +919,16 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "diff memset: %s", cudaGetErrorString(e));
   abcd_status s;
   const float alpha_min = make_opts(opts).alpha_min;
+  int tile_bits = 1;
+  while ((1LL << tile_bits) < n_tiles) ++tile_bits;
+  // digit counts of the tile sort's passes, made with the tile ranges
+  const SortPasses tile_passes = make_passes(0, tile_bits);
+  unsigned* tile_gh = ctx->ws.os_gh + 4 * kRadixBins;
   if ((s = check_launch(ctx, "keys_rects_kernel",
                         launch_pdl(keys_rects_kernel, dim3((n + 255) / 256), dim3(256), 0, ctx->stream,
                                    (const float*)proj->depth, (const int*)proj->radius,
                                    (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
-                                   ctx->ws.rects))))
+                                   ctx->ws.rects, ctx->ws.os_gh, 2 * 4 * kRadixBins))))
     return s;
   // the depth sort only needs the keys: it runs on the side stream while the tile rows and
   // ranges are made here
@@ -795,9 +937,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort fork: %s", cudaGetErrorString(e));
   u64* by_depth = nullptr;
   {
-    const int G = std::min(kMaxRadixBlocks, std::max(16, (n + 2047) / 2048));
-    if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, 32,
-                             64, G, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom)))
+    if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, n,
+                             32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom)))
       return s;
   }
   e = cudaEventRecord(ctx->ev_join, ctx->side);
@@ -828,14 +969,15 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       if ((s = check_launch(ctx, "ranges_order_kernel",
                             launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->stream,
                                        (const int*)ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges,
-                                       ctx->ws.tile_order))))
+                                       ctx->ws.tile_order, tile_passes, tile_gh))))
         return s;
       ctx->order_ranges = out->ranges;           // the order belongs to these ranges
       ctx->order_tiles = n_tiles;
     } else {
       if ((s = check_launch(ctx, "ranges_from_diff_kernel",
                             launch_pdl(ranges_from_diff_kernel, dim3(1), dim3(1024), 0, ctx->stream,
-                                       ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges))))
+                                       ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges,
+                                       tile_passes, tile_gh))))
         return s;
     }
   }
@@ -851,8 +993,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                         launch_pdl(scan_blocks_kernel, dim3(1), dim3(1024), 0, ctx->stream,
                                    ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status))))
     return s;
-  int tile_bits = 1;
-  while ((1LL << tile_bits) < n_tiles) ++tile_bits;
   int id_bits = 1;
   while ((1LL << id_bits) < n) ++id_bits;
   // K lives on the device: the tile passes take the largest grid; blocks past K exit at once.
@@ -870,8 +1010,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                      (const long long*)out->count, cap, tiles_x, alpha_min, id_bits,
                                      pairs, Ge))))
       return s;
-    return radix_sort<unsigned>(ctx, ctx->stream, pairs, pairs_b, 0, out->count, cap, id_bits,
-                                id_bits + tile_bits, kMaxRadixBlocks, nullptr, out->ids,
+    return radix_sort<unsigned>(ctx, ctx->stream, pairs, pairs_b, 0, out->count, cap, cap, id_bits,
+                                id_bits + tile_bits, 1, true, nullptr, out->ids,
                                 (1u << id_bits) - 1u, kTileMatchFrom);
   }
   if ((s = emit_smem_attr<u64>(ctx))) return s;
@@ -885,6 +1025,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    ctx->ws.pairs[0], Ge))))
     return s;
   return radix_sort<u64>(ctx, ctx->stream, ctx->ws.pairs[0], ctx->ws.pairs[1], 0, out->count, cap,
-                         32, 32 + tile_bits, kMaxRadixBlocks, nullptr, out->ids, 0xffffffffu,
+                         cap, 32, 32 + tile_bits, 1, true, nullptr, out->ids, 0xffffffffu,
                          kTileMatchFrom);
 }

@@ -143,7 +143,11 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.dsort[1] = (unsigned long long*)take(8ull * (size_t)max_g);
   w.pairs[0] = (unsigned long long*)take(8ull * (size_t)max_pairs);
   w.pairs[1] = (unsigned long long*)take(8ull * (size_t)max_pairs);
-  w.hist = (unsigned*)take(4ull * kRadixBins * (kMaxRadixBlocks + 1));
+  w.os_gh = (unsigned*)take(4ull * 2 * 4 * kRadixBins);
+  w.os_ctr = (unsigned*)take(256);
+  // sort tiles hold 2048 32-bit or 1024 64-bit items
+  w.os_tiles = (std::max<long long>(max_pairs, max_g) + 1023) / 1024 + 1;
+  w.os_state = (unsigned long long*)take(8ull * kRadixBins * (size_t)w.os_tiles);
   w.rects = (int4*)take(16ull * (size_t)max_g);
   w.counts = (unsigned*)take(4ull * (size_t)max_g);
   w.diff_bytes = 4ull * kMaxDiffCells;
@@ -184,6 +188,10 @@ abcd_status abcd_set_workspace(abcd_ctx* ctx, void* ptr, size_t bytes, int max_g
   ctx->max_pixels = max_pixels;
   layout(ctx->ws_base, max_gaussians, max_pairs, max_pixels, &ctx->ws);
   cudaError_t e = cudaMemsetAsync(ctx->ws.status, 0, 256, ctx->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.os_ctr, 0, 256, ctx->stream);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(ctx->ws.os_state, 0, 8ull * kRadixBins * (size_t)ctx->ws.os_tiles, ctx->stream);
+  ctx->os_epoch = 0;
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "clearing status: %s", cudaGetErrorString(e));
   return ABCD_OK;
 }
