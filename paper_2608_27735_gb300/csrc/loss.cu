@@ -23,16 +23,22 @@ namespace {
 
 constexpr int TW = 64;            // output tile (pixels)
 constexpr int TH = 28;
-constexpr int RUN = 8;            // outputs per thread per window pass
+// Outputs per thread in each window pass (a run reads RUN + 10 staged values), chosen so that
+// every pass is one round over the CTA's 480 threads with few idle: 480, 444, 418 and 448 runs.
+constexpr int RUN = 8;            // horizontal moments
+constexpr int RUN_V = 7;          // vertical moments
+constexpr int RUN_H3 = 6;         // horizontal windows of A, B, C
+constexpr int RUN_V3 = 4;         // vertical windows of A, B, C
 constexpr int IW = TW + 20, IH = TH + 20;    // inputs: tile + 10-pixel halo
 constexpr int MW = TW + 10, MH = TH + 10;    // windowed moments: tile + 5-pixel halo
 constexpr int HSEG = (MW + RUN - 1) / RUN;   // column runs of the horizontal moment pass
-constexpr int VSEG = (MH + RUN - 1) / RUN;   // row runs of the vertical moment pass
-constexpr int HSEG3 = TW / RUN;              // column runs of the horizontal A, B, C pass
-constexpr int VSEG3 = (TH + RUN - 1) / RUN;  // row runs of the vertical A, B, C pass
+constexpr int VSEG = (MH + RUN_V - 1) / RUN_V;     // row runs of the vertical moment pass
+constexpr int HSEG3 = (TW + RUN_H3 - 1) / RUN_H3;  // column runs of the horizontal A, B, C pass
+constexpr int VSEG3 = (TH + RUN_V3 - 1) / RUN_V3;  // row runs of the vertical A, B, C pass
 constexpr int kThreads = 480;                // 15 warps: one horizontal moment run per thread
-static_assert(IH * HSEG <= kThreads, "the horizontal moment pass is one round");
-static_assert(TW % RUN == 0 && MH >= RUN && TH >= RUN, "run tiling");
+static_assert(IH * HSEG <= kThreads && MW * VSEG <= kThreads && MH * HSEG3 <= kThreads &&
+              TW * VSEG3 <= kThreads, "every window pass is one round");
+static_assert(MH >= RUN_V && TW >= RUN_H3 && TH >= RUN_V3, "run tiling");
 // Row pitches are odd (consecutive lanes take consecutive rows in the horizontal passes and
 // consecutive columns in the vertical ones: no bank conflicts, also for the 8-byte pairs) and
 // wide enough that a horizontal run never reads past its row (values read beyond the valid
@@ -54,7 +60,7 @@ constexpr int kSmemFloats = kR0 + kR1;
 static_assert(IP >= IW && MP >= MW, "padded pitches");
 static_assert(3 * MH * MP <= kR0, "A, B, C fit in the input region");
 static_assert(3 * MH * TP <= kR1, "windows of A, B, C fit in the moment region");
-static_assert((HSEG3 - 1) * RUN + RUN + 10 <= MP, "horizontal A, B, C runs stay in a row");
+static_assert(TW - RUN_H3 + RUN_H3 + 10 <= MW, "horizontal A, B, C runs stay in the valid columns");
 static_assert(kR0 % 2 == 0 && (2 * MH * MP) % 2 == 0 && (2 * IH * MP) % 2 == 0, "pairs 8-byte aligned");
 static_assert(sizeof(float) * kSmemFloats <= 110 * 1024, "two CTAs per SM");
 
@@ -62,11 +68,12 @@ struct Window {
   float w[11];      // normalised 11-tap Gaussian, sigma 1.5
 };
 
-// RUN outputs of an 11-tap window from RUN + 10 staged pairs / values.
-__device__ __forceinline__ void window_pairs(const float2 (&v)[RUN + 10], const Window& win,
-                                             float2 (&out)[RUN]) {
+// N outputs of an 11-tap window from N + 10 staged pairs / values.
+template <int N>
+__device__ __forceinline__ void window_pairs(const float2 (&v)[N + 10], const Window& win,
+                                             float2 (&out)[N]) {
 #pragma unroll
-  for (int o = 0; o < RUN; ++o) {
+  for (int o = 0; o < N; ++o) {
     float2 a = make_float2(0.f, 0.f);
 #pragma unroll
     for (int t = 0; t < 11; ++t) a = __ffma2_rn(make_float2(win.w[t], win.w[t]), v[o + t], a);
@@ -74,10 +81,11 @@ __device__ __forceinline__ void window_pairs(const float2 (&v)[RUN + 10], const 
   }
 }
 
-__device__ __forceinline__ void window_scalars(const float (&v)[RUN + 10], const Window& win,
-                                               float (&out)[RUN]) {
+template <int N>
+__device__ __forceinline__ void window_scalars(const float (&v)[N + 10], const Window& win,
+                                               float (&out)[N]) {
 #pragma unroll
-  for (int o = 0; o < RUN; ++o) {
+  for (int o = 0; o < N; ++o) {
     float a = 0.f;
 #pragma unroll
     for (int t = 0; t < 11; ++t) a = fmaf(win.w[t], v[o + t], a);
@@ -104,17 +112,29 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
   const float inv = 1.f / (3.f * (float)W * (float)H);
   const float C1 = 0.01f * 0.01f, C2 = 0.03f * 0.03f;
   float l1 = 0.f, ssim = 0.f;
-  // ---- inputs with a 10-pixel halo, zero outside the image
-  for (int k = threadIdx.x; k < IH * IP; k += kThreads) {
-    const int r = k / IP, c = k - r * IP;
-    const int gy = oy - 10 + r, gx = ox - 10 + c;
-    float xv = 0.f, yv = 0.f;
-    if (c < IW && gx >= 0 && gx < W && gy >= 0 && gy < H) {
-      const long long p = (long long)gy * W + gx;
-      xv = __ldg(xin + 4 * p + ch);
-      yv = __ldg(yin + 3 * p + ch);
+  // ---- inputs with a 10-pixel halo, zero outside the image (all loads issued before the
+  // first store: one memory round trip)
+  {
+    constexpr int kLoads = (IH * IP + kThreads - 1) / kThreads;
+    float xv[kLoads], yv[kLoads];
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) {
+      const int k = threadIdx.x + j * kThreads;
+      const int r = k / IP, c = k - r * IP;
+      const int gy = oy - 10 + r, gx = ox - 10 + c;
+      xv[j] = 0.f;
+      yv[j] = 0.f;
+      if (k < IH * IP && c < IW && gx >= 0 && gx < W && gy >= 0 && gy < H) {
+        const long long p = (long long)gy * W + gx;
+        xv[j] = __ldg(xin + 4 * p + ch);
+        yv[j] = __ldg(yin + 3 * p + ch);
+      }
     }
-    sXY[k] = make_float2(xv, yv);
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) {
+      const int k = threadIdx.x + j * kThreads;
+      if (k < IH * IP) sXY[k] = make_float2(xv[j], yv[j]);
+    }
   }
   __syncthreads();
   // ---- horizontal windows of (x, y), (x^2, y^2) and xy: RUN outputs per run
@@ -123,7 +143,7 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
     float2 v[RUN + 10], o2[RUN];
 #pragma unroll
     for (int t = 0; t < RUN + 10; ++t) v[t] = sXY[r * IP + c0 + t];
-    window_pairs(v, win, o2);
+    window_pairs<RUN>(v, win, o2);
 #pragma unroll
     for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hM[r * MP + c0 + o] = o2[o];
     float p[RUN + 10], o1[RUN];
@@ -132,38 +152,38 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
       p[t] = v[t].x * v[t].y;
       v[t] = __fmul2_rn(v[t], v[t]);
     }
-    window_pairs(v, win, o2);
+    window_pairs<RUN>(v, win, o2);
 #pragma unroll
     for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hS[r * MP + c0 + o] = o2[o];
-    window_scalars(p, win, o1);
+    window_scalars<RUN>(p, win, o1);
 #pragma unroll
     for (int o = 0; o < RUN; ++o) if (c0 + o < MW) hC[r * MP + c0 + o] = o1[o];
   }
   __syncthreads();
   // ---- vertical windows -> moments -> SSIM and its partials A, B, C (zero off-image)
   for (int it = threadIdx.x; it < MW * VSEG; it += kThreads) {
-    const int c = it % MW, k0 = (it / MW) * RUN;
-    const int r0 = min(k0, MH - RUN);              // the last run starts early ...
+    const int c = it % MW, k0 = (it / MW) * RUN_V;
+    const int r0 = min(k0, MH - RUN_V);            // the last run starts early ...
     const int o0 = k0 - r0;                        // ... and skips what the run before made
-    float2 mm[RUN], ss[RUN];
-    float mc[RUN];
+    float2 mm[RUN_V], ss[RUN_V];
+    float mc[RUN_V];
     {
-      float2 col[RUN + 10];
+      float2 col[RUN_V + 10];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) col[t] = hM[(r0 + t) * MP + c];
-      window_pairs(col, win, mm);
+      for (int t = 0; t < RUN_V + 10; ++t) col[t] = hM[(r0 + t) * MP + c];
+      window_pairs<RUN_V>(col, win, mm);
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) col[t] = hS[(r0 + t) * MP + c];
-      window_pairs(col, win, ss);
+      for (int t = 0; t < RUN_V + 10; ++t) col[t] = hS[(r0 + t) * MP + c];
+      window_pairs<RUN_V>(col, win, ss);
     }
     {
-      float col[RUN + 10];
+      float col[RUN_V + 10];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) col[t] = hC[(r0 + t) * MP + c];
-      window_scalars(col, win, mc);
+      for (int t = 0; t < RUN_V + 10; ++t) col[t] = hC[(r0 + t) * MP + c];
+      window_scalars<RUN_V>(col, win, mc);
     }
 #pragma unroll
-    for (int o = 0; o < RUN; ++o) {
+    for (int o = 0; o < RUN_V; ++o) {
       if (o < o0) continue;
       const int r = r0 + o;
       const int gy = oy - 5 + r, gx = ox - 5 + c;
@@ -189,45 +209,46 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
   __syncthreads();
   // ---- horizontal windows of (A, B) and C: [MH][TW]
   for (int it = threadIdx.x; it < MH * HSEG3; it += kThreads) {
-    const int r = it % MH, c0 = (it / MH) * RUN;   // consecutive lanes: consecutive rows
+    const int r = it % MH, k0 = (it / MH) * RUN_H3;   // consecutive lanes: consecutive rows
+    const int c0 = min(k0, TW - RUN_H3), o0 = k0 - c0;
     {
-      float2 v[RUN + 10], o2[RUN];
+      float2 v[RUN_H3 + 10], o2[RUN_H3];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) v[t] = aAB[r * MP + c0 + t];
-      window_pairs(v, win, o2);
+      for (int t = 0; t < RUN_H3 + 10; ++t) v[t] = aAB[r * MP + c0 + t];
+      window_pairs<RUN_H3>(v, win, o2);
 #pragma unroll
-      for (int o = 0; o < RUN; ++o) gAB[r * TP + c0 + o] = o2[o];
+      for (int o = 0; o < RUN_H3; ++o) if (o >= o0) gAB[r * TP + c0 + o] = o2[o];
     }
     {
-      float v[RUN + 10], o1[RUN];
+      float v[RUN_H3 + 10], o1[RUN_H3];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) v[t] = aC[r * MP + c0 + t];
-      window_scalars(v, win, o1);
+      for (int t = 0; t < RUN_H3 + 10; ++t) v[t] = aC[r * MP + c0 + t];
+      window_scalars<RUN_H3>(v, win, o1);
 #pragma unroll
-      for (int o = 0; o < RUN; ++o) gC[r * TP + c0 + o] = o1[o];
+      for (int o = 0; o < RUN_H3; ++o) if (o >= o0) gC[r * TP + c0 + o] = o1[o];
     }
   }
   __syncthreads();
   // ---- vertical windows and the gradient on the output tile
   for (int it = threadIdx.x; it < TW * VSEG3; it += kThreads) {
-    const int c = it % TW, k0 = (it / TW) * RUN;
-    const int r0 = min(k0, TH - RUN), o0 = k0 - r0;
-    float2 gab[RUN];
-    float gc[RUN];
+    const int c = it % TW, k0 = (it / TW) * RUN_V3;
+    const int r0 = min(k0, TH - RUN_V3), o0 = k0 - r0;
+    float2 gab[RUN_V3];
+    float gc[RUN_V3];
     {
-      float2 v[RUN + 10];
+      float2 v[RUN_V3 + 10];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) v[t] = gAB[(r0 + t) * TP + c];
-      window_pairs(v, win, gab);
+      for (int t = 0; t < RUN_V3 + 10; ++t) v[t] = gAB[(r0 + t) * TP + c];
+      window_pairs<RUN_V3>(v, win, gab);
     }
     {
-      float v[RUN + 10];
+      float v[RUN_V3 + 10];
 #pragma unroll
-      for (int t = 0; t < RUN + 10; ++t) v[t] = gC[(r0 + t) * TP + c];
-      window_scalars(v, win, gc);
+      for (int t = 0; t < RUN_V3 + 10; ++t) v[t] = gC[(r0 + t) * TP + c];
+      window_scalars<RUN_V3>(v, win, gc);
     }
 #pragma unroll
-    for (int o = 0; o < RUN; ++o) {
+    for (int o = 0; o < RUN_V3; ++o) {
       const int gy = oy + r0 + o, gx = ox + c;
       if (o < o0 || gx >= W || gy >= H) continue;
       const long long q = (long long)gy * W + gx;
