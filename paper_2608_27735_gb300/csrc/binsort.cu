@@ -20,8 +20,8 @@
 //   3. exclusive scan of the pair counts in depth order: every Gaussian's output offset;
 //   4. emission of (tile << id_bits | id) items in depth order, 32-bit when tile and id bits
 //      fit (else 64-bit); the runs are recomputed with the same round-to-nearest arithmetic,
-//      so they match step 1 bit for bit; each warp's contiguous output is built in shared
-//      memory and written out coalesced;
+//      so they match step 1 bit for bit; each warp writes its Gaussians' contiguous output in
+//      order, consecutive lanes on consecutive pairs;
 //   5. stable LSD radix sort of the K items on the tile bits only, in passes of equal width,
 //      which keeps depth order inside each tile; the last pass writes ids.
 // Radix sorts are one-sweep: one kernel counts the digits of all passes, then each pass is a
@@ -693,15 +693,34 @@ ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, long long cap, un
 }
 
 // ---- emission of (tile << id_bits | id) in depth order.  A warp takes 32 consecutive
-// Gaussians of the depth order, whose pairs fill one contiguous range of the output; it builds
-// that range in its shared-memory buffer when it fits (else writes in place) and copies it out
-// with coalesced stores.  A lane writes the pairs of its own Gaussian when it has at most
-// kEmitSmall (its rows one after the other); the warp writes the larger ones together, one at a
-// time: lanes compute the row runs, a warp scan places them, and consecutive lanes take
-// consecutive pairs (the row of pair k found by a search over the scan).
-constexpr int kEmitSmall = 64;
-constexpr int kEmitBufBytes = 8192;             // per warp
+// Gaussians of the depth order, whose pairs fill one contiguous range of the output, and
+// writes that range in order with coalesced stores, all lanes busy whatever the Gaussians'
+// sizes: the warp's (Gaussian, tile row) pairs are taken 32 at a time (lane l: pair l of the
+// round, its Gaussian found by a search over the scan of row counts), each lane computes its
+// row's run of tiles, a warp scan places the runs, and consecutive lanes take consecutive
+// output pairs (the run of pair k found by a search over that scan).
 constexpr int kEmitThreads = 256;
+
+// Lanes 0..31 hold an inclusive scan `incl`; returns the number of lanes whose value is <= k
+// (clamped to 31): the lane whose range holds k.  Every lane must call it.
+__device__ __forceinline__ int scan_search(unsigned incl, unsigned k) {
+  int rl = 0;
+#pragma unroll
+  for (int step = 16; step > 0; step >>= 1) {
+    const unsigned v = __shfl_sync(0xffffffffu, incl, rl + step - 1);
+    if (v <= k) rl += step;
+  }
+  return min(rl, 31);
+}
+
+__device__ __forceinline__ unsigned warp_inclusive_scan(unsigned v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned y = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += y;
+  }
+  return v;
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kEmitThreads)
@@ -709,13 +728,13 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
             const unsigned* counts, const unsigned long long* block_off, const long long* count,
             long long cap, int tiles_x, float alpha_min, int id_bits, T* pairs, int G) {
   pdl_prologue();
-  constexpr unsigned kBuf = kEmitBufBytes / sizeof(T);
-  extern __shared__ __align__(16) unsigned char emit_smem[];
+  __shared__ Splat s_sp[kEmitThreads];
+  __shared__ int4 s_q[kEmitThreads];
+  __shared__ unsigned s_id[kEmitThreads];
   if (*count > cap) return;
   long long lo, hi;
   block_range(n, G, &lo, &hi);
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  T* buf = reinterpret_cast<T*>(emit_smem) + (size_t)w * kBuf;
   unsigned long long run = block_off[blockIdx.x];
   for (long long base = lo; base < hi; base += blockDim.x) {
     const long long i = base + threadIdx.x;
@@ -730,82 +749,48 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
     unsigned long long tot = 0;
     const unsigned long long off = run + block_exclusive_scan(t, &tot);
     run += tot;
+    s_sp[threadIdx.x] = sm_;
+    s_q[threadIdx.x] = qm;
+    s_id[threadIdx.x] = id;
     const unsigned long long off0 = __shfl_sync(0xffffffffu, off, 0);
-    const unsigned R = (unsigned)(__shfl_sync(0xffffffffu, off + t, 31) - off0);
-    const bool staged = R <= kBuf;                   // warp-uniform
-    T* out = staged ? buf : pairs + off0;            // this warp's range, from off0
-    if (t > 0 && t <= (unsigned)kEmitSmall) {
-      unsigned at = (unsigned)(off - off0);
-      const unsigned stop = at + t;
-      for (int ty = qm.y; ty < qm.w && at < stop; ++ty) {
-        const int2 r = row_run(sm_, qm, ty);
-        for (int x = r.x; x < r.y && at < stop; ++x)
-          out[at++] = ((T)(unsigned)(ty * tiles_x + x) << id_bits) | (T)id;
-      }
-    }
-    unsigned big = __ballot_sync(0xffffffffu, t > (unsigned)kEmitSmall);
-    while (big) {
-      const int j = __ffs(big) - 1;
-      big &= big - 1;
-      const unsigned tj = __shfl_sync(0xffffffffu, t, j);
-      const unsigned idj = __shfl_sync(0xffffffffu, id, j);
-      const unsigned oj = (unsigned)(__shfl_sync(0xffffffffu, off, j) - off0);
-      // lane j prepared Gaussian j: broadcast its rectangle and ellipse
-      const int4 q = make_int4(__shfl_sync(0xffffffffu, qm.x, j), __shfl_sync(0xffffffffu, qm.y, j),
-                               __shfl_sync(0xffffffffu, qm.z, j), __shfl_sync(0xffffffffu, qm.w, j));
-      Splat s;
-      s.u = __shfl_sync(0xffffffffu, sm_.u, j);
-      s.v = __shfl_sync(0xffffffffu, sm_.v, j);
-      s.hb = __shfl_sync(0xffffffffu, sm_.hb, j);
-      s.lim = __shfl_sync(0xffffffffu, sm_.lim, j);
-      s.ym = __shfl_sync(0xffffffffu, sm_.ym, j);
-      s.dyl = __shfl_sync(0xffffffffu, sm_.dyl, j);
-      s.fal = __shfl_sync(0xffffffffu, sm_.fal, j);
-      s.det4 = __shfl_sync(0xffffffffu, sm_.det4, j);
-      s.inv2a = __shfl_sync(0xffffffffu, sm_.inv2a, j);
-      unsigned done = 0;
-      for (int y0 = q.y; y0 < q.w && done < tj; y0 += 32) {
-        const int ty = y0 + lane;
-        int2 r = make_int2(0, 0);
-        if (ty < q.w) r = row_run(s, q, ty);
-        const unsigned c = (unsigned)(r.y - r.x);
-        unsigned incl = c;
-        for (int o = 1; o < 32; o <<= 1) {
-          const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += y;
-        }
-        const unsigned total = __shfl_sync(0xffffffffu, incl, 31);
-        for (unsigned k0 = 0; k0 < total; k0 += 32) {     // uniform trip count: every lane
-          const unsigned k = k0 + lane;                      // takes part in the shuffles
-          // row holding pair k: the number of lanes whose inclusive count is <= k
-          int rl = 0;
-          for (int step = 16; step > 0; step >>= 1) {
-            const unsigned v = __shfl_sync(0xffffffffu, incl, rl + step - 1);
-            if (v <= k) rl += step;
-          }
-          rl = min(rl, 31);
-          const unsigned before = __shfl_sync(0xffffffffu, incl - c, rl);
-          const int xa = __shfl_sync(0xffffffffu, r.x, rl);
-          const unsigned at = done + k;
-          if (k < total && at < tj)
-            out[oj + at] = ((T)(unsigned)((y0 + rl) * tiles_x + xa + (int)(k - before)) << id_bits) | (T)idj;
-        }
-        done += total;
-      }
-    }
+    const unsigned R = (unsigned)(__shfl_sync(0xffffffffu, off + t, 31) - off0);   // warp's pairs
+    const unsigned rows = t > 0 ? (unsigned)(qm.w - qm.y) : 0u;
+    const unsigned rincl = warp_inclusive_scan(rows, lane);
+    const unsigned P = __shfl_sync(0xffffffffu, rincl, 31);
     __syncwarp();
-    if (staged)
-      for (unsigned k = lane; k < R; k += 32) pairs[off0 + k] = buf[k];
-    __syncwarp();                                    // the buffer is reused by the next round
+    unsigned done = 0;                               // pairs written by this warp so far
+    for (unsigned p0 = 0; p0 < P; p0 += 32) {
+      const unsigned pr = p0 + lane;                 // this lane's (Gaussian, row) pair
+      const int j = scan_search(rincl, pr);
+      const unsigned jfirst = __shfl_sync(0xffffffffu, rincl - rows, j);
+      int2 r = make_int2(0, 0);
+      int ty = 0;
+      unsigned idj = 0;
+      if (pr < P) {
+        const int slot = w * 32 + j;
+        const int4 q = s_q[slot];
+        ty = q.y + (int)(pr - jfirst);
+        r = row_run(s_sp[slot], q, ty);
+        idj = s_id[slot];
+      }
+      const unsigned c = (unsigned)(r.y - r.x);
+      const unsigned cincl = warp_inclusive_scan(c, lane);
+      const unsigned total = __shfl_sync(0xffffffffu, cincl, 31);
+      for (unsigned k0 = 0; k0 < total; k0 += 32) {  // uniform trip count: every lane
+        const unsigned k = k0 + lane;                // takes part in the shuffles
+        const int rl = scan_search(cincl, k);
+        const unsigned before = __shfl_sync(0xffffffffu, cincl - c, rl);
+        const int xa = __shfl_sync(0xffffffffu, r.x, rl);
+        const int tyl = __shfl_sync(0xffffffffu, ty, rl);
+        const unsigned idl = __shfl_sync(0xffffffffu, idj, rl);
+        const unsigned at = done + k;
+        if (k < total && at < R)
+          pairs[off0 + at] = ((T)(unsigned)(tyl * tiles_x + xa + (int)(k - before)) << id_bits) | (T)idl;
+      }
+      done += total;
+    }
+    __syncthreads();                                 // s_sp, s_q, s_id are refilled next round
   }
-}
-
-constexpr size_t kEmitSmem = (size_t)kEmitBufBytes * (kEmitThreads / 32);
-
-template <typename T>
-abcd_status emit_smem_attr(abcd_ctx* ctx) {
-  const cudaError_t e = cudaFuncSetAttribute(emit_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kEmitSmem);
-  return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "emit smem: %s", cudaGetErrorString(e));
 }
 
 // Launches one pass for a digit of `bits` bits (4..8).
@@ -1000,9 +985,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (tile_bits + id_bits <= 32) {
     unsigned* pairs = reinterpret_cast<unsigned*>(ctx->ws.pairs[0]);
     unsigned* pairs_b = reinterpret_cast<unsigned*>(ctx->ws.pairs[1]);
-    if ((s = emit_smem_attr<unsigned>(ctx))) return s;
     if ((s = check_launch(ctx, "emit_kernel",
-                          launch_pdl(emit_kernel<unsigned>, dim3(Ge), dim3(kEmitThreads), kEmitSmem,
+                          launch_pdl(emit_kernel<unsigned>, dim3(Ge), dim3(kEmitThreads), 0,
                                      ctx->stream, (const u64*)by_depth, n, (const float2*)proj->uv,
                                      (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
                                      (const unsigned*)ctx->ws.counts,
@@ -1014,9 +998,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                 id_bits + tile_bits, 1, true, nullptr, out->ids,
                                 (1u << id_bits) - 1u, kTileMatchFrom);
   }
-  if ((s = emit_smem_attr<u64>(ctx))) return s;
   if ((s = check_launch(ctx, "emit_kernel",
-                        launch_pdl(emit_kernel<u64>, dim3(Ge), dim3(kEmitThreads), kEmitSmem,
+                        launch_pdl(emit_kernel<u64>, dim3(Ge), dim3(kEmitThreads), 0,
                                    ctx->stream, (const u64*)by_depth, n, (const float2*)proj->uv,
                                    (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
                                    (const unsigned*)ctx->ws.counts,
