@@ -160,8 +160,8 @@ def test_bin_sort_ragged_and_sh3(ctx, ragged):
 
 
 def test_bin_sort_many_gaussians(ctx):
-    """More Gaussians (270,000) than the one-cluster depth sort takes (2^18): the depth order
-    comes from the multi-kernel radix passes instead."""
+    """270,000 Gaussians: the depth sort's one-sweep passes span 132 tiles (long look-back
+    chains), and the tile sort sees ids of 19 bits."""
     s = sg.grid_scene((1, 1, 1), 5.0, 270_000, 0, seed=91)
     s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 96, 64, seed=91,
                                 height_jitter=1.0)
