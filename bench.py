@@ -511,14 +511,8 @@ def run_ours(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded scenegen, shaped like the paper's 200-camera grid scenes)",
-        "config": {"workload": f"scene-scale ABCD stage: 4x4x2 grid x {args.per_cell} Gaussians/cell "
-                               f"(SH3), {args.cams} cameras {args.width}x{args.height}, active cell "
-                               f"{ACTIVE_CELL}, T={args.T} steps per stage, L1+0.2 D-SSIM",
-                   "bench_step": "one ABCD stage: composite F/B for the observing cameras (K1), "
-                                 "T active-block steps (K2-K9), cache refresh (K10)",
-                   "T": args.T, "observing_cameras": len(st.observing), "active_gaussians": st.n,
-                   "pairs_mean": round(st.k_mean), "parallelism": f"replicas x{world}",
-                   "l2": "stage inputs exceed L2 (cached layers 52 GB read per stage)"},
+        "config": stage_config(args, st.n, world),
+        "pairs_mean": round(st.k_mean),
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
@@ -666,6 +660,18 @@ def cpu_baseline(args, log):
                       f"{dt:.1f} s"}
 
 
+def stage_config(args, n_active, world):
+    """The workload both arms name (their JSON lines carry the same config)."""
+    return {"workload": f"scene-scale ABCD stage: 4x4x2 grid x {args.per_cell} Gaussians/cell "
+                        f"(SH3), {args.cams} cameras {args.width}x{args.height}, active cell "
+                        f"{ACTIVE_CELL}, T={args.T} steps per stage, L1+0.2 D-SSIM",
+            "bench_step": "one ABCD stage: composite F/B for the observing cameras (K1), "
+                          "T active-block steps (K2-K9), cache refresh (K10)",
+            "T": args.T, "observing_cameras": args.cams, "active_gaussians": int(n_active),
+            "parallelism": f"replicas x{world}",
+            "l2": "stage inputs exceed L2 (cached layers 52 GB read per stage)"}
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -683,13 +689,14 @@ def run_reference(args):
         oracle_step(oracle, ga, cam, F, B, gt, state)
     dt = time.perf_counter() - t0
     v = args.steps / dt
-    sample = (f"each step: one active-block step of the scene-scale workload on one camera "
-              f"({ga.n} Gaussians, {args.width}x{args.height})")
+    sample = (f"each timed step: one active-block step (K2-K9) of this workload on one camera "
+              f"({ga.n} Gaussians, {args.width}x{args.height}); steps/s of the same unit as the "
+              f"other arm's value")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": round(v, 5), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt * 1e3 / args.steps, 1),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": "scene-scale active block, one camera per step"},
+        "data": "synthetic", "config": stage_config(args, ga.n, world),
         "cpu_baseline": {"value": round(v, 5), "unit": UNIT, "cores": oracle.cpu_threads(),
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(v, 5), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
