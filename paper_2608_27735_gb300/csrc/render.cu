@@ -40,7 +40,7 @@ constexpr int kSubPerTile = (kTile / kSub) * (kTile / kSub);
 static_assert(kSubPerTile == kRenderSubPerTile, "tile order expands to kRenderSubPerTile CTAs per tile");
 constexpr int kRounds = 2;                       // list entries per lane per staging group
 constexpr int kGroup = kSubThreads * kRounds;    // 64 entries loaded together
-constexpr int kBatch = 2 * kGroup;               // staged survivors per batch (at most)
+constexpr int kBatch = kGroup;                   // staged survivors per batch (at most)
 constexpr int kCkChunk = 128;                    // list positions per backward chunk
 constexpr int kItemCtasPerSm = 16;               // backward CTAs that replay listed chunks
 static_assert(kCkChunk % kGroup == 0, "checkpoints fall on staging group boundaries");
