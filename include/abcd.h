@@ -225,6 +225,44 @@ abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba, const flo
                              int width, int height, float lambda_ssim, float* loss_out,
                              float* dL_dout);
 
+/* ---- host tier of the layer cache (Section 2: the stored renders of the frozen
+ * partitions are kept in host memory and brought to the GPU when a stage composites them;
+ * refreshed renders go back).  Copies run on two copy streams of the context (host to
+ * device, device to host) and overlap the kernels on its stream; slots (e.g. one per camera)
+ * order them.  Host buffers should be pinned (cudaHostAlloc / cudaHostRegister); pageable
+ * memory makes a copy synchronous.  One cudaMemcpyAsync per call. ------------------------ */
+
+#define ABCD_MAX_CACHE_SLOTS 4096
+
+/* Queues a copy of `bytes` bytes from host_src (host) to dev_dst (device) for `slot`
+ * (0 <= slot < ABCD_MAX_CACHE_SLOTS).  It starts after the work that was queued on the
+ * context's stream before the slot's last abcd_cache_release (at once if there was none), so
+ * a slot's device data is not overwritten while a kernel still reads it.  Returns
+ * ABCD_ERR_INVALID_ARG for a null pointer, bytes == 0 or a bad slot (nothing queued),
+ * ABCD_ERR_CUDA if a copy or an event fails. */
+abcd_status abcd_cache_fetch(abcd_ctx* ctx, int slot, const void* host_src, void* dev_dst,
+                             size_t bytes);
+
+/* Makes the context's stream wait until every fetch and store of `slot` queued so far is
+ * done (nothing to wait for if there was none).  ABCD_ERR_INVALID_ARG for a bad slot. */
+abcd_status abcd_cache_wait(abcd_ctx* ctx, int slot);
+
+/* Marks the end of the reads of `slot`'s device data: later fetches of the slot start after
+ * the work queued on the context's stream so far.  ABCD_ERR_INVALID_ARG for a bad slot. */
+abcd_status abcd_cache_release(abcd_ctx* ctx, int slot);
+
+/* Queues a copy of `bytes` bytes from dev_src (device) to host_dst (host) for `slot` that
+ * starts after the work queued on the context's stream so far (a refreshed render going back
+ * to the host tier while the next stage computes); a later abcd_cache_wait(slot) also waits
+ * for it, so the device data is not rewritten before it has left.  ABCD_ERR_INVALID_ARG for a
+ * null pointer, bytes == 0 or a bad slot. */
+abcd_status abcd_cache_store(abcd_ctx* ctx, int slot, const void* dev_src, void* host_dst,
+                             size_t bytes);
+
+/* Waits until the context's queued fetches and stores are done (abcd_sync waits for its
+ * compute stream only). */
+abcd_status abcd_cache_sync(abcd_ctx* ctx);
+
 /* ---- host-side partition logic (Section 2: regular grid, assignment by mean) --------- */
 
 /* cell[i] = linear id (i + gx (j + gy k)) of the grid cell holding means[i] (host array,

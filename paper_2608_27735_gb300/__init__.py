@@ -21,6 +21,7 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "abcd.h")
 ABCD_OK, ABCD_ERR_INVALID_ARG, ABCD_ERR_CUDA, ABCD_ERR_CAPACITY, ABCD_ERR_TIMEOUT, \
     ABCD_ERR_WORKSPACE = range(6)
 ABCD_F16, ABCD_F32 = 0, 1
+ABCD_MAX_CACHE_SLOTS = 4096
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "CUDA", 3: "CAPACITY", 4: "TIMEOUT", 5: "WORKSPACE"}
 TILE = 16
 
@@ -94,6 +95,11 @@ _SIGS = {
                          C.c_float, C.c_float, C.c_float, C.c_int],
     "abcd_composite_cache": [C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p, C.c_int,
                              C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int],
+    "abcd_cache_fetch": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
+    "abcd_cache_wait": [C.c_void_p, C.c_int],
+    "abcd_cache_release": [C.c_void_p, C.c_int],
+    "abcd_cache_store": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
+    "abcd_cache_sync": [C.c_void_p],
     "abcd_assign_cells": [C.c_void_p, C.c_int, C.c_void_p, C.c_double, C.c_void_p, C.c_void_p],
     "abcd_partition_split": [C.c_void_p, C.c_void_p, C.c_double, C.c_void_p, C.c_int,
                              C.c_void_p, C.POINTER(C.c_int), C.c_void_p, C.POINTER(C.c_int)],
@@ -145,6 +151,12 @@ def _p(t):
     if t is None:
         return None
     assert t.is_cuda and t.is_contiguous(), "ABI arguments must be contiguous CUDA tensors"
+    return C.c_void_p(t.data_ptr())
+
+
+def _hp(t):
+    assert (not t.is_cuda) and t.is_contiguous() and t.is_pinned(), \
+        "host-tier buffers must be contiguous pinned host tensors"
     return C.c_void_p(t.data_ptr())
 
 
@@ -386,6 +398,31 @@ def abcd_composite_cache(ctx: Context, layers, order, split, width, height, F_ou
     ctx.check(lib().abcd_composite_cache(ctx.h, arr, L, int(layer_dtype), ordr, int(split),
                                          int(width), int(height), _p(F_out), _p(B_out),
                                          int(out_dtype)))
+
+
+def abcd_cache_fetch(ctx: Context, slot, host_src, dev_dst, nbytes=None):
+    """Queue host_src (pinned host tensor) -> dev_dst (CUDA tensor) for `slot`."""
+    n = host_src.numel() * host_src.element_size() if nbytes is None else int(nbytes)
+    ctx.check(lib().abcd_cache_fetch(ctx.h, int(slot), _hp(host_src), _p(dev_dst), n))
+
+
+def abcd_cache_wait(ctx: Context, slot):
+    ctx.check(lib().abcd_cache_wait(ctx.h, int(slot)))
+
+
+def abcd_cache_release(ctx: Context, slot):
+    ctx.check(lib().abcd_cache_release(ctx.h, int(slot)))
+
+
+def abcd_cache_store(ctx: Context, slot, dev_src, host_dst, nbytes=None):
+    """Queue dev_src (CUDA tensor) -> host_dst (pinned host tensor) for `slot`, after the
+    stream's work."""
+    n = dev_src.numel() * dev_src.element_size() if nbytes is None else int(nbytes)
+    ctx.check(lib().abcd_cache_store(ctx.h, int(slot), _p(dev_src), _hp(host_dst), n))
+
+
+def abcd_cache_sync(ctx: Context):
+    ctx.check(lib().abcd_cache_sync(ctx.h))
 
 
 def abcd_assign_cells(means_np, origin, side, dims):

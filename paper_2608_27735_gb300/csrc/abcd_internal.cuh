@@ -121,6 +121,13 @@ struct abcd_ctx {
   cudaStream_t stream = nullptr;
   cudaStream_t side = nullptr;          // forked work inside one call, joined before it returns
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // host tier of the layer cache (cache.cu): copy streams and per-slot events, made on first use
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  cudaEvent_t ev_store = nullptr;
+  cudaEvent_t* cache_ready = nullptr;           // [ABCD_MAX_CACHE_SLOTS]
+  cudaEvent_t* cache_released = nullptr;        // [ABCD_MAX_CACHE_SLOTS]
+  cudaEvent_t* cache_stored = nullptr;          // [ABCD_MAX_CACHE_SLOTS]
+  unsigned char* cache_has_release = nullptr;   // [ABCD_MAX_CACHE_SLOTS]
   int num_sms = 0;
   int radix_blocks = 0;
   char* ws_base = nullptr;
@@ -143,6 +150,7 @@ struct abcd_ctx {
 namespace abcd {
 
 abcd_status fail(abcd_ctx* ctx, abcd_status code, const char* fmt, ...);
+void cache_destroy(abcd_ctx* ctx);            // copy streams and slot events (cache.cu)
 abcd_status check_launch(abcd_ctx* ctx, const char* what);
 abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched);
 bool has_workspace(const abcd_ctx* ctx);

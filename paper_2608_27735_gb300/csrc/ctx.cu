@@ -120,6 +120,7 @@ abcd_status abcd_create(abcd_ctx** out, int device, void* stream) {
 
 abcd_status abcd_destroy(abcd_ctx* ctx) {
   if (!ctx) return ABCD_OK;
+  cache_destroy(ctx);
   if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
   if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
   if (ctx->side) cudaStreamDestroy(ctx->side);

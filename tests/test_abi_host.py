@@ -86,3 +86,18 @@ def test_no_cpu_fallback_without_gpu():
         pytest.skip("GPU present")
     with pytest.raises(RuntimeError):
         ab.Context(0)
+
+
+def test_cache_slot_count_matches_header():
+    import re
+    txt = open(ab.HEADER).read()
+    assert int(re.search(r"#define ABCD_MAX_CACHE_SLOTS (\d+)", txt).group(1)) == ab.ABCD_MAX_CACHE_SLOTS
+
+
+def test_cache_calls_reject_a_null_context(lib):
+    # argument checks come before any CUDA call (no GPU needed)
+    assert lib.abcd_cache_fetch(None, 0, None, None, 0) == ab.ABCD_ERR_INVALID_ARG
+    assert lib.abcd_cache_wait(None, 0) == ab.ABCD_ERR_INVALID_ARG
+    assert lib.abcd_cache_release(None, 0) == ab.ABCD_ERR_INVALID_ARG
+    assert lib.abcd_cache_store(None, 0, None, None, 0) == ab.ABCD_ERR_INVALID_ARG
+    assert lib.abcd_cache_sync(None) == ab.ABCD_ERR_INVALID_ARG

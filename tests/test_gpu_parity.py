@@ -387,6 +387,53 @@ def test_composite_cache_matches_oracle(ctx, dtype, out_dtype, H, W, L):
                 assert exact.mean() > 0.99
 
 
+def check_fb16(got, ref, L):
+    """fp16 composite output against the exact fold (fp32 accumulation, one rounding)."""
+    g = got.cpu().numpy()
+    m = L * 4 * 2.0 ** -24 * np.abs(ref)
+    lo, hi = (ref - m).astype(np.float16), (ref + m).astype(np.float16)
+    assert np.all((g >= lo) & (g <= hi))
+    exact = lo == hi
+    assert np.all(g[exact] == ref.astype(np.float16)[exact])
+
+
+def test_cache_host_tier_streams_layers(ctx):
+    """Host tier of the cache: two cameras' layers come from pinned host memory through ONE
+    device buffer (fetch on the copy stream, wait, composite, release), so the second fetch
+    must not land before the first composite has read the buffer; a composite goes back to
+    the host with a store."""
+    L, H, W = 6, 70, 90
+    cams = [sg.premultiplied_layers(L, H, W, seed=300 + c).astype(np.float16) for c in range(2)]
+    host = [torch.from_numpy(x).pin_memory() for x in cams]
+    dev = torch.empty(L, H, W, 4, dtype=torch.float16, device="cuda")
+    order = list(sg.random_permutation(L, seed=31))
+    split = 2
+    outs = []
+    for c in range(2):
+        ab.abcd_cache_fetch(ctx, 0, host[c], dev)
+        ab.abcd_cache_wait(ctx, 0)
+        Fo = torch.empty(H, W, 4, dtype=torch.float16, device="cuda")
+        Bo = torch.empty_like(Fo)
+        lay = [dev[k] for k in range(L)]
+        lay[order[split]] = None
+        ab.abcd_composite_cache(ctx, lay, order, split, W, H, Fo, Bo)
+        ab.abcd_cache_release(ctx, 0)
+        outs.append((Fo, Bo))
+    back = torch.empty(H, W, 4, dtype=torch.float16).pin_memory()
+    ab.abcd_cache_store(ctx, 1, outs[1][0], back)
+    ctx.sync()
+    ab.abcd_cache_sync(ctx)
+    for c in range(2):
+        src = cams[c].astype(np.float64)
+        check_fb16(outs[c][0], oracle.composite_layers(src, order[:split]), L)
+        check_fb16(outs[c][1], oracle.composite_layers(src, order[split + 1:]), L)
+    assert torch.equal(back, outs[1][0].cpu())
+    with pytest.raises(ab.AbcdError):
+        ab.abcd_cache_fetch(ctx, ab.ABCD_MAX_CACHE_SLOTS, host[0], dev)
+    with pytest.raises(ab.AbcdError):
+        ab.abcd_cache_wait(ctx, -1)
+
+
 def test_adam_matches_oracle(ctx, ragged):
     g = ragged.gaussians.subset(slice(0, 3001))
     theta = ab.Gaussians.from_numpy(g)
