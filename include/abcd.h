@@ -208,6 +208,34 @@ abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* layers, int L
                                  int layer_dtype, const int* order, int split, int width,
                                  int height, void* F_out, void* B_out, int out_dtype);
 
+/* Packed layers: the tile-sparse format of the cache (a lossless compression of the stored
+ * renders of Section 2, which are transparent wherever their partition puts no Gaussian).
+ * Over the 16x16-pixel tile grid of the image, tile_map[t] (int, [tiles]) is -1 for a tile
+ * that is not stored (every pixel (0, 0, 0, 0)), else the index of its block in `packed`:
+ * 16 x 16 fp16 RGBA pixels, row-major inside the tile (2 KB per block), blocks numbered in
+ * tile order.  Pixels of a stored border tile that fall outside the image are unspecified. */
+
+/* K10 into a packed layer: renders the active block alone (as abcd_render_composite_fwd's
+ * refresh_f16, F = B = transparent) and stores the tiles whose list (from abcd_bin_sort) is
+ * non-empty; a tile with an empty list renders (0, 0, 0, 0) exactly.  tile_map: device
+ * [tiles] int; packed: device, room for one block per tile, 16-byte aligned; count: device int
+ * receiving the number of stored tiles.  ABCD_ERR_INVALID_ARG for null or misaligned
+ * buffers. */
+abcd_status abcd_render_refresh_packed(abcd_ctx* ctx, const abcd_camera* cam,
+                                       const abcd_render_opts* opts, const abcd_projected* proj,
+                                       const abcd_tiles* tiles, int* tile_map, void* packed,
+                                       int* count);
+
+/* K1 over packed layers: the same folds as abcd_composite_cache (fp16 layers), with layer k
+ * given by tile_maps[k] and packed[k] (host arrays of L device pointers; NULL at the active
+ * position).  A tile a layer does not store is transparent for it, which leaves the fold
+ * unchanged, so the result equals abcd_composite_cache on the decoded layers bit for bit;
+ * only stored tiles are read. */
+abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_maps,
+                                        const void* const* packed, int L, const int* order,
+                                        int split, int width, int height, void* F_out,
+                                        void* B_out, int out_dtype);
+
 /* The loss of abcd_loss without a context or workspace, for callers that cannot allocate
  * device memory: code running inside a host application that owns every device allocation
  * (its own pool or arena, with raw cudaMalloc forbidden), or a caller that must not allocate

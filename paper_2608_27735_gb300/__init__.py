@@ -95,6 +95,10 @@ _SIGS = {
                          C.c_float, C.c_float, C.c_float, C.c_int],
     "abcd_composite_cache": [C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p, C.c_int,
                              C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int],
+    "abcd_render_refresh_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                   C.c_void_p, C.c_void_p, C.c_void_p],
+    "abcd_composite_cache_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
+                                    C.c_int, C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int],
     "abcd_cache_fetch": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
     "abcd_cache_wait": [C.c_void_p, C.c_int],
     "abcd_cache_release": [C.c_void_p, C.c_int],
@@ -398,6 +402,25 @@ def abcd_composite_cache(ctx: Context, layers, order, split, width, height, F_ou
     ctx.check(lib().abcd_composite_cache(ctx.h, arr, L, int(layer_dtype), ordr, int(split),
                                          int(width), int(height), _p(F_out), _p(B_out),
                                          int(out_dtype)))
+
+
+def abcd_render_refresh_packed(ctx: Context, cam, opts, proj, tiles, tile_map, packed, count):
+    """K10 into a packed layer: tile_map int32 [tiles], packed fp16 [tiles][16][16][4],
+    count int32 [1] (CUDA tensors)."""
+    p = proj.c(); t = tiles.c()
+    ctx.check(lib().abcd_render_refresh_packed(ctx.h, C.byref(cam), _opt(opts), C.byref(p),
+                                               C.byref(t), _p(tile_map), _p(packed), _p(count)))
+
+
+def abcd_composite_cache_packed(ctx: Context, tile_maps, packed, order, split, width, height,
+                                F_out, B_out, out_dtype=ABCD_F16):
+    """tile_maps / packed: lists of CUDA tensors (None at the active position)."""
+    L = len(tile_maps)
+    maps = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in tile_maps])
+    data = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in packed])
+    ordr = (C.c_int * max(1, L))(*[int(k) for k in order])
+    ctx.check(lib().abcd_composite_cache_packed(ctx.h, maps, data, L, ordr, int(split), int(width),
+                                                int(height), _p(F_out), _p(B_out), int(out_dtype)))
 
 
 def abcd_cache_fetch(ctx: Context, slot, host_src, dev_dst, nbytes=None):

@@ -167,3 +167,123 @@ extern "C" abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* la
               : launch_pdl(composite_kernel<1, false>, dim3(grid), dim3(256), 0, ctx->stream, lt, nf, nb, units, F_out, B_out, o16);
   return check_launch(ctx, "composite_kernel", e);
 }
+
+// ---- K1 over packed layers (the cache's tile-sparse format, see abcd_render_refresh_packed):
+// one CTA per 16x16 tile, two pixels per thread; a layer whose tile is not stored is
+// transparent, and folding (0, 0, 0, 0) leaves the accumulator unchanged, so skipping it gives
+// the dense result bit for bit.  Only the stored tiles are read.
+namespace abcd {
+namespace {
+
+struct PackedTable {
+  const int* map[kMaxLayers];       // front layers in order, then back layers in order
+  const uint4* data[kMaxLayers];    // 16-byte units: two fp16 RGBA pixels
+};
+
+constexpr int kPackedThreads = kTileThreads / 2;
+
+// acc (2 pixels) = acc over the two pixels of every layer in [k0, k1) stored at this tile
+__device__ __forceinline__ void fold_packed(const PackedTable& pt, int k0, int k1, int tile,
+                                            int unit, float* acc) {
+  int k = k0;
+  for (; k + 4 <= k1; k += 4) {
+    int m[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) m[j] = __ldg(pt.map[k + j] + tile);
+    uint4 r[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      r[j] = m[j] >= 0 ? __ldcs(pt.data[k + j] + (size_t)m[j] * kPackedThreads + unit) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (m[j] < 0) continue;
+      float v[8];
+      unpack_h8(r[j], v);
+      fold<2>(acc, v);
+    }
+  }
+  for (; k < k1; ++k) {
+    const int m = __ldg(pt.map[k] + tile);
+    if (m < 0) continue;
+    float v[8];
+    unpack_h8(__ldcs(pt.data[k] + (size_t)m * kPackedThreads + unit), v);
+    fold<2>(acc, v);
+  }
+}
+
+__device__ __forceinline__ void store_pixel_out(void* out, int f16, long long p, const float* acc) {
+  if (f16) {
+    const __half2 lo = __floats2half2_rn(acc[0], acc[1]), hi = __floats2half2_rn(acc[2], acc[3]);
+    reinterpret_cast<uint2*>(out)[p] = make_uint2(*reinterpret_cast<const unsigned*>(&lo),
+                                                  *reinterpret_cast<const unsigned*>(&hi));
+  } else {
+    reinterpret_cast<float4*>(out)[p] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  }
+}
+
+__global__ void __launch_bounds__(kPackedThreads)
+composite_packed_kernel(const __grid_constant__ PackedTable pt, int nf, int nb, int width,
+                        int height, int tiles_x, void* Fout, void* Bout, int out_f16) {
+  pdl_prologue();
+  const int tile = blockIdx.x;
+  const int unit = threadIdx.x;                       // pixels 2 unit, 2 unit + 1 of the tile
+  const int r = unit / (kTile / 2), c = 2 * (unit % (kTile / 2));
+  const int y = (tile / tiles_x) * kTile + r, x = (tile % tiles_x) * kTile + c;
+  for (int side = 0; side < 2; ++side) {
+    void* out = side ? Bout : Fout;
+    if (!out) continue;
+    float acc[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+    if (side == 0) fold_packed(pt, 0, nf, tile, unit, acc);
+    else fold_packed(pt, nf, nf + nb, tile, unit, acc);
+    if (y < height) {
+      if (x < width) store_pixel_out(out, out_f16, (long long)y * width + x, acc);
+      if (x + 1 < width) store_pixel_out(out, out_f16, (long long)y * width + x + 1, acc + 4);
+    }
+  }
+}
+
+}  // namespace
+}  // namespace abcd
+
+extern "C" abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_maps,
+                                                   const void* const* packed, int L,
+                                                   const int* order, int split, int width,
+                                                   int height, void* F_out, void* B_out,
+                                                   int out_dtype) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (L < 0 || L > kMaxLayers || (L > 0 && (!tile_maps || !packed || !order)) || split < 0 ||
+      split > L || width <= 0 || height <= 0)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache_packed: bad layer list, split or size");
+  if (out_dtype != ABCD_F16 && out_dtype != ABCD_F32)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache_packed: bad dtype");
+  PackedTable pt;
+  int nf = 0, nb = 0;
+  for (int k = 0; k < L; ++k) {
+    if (k == split) continue;
+    if (order[k] < 0 || order[k] >= L)
+      return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache_packed: order[%d] out of range", k);
+    const int* m = tile_maps[order[k]];
+    const void* d = packed[order[k]];
+    if (!m || !d) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache_packed: layer %d is NULL", order[k]);
+    if (((uintptr_t)d & 15) || ((uintptr_t)m & 3))
+      return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache_packed: layer %d misaligned", order[k]);
+    const int slot = k < split ? nf++ : -1;
+    if (slot >= 0) { pt.map[slot] = m; pt.data[slot] = (const uint4*)d; }
+  }
+  for (int k = split + 1; k < L; ++k) {
+    pt.map[nf + nb] = tile_maps[order[k]];
+    pt.data[nf + nb] = (const uint4*)packed[order[k]];
+    ++nb;
+  }
+  const uintptr_t oal = out_dtype == ABCD_F16 ? 7 : 15;
+  if (((uintptr_t)F_out & oal) || ((uintptr_t)B_out & oal))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_cache_packed: misaligned output");
+  if (!F_out && !B_out) return ABCD_OK;
+  const int tiles_x = (width + kTile - 1) / kTile, tiles_y = (height + kTile - 1) / kTile;
+  return check_launch(ctx, "composite_packed_kernel",
+                      launch_pdl(composite_packed_kernel, dim3(tiles_x * tiles_y),
+                                 dim3(kPackedThreads), 0, ctx->stream, pt, nf, nb, width, height,
+                                 tiles_x, F_out, B_out, out_dtype == ABCD_F16 ? 1 : 0));
+}

@@ -215,6 +215,8 @@ struct FwdArgs {
   float4* state_at;
   unsigned* n_last;
   uint2* refresh;      // fp16 x4 per pixel
+  uint2* refresh_packed;        // fp16 x4 per pixel of the tiles tile_map lists (packed layer)
+  const int* tile_map;
   const unsigned* tile_order;   // tiles, longest list first (nullptr: launch order)
   float4* ckpt;                 // render checkpoints (nullptr: none), see the workspace
   uint4* ck_items;
@@ -276,14 +278,19 @@ __device__ __forceinline__ void blend(PixF& p, float alpha, bool ok, float4 col,
   p.last = use ? __float_as_uint(col.w) + 1u : p.last;
 }
 
-__device__ __forceinline__ void store_pixel(const FwdArgs& a, long long p, const PixF& s) {
+__device__ __forceinline__ void store_pixel(const FwdArgs& a, long long p, const PixF& s, int qx,
+                                            int qy, int tile) {
   const float Aa = 1.f - s.T;
-  if (a.refresh) {
+  if (a.refresh || a.refresh_packed) {
     const __half2 lo = __floats2half2_rn(s.c0, s.c1), hi = __floats2half2_rn(s.c2, Aa);
     uint2 r;
     r.x = *reinterpret_cast<const unsigned*>(&lo);
     r.y = *reinterpret_cast<const unsigned*>(&hi);
-    a.refresh[p] = r;
+    if (a.refresh) a.refresh[p] = r;
+    if (a.refresh_packed) {
+      const int m = a.tile_map[tile];
+      if (m >= 0) a.refresh_packed[(size_t)m * kTileThreads + (qy % kTile) * kTile + qx % kTile] = r;
+    }
   }
   if (a.state_at) {
     a.state_at[p] = make_float4(s.c0, s.c1, s.c2, s.T);
@@ -368,8 +375,8 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
       a.ck_items[my_slot] = make_uint4((unsigned)blk, start, lane == n_items - 1 ? 0xffffffffu : start + kCkChunk, 0u);
     }
   }
-  if (bk.in0) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx0, p0);
-  if (bk.in1) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx1, p1);
+  if (bk.in0) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx0, p0, bk.qx0, bk.py, bk.tile);
+  if (bk.in1) store_pixel(a, (long long)bk.py * a.cam.width + bk.qx1, p1, bk.qx1, bk.py, bk.tile);
 }
 
 struct BwdArgs {
@@ -634,6 +641,8 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.state_at = state ? (float4*)state->A_T : nullptr;
   a.n_last = state ? state->n_last : nullptr;
   a.refresh = (uint2*)refresh_f16;
+  a.refresh_packed = nullptr;
+  a.tile_map = nullptr;
   const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
   a.tile_order = tile_order_for(ctx, tiles, n_tiles);
   a.ckpt = nullptr; a.ck_items = nullptr; a.ck_count = nullptr; a.ck_first = nullptr;
@@ -696,4 +705,90 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   return check_launch(ctx, "render_bwd_kernel",
                       launch_pdl(render_bwd_kernel, dim3(a.n_item_ctas + n_blocks), dim3(kSubThreads),
                                  0, ctx->stream, a));
+}
+
+// ---- packed layers (the cache's tile-sparse format): tile t of a layer is stored iff its
+// list is non-empty (a tile with no entry renders (0, 0, 0, 0) exactly), as the block
+// tile_map[t] of 16 x 16 fp16 RGBA pixels in row-major order; blocks are numbered in tile order.
+namespace abcd {
+namespace {
+
+__global__ void __launch_bounds__(1024)
+tile_map_kernel(const uint2* ranges, int n_tiles, int* tile_map, int* count) {
+  pdl_prologue();
+  const int per = (n_tiles + (int)blockDim.x - 1) / (int)blockDim.x;
+  const int lo = min(n_tiles, (int)threadIdx.x * per), hi = min(n_tiles, lo + per);
+  unsigned long long s = 0;
+  for (int t = lo; t < hi; ++t) s += ranges[t].y > ranges[t].x ? 1u : 0u;
+  unsigned long long total = 0;
+  __shared__ unsigned long long warp_sums[32];
+  // exclusive block scan of s
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  unsigned long long x = s;
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    const int nw = blockDim.x >> 5;
+    unsigned long long v = lane < nw ? warp_sums[lane] : 0ull;
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long y = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += y;
+    }
+    if (lane < nw) warp_sums[lane] = v;
+  }
+  __syncthreads();
+  unsigned long long run = (wid > 0 ? warp_sums[wid - 1] : 0ull) + x - s;
+  total = warp_sums[(blockDim.x >> 5) - 1];
+  for (int t = lo; t < hi; ++t) {
+    const bool used = ranges[t].y > ranges[t].x;
+    tile_map[t] = used ? (int)run : -1;
+    run += used ? 1u : 0u;
+  }
+  if (threadIdx.x == 0) *count = (int)total;
+}
+
+}  // namespace
+}  // namespace abcd
+
+extern "C" abcd_status abcd_render_refresh_packed(abcd_ctx* ctx, const abcd_camera* cam,
+                                                  const abcd_render_opts* opts,
+                                                  const abcd_projected* proj,
+                                                  const abcd_tiles* tiles, int* tile_map,
+                                                  void* packed, int* count) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!cam || cam->width <= 0 || cam->height <= 0 || !tiles || !tiles->ids || !tiles->ranges)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_refresh_packed: bad camera or tiles");
+  if (!proj_ok(proj)) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_refresh_packed: bad projected buffers");
+  if (!tile_map || !packed || !count || ((uintptr_t)packed & 15) || ((uintptr_t)tile_map & 3))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_refresh_packed: bad or misaligned output");
+  FwdArgs a;
+  a.cam = make_cam(cam, opts);
+  a.op = make_opts(opts);
+  a.uv = (const float2*)proj->uv;
+  a.co = (const float4*)proj->conic_opacity;
+  a.rgb = proj->rgb;
+  a.ids = tiles->ids;
+  a.ranges = (const uint2*)tiles->ranges;
+  a.F = nullptr; a.B = nullptr; a.fb_dtype = ABCD_F16;
+  for (int c = 0; c < 3; ++c) a.bg[c] = 0.f;
+  a.out = nullptr;
+  a.state_at = nullptr;
+  a.n_last = nullptr;
+  a.refresh = nullptr;
+  a.refresh_packed = (uint2*)packed;
+  a.tile_map = tile_map;
+  const int n_tiles = a.cam.tiles_x * a.cam.tiles_y, n_blocks = n_tiles * kSubPerTile;
+  a.tile_order = tile_order_for(ctx, tiles, n_tiles);
+  a.ckpt = nullptr; a.ck_items = nullptr; a.ck_count = nullptr; a.ck_first = nullptr;
+  a.ck_cap = 0;
+  abcd_status s = check_launch(ctx, "tile_map_kernel",
+                               launch_pdl(tile_map_kernel, dim3(1), dim3(1024), 0, ctx->stream,
+                                          (const uint2*)tiles->ranges, n_tiles, tile_map, count));
+  if (s) return s;
+  return check_launch(ctx, "render_fwd_kernel",
+                      launch_pdl(render_fwd_kernel, dim3(n_blocks), dim3(kSubThreads), 0, ctx->stream, a));
 }

@@ -434,6 +434,90 @@ def test_cache_host_tier_streams_layers(ctx):
         ab.abcd_cache_wait(ctx, -1)
 
 
+def pack_layer(dense, tiles_x, tiles_y):
+    """Test-side encoder of the packed layer format: (tile_map, packed) of a dense fp16
+    [H][W][4] layer, a tile stored iff any of its pixels is not all-zero bits."""
+    H, W = dense.shape[:2]
+    pad = np.zeros((tiles_y * 16, tiles_x * 16, 4), np.float16)
+    pad[:H, :W] = dense
+    blocks = pad.reshape(tiles_y, 16, tiles_x, 16, 4).transpose(0, 2, 1, 3, 4).reshape(-1, 16, 16, 4)
+    used = np.any(blocks.view(np.uint16) != 0, axis=(1, 2, 3))
+    tmap = np.where(used, np.cumsum(used) - 1, -1).astype(np.int32)
+    return tmap, np.ascontiguousarray(blocks[used])
+
+
+def test_refresh_packed_matches_dense_refresh(ctx, ragged):
+    """K10 into the packed format: the stored tiles are the dense refresh's, bit for bit, and
+    every tile left out is transparent in it."""
+    case = Case(ragged, 2, fb=False)
+    r = run_forward(ctx, case, want_state=False, refresh=True)
+    W, H = case.cam.width, case.cam.height
+    tx, ty = oracle.tiles_xy(W, H)
+    tmap = torch.full((tx * ty,), -7, dtype=torch.int32, device="cuda")
+    packed = torch.zeros(tx * ty, 16, 16, 4, dtype=torch.float16, device="cuda")
+    count = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ab.abcd_render_refresh_packed(ctx, r["cam"], None, r["proj"], r["tiles"], tmap, packed, count)
+    ctx.sync()
+    dense = r["refresh"].cpu().numpy()
+    m = tmap.cpu().numpy()
+    rng = r["tiles"].ranges.cpu().numpy().reshape(-1, 2).astype(np.int64)
+    used = rng[:, 1] > rng[:, 0]
+    assert np.array_equal(m >= 0, used) and int(count.item()) == int(used.sum())
+    assert np.array_equal(m[used], np.arange(used.sum()))
+    pk = packed.cpu().numpy()
+    pad = np.zeros((ty * 16, tx * 16, 4), np.float16)
+    pad[:H, :W] = dense
+    blocks = pad.reshape(ty, 16, tx, 16, 4).transpose(0, 2, 1, 3, 4).reshape(-1, 16, 16, 4)
+    inside = np.zeros((ty * 16, tx * 16), bool)
+    inside[:H, :W] = True
+    inb = inside.reshape(ty, 16, tx, 16).transpose(0, 2, 1, 3).reshape(-1, 16, 16)
+    for t in range(tx * ty):
+        if used[t]:
+            ok = inb[t]
+            assert np.array_equal(pk[m[t]][ok].view(np.uint16), blocks[t][ok].view(np.uint16)), t
+        else:
+            assert not np.any(blocks[t].view(np.uint16)), t
+
+
+def test_composite_packed_matches_dense(ctx):
+    """K1 over packed layers equals K1 over the dense layers bit for bit (a tile a layer leaves
+    out folds like its zeros), on a ragged image with layers that leave tiles out."""
+    L, H, W = 7, 75, 101
+    tx, ty = oracle.tiles_xy(W, H)
+    st = sg.premultiplied_layers(L, H, W, seed=17).astype(np.float16)
+    rng = np.random.default_rng(5)
+    for k in range(L):                      # blank a random third of each layer's tiles
+        for t in np.nonzero(rng.random(tx * ty) < 0.33)[0]:
+            y0, x0 = (t // tx) * 16, (t % tx) * 16
+            st[k, y0:y0 + 16, x0:x0 + 16] = 0
+    order = list(sg.random_permutation(L, seed=8))
+    maps, packs = [], []
+    for k in range(L):
+        m, pk = pack_layer(st[k], tx, ty)
+        maps.append(torch.from_numpy(m).cuda())
+        packs.append(torch.from_numpy(pk if len(pk) else np.zeros((1, 16, 16, 4), np.float16)).cuda())
+    dense = [torch.from_numpy(st[k]).cuda() for k in range(L)]
+    for split in (0, 3, L):
+        outs = []
+        for packed_path in (False, True):
+            Fo = torch.empty(H, W, 4, dtype=torch.float16, device="cuda")
+            Bo = torch.empty_like(Fo)
+            if packed_path:
+                mm, pp = list(maps), list(packs)
+                if split < L:
+                    mm[order[split]] = pp[order[split]] = None
+                ab.abcd_composite_cache_packed(ctx, mm, pp, order, split, W, H, Fo, Bo)
+            else:
+                lay = list(dense)
+                if split < L:
+                    lay[order[split]] = None
+                ab.abcd_composite_cache(ctx, lay, order, split, W, H, Fo, Bo)
+            outs.append((Fo, Bo))
+        ctx.sync()
+        for a_, b_ in zip(outs[0], outs[1]):
+            assert torch.equal(a_.view(torch.int16), b_.view(torch.int16)), split
+
+
 def test_adam_matches_oracle(ctx, ragged):
     g = ragged.gaussians.subset(slice(0, 3001))
     theta = ab.Gaussians.from_numpy(g)
