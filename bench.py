@@ -203,15 +203,40 @@ class Stage:
         self.tiles = ab.Tiles.alloc(cap, self.W, self.H, device)
         log(f"[bench] active block n={self.n}, pairs K mean {self.k_mean:.0f}; max over all "
             f"partitions {kmax}, capacity {cap}")
-        # cache of fp16 premultiplied renders, one per (camera, partition)
-        self.cache = torch.empty(C, self.n_parts, self.H, self.W, 4, dtype=torch.float16, device=device)
+        # cache of fp16 premultiplied renders, one per (camera, partition), in the packed
+        # (tile-sparse) format: per camera, the frozen partitions' stored tiles back to back
+        # (layer p at block offset self.pk_off[ci][p]) and the active partition's layer at
+        # full capacity (the refresh rewrites it); tile maps for all layers
         t1 = time.time()
-        for p in range(self.n_parts):
-            th = ab.Gaussians.from_numpy(g.subset(self.part_idx[p]), device)
-            for ci in range(C):
-                self.render_layer(th, ci, self.cache[ci, p])
-            self.ctx.sync()
-        log(f"[bench] cache of {C}x{self.n_parts} layers ({self.cache.numel() * 2 / 1e9:.1f} GB) in {time.time() - t1:.1f}s")
+        P, a = self.n_parts, self.active
+        self.n_t = ((self.W + 15) // 16) * ((self.H + 15) // 16)
+        self.pk_map = torch.empty(C, P, self.n_t, dtype=torch.int32, device=device)
+        self.pk_active = torch.empty(C, self.n_t, 16, 16, 4, dtype=torch.float16, device=device)
+        self.pk_count = torch.zeros(C, P, dtype=torch.int32, device=device)
+        ths = [ab.Gaussians.from_numpy(g.subset(self.part_idx[p]), device) for p in range(P)]
+        tmp = torch.empty(P, self.n_t, 16, 16, 4, dtype=torch.float16, device=device)
+        self.pk_frozen, self.pk_off = [], []
+        for ci in range(C):
+            for p in range(P):
+                self.render_packed(ths[p], ci, tmp[p] if p != a else self.pk_active[ci], p)
+            cnt = self.pk_count[ci].cpu().numpy()
+            off, run = [0] * P, 0
+            for p in range(P):
+                if p != a:
+                    off[p], run = run, run + int(cnt[p])
+            buf = torch.empty(max(run, 1), 16, 16, 4, dtype=torch.float16, device=device)
+            for p in range(P):
+                if p != a and cnt[p]:
+                    buf[off[p]:off[p] + int(cnt[p])].copy_(tmp[p][:int(cnt[p])])
+            self.pk_frozen.append(buf)
+            self.pk_off.append(off)
+        del tmp, ths
+        self.ctx.sync()
+        stored = sum(int(b.numel()) * 2 for b in self.pk_frozen)
+        self.cache_bytes = stored
+        log(f"[bench] cache of {C}x{P} layers: {stored / 1e9:.1f} GB of stored tiles for the frozen "
+            f"partitions ({100.0 * stored / (C * (P - 1) * self.n_t * 2048):.0f}% of the tiles) "
+            f"in {time.time() - t1:.1f}s")
         # targets: renders of the seed-perturbed scene
         t1 = time.time()
         self.gt = torch.empty(C, self.H, self.W, 3, device=device)
@@ -241,6 +266,23 @@ class Stage:
         ab.abcd_project(ctx, th, self.cams[ci], None, proj)
         ab.abcd_bin_sort(ctx, proj, th.n, self.cams[ci], tiles)
         ab.abcd_render_composite_fwd(ctx, self.cams[ci], None, proj, tiles, refresh_f16=dst)
+
+    def render_packed(self, th, ci, dst, p, w=None):
+        """K2-K4 and K10 into the packed layer dst (tile map and count of partition p)."""
+        ab = self.ab
+        ctx, proj, tiles = (self.ctx, self.proj, self.tiles) if w is None else (w["ctx"], w["proj"], w["tiles"])
+        ab.abcd_project(ctx, th, self.cams[ci], None, proj)
+        ab.abcd_bin_sort(ctx, proj, th.n, self.cams[ci], tiles)
+        ab.abcd_render_refresh_packed(ctx, self.cams[ci], None, proj, tiles, self.pk_map[ci, p], dst,
+                                      self.pk_count[ci, p:p + 1])
+
+    def packed_layers(self, ci):
+        """Tile maps and packed data of camera ci's layers (None at the active partition)."""
+        P, a = self.n_parts, self.active
+        maps = [self.pk_map[ci, p] for p in range(P)]
+        data = [self.pk_frozen[ci][self.pk_off[ci][p]:] if p != a else None for p in range(P)]
+        maps[a] = None
+        return maps, data
 
     def render_targets(self):
         torch, ab = self.torch, self.ab
@@ -277,15 +319,21 @@ class Stage:
         return int(self.order.pop())
 
     # ---- the three parts of a stage
-    def composite_all(self, layers=None, sampled_every=20):
+    def composite_all(self, sampled_every=20):
         ab = self.ab
         for j, ci in enumerate(self.observing):
+            self.composite_one(ci, j % sampled_every == 0)
+
+    def composite_one(self, ci, sampled=False):
+        if not hasattr(self, "_pk_tables"):
+            self._pk_tables = {}
+        pl = self._pk_tables.get(ci)
+        if pl is None:
             f, b = self.splits[ci]
-            src = self.cache[ci] if layers is None else layers(ci)
-            lay = [src[p] for p in range(self.n_parts)]
-            lay[self.active] = None
-            self._mark("composite", j % sampled_every == 0, ab.abcd_composite_cache, self.ctx, lay,
-                       f + [self.active] + b, len(f), self.W, self.H, self.F[ci], self.B[ci])
+            maps, data = self.packed_layers(ci)
+            pl = self._pk_tables[ci] = self.ab.PackedLayers(maps, data, f + [self.active] + b, len(f))
+        self._mark("composite", sampled, self.ab.abcd_composite_cache_packed_tables, self.ctx, pl,
+                   self.W, self.H, self.F[ci], self.B[ci])
 
     def step(self, t, stage_step):
         ab = self.ab
@@ -293,6 +341,13 @@ class Stage:
         cam = self.cams[ci]
         smp = (self.step_count % self.sample_every) == 0
         self.step_count += 1
+        if not smp:
+            # the whole step in one call (the sampled steps below time each kernel)
+            if not hasattr(self, "_train"):
+                self._train = ab.TrainStep(self.ctx, self.theta, self.grads, self.m, self.v,
+                                           self.proj, self.tiles, self.out, self.state, LR)
+            self._train(cam, self.F[ci], self.B[ci], self.gt[ci], self.loss[t:t + 1], stage_step + 1)
+            return
         self._mark("project", smp, ab.abcd_project, self.ctx, self.theta, cam, None, self.proj)
         self._mark("bin_sort", smp, ab.abcd_bin_sort, self.ctx, self.proj, self.n, cam, self.tiles)
         self._mark("render_fwd", smp, ab.abcd_render_composite_fwd, self.ctx, cam, None, self.proj,
@@ -325,7 +380,8 @@ class Stage:
         for w in self.side:
             w["ctx"].stream.wait_event(s)
         for j, ci in enumerate(self.observing):
-            self.render_layer(self.theta, ci, self.cache[ci, self.active], self.side[j % len(self.side)])
+            self.render_packed(self.theta, ci, self.pk_active[ci], self.active,
+                               self.side[j % len(self.side)])
         for w in self.side:
             self.stream.wait_event(torch_event(torch, w["ctx"].stream))
         e = torch_event(torch, self.stream)
@@ -367,7 +423,9 @@ def algorithmic(st: Stage, name, avg_ms, pairs_mean):
     if name == "loss":
         return "alu", LOSS_FLOP_PER_PX * npx / (avg_ms * 1e-3) / 1e12, "TFLOP/s"
     if name == "composite":
-        byts = (st.n_parts - 1) * 8 * npx + 2 * 8 * npx
+        # stored tiles of the frozen layers and their tile maps read, F and B written
+        C = len(st.cams)
+        byts = st.cache_bytes / C + (st.n_parts - 1) * st.n_t * 4 + 2 * 8 * npx
         return "hbm", byts / (avg_ms * 1e-3) / 1e9, "GB/s"
     if name == "adam":
         return "hbm", 7 * 4 * (14 + 3 * D) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
@@ -454,11 +512,14 @@ def run_ours(args):
     l0 = st.launches()
     torch.cuda.nvtx.range_push("abcd_timed")
     e0 = torch_event(torch, st.stream)
+    h0 = time.perf_counter()
     for _ in range(args.steps):
         st.run_stage()
+    host_ms = (time.perf_counter() - h0) * 1e3
     e1 = torch_event(torch, st.stream)
     torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
+    log(f"[bench] host issue time {host_ms / args.steps:.1f} ms per stage")
     barrier()
     launches = st.launches() - l0
     clocks = clk.stop()
@@ -529,40 +590,38 @@ def run_ours(args):
 
 def run_e2e(st: Stage, args, world, barrier):
     """The same stages with their inputs in pinned host memory (the host tier of the cache).
-    Every stage, each observing camera's frozen layers and target go host -> device on the
-    context's copy stream (abcd_cache_fetch); a camera's copies for the next stage start as
-    soon as this stage's composite of that camera has read its buffers (abcd_cache_release),
-    so they overlap this stage's steps, as in the steady state of a training loop.  The
-    refreshed layers go back on the other copy stream (abcd_cache_store); the parameters come
-    in and go back, and the per-step losses go back, on the compute stream."""
+    Every stage, each observing camera's frozen layers (tile maps and stored tiles of the
+    packed format) and target go host -> device on the context's copy stream
+    (abcd_cache_fetch); a camera's copies for the next stage start as soon as this stage's
+    composite of that camera has read its buffers (abcd_cache_release), so they overlap this
+    stage's steps, as in the steady state of a training loop.  The refreshed layers go back on
+    the other copy stream (abcd_cache_store); the parameters come in and go back, and the
+    per-step losses go back, on the compute stream."""
     torch, ab = st.torch, st.ab
     C = len(st.cams)
-    pool = min(8, C)                  # distinct pinned host buffers, cycled over the cameras
     P, a = st.n_parts, st.active
-    host_layers = torch.empty(pool, P, st.H, st.W, 4, dtype=torch.float16, pin_memory=True)
-    host_gt = torch.empty(pool, st.H, st.W, 3, dtype=torch.float32, pin_memory=True)
-    for k in range(pool):
-        host_layers[k].copy_(st.cache[k])
-        host_gt[k].copy_(st.gt[k])
+    host_frozen = [t.cpu().pin_memory() for t in st.pk_frozen]
+    host_maps = st.pk_map.cpu().pin_memory()
+    host_gt = st.gt.cpu().pin_memory()
     theta_host = [t.cpu().pin_memory() for t in st.theta.tensors()]
-    refreshed = torch.empty(pool, st.H, st.W, 4, dtype=torch.float16, pin_memory=True)
+    pool = min(8, C)
+    refreshed = torch.empty(pool, st.n_t, 16, 16, 4, dtype=torch.float16, pin_memory=True)
+    refreshed_map = torch.empty(pool, st.n_t, dtype=torch.int32, pin_memory=True)
     loss_host = torch.empty(args.T, dtype=torch.float32, pin_memory=True)
     gts = [st.gt, torch.empty_like(st.gt)]          # targets of this stage / the next one
-    layer_bytes = st.H * st.W * 4 * 2
     counted = {"h2d": 0, "d2h": 0}
 
     def fetch(ci, gt_dst):
         """Queues the host -> device copies of camera ci's inputs; returns their bytes."""
-        src = host_layers[ci % pool]
         n = 0
-        if a > 0:
-            ab.abcd_cache_fetch(st.ctx, ci, src[:a], st.cache[ci, :a])
-            n += a * layer_bytes
-        if a + 1 < P:
-            ab.abcd_cache_fetch(st.ctx, ci, src[a + 1:], st.cache[ci, a + 1:])
-            n += (P - a - 1) * layer_bytes
-        ab.abcd_cache_fetch(st.ctx, ci, host_gt[ci % pool], gt_dst[ci])
-        return n + host_gt[0].numel() * 4
+        for lo, hi in ((0, a), (a + 1, P)):
+            if hi > lo:
+                ab.abcd_cache_fetch(st.ctx, ci, host_maps[ci, lo:hi], st.pk_map[ci, lo:hi])
+                n += (hi - lo) * st.n_t * 4
+        ab.abcd_cache_fetch(st.ctx, ci, host_frozen[ci], st.pk_frozen[ci])
+        n += host_frozen[ci].numel() * 2
+        ab.abcd_cache_fetch(st.ctx, ci, host_gt[ci], gt_dst[ci])
+        return n + host_gt[ci].numel() * 4
 
     def stage(k):
         cur, nxt = gts[k % 2], gts[(k + 1) % 2]
@@ -575,10 +634,7 @@ def run_e2e(st: Stage, args, world, barrier):
                 tns.zero_()
         for ci in st.observing:
             ab.abcd_cache_wait(st.ctx, ci)           # this stage's layers and target landed
-            f, b = st.splits[ci]
-            lay = [st.cache[ci, p] for p in range(P)]
-            lay[a] = None
-            ab.abcd_composite_cache(st.ctx, lay, f + [a] + b, len(f), st.W, st.H, st.F[ci], st.B[ci])
+            st.composite_one(ci)
             ab.abcd_cache_release(st.ctx, ci)
             h2d += fetch(ci, nxt)                     # the next stage's, behind this composite
         st.gt = cur
@@ -588,8 +644,9 @@ def run_e2e(st: Stage, args, world, barrier):
         d2h += st.loss.numel() * 4
         st.refresh_all()
         for ci in st.observing:
-            ab.abcd_cache_store(st.ctx, ci, st.cache[ci, a], refreshed[ci % pool])
-            d2h += layer_bytes
+            ab.abcd_cache_store(st.ctx, ci, st.pk_active[ci], refreshed[ci % pool])
+            ab.abcd_cache_store(st.ctx, ci, st.pk_map[ci, a], refreshed_map[ci % pool])
+            d2h += st.pk_active[ci].numel() * 2 + st.n_t * 4
         for src, dst in zip(st.theta.tensors(), theta_host):
             dst.copy_(src, non_blocking=True)
             d2h += src.numel() * 4
@@ -605,14 +662,18 @@ def run_e2e(st: Stage, args, world, barrier):
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     e0 = torch_event(torch, st.stream)
+    h0 = time.perf_counter()
     for k in range(args.steps):
         stage(k + 1)
+    host_ms = (time.perf_counter() - h0) * 1e3
     e1 = torch_event(torch, st.stream)
     ab.abcd_cache_sync(st.ctx)
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
     barrier()
     ms = max(e0.elapsed_time(e1), wall * 1e3)
+    print(f"[bench] e2e: host issue time {host_ms / args.steps:.1f} ms, device {e0.elapsed_time(e1) / args.steps:.1f} ms, "
+          f"wall {wall * 1e3 / args.steps:.1f} ms per stage", file=sys.stderr, flush=True)
     ms_t = torch.tensor([ms], dtype=torch.float64, device="cuda")
     if world > 1:
         import torch.distributed as dist
@@ -621,9 +682,10 @@ def run_e2e(st: Stage, args, world, barrier):
     st.gt = gts[0]
     return {"value": round(args.steps * args.T * world / (ms / 1e3), 2), "unit": UNIT,
             "h2d_bytes_per_step": int(counted["h2d"]), "d2h_bytes_per_step": int(counted["d2h"]),
-            "note": "per stage: active parameters, observing cameras' frozen layers and targets "
-                    "host->device (layers and targets on the copy stream, one stage ahead); "
-                    "refreshed layers, parameters and losses device->host"}
+            "note": "per stage: active parameters, observing cameras' frozen layers (packed: tile "
+                    "maps and stored tiles) and targets host->device (layers and targets on the "
+                    "copy stream, one stage ahead); refreshed layers, parameters and losses "
+                    "device->host"}
 
 
 # ---------------------------------------------------------------------------------------
@@ -692,7 +754,8 @@ def stage_config(args, n_active, world):
                           "T active-block steps (K2-K9), cache refresh (K10)",
             "T": args.T, "observing_cameras": args.cams, "active_gaussians": int(n_active),
             "parallelism": f"replicas x{world}",
-            "l2": "stage inputs exceed L2 (cached layers 52 GB read per stage)"}
+            "l2": "stage inputs exceed L2 (every stage reads all observing cameras' stored "
+                  "layer tiles, many GB)"}
 
 
 def run_reference(args):

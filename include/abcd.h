@@ -196,6 +196,20 @@ abcd_status abcd_adam_active(abcd_ctx* ctx, abcd_gaussians* theta, const abcd_ga
                              abcd_gaussians* m, abcd_gaussians* v, const float lr[6],
                              float beta1, float beta2, float eps, int step);
 
+/* One active-block step of Section 2 in one call: K2 abcd_project, K3-K4 abcd_bin_sort, K5
+ * abcd_render_composite_fwd (out_rgba and state), K6-K8 abcd_backward with the loss against
+ * gt_rgb (its gradient in the workspace) into grads, K9 abcd_adam_active.  The same as calling
+ * those entry points in that order with these arguments; one call instead of six saves the
+ * caller's per-call cost on a step of about thirty launches.  The first failing call's status
+ * is returned (later ones are not made). */
+abcd_status abcd_train_step(abcd_ctx* ctx, abcd_gaussians* theta, abcd_gaussians* grads,
+                            abcd_gaussians* m, abcd_gaussians* v, const abcd_camera* cam,
+                            const abcd_render_opts* opts, abcd_projected* proj, abcd_tiles* tiles,
+                            const void* F, const void* B, int fb_dtype, const float* bg,
+                            float* out_rgba, abcd_fwd_state* state, const float* gt_rgb,
+                            float lambda_ssim, float* loss_out, const float lr[6], float beta1,
+                            float beta2, float eps, int step);
+
 /* K1. Depth-ordered over-compositing of cached per-partition renders into the foreground F and
  * background B of one camera (Section 2: the frozen partitions' stored renders, taken in the
  * camera's depth order, collapse into two RGBA images).  layers: host array of L device pointers to [H][W][4] premultiplied RGBA of

@@ -99,6 +99,9 @@ _SIGS = {
                                    C.c_void_p, C.c_void_p, C.c_void_p],
     "abcd_composite_cache_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
                                     C.c_int, C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int],
+    "abcd_train_step": [C.c_void_p] + [C.c_void_p] * 8 + [C.c_void_p, C.c_void_p, C.c_int,
+                         C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_float, C.c_void_p,
+                         C.c_void_p, C.c_float, C.c_float, C.c_float, C.c_int],
     "abcd_cache_fetch": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
     "abcd_cache_wait": [C.c_void_p, C.c_int],
     "abcd_cache_release": [C.c_void_p, C.c_int],
@@ -421,6 +424,50 @@ def abcd_composite_cache_packed(ctx: Context, tile_maps, packed, order, split, w
     ordr = (C.c_int * max(1, L))(*[int(k) for k in order])
     ctx.check(lib().abcd_composite_cache_packed(ctx.h, maps, data, L, ordr, int(split), int(width),
                                                 int(height), _p(F_out), _p(B_out), int(out_dtype)))
+
+
+class TrainStep:
+    """abcd_train_step with the argument structs built once: the buffers of a training loop
+    stay put, so only the camera, F, B, target, loss slot and step change per call."""
+
+    def __init__(self, ctx: Context, theta, grads, m, v, proj, tiles, out_rgba, state, lr,
+                 beta1=0.9, beta2=0.999, eps=1e-15, lambda_ssim=0.2, opts=None, bg=None):
+        self.ctx = ctx
+        self.structs = [theta.c(), grads.c(), m.c(), v.c(), proj.c(), tiles.c(), state.c()]
+        self.refs = [C.byref(x) for x in self.structs]
+        self.opts = _opt(opts)
+        self.bg = _bg(bg)
+        self.out = _p(out_rgba)
+        self.lr = (C.c_float * 6)(*[float(x) for x in lr])
+        self.beta1, self.beta2, self.eps, self.lam = float(beta1), float(beta2), float(eps), float(lambda_ssim)
+        self.keep = (theta, grads, m, v, proj, tiles, out_rgba, state)
+
+    def __call__(self, cam, F, B, gt_rgb, loss_out, step, fb_dtype=ABCD_F16):
+        th, gr, mm, vv, pr, ti, st = self.refs
+        self.ctx.check(lib().abcd_train_step(
+            self.ctx.h, th, gr, mm, vv, C.byref(cam), self.opts, pr, ti, _p(F), _p(B), int(fb_dtype),
+            self.bg, self.out, st, _p(gt_rgb), self.lam, _p(loss_out), self.lr, self.beta1,
+            self.beta2, self.eps, int(step)))
+
+
+class PackedLayers:
+    """The pointer tables of one camera's packed layers, built once for repeated composites
+    (the per-call conversion of 2 L tensors is host time a stage spends per camera)."""
+
+    def __init__(self, tile_maps, packed, order, split):
+        L = len(tile_maps)
+        self.L, self.split = L, int(split)
+        self.maps = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in tile_maps])
+        self.data = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in packed])
+        self.order = (C.c_int * max(1, L))(*[int(k) for k in order])
+        self.keep = (tile_maps, packed)          # the tensors must outlive the tables
+
+
+def abcd_composite_cache_packed_tables(ctx: Context, pl: PackedLayers, width, height, F_out, B_out,
+                                       out_dtype=ABCD_F16):
+    ctx.check(lib().abcd_composite_cache_packed(ctx.h, pl.maps, pl.data, pl.L, pl.order, pl.split,
+                                                int(width), int(height), _p(F_out), _p(B_out),
+                                                int(out_dtype)))
 
 
 def abcd_cache_fetch(ctx: Context, slot, host_src, dev_dst, nbytes=None):

@@ -33,3 +33,27 @@ extern "C" abcd_status abcd_backward(abcd_ctx* ctx, const abcd_gaussians* theta,
     return s;
   return abcd_project_backward(ctx, theta, cam, opts, ctx->ws.grad2d, grads);
 }
+
+extern "C" abcd_status abcd_train_step(abcd_ctx* ctx, abcd_gaussians* theta, abcd_gaussians* grads,
+                                       abcd_gaussians* m, abcd_gaussians* v,
+                                       const abcd_camera* cam, const abcd_render_opts* opts,
+                                       abcd_projected* proj, abcd_tiles* tiles, const void* F,
+                                       const void* B, int fb_dtype, const float* bg,
+                                       float* out_rgba, abcd_fwd_state* state,
+                                       const float* gt_rgb, float lambda_ssim, float* loss_out,
+                                       const float lr[6], float beta1, float beta2, float eps,
+                                       int step) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!theta || !grads || !m || !v || !cam || !proj || !tiles || !out_rgba || !state || !gt_rgb || !lr)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_train_step: null argument");
+  abcd_status s;
+  if ((s = abcd_project(ctx, theta, cam, opts, proj))) return s;
+  if ((s = abcd_bin_sort(ctx, proj, theta->n, cam, opts, tiles))) return s;
+  if ((s = abcd_render_composite_fwd(ctx, cam, opts, proj, tiles, F, B, fb_dtype, bg, out_rgba,
+                                     state, nullptr)))
+    return s;
+  if ((s = abcd_backward(ctx, theta, cam, opts, proj, tiles, F, B, fb_dtype, bg, out_rgba, state,
+                         gt_rgb, lambda_ssim, loss_out, nullptr, grads)))
+    return s;
+  return abcd_adam_active(ctx, theta, grads, m, v, lr, beta1, beta2, eps, step);
+}

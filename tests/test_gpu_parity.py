@@ -565,6 +565,46 @@ def _full_step(ctx, scene, case):
     return loss.item(), L, grads, ref, R
 
 
+def test_train_step_matches_separate_calls(ctx, tiny):
+    """abcd_train_step (the six entry points of a step in one call) gives the same loss and,
+    up to the order of the backward's atomic sums, the same parameters and Adam moments as
+    calling project, bin_sort, render, backward and Adam one by one."""
+    case = Case(tiny, 1, fb=True)
+    H, W = case.cam.height, case.cam.width
+    cam = ab.camera(case.cam)
+    gt = torch.from_numpy(sg.random_image(H, W, 3, seed=77)).cuda()
+    F = torch.from_numpy(case.F).cuda()
+    B = torch.from_numpy(case.B).cuda()
+    lr = [1e-3, 5e-3, 1e-3, 0.025, 2.5e-3, 1.25e-4]
+    res = []
+    for fused in (False, True):
+        theta = ab.Gaussians.from_numpy(case.g)
+        grads, m, v = (ab.Gaussians.zeros_like(theta) for _ in range(3))
+        proj = ab.Projected.alloc(theta.n)
+        tiles = ab.Tiles.alloc(1_000_000, W, H)
+        out = torch.empty(H, W, 4, device="cuda")
+        st = ab.FwdState.alloc(W, H)
+        loss = torch.zeros(2, device="cuda")
+        step = ab.TrainStep(ctx, theta, grads, m, v, proj, tiles, out, st, lr)
+        for k in range(2):
+            if fused:
+                step(cam, F, B, gt, loss[k:k + 1], k + 1)
+            else:
+                ab.abcd_project(ctx, theta, cam, None, proj)
+                ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+                ab.abcd_render_composite_fwd(ctx, cam, None, proj, tiles, F, B, ab.ABCD_F16, None,
+                                             out, st)
+                ab.abcd_backward(ctx, theta, cam, None, proj, tiles, F, B, ab.ABCD_F16, None, out,
+                                 st, gt, 0.2, loss[k:k + 1], None, grads)
+                ab.abcd_adam_active(ctx, theta, grads, m, v, lr, 0.9, 0.999, 1e-15, k + 1)
+        ctx.sync()
+        res.append((loss.cpu(), [t.cpu() for t in theta.tensors() + m.tensors() + v.tensors()]))
+    assert torch.equal(res[0][0][:1], res[1][0][:1])            # first loss: same inputs
+    assert torch.allclose(res[0][0], res[1][0], rtol=1e-5, atol=0)
+    for a_, b_ in zip(res[0][1], res[1][1]):
+        assert torch.allclose(a_, b_, rtol=1e-4, atol=1e-7)
+
+
 @pytest.mark.parametrize("seed,cam_idx", [(1001, 0), (1005, 1)])
 def test_full_step_matches_oracle(ctx, seed, cam_idx):
     """project -> bin/sort -> render + composite -> L1 + 0.2 D-SSIM -> backward, element-wise.
