@@ -267,14 +267,19 @@ class Stage:
         ab.abcd_bin_sort(ctx, proj, th.n, self.cams[ci], tiles)
         ab.abcd_render_composite_fwd(ctx, self.cams[ci], None, proj, tiles, refresh_f16=dst)
 
-    def render_packed(self, th, ci, dst, p, w=None):
-        """K2-K4 and K10 into the packed layer dst (tile map and count of partition p)."""
+    def render_packed(self, th, ci, dst, p, w=None, map_dst=None, cnt_dst=None):
+        """K2-K4 and K10 into the packed layer dst (tile map and count of partition p, or into
+        map_dst / cnt_dst), in one library call."""
         ab = self.ab
-        ctx, proj, tiles = (self.ctx, self.proj, self.tiles) if w is None else (w["ctx"], w["proj"], w["tiles"])
-        ab.abcd_project(ctx, th, self.cams[ci], None, proj)
-        ab.abcd_bin_sort(ctx, proj, th.n, self.cams[ci], tiles)
-        ab.abcd_render_refresh_packed(ctx, self.cams[ci], None, proj, tiles, self.pk_map[ci, p], dst,
-                                      self.pk_count[ci, p:p + 1])
+        holder = self.__dict__ if w is None else w
+        fn = holder.get("_refresh") if th is self.theta else None
+        if fn is None:
+            ctx, proj, tiles = (self.ctx, self.proj, self.tiles) if w is None else (w["ctx"], w["proj"], w["tiles"])
+            fn = ab.RefreshLayer(ctx, th, proj, tiles)
+            if th is self.theta:
+                holder["_refresh"] = fn
+        fn(self.cams[ci], self.pk_map[ci, p] if map_dst is None else map_dst, dst,
+           self.pk_count[ci, p:p + 1] if cnt_dst is None else cnt_dst)
 
     def packed_layers(self, ci):
         """Tile maps and packed data of camera ci's layers (None at the active partition)."""
@@ -564,6 +569,9 @@ def run_ours(args):
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(st, args, world, barrier)
+    streaming = None
+    if not args.no_e2e:
+        streaming = run_streaming(st, args, world, barrier)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, log)
@@ -577,6 +585,7 @@ def run_ours(args):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
+        "streaming_one_fb_pair": streaming,
         "gpu_launches": int(launches),
         "clocks": clocks,
         "ops": {k: {"avg_ms": round(v["avg_ms"], 4), "share": round(share[k], 4)} for k, v in ops.items()},
@@ -686,6 +695,128 @@ def run_e2e(st: Stage, args, world, barrier):
                     "maps and stored tiles) and targets host->device (layers and targets on the "
                     "copy stream, one stage ahead); refreshed layers, parameters and losses "
                     "device->host"}
+
+
+def run_streaming(st: Stage, args, world, barrier):
+    """One F/B pair at a time (the host tier's streaming mode): no camera's layers, F, B or
+    target stay on the device between steps.  For each step the sampled camera's frozen
+    layers (packed) and target come from pinned host memory into one of two device slots,
+    are composited into that slot's F/B pair, and the step runs; the next camera's copies are
+    queued before the step, so they overlap it.  The refresh renders each camera's active
+    layer into one of two device buffers and stores it back.  Device bytes for the cache, F,
+    B and targets: two slots, whatever the number of cameras or partitions."""
+    torch, ab = st.torch, st.ab
+    P, a = st.n_parts, st.active
+    host_frozen = [t.cpu().pin_memory() for t in st.pk_frozen]
+    host_maps = st.pk_map.cpu().pin_memory()
+    host_gt = st.gt.cpu().pin_memory()
+    theta_host = [t.cpu().pin_memory() for t in st.theta.tensors()]
+    loss_host = torch.empty(args.T, dtype=torch.float32, pin_memory=True)
+    cap = max(t.shape[0] for t in st.pk_frozen)
+    dev = st.dev
+    slots = [dict(frozen=torch.empty(cap, 16, 16, 4, dtype=torch.float16, device=dev),
+                  maps=torch.empty(P, st.n_t, dtype=torch.int32, device=dev),
+                  gt=torch.empty(st.H, st.W, 3, device=dev),
+                  F=torch.empty(st.H, st.W, 4, dtype=torch.float16, device=dev),
+                  B=torch.empty(st.H, st.W, 4, dtype=torch.float16, device=dev)) for _ in range(2)]
+    # refresh: each side context renders into its own two buffers and stores them back
+    for w in st.side:
+        w["active"] = [torch.empty(st.n_t, 16, 16, 4, dtype=torch.float16, device=dev) for _ in range(2)]
+        w["back"] = [torch.empty(st.n_t, 16, 16, 4, dtype=torch.float16, pin_memory=True) for _ in range(2)]
+        w["back_map"] = [torch.empty(st.n_t, dtype=torch.int32, pin_memory=True) for _ in range(2)]
+        w["active_map"] = [torch.empty(st.n_t, dtype=torch.int32, device=dev) for _ in range(2)]
+        w["active_cnt"] = torch.zeros(2, dtype=torch.int32, device=dev)
+    dev_bytes = sum(sum(v.numel() * v.element_size() for v in s_.values()) for s_ in slots) + \
+        sum(x.numel() * x.element_size() for w in st.side for x in w["active"] + w["active_map"])
+    train = ab.TrainStep(st.ctx, st.theta, st.grads, st.m, st.v, st.proj, st.tiles, st.out,
+                         st.state, LR)
+    rng = np.random.default_rng(11)
+
+    def fetch(k, ci):
+        sl = slots[k]
+        for lo, hi in ((0, a), (a + 1, P)):
+            if hi > lo:
+                ab.abcd_cache_fetch(st.ctx, k, host_maps[ci, lo:hi], sl["maps"][lo:hi])
+        n = host_frozen[ci].shape[0]
+        ab.abcd_cache_fetch(st.ctx, k, host_frozen[ci], sl["frozen"][:n])
+        ab.abcd_cache_fetch(st.ctx, k, host_gt[ci], sl["gt"])
+
+    def composite(k, ci):
+        sl = slots[k]
+        f, b = st.splits[ci]
+        maps = [sl["maps"][p] if p != a else None for p in range(P)]
+        data = [sl["frozen"][st.pk_off[ci][p]:] if p != a else None for p in range(P)]
+        ab.abcd_composite_cache_packed(st.ctx, maps, data, f + [a] + b, len(f), st.W, st.H,
+                                       sl["F"], sl["B"])
+
+    def stage():
+        for dst, src in zip(st.theta.tensors(), theta_host):
+            dst.copy_(src, non_blocking=True)
+        for x in (st.m, st.v):
+            for tns in x.tensors():
+                tns.zero_()
+        order = []
+        while len(order) < args.T:
+            order += list(rng.permutation(st.observing))
+        fetch(0, order[0])
+        for t in range(args.T):
+            k = t % 2
+            ab.abcd_cache_wait(st.ctx, k)
+            composite(k, order[t])
+            if t + 1 < args.T:
+                fetch(1 - k, order[t + 1])        # behind the step that last used that slot
+            train(st.cams[order[t]], slots[k]["F"], slots[k]["B"], slots[k]["gt"],
+                  st.loss[t:t + 1], t + 1)
+            ab.abcd_cache_release(st.ctx, k)
+        loss_host.copy_(st.loss, non_blocking=True)
+        fork = torch_event(torch, st.stream)
+        for w in st.side:
+            w["ctx"].stream.wait_event(fork)
+        nw = len(st.side)
+        for j, ci in enumerate(st.observing):
+            w = st.side[j % nw]
+            k = (j // nw) % 2
+            ab.abcd_cache_wait(w["ctx"], k)        # this buffer's previous store has left
+            st.render_packed(st.theta, ci, w["active"][k], a, w, w["active_map"][k],
+                             w["active_cnt"][k:k + 1])
+            ab.abcd_cache_store(w["ctx"], k, w["active"][k], w["back"][k])
+            ab.abcd_cache_store(w["ctx"], k, w["active_map"][k], w["back_map"][k])
+        for w in st.side:
+            st.stream.wait_event(torch_event(torch, w["ctx"].stream))
+        for src, dst in zip(st.theta.tensors(), theta_host):
+            dst.copy_(src, non_blocking=True)
+
+    stage()
+    torch.cuda.synchronize()
+    st.sample_every = 10 ** 9
+    barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    e0 = torch_event(torch, st.stream)
+    for _ in range(args.steps):
+        stage()
+    e1 = torch_event(torch, st.stream)
+    ab.abcd_cache_sync(st.ctx)
+    for w in st.side:
+        ab.abcd_cache_sync(w["ctx"])
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    barrier()
+    ms = max(e0.elapsed_time(e1), wall * 1e3)
+    ms_t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+    ms = float(ms_t.item())
+    per_step = sum(host_frozen[c].numel() * 2 + (P - 1) * st.n_t * 4 + host_gt[c].numel() * 4
+                   for c in st.observing) / len(st.observing)
+    return {"value": round(args.steps * args.T * world / (ms / 1e3), 2), "unit": UNIT,
+            "device_bytes_cache_fb_targets": int(dev_bytes),
+            "h2d_bytes_per_active_step": int(per_step),
+            "note": "one F/B pair at a time: per step the sampled camera's packed frozen layers "
+                    "and target are copied from pinned host memory (one step ahead) and "
+                    "composited; the refresh stores each camera's layer back; the device holds "
+                    "two slots whatever the number of cameras and partitions"}
 
 
 # ---------------------------------------------------------------------------------------

@@ -240,6 +240,13 @@ abcd_status abcd_render_refresh_packed(abcd_ctx* ctx, const abcd_camera* cam,
                                        const abcd_tiles* tiles, int* tile_map, void* packed,
                                        int* count);
 
+/* K10 for one camera in one call: abcd_project, abcd_bin_sort and
+ * abcd_render_refresh_packed with these arguments, in that order (the first failing call's
+ * status is returned). */
+abcd_status abcd_refresh_layer(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_camera* cam,
+                               const abcd_render_opts* opts, abcd_projected* proj,
+                               abcd_tiles* tiles, int* tile_map, void* packed, int* count);
+
 /* K1 over packed layers: the same folds as abcd_composite_cache (fp16 layers), with layer k
  * given by tile_maps[k] and packed[k] (host arrays of L device pointers; NULL at the active
  * position).  A tile a layer does not store is transparent for it, which leaves the fold

@@ -102,6 +102,7 @@ _SIGS = {
     "abcd_train_step": [C.c_void_p] + [C.c_void_p] * 8 + [C.c_void_p, C.c_void_p, C.c_int,
                          C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_float, C.c_void_p,
                          C.c_void_p, C.c_float, C.c_float, C.c_float, C.c_int],
+    "abcd_refresh_layer": [C.c_void_p] * 9,
     "abcd_cache_fetch": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
     "abcd_cache_wait": [C.c_void_p, C.c_int],
     "abcd_cache_release": [C.c_void_p, C.c_int],
@@ -448,6 +449,22 @@ class TrainStep:
             self.ctx.h, th, gr, mm, vv, C.byref(cam), self.opts, pr, ti, _p(F), _p(B), int(fb_dtype),
             self.bg, self.out, st, _p(gt_rgb), self.lam, _p(loss_out), self.lr, self.beta1,
             self.beta2, self.eps, int(step)))
+
+
+class RefreshLayer:
+    """abcd_refresh_layer with the argument structs of one context's buffers built once."""
+
+    def __init__(self, ctx: Context, theta, proj, tiles, opts=None):
+        self.ctx = ctx
+        self.structs = [theta.c(), proj.c(), tiles.c()]
+        self.refs = [C.byref(x) for x in self.structs]
+        self.opts = _opt(opts)
+        self.keep = (theta, proj, tiles)
+
+    def __call__(self, cam, tile_map, packed, count):
+        th, pr, ti = self.refs
+        self.ctx.check(lib().abcd_refresh_layer(self.ctx.h, th, C.byref(cam), self.opts, pr, ti,
+                                                _p(tile_map), _p(packed), _p(count)))
 
 
 class PackedLayers:

@@ -57,3 +57,16 @@ extern "C" abcd_status abcd_train_step(abcd_ctx* ctx, abcd_gaussians* theta, abc
     return s;
   return abcd_adam_active(ctx, theta, grads, m, v, lr, beta1, beta2, eps, step);
 }
+
+extern "C" abcd_status abcd_refresh_layer(abcd_ctx* ctx, const abcd_gaussians* theta,
+                                          const abcd_camera* cam, const abcd_render_opts* opts,
+                                          abcd_projected* proj, abcd_tiles* tiles, int* tile_map,
+                                          void* packed, int* count) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!theta || !cam || !proj || !tiles)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_refresh_layer: null argument");
+  abcd_status s;
+  if ((s = abcd_project(ctx, theta, cam, opts, proj))) return s;
+  if ((s = abcd_bin_sort(ctx, proj, theta->n, cam, opts, tiles))) return s;
+  return abcd_render_refresh_packed(ctx, cam, opts, proj, tiles, tile_map, packed, count);
+}

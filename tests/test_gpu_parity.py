@@ -457,7 +457,14 @@ def test_refresh_packed_matches_dense_refresh(ctx, ragged):
     packed = torch.zeros(tx * ty, 16, 16, 4, dtype=torch.float16, device="cuda")
     count = torch.zeros(1, dtype=torch.int32, device="cuda")
     ab.abcd_render_refresh_packed(ctx, r["cam"], None, r["proj"], r["tiles"], tmap, packed, count)
+    # the one-call form (project, bin_sort, packed refresh) gives the same bytes
+    tmap2, packed2, count2 = torch.full_like(tmap, -7), torch.zeros_like(packed), torch.zeros_like(count)
+    ab.RefreshLayer(ctx, r["theta"], ab.Projected.alloc(r["theta"].n),
+                    ab.Tiles.alloc(4_000_000, W, H))(r["cam"], tmap2, packed2, count2)
     ctx.sync()
+    assert torch.equal(tmap, tmap2) and torch.equal(count, count2)
+    used2 = (tmap2 >= 0).nonzero().numel()
+    assert torch.equal(packed2[:used2].view(torch.int16), packed[:used2].view(torch.int16))
     dense = r["refresh"].cpu().numpy()
     m = tmap.cpu().numpy()
     rng = r["tiles"].ranges.cpu().numpy().reshape(-1, 2).astype(np.int64)
