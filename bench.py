@@ -572,6 +572,15 @@ def run_ours(args):
     streaming = None
     if not args.no_e2e:
         streaming = run_streaming(st, args, world, barrier)
+    quality = None
+    if rank == 0 and not args.no_e2e:
+        # Section 3's comparison on a small seeded scene (about a second of GPU time)
+        from paper_2608_27735_gb300.bcd import quality_experiment
+        h = quality_experiment()
+        quality = {k: [round(x, 5) for x in v] for k, v in h.items()}
+        quality["note"] = ("eval loss (L1 + 0.2 D-SSIM of the full composited render, mean over 8 "
+                           "cameras) after 0..3 cycles; 2x2x1 grid, 4000 Gaussians, equal step "
+                           "counts; full_scene = one block")
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, log)
@@ -586,6 +595,7 @@ def run_ours(args):
         "cpu_baseline": cpu,
         "e2e": e2e,
         "streaming_one_fb_pair": streaming,
+        "bcd_quality": quality,
         "gpu_launches": int(launches),
         "clocks": clocks,
         "ops": {k: {"avg_ms": round(v["avg_ms"], 4), "share": round(share[k], 4)} for k, v in ops.items()},

@@ -1,0 +1,43 @@
+"""The block coordinate descent schedule over every block (Section 2) and the comparison of
+Section 3 on a seeded synthetic scene: ABCD approaches full-scene training, the ablated
+variant (blocks trained without F and B) does not."""
+import numpy as np
+import pytest
+
+import paper_2608_27735_gb300 as ab
+from paper_2608_27735_gb300 import scenegen as sg
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+def test_abcd_matches_full_scene_quality_and_ablation_does_not():
+    ab.build()
+    from paper_2608_27735_gb300.bcd import quality_experiment
+    h = quality_experiment(T=100, cycles=3)
+    full, abcd, abl = h["full_scene"], h["abcd"], h["ablated"]
+    assert full[-1] < 0.15 * full[0]
+    assert abcd[-1] < 0.15 * abcd[0]
+    assert abcd[-1] < 3.0 * full[-1]
+    assert abl[-1] > 0.5 * abl[0] and abl[-1] > 5.0 * abcd[-1]
+    # ABCD starts from the layered render of the same scene as the ablated variant
+    assert abcd[0] == pytest.approx(abl[0], rel=1e-6)
+
+
+def test_one_block_abcd_is_plain_training():
+    """On a one-block grid F and B are transparent, so ABCD and its ablation run the same
+    steps: the same losses up to the order of the backward's atomic sums."""
+    ab.build()
+    from paper_2608_27735_gb300.bcd import BCD, default_lr
+    s = sg.grid_scene((1, 1, 1), 5.0, 600, 0, seed=7)
+    s.cameras = sg.ring_cameras(4, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 64, 48, seed=7)
+    tg = np.stack([sg.random_image(48, 64, 3, seed=20 + k) for k in range(4)]).astype(np.float32)
+    res = []
+    for mode in ("abcd", "ablated"):
+        run = BCD(s.gaussians, (1, 1, 1), s.grid.origin, 5.0, s.cameras, tg, 40, default_lr(5.0),
+                  mode=mode, seed=3)
+        run.cycle()
+        res.append((run.loss.cpu().numpy(), run.eval_loss()))
+    np.testing.assert_allclose(res[0][0], res[1][0], rtol=1e-4)
+    assert res[0][1] == pytest.approx(res[1][1], rel=1e-4)
