@@ -288,6 +288,26 @@ def backward(splats: SplatSet, offsets, ids, width, height, G, F=None, B=None, b
     return grad2d
 
 
+def backward_pixels(splats: SplatSet, offsets, ids, width, height, G, pixels, F=None, B=None,
+                    bg=None, opts=None):
+    """backward() over the listed pixels only (linear indices): equal to it when G vanishes
+    at every other pixel (each pixel's terms carry a factor of G)."""
+    opts = opts or default_opts()
+    H, W = height, width
+    offsets = np.ascontiguousarray(offsets, dtype=np.int64)
+    ids = np.ascontiguousarray(ids, dtype=np.int32)
+    F, B = _img(F, H, W), _img(B, H, W)
+    bgv = None if bg is None else _f64(bg)
+    Gv = _img(G, H, W, 3)
+    pix = np.ascontiguousarray(np.sort(np.asarray(pixels, dtype=np.int64)), dtype=np.int32)
+    grad2d = np.zeros((splats.s.n, 9))
+    rc = lib().orc_backward_pixels(C.byref(splats.s), _p(offsets), _p(ids), W, H, C.byref(opts),
+                                   _p(F), _p(B), _p(bgv), _p(Gv), _p(pix), int(pix.shape[0]),
+                                   _p(grad2d))
+    assert rc == 0
+    return grad2d
+
+
 def composite_layers(layers, order):
     """Left fold of 'over' over layers[order[k]]; layers [L, H, W, 4] -> [H, W, 4]."""
     layers = _f64(layers)

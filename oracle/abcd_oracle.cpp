@@ -600,6 +600,27 @@ int orc_backward_image(const orc_splats* s, const long long* offsets, const int*
   return 0;
 }
 
+int orc_backward_pixels(const orc_splats* s, const long long* offsets, const int* ids,
+                        int width, int height, const orc_opts* o, const double* F,
+                        const double* B, const double* bg, const double* G,
+                        const int* pixels, int n_pixels, double* grad2d) {
+  // the same sum as orc_backward_image over the listed pixels only: a pixel whose upstream
+  // gradient G is zero adds exactly zero to every component, so for a G that vanishes
+  // outside the list the two agree
+  const int tx = (width + o->tile - 1) / o->tile;
+  std::memset(grad2d, 0, sizeof(double) * 9 * (size_t)s->n);
+  for (int k = 0; k < n_pixels; ++k) {
+    const int p = pixels[k];
+    if (p < 0 || p >= width * height) return 1;
+    const int px = p % width, py = p / width;
+    const long long t = (long long)(py / o->tile) * tx + (px / o->tile);
+    orc_backward_pixel(s, ids + offsets[t], (int)(offsets[t + 1] - offsets[t]), px, py, o,
+                       F ? F + 4 * (size_t)p : nullptr, B ? B + 4 * (size_t)p : nullptr, bg,
+                       nullptr, 0, G + 3 * (size_t)p, grad2d);
+  }
+  return 0;
+}
+
 int orc_composite_layers(int n_pixels, const double* layers, const int* order, int count,
                          double* out) {
 #pragma omp parallel for schedule(static)

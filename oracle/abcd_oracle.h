@@ -151,6 +151,13 @@ int orc_backward_image(const orc_splats* s, const long long* offsets, const int*
                        const double* B, const double* bg, const double* G /*[H][W][3]*/,
                        double* grad2d /*[n][9], overwritten*/);
 
+/* orc_backward_image restricted to the pixels listed (linear indices, ascending); equal to it
+ * when G is zero at every other pixel.  Returns 1 for an index outside the image. */
+int orc_backward_pixels(const orc_splats* s, const long long* offsets, const int* ids,
+                        int width, int height, const orc_opts* o, const double* F,
+                        const double* B, const double* bg, const double* G,
+                        const int* pixels, int n_pixels, double* grad2d);
+
 /* Left fold of X over Y = X + (1 - X.a) * Y over layers[order[k]] for k in the given
  * sequence, starting from transparent.  layers: [L][P][4]. out: [P][4]. */
 int orc_composite_layers(int n_pixels, const double* layers, const int* order, int count,

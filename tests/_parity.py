@@ -93,7 +93,7 @@ def _in(rect, x, y):
 LOG2E = 1.4426950408889634
 
 
-def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, delta=1e-4):
+def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, delta=1e-4, tiles=None):
     """Entries (Gaussian, tile) the GPU may list or not.
 
     The oracle lists tile t of Gaussian g when t is in g's square and the least sigma over
@@ -101,35 +101,49 @@ def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, delta=1e-4
     log2 units with a margin: kept when sigma' * 0.999 <= (1.001 thr' + 0.01) * 1.001.
     Returns (opt_list, opt_render): tile -> set of ids whose listing may differ, and the
     subset where the Gaussian might still reach alpha_min at a pixel (render alternatives
-    needed); the rest of opt_list is skipped by every pixel either way."""
+    needed); the rest of opt_list is skipped by every pixel either way.  tiles: only these
+    tiles (all if None)."""
     tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
     opt_list, opt_render = {}, {}
-    for g in np.nonzero(np.any(hi != 0, axis=1) & (P["depth"] > 0.2))[0]:
+
+    def visit(g, x, y):
         o = P["opacity"][g]
         u, v = P["uv"][g]
         thr = math.log(o / alpha_min) * LOG2E if o >= alpha_min else -1.0
         lim = (thr * 1.001 + 0.01) * 1.001 if thr >= 0 else -1.0
-        for y in range(hi[g, 1], hi[g, 3]):
-            for x in range(hi[g, 0], hi[g, 2]):
-                m = LOG2E * oracle.box_min_sigma(P["conic"][g], x * tile + 0.5 - u,
-                                                 x * tile + tile - 0.5 - u,
-                                                 y * tile + 0.5 - v, y * tile + tile - 0.5 - v)
-                in_sq_certain = _in(lo[g], x, y)
-                keep_certain = thr >= 0 and m <= thr * (1 - delta) - delta
-                keep_possible = thr >= 0 and m * 0.999 <= lim * (1 + delta) + delta
-                if (in_sq_certain and keep_certain) or not keep_possible:
-                    continue
-                t = y * tx + x
-                opt_list.setdefault(t, set()).add(int(g))
-                if thr >= 0 and m <= thr * (1 + delta) + delta:
-                    opt_render.setdefault(t, set()).add(int(g))
+        m = LOG2E * oracle.box_min_sigma(P["conic"][g], x * tile + 0.5 - u,
+                                         x * tile + tile - 0.5 - u,
+                                         y * tile + 0.5 - v, y * tile + tile - 0.5 - v)
+        in_sq_certain = _in(lo[g], x, y)
+        keep_certain = thr >= 0 and m <= thr * (1 - delta) - delta
+        keep_possible = thr >= 0 and m * 0.999 <= lim * (1 + delta) + delta
+        if (in_sq_certain and keep_certain) or not keep_possible:
+            return
+        t = y * tx + x
+        opt_list.setdefault(t, set()).add(int(g))
+        if thr >= 0 and m <= thr * (1 + delta) + delta:
+            opt_render.setdefault(t, set()).add(int(g))
+
+    live = np.any(hi != 0, axis=1) & (P["depth"] > 0.2)
+    if tiles is None:
+        for g in np.nonzero(live)[0]:
+            for y in range(hi[g, 1], hi[g, 3]):
+                for x in range(hi[g, 0], hi[g, 2]):
+                    visit(g, x, y)
+    else:
+        for t in sorted(set(int(t) for t in tiles)):
+            x, y = t % tx, t // tx
+            cand = live & (hi[:, 0] <= x) & (x < hi[:, 2]) & (hi[:, 1] <= y) & (y < hi[:, 3])
+            for g in np.nonzero(cand)[0]:
+                visit(g, x, y)
     return opt_list, opt_render
 
 
-def check_tile_lists(gpu_ranges, gpu_ids, off, ids, P, opt, n_tiles):
-    """GPU lists == oracle lists up to optional members, sorted by (fp32 depth, id)."""
+def check_tile_lists(gpu_ranges, gpu_ids, off, ids, P, opt, n_tiles, tiles=None):
+    """GPU lists == oracle lists up to optional members, sorted by (fp32 depth, id); over the
+    given tiles (all if None)."""
     keys = P["depth_key"].astype(np.int64)
-    for t in range(n_tiles):
+    for t in (range(n_tiles) if tiles is None else tiles):
         s, e = int(gpu_ranges[t, 0]), int(gpu_ranges[t, 1])
         L = [int(v) for v in gpu_ids[s:e]] if e > s else []
         O = [int(v) for v in ids[off[t]:off[t + 1]]]

@@ -282,6 +282,26 @@ def test_render_invariants_tiny_scene():
     assert (R["n_used"] > 0).mean() > 0.3
 
 
+def test_backward_over_a_pixel_list_equals_the_full_backward():
+    """The restricted backward (the sampled full-size tests use it) is the full one when the
+    upstream gradient vanishes off the list: every term of a pixel carries a factor of G."""
+    s = sg.tiny_scene()
+    cam = s.cameras[2]
+    g = s.gaussians.subset(slice(0, 3000))
+    P = oracle.project(g, cam)
+    off, ids = oracle.tile_lists(P, cam.width, cam.height)
+    sp = oracle.SplatSet.from_proj(P)
+    rng = np.random.default_rng(12)
+    pix = rng.choice(cam.width * cam.height, 900, replace=False)
+    G = np.zeros((cam.height, cam.width, 3))
+    G.reshape(-1, 3)[pix] = rng.normal(size=(900, 3))
+    F = sg.premultiplied_layers(2, cam.height, cam.width, seed=4).astype(np.float64)
+    full = oracle.backward(sp, off, ids, cam.width, cam.height, G, F=F[0], B=F[1])
+    part = oracle.backward_pixels(sp, off, ids, cam.width, cam.height, G, pix, F=F[0], B=F[1])
+    assert np.abs(full).max() > 0
+    np.testing.assert_array_equal(part, full)
+
+
 def _layer_lists(P, cells, part_order, tx, ty):
     """Per-tile lists of the explicit render of the given partitions, layered in order."""
     per = []
