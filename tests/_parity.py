@@ -56,33 +56,56 @@ def splats_with_margins(g, cam, P):
                                      eps_alpha=EPS_ALPHA, eps_step=EPS_STEP)
 
 
-def rect_bounds(P, cam, m_uv, tile=16):
-    """Smallest and largest tile rectangle any admissible fp32 rounding can give."""
+def near_tiles(P, cam, m_uv, tiles, tile=16):
+    """Gaussians whose tile rectangle, under any admissible fp32 rounding, may meet one of
+    `tiles` (a superset: every other Gaussian is listed in none of them either way)."""
+    tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
+    ind = np.zeros((ty + 1, tx + 1), np.int64)
+    for t in tiles:
+        ind[t // tx + 1, t % tx + 1] = 1
+    S = ind.cumsum(0).cumsum(1)
+    r = np.ceil(P["radius_exact"] * (1 + 1e-5)) + 1
+    u, v = P["uv"][:, 0], P["uv"][:, 1]
+    cl = lambda a, m: np.clip(a, 0, m).astype(np.int64)
+    x0 = cl(np.floor((u - m_uv[:, 0] - r) / tile), tx)
+    x1 = cl(np.floor((u + m_uv[:, 0] + r) / tile) + 1, tx)
+    y0 = cl(np.floor((v - m_uv[:, 1] - r) / tile), ty)
+    y1 = cl(np.floor((v + m_uv[:, 1] + r) / tile) + 1, ty)
+    cnt = S[y1, x1] - S[y0, x1] - S[y1, x0] + S[y0, x0]
+    live = (P["depth"] > 0.2) & (P["radius_exact"] > 0)
+    return np.nonzero(live & (cnt > 0))[0]
+
+
+def rect_bounds(P, cam, m_uv, tile=16, idx=None):
+    """Smallest and largest tile rectangle any admissible fp32 rounding can give (for the
+    Gaussians idx only, all if None; the others get empty rectangles).  The candidates are
+    the rectangles of both roundings of the radius (ceil of 3 sqrt(lambda_max) at its
+    relative uncertainty) and of the corners of the (u, v) uncertainty box."""
     tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
     n = P["visible"].shape[0]
     lo = np.zeros((n, 4), np.int64)
     hi = np.zeros((n, 4), np.int64)
     amb_radius = np.zeros(n, bool)
-    for i in range(n):
-        if P["depth"][i] <= 0.2 or P["radius_exact"][i] == 0:
-            continue
-        re = P["radius_exact"][i]
-        rs = {math.ceil(re * (1 - 1e-5)), math.ceil(re * (1 + 1e-5))}
-        amb_radius[i] = len(rs) > 1
-        u, v = P["uv"][i]
-        du, dv = m_uv[i]
-        cands = []
-        for r in rs:
-            for uu in (u - du, u + du):
-                for vv in (v - dv, v + dv):
-                    x0 = min(max(math.floor((uu - r) / tile), 0), tx)
-                    y0 = min(max(math.floor((vv - r) / tile), 0), ty)
-                    x1 = min(max(math.floor((uu + r) / tile) + 1, 0), tx)
-                    y1 = min(max(math.floor((vv + r) / tile) + 1, 0), ty)
-                    cands.append((x0, y0, x1, y1))
-        c = np.array(cands)
-        lo[i] = [c[:, 0].max(), c[:, 1].max(), c[:, 2].min(), c[:, 3].min()]
-        hi[i] = [c[:, 0].min(), c[:, 1].min(), c[:, 2].max(), c[:, 3].max()]
+    sel = np.arange(n) if idx is None else np.asarray(idx, np.int64)
+    sel = sel[(P["depth"][sel] > 0.2) & (P["radius_exact"][sel] != 0)]
+    if sel.size == 0:
+        return lo, hi, amb_radius
+    re = P["radius_exact"][sel].astype(np.float64)
+    r_lo, r_hi = np.ceil(re * (1 - 1e-5)), np.ceil(re * (1 + 1e-5))
+    amb_radius[sel] = r_lo != r_hi
+    u, v = P["uv"][sel, 0].astype(np.float64), P["uv"][sel, 1].astype(np.float64)
+    du, dv = m_uv[sel, 0], m_uv[sel, 1]
+    cx0, cy0, cx1, cy1 = [], [], [], []
+    for r in (r_lo, r_hi):
+        for uu in (u - du, u + du):
+            for vv in (v - dv, v + dv):
+                cx0.append(np.clip(np.floor((uu - r) / tile), 0, tx))
+                cy0.append(np.clip(np.floor((vv - r) / tile), 0, ty))
+                cx1.append(np.clip(np.floor((uu + r) / tile) + 1, 0, tx))
+                cy1.append(np.clip(np.floor((vv + r) / tile) + 1, 0, ty))
+    cx0, cy0, cx1, cy1 = (np.stack(c).astype(np.int64) for c in (cx0, cy0, cx1, cy1))
+    lo[sel] = np.stack([cx0.max(0), cy0.max(0), cx1.min(0), cy1.min(0)], 1)
+    hi[sel] = np.stack([cx0.min(0), cy0.min(0), cx1.max(0), cy1.max(0)], 1)
     return lo, hi, amb_radius
 
 
