@@ -163,6 +163,17 @@ __device__ __forceinline__ int stage_fill(const unsigned* ids, unsigned start, i
     }
     next += kGroup;
   }
+  // the blend loops read up to one (forward) or two (backward) slots past the last survivor
+  // as masked-out entries: they must hold finite zeros, not another kernel's leftovers (a
+  // zero weight times a non-finite value is not zero)
+  constexpr int kPad = WITH_ID ? 2 : 1;
+  constexpr int kSlots = WITH_ID ? kBatch + 2 : kBatch;
+  if (lane < kPad && total + lane < kSlots) {
+    s_uv[total + lane] = make_float2(0.f, 0.f);
+    s_co[total + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+    s_rgb[total + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (WITH_ID) s_id[total + lane] = 0u;
+  }
   __syncwarp();
   return total;
 }
