@@ -169,7 +169,8 @@ extern "C" abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* la
 }
 
 // ---- K1 over packed layers (the cache's tile-sparse format, see abcd_render_refresh_packed):
-// one CTA per 16x16 tile, two pixels per thread; a layer whose tile is not stored is
+// one CTA per 16x16 tile, two pixels per thread, the tile's map entries of all layers read
+// once into shared memory; a layer whose tile is not stored is
 // transparent, and folding (0, 0, 0, 0) leaves the accumulator unchanged, so skipping it gives
 // the dense result bit for bit.  Only the stored tiles are read.
 namespace abcd {
@@ -182,31 +183,32 @@ struct PackedTable {
 
 constexpr int kPackedThreads = kTileThreads / 2;
 
-// acc (2 pixels) = acc over the two pixels of every layer in [k0, k1) stored at this tile
-__device__ __forceinline__ void fold_packed(const PackedTable& pt, int k0, int k1, int tile,
+// acc (2 pixels) = acc over the two pixels of every layer in [k0, k1) stored at this tile;
+// m: the tile's block index in every layer (shared memory, -1: not stored).  Eight layers'
+// loads are in flight before they are folded.
+constexpr int kPackedInFlight = 8;
+
+__device__ __forceinline__ void fold_packed(const PackedTable& pt, const int* m, int k0, int k1,
                                             int unit, float* acc) {
   int k = k0;
-  for (; k + 4 <= k1; k += 4) {
-    int m[4];
+  for (; k + kPackedInFlight <= k1; k += kPackedInFlight) {
+    uint4 r[kPackedInFlight];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) m[j] = __ldg(pt.map[k + j] + tile);
-    uint4 r[4];
+    for (int j = 0; j < kPackedInFlight; ++j)
+      r[j] = m[k + j] >= 0 ? __ldcs(pt.data[k + j] + (size_t)m[k + j] * kPackedThreads + unit)
+                           : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      r[j] = m[j] >= 0 ? __ldcs(pt.data[k + j] + (size_t)m[j] * kPackedThreads + unit) : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (m[j] < 0) continue;
+    for (int j = 0; j < kPackedInFlight; ++j) {
+      if (m[k + j] < 0) continue;
       float v[8];
       unpack_h8(r[j], v);
       fold<2>(acc, v);
     }
   }
   for (; k < k1; ++k) {
-    const int m = __ldg(pt.map[k] + tile);
-    if (m < 0) continue;
+    if (m[k] < 0) continue;
     float v[8];
-    unpack_h8(__ldcs(pt.data[k] + (size_t)m * kPackedThreads + unit), v);
+    unpack_h8(__ldcs(pt.data[k] + (size_t)m[k] * kPackedThreads + unit), v);
     fold<2>(acc, v);
   }
 }
@@ -225,8 +227,11 @@ __global__ void __launch_bounds__(kPackedThreads)
 composite_packed_kernel(const __grid_constant__ PackedTable pt, int nf, int nb, int width,
                         int height, int tiles_x, void* Fout, void* Bout, int out_f16) {
   pdl_prologue();
+  __shared__ int s_map[kMaxLayers];
   const int tile = blockIdx.x;
   const int unit = threadIdx.x;                       // pixels 2 unit, 2 unit + 1 of the tile
+  for (int k = threadIdx.x; k < nf + nb; k += blockDim.x) s_map[k] = __ldg(pt.map[k] + tile);
+  __syncthreads();
   const int r = unit / (kTile / 2), c = 2 * (unit % (kTile / 2));
   const int y = (tile / tiles_x) * kTile + r, x = (tile % tiles_x) * kTile + c;
   for (int side = 0; side < 2; ++side) {
@@ -235,8 +240,8 @@ composite_packed_kernel(const __grid_constant__ PackedTable pt, int nf, int nb, 
     float acc[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    if (side == 0) fold_packed(pt, 0, nf, tile, unit, acc);
-    else fold_packed(pt, nf, nf + nb, tile, unit, acc);
+    if (side == 0) fold_packed(pt, s_map, 0, nf, unit, acc);
+    else fold_packed(pt, s_map, nf, nf + nb, unit, acc);
     if (y < height) {
       if (x < width) store_pixel_out(out, out_f16, (long long)y * width + x, acc);
       if (x + 1 < width) store_pixel_out(out, out_f16, (long long)y * width + x + 1, acc + 4);

@@ -193,7 +193,7 @@ loss_kernel(const float* __restrict__ xin, const float* __restrict__ yin, int W,
         const float vx = ss[o].x - mx * mx, vy = ss[o].y - my * my, cxy = mc[o] - mx * my;
         const float N1 = 2.f * mx * my + C1, N2 = 2.f * cxy + C2;
         const float D1 = mx * mx + my * my + C1, D2 = vx + vy + C2;
-        const float iD = __frcp_rn(D1 * D2);
+        const float iD = __fdividef(1.f, D1 * D2);   // fast reciprocal (about 2 ulp)
         const float S = N1 * N2 * iD;
         const float dvx = -S * (D1 * iD);           // -S / D2
         const float dcxy = 2.f * N1 * iD;
