@@ -44,7 +44,7 @@ BWD_FLOP_PER_PAIR = 68      # recompute + d alpha + colour, opacity, mean and co
 LOSS_FLOP_PER_PX = 1000     # five 11-tap windows twice (separable), SSIM terms, 3 channels
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=3, help="timed ABCD stages")
@@ -58,7 +58,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sample-every", type=int, default=10, help="per-op event sampling stride")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def dist_env():
@@ -66,6 +66,23 @@ def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return rank, world, local
+
+
+def max_over_ranks(ms, world):
+    """The slowest rank's time: replicas report the whole job's throughput over it."""
+    if world <= 1:
+        return float(ms)
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_value(stages, T, world, ms):
+    """Active-block steps/s of the whole job: every rank runs `stages` stages of T steps."""
+    return stages * T * world / (ms / 1e3)
 
 
 # ---------------------------------------------------------------------------------------
@@ -530,13 +547,8 @@ def run_ours(args):
     clocks = clk.stop()
     st.ctx.sync()
     ms = e0.elapsed_time(e1)
-    ms_t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        import torch.distributed as dist
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms = float(ms_t.item())
-    steps_total = args.steps * args.T * world
-    value = steps_total / (ms / 1e3)
+    ms = max_over_ranks(ms, world)
+    value = replica_value(args.steps, args.T, world, ms)
     # per-op breakdown from the sampled events
     ops = {}
     for name, evs in st.events.items():
@@ -693,11 +705,7 @@ def run_e2e(st: Stage, args, world, barrier):
     ms = max(e0.elapsed_time(e1), wall * 1e3)
     print(f"[bench] e2e: host issue time {host_ms / args.steps:.1f} ms, device {e0.elapsed_time(e1) / args.steps:.1f} ms, "
           f"wall {wall * 1e3 / args.steps:.1f} ms per stage", file=sys.stderr, flush=True)
-    ms_t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        import torch.distributed as dist
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms = float(ms_t.item())
+    ms = max_over_ranks(ms, world)
     st.gt = gts[0]
     return {"value": round(args.steps * args.T * world / (ms / 1e3), 2), "unit": UNIT,
             "h2d_bytes_per_step": int(counted["h2d"]), "d2h_bytes_per_step": int(counted["d2h"]),
@@ -813,11 +821,7 @@ def run_streaming(st: Stage, args, world, barrier):
     wall = time.perf_counter() - t0
     barrier()
     ms = max(e0.elapsed_time(e1), wall * 1e3)
-    ms_t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        import torch.distributed as dist
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms = float(ms_t.item())
+    ms = max_over_ranks(ms, world)
     per_step = sum(host_frozen[c].numel() * 2 + (P - 1) * st.n_t * 4 + host_gt[c].numel() * 4
                    for c in st.observing) / len(st.observing)
     return {"value": round(args.steps * args.T * world / (ms / 1e3), 2), "unit": UNIT,
