@@ -318,6 +318,18 @@ def composite_layers(layers, order):
     return out
 
 
+def layer_visibility(layers, order):
+    """(visible[L], coverage[L]) of layers [L, H, W, 4] taken in `order` (front to back)."""
+    layers = _f64(layers)
+    L, H, W, _ = layers.shape
+    order = np.ascontiguousarray(order, dtype=np.int32)
+    vis, cov = np.zeros(L), np.zeros(L)
+    rc = lib().orc_layer_visibility(H * W, L, _p(layers), _p(order), int(order.shape[0]),
+                                    _p(vis), _p(cov))
+    assert rc == 0, "repeated or out-of-range layer index"
+    return vis, cov
+
+
 def loss(x, y, lam, with_grad=True):
     x, y = _f64(x), _f64(y)
     H, W, _ = x.shape

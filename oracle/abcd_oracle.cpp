@@ -635,6 +635,30 @@ int orc_composite_layers(int n_pixels, const double* layers, const int* order, i
   return 0;
 }
 
+int orc_layer_visibility(int n_pixels, int n_layers, const double* layers, const int* order,
+                         int count, double* visible, double* coverage) {
+  std::vector<char> seen(n_layers > 0 ? n_layers : 0, 0);
+  for (int k = 0; k < count; ++k) {
+    if (order[k] < 0 || order[k] >= n_layers || seen[order[k]]) return 1;
+    seen[order[k]] = 1;
+  }
+  for (int j = 0; j < n_layers; ++j) visible[j] = coverage[j] = 0.0;
+  for (int k = 0; k < count; ++k) {
+    const int j = order[k];
+    double vis = 0.0, cov = 0.0;
+    for (int p = 0; p < n_pixels; ++p) {
+      double T = 1.0;                          // transmittance of the layers in front of j
+      for (int i = 0; i < k; ++i) T *= 1.0 - layers[((size_t)order[i] * n_pixels + p) * 4 + 3];
+      const double a = layers[((size_t)j * n_pixels + p) * 4 + 3];
+      vis += a * T;
+      cov += a;
+    }
+    visible[j] = vis / n_pixels;
+    coverage[j] = cov / n_pixels;
+  }
+  return 0;
+}
+
 int orc_ssim_map(int width, int height, const double* x, const double* y, double* map) {
   const double C1 = 0.01 * 0.01, C2 = 0.03 * 0.03;
   double w[11];

@@ -22,6 +22,8 @@
  *   orc_render_pixel/image closed form, invariants, associativity identity
  *   orc_backward_pixel/... central finite differences (fp64), incl. the F/B alpha term
  *   orc_composite_layers   constant-layer closed form, split invariance
+ *   orc_layer_visibility   telescoping identity against the composite's alpha, opaque and
+ *                          single-layer cases, the culling error bound
  *   orc_loss               SSIM(x,x)=1, scipy 2-D correlation, finite differences
  *   orc_adam               first-step closed form, hand-computed second step
  *   orc_assign_cells / orc_partition_split   brute-force ray sampling of the depth order
@@ -162,6 +164,15 @@ int orc_backward_pixels(const orc_splats* s, const long long* offsets, const int
  * sequence, starting from transparent.  layers: [L][P][4]. out: [P][4]. */
 int orc_composite_layers(int n_pixels, const double* layers, const int* order, int count,
                          double* out);
+
+/* Visibility of each layer of one camera's depth order (Section 5: visibility thresholds and
+ * occlusion culling of camera-partition pairs).  For the layer at position k of the order,
+ * with alpha_k its alpha and T_k the product of (1 - alpha) over the layers before it:
+ * visible[order[k]] = mean over pixels of alpha_k T_k, coverage[order[k]] = mean of alpha_k;
+ * layers not listed get 0.  layers: [L][P][4]; order: count distinct indices below L.
+ * Returns 1 for a repeated or out-of-range index. */
+int orc_layer_visibility(int n_pixels, int n_layers, const double* layers, const int* order,
+                         int count, double* visible, double* coverage);
 
 /* (1 - lam) * mean|x - y| + lam * (1 - mean SSIM(x, y)), 11x11 Gaussian window (sigma 1.5),
  * zero padding, C1 = 0.01^2, C2 = 0.03^2; x, y: [H][W][3].  grad (may be NULL) = dL/dx. */

@@ -369,6 +369,62 @@ def test_over_constant_layers_golden():
     np.testing.assert_array_equal(out[0, 0], expect)
 
 
+def _premultiplied_layers(rng, L, H, W, clear=0.3):
+    """Random premultiplied RGBA layers (colour <= alpha), each with a share of clear pixels."""
+    a = rng.uniform(0, 1, (L, H, W, 1)) * (rng.uniform(0, 1, (L, H, W, 1)) > clear)
+    return np.concatenate([a * rng.uniform(0, 1, (L, H, W, 3)), a], -1)
+
+
+def test_visibility_constant_layers_closed_form():
+    """Constant alphas 0.5, 0.25, 0.8 taken in the order 2, 0, 1: each layer's visible share is
+    its alpha times the transmittance of the layers before it, worked by hand."""
+    alphas = [0.5, 0.25, 0.8]
+    st = np.stack([np.full((3, 5, 4), a) for a in alphas])
+    vis, cov = oracle.layer_visibility(st, [2, 0, 1])
+    np.testing.assert_allclose(cov, alphas, rtol=0, atol=1e-15)
+    np.testing.assert_allclose(vis, [0.5 * 0.2, 0.25 * 0.2 * 0.5, 0.8], rtol=0, atol=1e-15)
+    # a layer left out of the order has neither; an opaque layer hides everything behind it
+    vis, cov = oracle.layer_visibility(st, [1])
+    np.testing.assert_allclose(vis, [0, 0.25, 0], atol=1e-15)
+    np.testing.assert_allclose(cov, [0, 0.25, 0], atol=1e-15)
+    opaque = np.concatenate([st, np.ones((1, 3, 5, 4))])
+    vis, cov = oracle.layer_visibility(opaque, [3, 0, 1, 2])
+    np.testing.assert_allclose(vis, [0, 0, 0, 1], atol=1e-15)
+    np.testing.assert_allclose(cov, alphas + [1.0], atol=1e-15)
+
+
+def test_visibility_telescopes_to_the_composite_alpha():
+    """1 - prod(1 - a_k) = sum_k a_k prod_{i<k} (1 - a_i): the visible shares of all layers add
+    up to the mean alpha of their composite (checked against composite_layers)."""
+    rng = np.random.default_rng(11)
+    st = _premultiplied_layers(rng, 7, 9, 13)
+    for order in ([0, 1, 2, 3, 4, 5, 6], [6, 2, 4, 0, 5, 1, 3], [3, 1, 5]):
+        vis, cov = oracle.layer_visibility(st, order)
+        comp = oracle.composite_layers(st, order)
+        assert abs(vis.sum() - comp[..., 3].mean()) < 1e-13, order
+        np.testing.assert_allclose(cov[order], st[order][..., 3].mean(axis=(1, 2)), atol=1e-15)
+        assert np.all(vis <= cov + 1e-15)
+
+
+def test_culling_error_bound():
+    """Leaving a set D of layers out of the composite changes every channel of every pixel by
+    at most sum_{j in D} a_j T_j when colours are premultiplied and at most alpha: the mean
+    error of the culled composite is at most the sum of the dropped layers' visible shares."""
+    rng = np.random.default_rng(12)
+    st = _premultiplied_layers(rng, 6, 11, 10)
+    order = [4, 0, 5, 2, 1, 3]
+    vis, _ = oracle.layer_visibility(st, order)
+    full = oracle.composite_layers(st, order)
+    for drop in ({0}, {4}, {3}, {0, 2}, {4, 5, 1}, set(order)):
+        kept = [j for j in order if j not in drop]
+        culled = oracle.composite_layers(st, kept) if kept else np.zeros_like(full)
+        err = np.abs(full - culled).mean(axis=(0, 1))
+        bound = sum(vis[j] for j in drop)
+        assert np.all(err <= bound + 1e-13), (drop, err, bound)
+        if drop == set(order):          # nothing kept: the alpha error is the bound exactly
+            assert abs(err[3] - bound) < 1e-13
+
+
 def test_bg_and_fb_in_closed_form():
     """Empty active block: out = F over B (+ (1 - out.a) bg)."""
     rng = np.random.default_rng(1)
