@@ -642,19 +642,20 @@ int orc_layer_visibility(int n_pixels, int n_layers, const double* layers, const
     if (order[k] < 0 || order[k] >= n_layers || seen[order[k]]) return 1;
     seen[order[k]] = 1;
   }
-  for (int j = 0; j < n_layers; ++j) visible[j] = coverage[j] = 0.0;
-  for (int k = 0; k < count; ++k) {
-    const int j = order[k];
-    double vis = 0.0, cov = 0.0;
-    for (int p = 0; p < n_pixels; ++p) {
-      double T = 1.0;                          // transmittance of the layers in front of j
-      for (int i = 0; i < k; ++i) T *= 1.0 - layers[((size_t)order[i] * n_pixels + p) * 4 + 3];
+  std::vector<double> vis(n_layers > 0 ? n_layers : 0, 0.0), cov(vis);
+  for (int p = 0; p < n_pixels; ++p) {
+    double T = 1.0;                  // product of (1 - alpha) over the layers walked so far
+    for (int k = 0; k < count; ++k) {
+      const int j = order[k];
       const double a = layers[((size_t)j * n_pixels + p) * 4 + 3];
-      vis += a * T;
-      cov += a;
+      vis[j] += a * T;
+      cov[j] += a;
+      T *= 1.0 - a;
     }
-    visible[j] = vis / n_pixels;
-    coverage[j] = cov / n_pixels;
+  }
+  for (int j = 0; j < n_layers; ++j) {
+    visible[j] = vis[j] / n_pixels;
+    coverage[j] = cov[j] / n_pixels;
   }
   return 0;
 }
