@@ -584,6 +584,7 @@ def run_ours(args):
     streaming = None
     if not args.no_e2e:
         streaming = run_streaming(st, args, world, barrier)
+    visibility = run_visibility(st)
     quality = None
     if rank == 0 and not args.no_e2e:
         # Section 3's comparison on a small seeded scene (about a second of GPU time)
@@ -592,7 +593,8 @@ def run_ours(args):
         quality = {k: [round(x, 5) for x in v] for k, v in h.items()}
         quality["note"] = ("eval loss (L1 + 0.2 D-SSIM of the full composited render, mean over 8 "
                            "cameras) after 0..3 cycles; 2x2x1 grid, 4000 Gaussians, equal step "
-                           "counts; full_scene = one block")
+                           "counts; full_scene = one block; abcd_culled = camera-partition pairs "
+                           "below a 1% visible share dropped")
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, log)
@@ -608,6 +610,7 @@ def run_ours(args):
         "e2e": e2e,
         "streaming_one_fb_pair": streaming,
         "bcd_quality": quality,
+        "visibility_culling": visibility,
         "gpu_launches": int(launches),
         "clocks": clocks,
         "ops": {k: {"avg_ms": round(v["avg_ms"], 4), "share": round(share[k], 4)} for k, v in ops.items()},
@@ -617,6 +620,64 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+TAU_VISIBLE = 1e-3
+
+
+def run_visibility(st: Stage, reps=3):
+    """Section 5's visibility threshold and occlusion culling on the stage's cache: every
+    observing camera's layers (the active one as last refreshed) in its depth order, one
+    abcd_layer_visibility_packed call per camera, timed on the context's stream; the pairs
+    whose visible share is below TAU_VISIBLE, the stored bytes they hold and the bound on the
+    composite error that dropping them gives.  The calls read every camera's stored tiles in
+    turn (many GB, no L2 reuse)."""
+    torch, ab = st.torch, st.ab
+    P, a = st.n_parts, st.active
+    cams = st.observing
+    C = len(cams)
+    vis = torch.empty(C, P, dtype=torch.float64, device=st.dev)
+    cov = torch.empty_like(vis)
+    tables = []
+    for ci in cams:
+        f, b = st.splits[ci]
+        maps = [st.pk_map[ci, p] for p in range(P)]
+        data = [st.pk_frozen[ci][st.pk_off[ci][p]:] if p != a else st.pk_active[ci] for p in range(P)]
+        tables.append(ab.PackedLayers(maps, data, f + [a] + b, P))
+
+    def sweep():
+        for j in range(C):
+            ab.abcd_layer_visibility_tables(st.ctx, tables[j], st.W, st.H, vis[j], cov[j])
+
+    sweep()
+    st.ctx.sync()
+    e0 = torch_event(torch, st.stream)
+    for _ in range(reps):
+        sweep()
+    e1 = torch_event(torch, st.stream)
+    st.ctx.sync()
+    us = e0.elapsed_time(e1) * 1e3 / (reps * C)
+    v, c = vis.cpu().numpy(), cov.cpu().numpy()
+    keep = ab.cull_pairs(v, c, TAU_VISIBLE)
+    keep[:, a] = True                     # the active block's own pairs are being trained
+    counts = st.pk_count.cpu().numpy()[cams].astype(np.int64)
+    stored = int(counts.sum()) * 2048
+    per_cam = stored / C + P * st.n_t * 4
+    frozen = np.ones(P, bool)
+    frozen[a] = False
+    culled = (~keep) & frozen[None, :]
+    culled_bytes = int(counts[culled].sum()) * 2048
+    bound = float(np.where(culled, v, 0.0).sum(axis=1).max())
+    peaks = load_peaks()
+    peak = peaks["hbm_gbs"] if peaks else 6800.0
+    gbs = per_cam / (us * 1e-6) / 1e9
+    return {"tau_visible": TAU_VISIBLE, "pairs": C * (P - 1), "culled_pairs": int(culled.sum()),
+            "frozen_cache_bytes": int(st.cache_bytes), "culled_bytes": culled_bytes,
+            "max_mean_error_bound": round(bound, 6),
+            "mean_visible_of_culled": round(float(v[culled].mean()), 7) if culled.any() else None,
+            "us_per_camera": round(us, 2), "algorithmic_bytes_per_camera": int(per_cam),
+            "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4),
+            "kernel": "visibility_kernel<true>"}
 
 
 def run_e2e(st: Stage, args, world, barrier):

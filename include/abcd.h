@@ -257,6 +257,33 @@ abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_ma
                                         int split, int width, int height, void* F_out,
                                         void* B_out, int out_dtype);
 
+/* Visibility of the cached layers of one camera, for the visibility thresholds and occlusion
+ * culling of camera-partition pairs that Section 5 proposes.  The layers are taken in `order`
+ * (host, `count` distinct indices below L, front to back; a layer left out counts as absent).
+ * For the layer at position k, with alpha_k its alpha and T_k the product of (1 - alpha) over
+ * the layers before it:
+ *   visible[order[k]]  = mean over the W x H pixels of alpha_k T_k (its share of the composite),
+ *   coverage[order[k]] = mean of alpha_k (its image area, occluders ignored);
+ * both 0 for layers not in the order.  Leaving a set D of layers out of the composite changes
+ * every channel of every pixel by at most the sum over D of alpha_j T_j (premultiplied colours
+ * at most alpha), so the sum of the dropped layers' visible shares bounds the mean error of
+ * the culled composite.  layers: host array of L device pointers to fp16 [H][W][4]
+ * premultiplied RGBA (8-byte aligned); visible, coverage: device double [L] (coverage may be
+ * NULL), overwritten.  The sums are exact in 24-bit fixed point per pixel value (result
+ * independent of the order of the additions); they use the context's workspace (ABCD_ERR_WORKSPACE
+ * without one).  L <= 256; ABCD_ERR_INVALID_ARG for a repeated or out-of-range index, a NULL
+ * or misaligned layer or output. */
+abcd_status abcd_layer_visibility(abcd_ctx* ctx, const void* const* layers, int L,
+                                  const int* order, int count, int width, int height,
+                                  double* visible, double* coverage);
+
+/* abcd_layer_visibility over packed layers (tile_maps[k], packed[k] as for
+ * abcd_composite_cache_packed); a tile a layer does not store is transparent. */
+abcd_status abcd_layer_visibility_packed(abcd_ctx* ctx, const int* const* tile_maps,
+                                         const void* const* packed, int L, const int* order,
+                                         int count, int width, int height, double* visible,
+                                         double* coverage);
+
 /* The loss of abcd_loss without a context or workspace, for callers that cannot allocate
  * device memory: code running inside a host application that owns every device allocation
  * (its own pool or arena, with raw cudaMalloc forbidden), or a caller that must not allocate

@@ -99,6 +99,10 @@ _SIGS = {
                                    C.c_void_p, C.c_void_p, C.c_void_p],
     "abcd_composite_cache_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
                                     C.c_int, C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int],
+    "abcd_layer_visibility": [C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_int, C.c_int,
+                              C.c_int, C.c_void_p, C.c_void_p],
+    "abcd_layer_visibility_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
+                                     C.c_int, C.c_int, C.c_int, C.c_void_p, C.c_void_p],
     "abcd_train_step": [C.c_void_p] + [C.c_void_p] * 8 + [C.c_void_p, C.c_void_p, C.c_int,
                          C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_float, C.c_void_p,
                          C.c_void_p, C.c_float, C.c_float, C.c_float, C.c_int],
@@ -425,6 +429,45 @@ def abcd_composite_cache_packed(ctx: Context, tile_maps, packed, order, split, w
     ordr = (C.c_int * max(1, L))(*[int(k) for k in order])
     ctx.check(lib().abcd_composite_cache_packed(ctx.h, maps, data, L, ordr, int(split), int(width),
                                                 int(height), _p(F_out), _p(B_out), int(out_dtype)))
+
+
+def abcd_layer_visibility(ctx: Context, layers, order, width, height, visible, coverage=None):
+    """layers: list of L fp16 CUDA tensors [H][W][4] (None for a layer not in `order`); order:
+    the layers front to back; visible / coverage: float64 CUDA tensors [L]."""
+    L = len(layers)
+    arr = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in layers])
+    ordr = (C.c_int * max(1, len(order)))(*[int(k) for k in order])
+    ctx.check(lib().abcd_layer_visibility(ctx.h, arr, L, ordr, len(order), int(width), int(height),
+                                          _p(visible), _p(coverage)))
+
+
+def abcd_layer_visibility_packed(ctx: Context, tile_maps, packed, order, width, height, visible,
+                                 coverage=None):
+    """The same over packed layers (tile_maps / packed: lists of CUDA tensors)."""
+    L = len(tile_maps)
+    maps = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in tile_maps])
+    data = (C.c_void_p * max(1, L))(*[(t.data_ptr() if t is not None else None) for t in packed])
+    ordr = (C.c_int * max(1, len(order)))(*[int(k) for k in order])
+    ctx.check(lib().abcd_layer_visibility_packed(ctx.h, maps, data, L, ordr, len(order), int(width),
+                                                 int(height), _p(visible), _p(coverage)))
+
+
+def abcd_layer_visibility_tables(ctx: Context, pl, width, height, visible, coverage=None):
+    """abcd_layer_visibility_packed over the tables of a PackedLayers built with split = L
+    (every layer of the order, front to back)."""
+    ctx.check(lib().abcd_layer_visibility_packed(ctx.h, pl.maps, pl.data, pl.L, pl.order, pl.L,
+                                                 int(width), int(height), _p(visible),
+                                                 _p(coverage)))
+
+
+def cull_pairs(visible, coverage, tau_visible, tau_area=0.0):
+    """Camera-partition pairs to keep (Section 5's visibility threshold and occlusion culling):
+    a layer stays when its visible share of the composite is at least tau_visible and its
+    image area at least tau_area.  The dropped layers' visible shares add up to a bound on the
+    mean per-channel error of the culled composite.  Host arrays in, boolean mask out."""
+    import numpy as np
+    v, c = np.asarray(visible, dtype=np.float64), np.asarray(coverage, dtype=np.float64)
+    return (v >= float(tau_visible)) & (c >= float(tau_area))
 
 
 class TrainStep:

@@ -14,8 +14,9 @@ from __future__ import annotations
 import numpy as np
 
 from . import (ABCD_F16, ABCD_F32, Context, FwdState, Gaussians, Projected, Tiles, TrainStep,
-               abcd_assign_cells, abcd_composite_cache, abcd_loss, abcd_partition_split,
-               abcd_project, abcd_bin_sort, abcd_render_composite_fwd, camera, _torch)
+               abcd_assign_cells, abcd_composite_cache, abcd_layer_visibility, abcd_loss,
+               abcd_partition_split, abcd_project, abcd_bin_sort, abcd_render_composite_fwd,
+               camera, cull_pairs, _torch)
 
 # Adam learning rates per group (means, log-scales, quaternions, opacity logits, SH degree 0,
 # higher SH degrees): 3DGS-style defaults, the means' scaled by the scene extent.
@@ -28,10 +29,15 @@ class BCD:
 
     gaussians: scenegen.Gaussians of the whole scene; dims, origin, side: the grid; cameras:
     objects with R, t, fx, fy, cx, cy, width, height, position; targets: float32 [C][H][W][3];
-    mode: "abcd" (F and B from the cache) or "ablated" (F = B = transparent)."""
+    mode: "abcd" (F and B from the cache) or "ablated" (F = B = transparent).  cull_tau: the
+    visibility threshold of Section 5's culling of camera-partition pairs (None: no culling):
+    after every refresh each camera's layers are measured (abcd_layer_visibility) and a pair
+    whose visible share of the camera's composite is below cull_tau is dropped, from F and B
+    of the other blocks' stages and from the cameras its own block trains on, until a later
+    measurement brings it back."""
 
     def __init__(self, gaussians, dims, origin, side, cameras, targets, T, lr, mode="abcd",
-                 device=0, seed=0, lambda_ssim=0.2, max_pairs=2_000_000):
+                 device=0, seed=0, lambda_ssim=0.2, max_pairs=2_000_000, cull_tau=None):
         assert mode in ("abcd", "ablated")
         torch = _torch()
         self.torch, self.mode, self.T = torch, mode, int(T)
@@ -70,31 +76,63 @@ class BCD:
         self.queue = []
         self.loss = torch.zeros(max(1, self.T), device="cuda")
         self.steps_done = 0
+        self.cull_tau = cull_tau
+        self.keep = np.ones((C, n_blocks), bool)     # camera-partition pairs in use
+        self.visible = np.zeros((C, n_blocks))
         for b in self.blocks:
-            self.refresh(b)
+            self.refresh(b, measure=False)
+        self.measure_visibility()
 
     # ---- pieces of a stage
-    def refresh(self, b):
-        """Re-renders block b's cached layer for every camera (K2-K5, refresh output)."""
+    def refresh(self, b, measure=True):
+        """Re-renders block b's cached layer for every camera (K2-K5, refresh output), then
+        (with culling) measures the cameras' layers again."""
         th = self.theta[b]
         for ci, cam in enumerate(self.cams):
             abcd_project(self.ctx, th, cam, None, self.proj)
             abcd_bin_sort(self.ctx, self.proj, th.n, cam, self.tiles)
             abcd_render_composite_fwd(self.ctx, cam, None, self.proj, self.tiles,
                                       refresh_f16=self.layers[ci, b])
+        if measure:
+            self.measure_visibility()
+
+    def measure_visibility(self):
+        """Visible share of every camera-partition pair in its camera's composite of all
+        cached layers, and the pairs kept at the threshold."""
+        if self.cull_tau is None:
+            return
+        torch = self.torch
+        C, n_blocks = self.keep.shape
+        vis = torch.empty(C, n_blocks, dtype=torch.float64, device="cuda")
+        cov = torch.empty_like(vis)
+        for ci in range(C):
+            order, _ = self.order[ci, 0]
+            abcd_layer_visibility(self.ctx, [self.layers[ci, k] for k in range(n_blocks)], order,
+                                  self.W, self.H, vis[ci], cov[ci])
+        self.visible = vis.cpu().numpy()
+        self.keep = cull_pairs(self.visible, cov.cpu().numpy(), self.cull_tau)
 
     def composite(self, b):
-        """F and B of every camera around active block b, from the cached layers (K1)."""
-        n_blocks = self.layers.shape[1]
+        """F and B of every camera around active block b, from the cached layers of the pairs
+        in use (K1)."""
         for ci in range(len(self.cams)):
-            order, split = self.order[ci, b]
-            lay = [self.layers[ci, k] for k in range(n_blocks)]
-            lay[b] = None
-            abcd_composite_cache(self.ctx, lay, order, split, self.W, self.H, self.F[ci], self.B[ci])
+            order, _ = self.order[ci, b]
+            kept = [k for k in order if k == b or self.keep[ci, k]]
+            split = kept.index(b)
+            lay = [self.layers[ci, k] if k != b else None for k in kept]
+            abcd_composite_cache(self.ctx, lay, list(range(len(kept))), split, self.W, self.H,
+                                 self.F[ci], self.B[ci])
 
-    def next_camera(self):
-        if not self.queue:                   # shuffle without replacement, reshuffled when used up
-            self.queue = list(self.rng.permutation(len(self.cams)))
+    def cameras_of(self, b):
+        """Cameras block b trains on: those whose pair with b is in use."""
+        return [ci for ci in range(len(self.cams)) if self.keep[ci, b]]
+
+    def next_camera(self, allowed=None):
+        """Shuffle without replacement over the allowed cameras, reshuffled when used up."""
+        allowed = list(range(len(self.cams))) if allowed is None else list(allowed)
+        self.queue = [ci for ci in self.queue if ci in allowed]
+        if not self.queue:
+            self.queue = [allowed[i] for i in self.rng.permutation(len(allowed))]
         return int(self.queue.pop())
 
     def stage(self, b):
@@ -105,12 +143,13 @@ class BCD:
             self.composite(b)
         step = TrainStep(self.ctx, th, grads, m, v, self.proj, self.tiles, self.out, self.state,
                          self.lr, lambda_ssim=self.lam)
-        for t in range(self.T):
-            ci = self.next_camera()
+        allowed = self.cameras_of(b)
+        for t in range(self.T if allowed else 0):
+            ci = self.next_camera(allowed)
             F = self.F[ci] if self.mode == "abcd" else None
             B = self.B[ci] if self.mode == "abcd" else None
             step(self.cams[ci], F, B, self.gt[ci], self.loss[t:t + 1], t + 1)
-        self.steps_done += self.T
+        self.steps_done += self.T if allowed else 0
         self.refresh(b)
 
     def cycle(self):
@@ -140,11 +179,14 @@ class BCD:
         return float(acc.mean().item())
 
 
-def quality_experiment(T=100, cycles=3, per_cell=1000, n_cams=8, width=96, height=72, seed=2024):
+def quality_experiment(T=100, cycles=3, per_cell=1000, n_cams=8, width=96, height=72, seed=2024,
+                       cull_tau=0.01):
     """Section 3's comparison on a seeded synthetic scene (a 2x2x1 grid of side 5, SH degree
     0): full-scene training (one block, 4 T steps per cycle), ABCD and the ablated variant (4
     blocks, T steps each per cycle), the same number of steps in all three, against targets
-    rendered from a perturbed copy of the scene.  Returns {name: [eval loss after 0..cycles]}."""
+    rendered from a perturbed copy of the scene; and ABCD with the camera-partition pairs
+    culled at visible share cull_tau (Section 5), which trains each block on the cameras that
+    see it.  Returns {name: [eval loss after 0..cycles]}; the eval renders every layer."""
     from . import scenegen as sg
     dims, side = (2, 2, 1), 5.0
     s = sg.grid_scene(dims, side, per_cell, 0, seed=seed)
@@ -156,11 +198,12 @@ def quality_experiment(T=100, cycles=3, per_cell=1000, n_cams=8, width=96, heigh
               s.cameras, blank, 0, default_lr(2 * side))
     targets = np.stack([ref.render_full(ci)[..., :3].cpu().numpy() for ci in range(n_cams)])
     out = {}
-    for name, d, sd, mode, t in (("full_scene", (1, 1, 1), 2 * side, "abcd", 4 * T),
-                                 ("abcd", dims, side, "abcd", T),
-                                 ("ablated", dims, side, "ablated", T)):
+    for name, d, sd, mode, t, tau in (("full_scene", (1, 1, 1), 2 * side, "abcd", 4 * T, None),
+                                      ("abcd", dims, side, "abcd", T, None),
+                                      ("ablated", dims, side, "ablated", T, None),
+                                      ("abcd_culled", dims, side, "abcd", T, cull_tau)):
         run = BCD(s.gaussians, d, origin, sd, s.cameras, targets, t, default_lr(2 * side),
-                  mode=mode, seed=seed + 2)
+                  mode=mode, seed=seed + 2, cull_tau=tau)
         hist = [run.eval_loss()]
         for _ in range(cycles):
             run.cycle()

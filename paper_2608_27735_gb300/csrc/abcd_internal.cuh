@@ -19,6 +19,7 @@ constexpr int kMaxRadixBlocks = 1024;     // upper bound used to size the histog
 constexpr int kMaxLossBlocks = 1 << 16;
 constexpr int kMaxLayers = 256;
 constexpr long long kMaxDiffCells = 1LL << 20;   // (tiles_x + 1) * (tiles_y + 1)
+constexpr int kVisSumCopies = 8;          // copies of the layer visibility sums
 
 // Device status bits (OR-ed into the status word; abcd_sync reports the lowest set code).
 constexpr unsigned kStatusCapacity = 1u << ABCD_ERR_CAPACITY;
@@ -64,6 +65,8 @@ struct Workspace {
   unsigned* ck_count;               // items allocated by the last forward with a state
   unsigned* ck_first;               // [4 max_tiles] end of each block's first chunk, or ~0
   int ck_cap;
+  unsigned long long* vis_sums;     // [kVisSumCopies][2][kMaxLayers] layer visibility sums (zero between calls)
+  unsigned* vis_ticket;             // CTAs of the visibility call that finished
 };
 
 constexpr int kRenderSubPerTile = 4;      // render CTAs (8x8 pixel blocks) per 16x16 tile

@@ -7,6 +7,8 @@
 // accumulator stays in registers across layers, F and B are written once.  Four layers are
 // loaded before they are folded so each thread keeps 64 bytes in flight.  The grid is a
 // multiple of the SM count and strides over pixel pairs.
+#include <algorithm>
+
 #include "abcd_internal.cuh"
 
 namespace abcd {
@@ -170,24 +172,73 @@ extern "C" abcd_status abcd_composite_cache(abcd_ctx* ctx, const void* const* la
 
 // ---- K1 over packed layers (the cache's tile-sparse format, see abcd_render_refresh_packed):
 // one CTA per 16x16 tile, two pixels per thread, the tile's map entries of all layers read
-// once into shared memory; a layer whose tile is not stored is
-// transparent, and folding (0, 0, 0, 0) leaves the accumulator unchanged, so skipping it gives
-// the dense result bit for bit.  Only the stored tiles are read.
+// once into shared memory; a layer whose tile is not stored is transparent, and folding
+// (0, 0, 0, 0) leaves the accumulator unchanged, so skipping it gives the dense result bit for
+// bit.  Only the stored tiles are read.
 namespace abcd {
 namespace {
 
 struct PackedTable {
   const int* map[kMaxLayers];       // front layers in order, then back layers in order
-  const uint4* data[kMaxLayers];    // 16-byte units: two fp16 RGBA pixels
+  const uint4* data[kMaxLayers];    // 2 KB blocks of 16-byte units: two fp16 RGBA pixels
 };
 
 constexpr int kPackedThreads = kTileThreads / 2;
+constexpr int kPackedInFlight = 8;
+
+// The positions k in [0, n) with s_map[k] >= 0, in order, into s_list; returns how many (every
+// thread).  Warp 0 compacts with ballots; the caller's next __syncthreads publishes s_list.
+__device__ __forceinline__ void compact_stored(const int* s_map, int n, int* s_list,
+                                               int* s_count) {
+  if (threadIdx.x >= 32) return;
+  const int lane = threadIdx.x;
+  int run = 0;
+  for (int k0 = 0; k0 < n; k0 += 32) {
+    const bool st = k0 + lane < n && s_map[k0 + lane] >= 0;
+    const unsigned b = __ballot_sync(0xffffffffu, st);
+    if (st) s_list[run + __popc(b & ((1u << lane) - 1u))] = k0 + lane;
+    run += __popc(b);
+  }
+  if (lane == 0) *s_count = run;
+}
+
+// Calls fn(k, v) in order for the listed positions s_list[j0 .. j1) (v: this thread's 16-byte
+// unit of layer k's block at the tile), the loads of kPackedInFlight blocks in flight before
+// they are used.
+template <typename Fn>
+__device__ __forceinline__ void for_each_listed(const uint4* const* data, const int* s_map,
+                                                const int* s_list, int j0, int j1, Fn fn) {
+  const int unit = threadIdx.x;
+  int j = j0;
+  for (; j + kPackedInFlight <= j1; j += kPackedInFlight) {
+    uint4 r[kPackedInFlight];
+#pragma unroll
+    for (int i = 0; i < kPackedInFlight; ++i) {
+      const int k = s_list[j + i];
+      r[i] = __ldcs(data[k] + (size_t)s_map[k] * kPackedThreads + unit);
+    }
+#pragma unroll
+    for (int i = 0; i < kPackedInFlight; ++i) fn(s_list[j + i], r[i]);
+  }
+  if (j < j1) {
+    uint4 r[kPackedInFlight];
+#pragma unroll
+    for (int i = 0; i < kPackedInFlight; ++i) {
+      if (j + i >= j1) break;
+      const int k = s_list[j + i];
+      r[i] = __ldcs(data[k] + (size_t)s_map[k] * kPackedThreads + unit);
+    }
+#pragma unroll
+    for (int i = 0; i < kPackedInFlight; ++i) {
+      if (j + i >= j1) break;
+      fn(s_list[j + i], r[i]);
+    }
+  }
+}
 
 // acc (2 pixels) = acc over the two pixels of every layer in [k0, k1) stored at this tile;
 // m: the tile's block index in every layer (shared memory, -1: not stored).  Eight layers'
 // loads are in flight before they are folded.
-constexpr int kPackedInFlight = 8;
-
 __device__ __forceinline__ void fold_packed(const PackedTable& pt, const int* m, int k0, int k1,
                                             int unit, float* acc) {
   int k = k0;
@@ -291,4 +342,206 @@ extern "C" abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* con
                       launch_pdl(composite_packed_kernel, dim3(tiles_x * tiles_y),
                                  dim3(kPackedThreads), 0, ctx->stream, pt, nf, nb, width, height,
                                  tiles_x, F_out, B_out, out_dtype == ABCD_F16 ? 1 : 0));
+}
+
+// ---- visibility of the layers of one camera's depth order (Section 5: visibility thresholds
+// and occlusion culling of camera-partition pairs).  For the layer at position k, with alpha_k
+// its alpha and T_k the product of (1 - alpha) over the layers before it, visible = mean over
+// pixels of alpha_k T_k and coverage = mean of alpha_k.  Leaving a set D of layers out of the
+// composite changes every channel of every pixel by at most the sum over D of alpha_j T_j
+// (colours premultiplied and at most alpha), so the dropped layers' visible shares bound the
+// mean error of a culled composite.
+// One CTA per 16x16 tile at a time (a grid that strides over tiles), two pixels per thread, T
+// in registers across the order.  Sums are exact: every value is rounded to 24-bit fixed point
+// and added as an integer (a warp reduction, then 64-bit shared and global accumulators), so
+// the result does not depend on the order of the additions; CTAs add to one of kVisCopies
+// copies of the global sums (fewer atomics on one address) and the last CTA to finish adds the
+// copies, converts them to means and clears them for the next call.
+namespace abcd {
+namespace {
+
+constexpr float kVisScale = 16777216.f;       // 2^24
+constexpr int kVisInFlight = 8;               // layers whose loads are in flight together
+constexpr int kVisCopies = kVisSumCopies;     // global accumulators (CTA b adds to copy b % 8)
+
+struct VisTable {
+  const int* map[kMaxLayers];                 // packed: tile map per position of the order
+  const uint4* data[kMaxLayers];              // packed: 2 KB blocks; dense: half [H][W][4]
+  int layer[kMaxLayers];                      // layer index at each position
+};
+
+// Adds one layer's contribution at the thread's two pixels (alphas a0, a1) to the CTA's sums
+// of position k, then takes the layer's transmittance factor into T0, T1.  Warp-uniform k.
+__device__ __forceinline__ void vis_accumulate(float a0, float a1, float& T0, float& T1, int k,
+                                               unsigned long long (*s_sum)[kMaxLayers]) {
+  const unsigned vf = __float2uint_rn(a0 * T0 * kVisScale) + __float2uint_rn(a1 * T1 * kVisScale);
+  const unsigned cf = __float2uint_rn(a0 * kVisScale) + __float2uint_rn(a1 * kVisScale);
+  T0 *= 1.f - a0;
+  T1 *= 1.f - a1;
+  const unsigned vs = __reduce_add_sync(0xffffffffu, vf);
+  const unsigned cs = __reduce_add_sync(0xffffffffu, cf);
+  if ((threadIdx.x & 31) == 0) {
+    if (vs) atomicAdd(&s_sum[0][k], (unsigned long long)vs);
+    if (cs) atomicAdd(&s_sum[1][k], (unsigned long long)cs);
+  }
+}
+
+__device__ __forceinline__ float alpha_hi(unsigned w) {
+  return __high2float(*reinterpret_cast<const __half2*>(&w));
+}
+
+template <bool PACKED>
+__global__ void __launch_bounds__(kPackedThreads, 10)
+visibility_kernel(const __grid_constant__ VisTable vt, int count, int L, int width, int height,
+                  int tiles_x, int n_tiles, unsigned long long* sums, unsigned* ticket,
+                  double* visible, double* coverage) {
+  pdl_prologue();
+  __shared__ unsigned long long s_sum[2][kMaxLayers];
+  __shared__ int s_map[kMaxLayers];
+  __shared__ int s_list[kMaxLayers];
+  __shared__ int s_count;
+  __shared__ bool s_last;
+  for (int k = threadIdx.x; k < count; k += blockDim.x) { s_sum[0][k] = 0ull; s_sum[1][k] = 0ull; }
+  const int unit = threadIdx.x;
+  const int r = unit / (kTile / 2), c = 2 * (unit % (kTile / 2));
+  for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    __syncthreads();                                   // s_map, s_list of the previous tile done
+    if (PACKED) {
+      for (int k = threadIdx.x; k < count; k += blockDim.x) s_map[k] = __ldg(vt.map[k] + tile);
+      __syncthreads();
+      compact_stored(s_map, count, s_list, &s_count);
+    }
+    __syncthreads();
+    const int y = (tile / tiles_x) * kTile + r, x = (tile % tiles_x) * kTile + c;
+    const bool in0 = y < height && x < width, in1 = y < height && x + 1 < width;
+    float T0 = 1.f, T1 = 1.f;
+    if (PACKED) {
+      for_each_listed(vt.data, s_map, s_list, 0, s_count, [&](int k, uint4 u) {
+        vis_accumulate(in0 ? alpha_hi(u.y) : 0.f, in1 ? alpha_hi(u.w) : 0.f, T0, T1, k, s_sum);
+      });
+      continue;
+    }
+    const long long p = (long long)y * width + x;
+    for (int k0 = 0; k0 < count; k0 += kVisInFlight) {
+      // the loads of kVisInFlight layers are issued before any is used (they do not depend on
+      // T), so a tile waits for memory once per group instead of once per layer
+      unsigned w0[kVisInFlight], w1[kVisInFlight];
+#pragma unroll
+      for (int j = 0; j < kVisInFlight; ++j) {
+        w0[j] = w1[j] = 0u;
+        const int k = k0 + j;
+        if (k >= count) continue;
+        const uint2* d = reinterpret_cast<const uint2*>(vt.data[k]);
+        if (in0) w0[j] = __ldcs(d + p).y;
+        if (in1) w1[j] = __ldcs(d + p + 1).y;
+      }
+#pragma unroll
+      for (int j = 0; j < kVisInFlight; ++j)
+        if (k0 + j < count)
+          vis_accumulate(alpha_hi(w0[j]), alpha_hi(w1[j]), T0, T1, k0 + j, s_sum);
+    }
+  }
+  __syncthreads();
+  unsigned long long* mine = sums + (size_t)(blockIdx.x % kVisCopies) * 2 * kMaxLayers;
+  for (int k = threadIdx.x; k < count; k += blockDim.x) {
+    if (s_sum[0][k]) atomicAdd(mine + k, s_sum[0][k]);
+    if (s_sum[1][k]) atomicAdd(mine + kMaxLayers + k, s_sum[1][k]);
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const double inv = 1.0 / ((double)kVisScale * (double)width * (double)height);
+  for (int j = threadIdx.x; j < L; j += blockDim.x) {
+    visible[j] = 0.0;
+    if (coverage) coverage[j] = 0.0;
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < count; k += blockDim.x) {
+    unsigned long long v = 0ull, cv = 0ull;
+    for (int cp = 0; cp < kVisCopies; ++cp) {
+      v += atomicExch(sums + (size_t)cp * 2 * kMaxLayers + k, 0ull);
+      cv += atomicExch(sums + (size_t)cp * 2 * kMaxLayers + kMaxLayers + k, 0ull);
+    }
+    visible[vt.layer[k]] = (double)v * inv;
+    if (coverage) coverage[vt.layer[k]] = (double)cv * inv;
+  }
+  if (threadIdx.x == 0) *ticket = 0u;
+}
+
+// Checks the order and the outputs, fills vt.layer and launches.
+abcd_status visibility_launch(abcd_ctx* ctx, const char* who, VisTable& vt, bool packed, int L,
+                              const int* order, int count, int width, int height,
+                              double* visible, double* coverage) {
+  if (!visible || ((uintptr_t)visible & 7) || ((uintptr_t)coverage & 7))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "%s: null or misaligned output", who);
+  const int tiles_x = (width + kTile - 1) / kTile, tiles_y = (height + kTile - 1) / kTile;
+  const int n_tiles = tiles_x * tiles_y;
+  const int grid = std::max(1, std::min(n_tiles, 8 * ctx->num_sms));
+  const auto kernel = packed ? visibility_kernel<true> : visibility_kernel<false>;
+  return check_launch(ctx, "visibility_kernel",
+                      launch_pdl(kernel, dim3(grid), dim3(kPackedThreads), 0, ctx->stream, vt,
+                                 count, L, width, height, tiles_x, n_tiles, ctx->ws.vis_sums,
+                                 ctx->ws.vis_ticket, visible, coverage));
+}
+
+// The order: count distinct indices below L.
+bool valid_order(const int* order, int count, int L) {
+  unsigned char seen[kMaxLayers] = {0};
+  for (int k = 0; k < count; ++k) {
+    if (order[k] < 0 || order[k] >= L || seen[order[k]]) return false;
+    seen[order[k]] = 1;
+  }
+  return true;
+}
+
+}  // namespace
+}  // namespace abcd
+
+extern "C" abcd_status abcd_layer_visibility(abcd_ctx* ctx, const void* const* layers, int L,
+                                             const int* order, int count, int width, int height,
+                                             double* visible, double* coverage) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!has_workspace(ctx)) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_layer_visibility: no workspace");
+  if (L < 0 || L > kMaxLayers || count < 0 || count > L || (count > 0 && (!layers || !order)) ||
+      width <= 0 || height <= 0 || !valid_order(order, count, L))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_layer_visibility: bad layer list, order or size");
+  VisTable vt;
+  for (int k = 0; k < count; ++k) {
+    const void* p = layers[order[k]];
+    if (!p || ((uintptr_t)p & 7))
+      return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_layer_visibility: layer %d is NULL or misaligned", order[k]);
+    vt.map[k] = nullptr;
+    vt.data[k] = static_cast<const uint4*>(p);
+    vt.layer[k] = order[k];
+  }
+  return visibility_launch(ctx, "abcd_layer_visibility", vt, false, L, order, count, width,
+                           height, visible, coverage);
+}
+
+extern "C" abcd_status abcd_layer_visibility_packed(abcd_ctx* ctx, const int* const* tile_maps,
+                                                    const void* const* packed, int L,
+                                                    const int* order, int count, int width,
+                                                    int height, double* visible,
+                                                    double* coverage) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (!has_workspace(ctx)) return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_layer_visibility_packed: no workspace");
+  if (L < 0 || L > kMaxLayers || count < 0 || count > L ||
+      (count > 0 && (!tile_maps || !packed || !order)) || width <= 0 || height <= 0 ||
+      !valid_order(order, count, L))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_layer_visibility_packed: bad layer list, order or size");
+  VisTable vt;
+  for (int k = 0; k < count; ++k) {
+    const int* m = tile_maps[order[k]];
+    const void* d = packed[order[k]];
+    if (!m || !d || ((uintptr_t)d & 15) || ((uintptr_t)m & 3))
+      return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_layer_visibility_packed: layer %d is NULL or misaligned", order[k]);
+    vt.map[k] = m;
+    vt.data[k] = static_cast<const uint4*>(d);
+    vt.layer[k] = order[k];
+  }
+  return visibility_launch(ctx, "abcd_layer_visibility_packed", vt, true, L, order, count,
+                           width, height, visible, coverage);
 }

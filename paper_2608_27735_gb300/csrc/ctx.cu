@@ -164,6 +164,8 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.ck_items = (uint4*)take(16ull * (size_t)w.ck_cap);
   w.ck_count = (unsigned*)take(256);
   w.ck_first = (unsigned*)take(4ull * 4 * (size_t)w.max_tiles);
+  w.vis_sums = (unsigned long long*)take(8ull * kVisSumCopies * 2 * kMaxLayers);
+  w.vis_ticket = (unsigned*)take(256);
   if (ws) *ws = w;
   return off;
 }
@@ -190,6 +192,8 @@ abcd_status abcd_set_workspace(abcd_ctx* ctx, void* ptr, size_t bytes, int max_g
   layout(ctx->ws_base, max_gaussians, max_pairs, max_pixels, &ctx->ws);
   cudaError_t e = cudaMemsetAsync(ctx->ws.status, 0, 256, ctx->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.os_ctr, 0, 256, ctx->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.vis_sums, 0, 8ull * kVisSumCopies * 2 * kMaxLayers, ctx->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.vis_ticket, 0, 256, ctx->stream);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(ctx->ws.os_state, 0, 8ull * kRadixBins * (size_t)ctx->ws.os_tiles, ctx->stream);
   ctx->os_epoch = 0;

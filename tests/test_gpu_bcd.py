@@ -23,6 +23,35 @@ def test_abcd_matches_full_scene_quality_and_ablation_does_not():
     assert abl[-1] > 0.5 * abl[0] and abl[-1] > 5.0 * abcd[-1]
     # ABCD starts from the layered render of the same scene as the ablated variant
     assert abcd[0] == pytest.approx(abl[0], rel=1e-6)
+    # culling the camera-partition pairs below a 1% visible share keeps ABCD's quality far
+    # from the ablation's
+    cul = h["abcd_culled"]
+    assert cul[0] == pytest.approx(abcd[0], rel=1e-6)
+    assert cul[-1] < 0.5 * abl[-1] and cul[-1] < 0.3 * cul[0]
+
+
+def test_culling_at_zero_threshold_changes_nothing():
+    """With a threshold of 0 every pair is kept: the stage composites the same layers in the
+    same order and trains on the same cameras as without culling."""
+    ab.build()
+    from paper_2608_27735_gb300.bcd import BCD, default_lr
+    s = sg.grid_scene((2, 1, 1), 5.0, 500, 0, seed=9)
+    s.cameras = sg.ring_cameras(4, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 64, 48, seed=9)
+    tg = np.stack([sg.random_image(48, 64, 3, seed=40 + k) for k in range(4)]).astype(np.float32)
+    res = []
+    for tau in (None, 0.0):
+        run = BCD(s.gaussians, (2, 1, 1), s.grid.origin, 5.0, s.cameras, tg, 20, default_lr(10.0),
+                  seed=4, cull_tau=tau)
+        run.stage(run.blocks[0])
+        res.append((run.loss.cpu().numpy(), run.F.cpu().numpy(), run.B.cpu().numpy(), run))
+    np.testing.assert_allclose(res[0][0], res[1][0], rtol=1e-4)
+    assert np.array_equal(res[0][1], res[1][1]) and np.array_equal(res[0][2], res[1][2])
+    run = res[1][3]
+    assert run.keep.all() and run.visible.shape == run.keep.shape
+    # every camera's visible shares add up to the mean alpha of its full composite
+    for ci in range(4):
+        full = run.render_full(ci)[..., 3].double().mean().item()
+        assert run.visible[ci].sum() == pytest.approx(full, abs=4 * 2.0 ** -23 + 1e-6)
 
 
 def test_one_block_abcd_is_plain_training():

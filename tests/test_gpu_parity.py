@@ -525,6 +525,99 @@ def test_composite_packed_matches_dense(ctx):
             assert torch.equal(a_.view(torch.int16), b_.view(torch.int16)), split
 
 
+def _blank_tiles(st, tx, ty, share, seed):
+    """Zero a random share of each layer's 16x16 tiles (the layers' transparent regions)."""
+    rng = np.random.default_rng(seed)
+    for k in range(st.shape[0]):
+        for t in np.nonzero(rng.random(tx * ty) < share)[0]:
+            y0, x0 = (t // tx) * 16, (t % tx) * 16
+            st[k, y0:y0 + 16, x0:x0 + 16] = 0
+    return st
+
+
+def visibility_tol(count):
+    """Mean of values rounded to 2^-24 fixed point (2^-25 each) after fp32 transmittance
+    products of up to count factors (relative error <= count 2^-24)."""
+    return 2.0 ** -24 + count * 2.0 ** -23
+
+
+@pytest.mark.parametrize("H,W,L", [(37, 53, 9), (75, 101, 40), (16, 16, 1)])
+def test_layer_visibility_matches_oracle(ctx, H, W, L):
+    """Visible share and coverage of each layer of a depth order (dense and packed layers)
+    against the oracle; the sums are exact integers, so packed equals dense bit for bit and a
+    repeated call returns the same bits (the accumulators are cleared between calls)."""
+    tx, ty = oracle.tiles_xy(W, H)
+    st = _blank_tiles(sg.premultiplied_layers(L, H, W, seed=40 + L).astype(np.float16), tx, ty,
+                      0.3, 6)
+    src = st.astype(np.float64)
+    dense = [torch.from_numpy(st[k]).cuda() for k in range(L)]
+    maps, packs = [], []
+    for k in range(L):
+        m, pk = pack_layer(st[k], tx, ty)
+        maps.append(torch.from_numpy(m).cuda())
+        packs.append(torch.from_numpy(pk if len(pk) else np.zeros((1, 16, 16, 4), np.float16)).cuda())
+    perm = list(sg.random_permutation(L, seed=H))
+    for order in (perm, perm[: max(1, L // 2)], []):
+        vr, cr = oracle.layer_visibility(src, order)
+        got = []
+        for packed_path in (False, True, True):
+            vis = torch.full((L,), -1.0, dtype=torch.float64, device="cuda")
+            cov = torch.full((L,), -1.0, dtype=torch.float64, device="cuda")
+            if packed_path:
+                ab.abcd_layer_visibility_packed(ctx, maps, packs, order, W, H, vis, cov)
+            else:
+                ab.abcd_layer_visibility(ctx, dense, order, W, H, vis, cov)
+            ctx.sync()
+            got.append((vis.cpu().numpy(), cov.cpu().numpy()))
+        tol = visibility_tol(len(order))
+        np.testing.assert_allclose(got[0][0], vr, rtol=0, atol=tol)
+        np.testing.assert_allclose(got[0][1], cr, rtol=0, atol=tol)
+        for g in got[1:]:
+            assert np.array_equal(g[0], got[0][0]) and np.array_equal(g[1], got[0][1])
+
+
+def test_layer_visibility_occlusion_and_errors(ctx):
+    """An opaque layer in front hides every layer behind it exactly; coverage ignores it; a
+    culled composite stays within the bound the dropped layers' visible shares give; bad
+    orders are refused before any launch."""
+    L, H, W = 5, 40, 50
+    st = sg.premultiplied_layers(L, H, W, seed=77).astype(np.float16)
+    st[2, :, :, :] = 0
+    st[2, :, :, 3] = 1                       # an opaque black layer
+    dense = [torch.from_numpy(st[k]).cuda() for k in range(L)]
+    vis = torch.empty(L, dtype=torch.float64, device="cuda")
+    cov = torch.empty(L, dtype=torch.float64, device="cuda")
+    ab.abcd_layer_visibility(ctx, dense, [4, 2, 0, 1, 3], W, H, vis, cov)
+    ctx.sync()
+    v, c = vis.cpu().numpy(), cov.cpu().numpy()
+    assert v[0] == 0 and v[1] == 0 and v[3] == 0 and v[2] > 0
+    np.testing.assert_allclose(c, st[..., 3].astype(np.float64).mean(axis=(1, 2)), atol=visibility_tol(L))
+    # culling by a threshold: the culled composite (abcd_composite_cache over the kept layers)
+    # is within the dropped layers' visible shares of the full one, channel by channel
+    st = sg.premultiplied_layers(L, H, W, seed=78).astype(np.float16)
+    st[1] *= np.float16(0.01)
+    st[3] *= np.float16(0.02)
+    dense = [torch.from_numpy(st[k]).cuda() for k in range(L)]
+    order = [0, 1, 2, 3, 4]
+    ab.abcd_layer_visibility(ctx, dense, order, W, H, vis, cov)
+    full = torch.empty(H, W, 4, device="cuda")
+    ab.abcd_composite_cache(ctx, dense, order, L, W, H, full, None, ab.ABCD_F16, ab.ABCD_F32)
+    ctx.sync()
+    v, c = vis.cpu().numpy(), cov.cpu().numpy()
+    keep = ab.cull_pairs(v, c, tau_visible=0.02)
+    assert not keep[1] and not keep[3] and keep[[0, 2, 4]].all()
+    kept = [j for j in order if keep[j]]
+    culled = torch.empty(H, W, 4, device="cuda")
+    ab.abcd_composite_cache(ctx, [dense[j] for j in kept], list(range(len(kept))), len(kept),
+                            W, H, culled, None, ab.ABCD_F16, ab.ABCD_F32)
+    ctx.sync()
+    err = (full - culled).abs().double().mean(dim=(0, 1)).cpu().numpy()
+    assert np.all(err <= v[~keep].sum() + 1e-6), (err, v[~keep])
+    for bad in ([0, 0], [0, 5], [-1]):
+        with pytest.raises(ab.AbcdError):
+            ab.abcd_layer_visibility(ctx, dense, bad, W, H, vis, cov)
+
+
 def test_adam_matches_oracle(ctx, ragged):
     g = ragged.gaussians.subset(slice(0, 3001))
     theta = ab.Gaussians.from_numpy(g)
