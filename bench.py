@@ -594,7 +594,8 @@ def run_ours(args):
         quality["note"] = ("eval loss (L1 + 0.2 D-SSIM of the full composited render, mean over 8 "
                            "cameras) after 0..3 cycles; 2x2x1 grid, 4000 Gaussians, equal step "
                            "counts; full_scene = one block; abcd_culled = camera-partition pairs "
-                           "below a 1% visible share dropped")
+                           "below a 1% visible share dropped; abcd_overlap = overlapping "
+                           "boundary region of width 1 (a fifth of a cell)")
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, log)

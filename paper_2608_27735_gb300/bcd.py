@@ -14,9 +14,9 @@ from __future__ import annotations
 import numpy as np
 
 from . import (ABCD_F16, ABCD_F32, Context, FwdState, Gaussians, Projected, Tiles, TrainStep,
-               abcd_assign_cells, abcd_composite_cache, abcd_layer_visibility, abcd_loss,
-               abcd_partition_split, abcd_project, abcd_bin_sort, abcd_render_composite_fwd,
-               camera, cull_pairs, _torch)
+               abcd_adam_active, abcd_assign_cells, abcd_backward, abcd_composite_cache,
+               abcd_layer_visibility, abcd_loss, abcd_partition_split, abcd_project,
+               abcd_bin_sort, abcd_render_composite_fwd, camera, cull_pairs, _torch)
 
 # Adam learning rates per group (means, log-scales, quaternions, opacity logits, SH degree 0,
 # higher SH degrees): 3DGS-style defaults, the means' scaled by the scene extent.
@@ -34,10 +34,16 @@ class BCD:
     after every refresh each camera's layers are measured (abcd_layer_visibility) and a pair
     whose visible share of the camera's composite is below cull_tau is dropped, from F and B
     of the other blocks' stages and from the cameras its own block trains on, until a later
-    measurement brings it back."""
+    measurement brings it back.  overlap: the width of the overlapping boundary region that
+    Section 5 proposes (0: none).  Membership stays by the mean, but a block's stage renders,
+    with the block, the other blocks' Gaussians whose means lie within `overlap` of its cell
+    (its halo: frozen, sorted by depth together with the block's own, no gradient step), and
+    for every camera F and B take each donor block's layer re-rendered without them, so every
+    Gaussian is drawn once and the ones near the block's faces in their true depth order."""
 
     def __init__(self, gaussians, dims, origin, side, cameras, targets, T, lr, mode="abcd",
-                 device=0, seed=0, lambda_ssim=0.2, max_pairs=2_000_000, cull_tau=None):
+                 device=0, seed=0, lambda_ssim=0.2, max_pairs=2_000_000, cull_tau=None,
+                 overlap=0.0):
         assert mode in ("abcd", "ablated")
         torch = _torch()
         self.torch, self.mode, self.T = torch, mode, int(T)
@@ -51,7 +57,12 @@ class BCD:
         self.members = [np.nonzero(cells == b)[0] for b in range(n_blocks)]
         self.blocks = [b for b in range(n_blocks) if len(self.members[b])]
         self.theta = {b: Gaussians.from_numpy(gaussians.subset(self.members[b])) for b in self.blocks}
-        n_max = max(len(self.members[b]) for b in self.blocks)
+        # halo of each block: {donor block: positions in the donor's parameters}
+        self.overlap = float(overlap)
+        self.halo = {b: self._halo(b, np.asarray(gaussians.means, np.float64))
+                     for b in self.blocks} if self.overlap > 0 else {b: {} for b in self.blocks}
+        n_max = max(len(self.members[b]) + sum(len(v) for v in self.halo[b].values())
+                    for b in self.blocks)
         self.cams_np = list(cameras)
         self.cams = [camera(c) for c in cameras]
         W, H = int(cameras[0].width), int(cameras[0].height)
@@ -82,6 +93,48 @@ class BCD:
         for b in self.blocks:
             self.refresh(b, measure=False)
         self.measure_visibility()
+
+    def _halo(self, b, means):
+        """Other blocks' Gaussians whose means lie within self.overlap of block b's cell."""
+        gx, gy, _ = self.dims
+        ix, iy, iz = b % gx, (b // gx) % gy, b // (gx * gy)
+        lo = np.asarray(self.origin) + self.side * np.array([ix, iy, iz], np.float64)
+        hi = lo + self.side
+        out = {}
+        for q in self.blocks:
+            if q == b:
+                continue
+            mq = means[self.members[q]]
+            near = np.all((mq >= lo - self.overlap) & (mq <= hi + self.overlap), axis=1)
+            if near.any():
+                out[q] = np.nonzero(near)[0]
+        return out
+
+    def _take(self, g, pos):
+        """Gaussians at positions pos (host int array) of g, as new device tensors."""
+        idx = self.torch.as_tensor(pos, dtype=self.torch.long, device="cuda")
+        return Gaussians(*(t.index_select(0, idx) for t in g.tensors()), g.sh_degree)
+
+    def _stage_theta(self, b):
+        """Block b followed by its halo (one buffer), or block b itself without a halo."""
+        th = self.theta[b]
+        if not self.halo[b]:
+            return th
+        parts = [th] + [self._take(self.theta[q], pos) for q, pos in self.halo[b].items()]
+        return Gaussians(*(self.torch.cat([p.tensors()[k] for p in parts]).contiguous()
+                           for k in range(5)), th.sh_degree)
+
+    def _core_layer(self, q, pos, ci, dst):
+        """Donor block q's layer for camera ci without its Gaussians at positions pos."""
+        keep = np.setdiff1d(np.arange(self.theta[q].n), pos)
+        g = self._take(self.theta[q], keep)
+        if g.n == 0:
+            dst.zero_()
+            return
+        abcd_project(self.ctx, g, self.cams[ci], None, self.proj)
+        abcd_bin_sort(self.ctx, self.proj, g.n, self.cams[ci], self.tiles)
+        abcd_render_composite_fwd(self.ctx, self.cams[ci], None, self.proj, self.tiles,
+                                  refresh_f16=dst)
 
     # ---- pieces of a stage
     def refresh(self, b, measure=True):
@@ -114,12 +167,18 @@ class BCD:
 
     def composite(self, b):
         """F and B of every camera around active block b, from the cached layers of the pairs
-        in use (K1)."""
+        in use (K1); with a halo, each donor block's layer is its layer without the halo."""
+        core = self.torch.empty(len(self.halo[b]), self.H, self.W, 4, dtype=self.torch.float16,
+                                device="cuda")
         for ci in range(len(self.cams)):
             order, _ = self.order[ci, b]
             kept = [k for k in order if k == b or self.keep[ci, k]]
             split = kept.index(b)
             lay = [self.layers[ci, k] if k != b else None for k in kept]
+            for j, (q, pos) in enumerate(self.halo[b].items()):
+                if q in kept:
+                    self._core_layer(q, pos, ci, core[j])
+                    lay[kept.index(q)] = core[j]
             abcd_composite_cache(self.ctx, lay, list(range(len(kept))), split, self.W, self.H,
                                  self.F[ci], self.B[ci])
 
@@ -137,20 +196,58 @@ class BCD:
 
     def stage(self, b):
         th = self.theta[b]
-        torch = self.torch
         grads, m, v = (Gaussians.zeros_like(th) for _ in range(3))   # Adam state per stage
         if self.mode == "abcd":
             self.composite(b)
-        step = TrainStep(self.ctx, th, grads, m, v, self.proj, self.tiles, self.out, self.state,
-                         self.lr, lambda_ssim=self.lam)
         allowed = self.cameras_of(b)
-        for t in range(self.T if allowed else 0):
-            ci = self.next_camera(allowed)
-            F = self.F[ci] if self.mode == "abcd" else None
-            B = self.B[ci] if self.mode == "abcd" else None
-            step(self.cams[ci], F, B, self.gt[ci], self.loss[t:t + 1], t + 1)
+        if self.halo[b]:
+            # the block and its frozen halo are rendered together; Adam updates the block's
+            # rows (the first th.n of every array) only
+            ths = self._stage_theta(b)
+            gs = Gaussians.zeros_like(ths)
+            head = lambda g: Gaussians(*(t[:th.n] for t in g.tensors()), g.sh_degree)
+            for t in range(self.T if allowed else 0):
+                ci = self.next_camera(allowed)
+                cam = self.cams[ci]
+                F = self.F[ci] if self.mode == "abcd" else None
+                B = self.B[ci] if self.mode == "abcd" else None
+                abcd_project(self.ctx, ths, cam, None, self.proj)
+                abcd_bin_sort(self.ctx, self.proj, ths.n, cam, self.tiles)
+                abcd_render_composite_fwd(self.ctx, cam, None, self.proj, self.tiles, F, B,
+                                          ABCD_F16, None, self.out, self.state)
+                abcd_backward(self.ctx, ths, cam, None, self.proj, self.tiles, F, B, ABCD_F16,
+                              None, self.out, self.state, self.gt[ci], self.lam,
+                              self.loss[t:t + 1], None, gs)
+                abcd_adam_active(self.ctx, head(ths), head(gs), m, v, self.lr, 0.9, 0.999,
+                                 1e-15, t + 1)
+            for a_, s_ in zip(th.tensors(), ths.tensors()):
+                a_.copy_(s_[:th.n])
+        else:
+            step = TrainStep(self.ctx, th, grads, m, v, self.proj, self.tiles, self.out,
+                             self.state, self.lr, lambda_ssim=self.lam)
+            for t in range(self.T if allowed else 0):
+                ci = self.next_camera(allowed)
+                F = self.F[ci] if self.mode == "abcd" else None
+                B = self.B[ci] if self.mode == "abcd" else None
+                step(self.cams[ci], F, B, self.gt[ci], self.loss[t:t + 1], t + 1)
         self.steps_done += self.T if allowed else 0
         self.refresh(b)
+
+    def stage_render(self, b, ci):
+        """The composite the first step of block b's stage renders for camera ci (F over the
+        block, with its halo, over B), fp32 RGBA; the parameters are left unchanged."""
+        if self.mode == "abcd":
+            self.composite(b)
+        ths = self._stage_theta(b)
+        cam = self.cams[ci]
+        F = self.F[ci] if self.mode == "abcd" else None
+        B = self.B[ci] if self.mode == "abcd" else None
+        abcd_project(self.ctx, ths, cam, None, self.proj)
+        abcd_bin_sort(self.ctx, self.proj, ths.n, cam, self.tiles)
+        out = self.torch.empty(self.H, self.W, 4, device="cuda")
+        abcd_render_composite_fwd(self.ctx, cam, None, self.proj, self.tiles, F, B, ABCD_F16,
+                                  None, out, None)
+        return out
 
     def cycle(self):
         for b in self.blocks:
@@ -180,13 +277,14 @@ class BCD:
 
 
 def quality_experiment(T=100, cycles=3, per_cell=1000, n_cams=8, width=96, height=72, seed=2024,
-                       cull_tau=0.01):
+                       cull_tau=0.01, overlap=1.0):
     """Section 3's comparison on a seeded synthetic scene (a 2x2x1 grid of side 5, SH degree
     0): full-scene training (one block, 4 T steps per cycle), ABCD and the ablated variant (4
     blocks, T steps each per cycle), the same number of steps in all three, against targets
     rendered from a perturbed copy of the scene; and ABCD with the camera-partition pairs
     culled at visible share cull_tau (Section 5), which trains each block on the cameras that
-    see it.  Returns {name: [eval loss after 0..cycles]}; the eval renders every layer."""
+    see it, and ABCD with an overlapping boundary region of width `overlap` (Section 5).
+    Returns {name: [eval loss after 0..cycles]}; the eval renders every layer."""
     from . import scenegen as sg
     dims, side = (2, 2, 1), 5.0
     s = sg.grid_scene(dims, side, per_cell, 0, seed=seed)
@@ -198,12 +296,14 @@ def quality_experiment(T=100, cycles=3, per_cell=1000, n_cams=8, width=96, heigh
               s.cameras, blank, 0, default_lr(2 * side))
     targets = np.stack([ref.render_full(ci)[..., :3].cpu().numpy() for ci in range(n_cams)])
     out = {}
-    for name, d, sd, mode, t, tau in (("full_scene", (1, 1, 1), 2 * side, "abcd", 4 * T, None),
-                                      ("abcd", dims, side, "abcd", T, None),
-                                      ("ablated", dims, side, "ablated", T, None),
-                                      ("abcd_culled", dims, side, "abcd", T, cull_tau)):
+    for name, d, sd, mode, t, tau, ov in (
+            ("full_scene", (1, 1, 1), 2 * side, "abcd", 4 * T, None, 0.0),
+            ("abcd", dims, side, "abcd", T, None, 0.0),
+            ("ablated", dims, side, "ablated", T, None, 0.0),
+            ("abcd_culled", dims, side, "abcd", T, cull_tau, 0.0),
+            ("abcd_overlap", dims, side, "abcd", T, None, overlap)):
         run = BCD(s.gaussians, d, origin, sd, s.cameras, targets, t, default_lr(2 * side),
-                  mode=mode, seed=seed + 2, cull_tau=tau)
+                  mode=mode, seed=seed + 2, cull_tau=tau, overlap=ov)
         hist = [run.eval_loss()]
         for _ in range(cycles):
             run.cycle()
