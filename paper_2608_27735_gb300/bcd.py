@@ -24,6 +24,25 @@ def default_lr(extent):
     return [1.6e-4 * extent, 5e-3, 1e-3, 0.025, 2.5e-3, 2.5e-3 / 20]
 
 
+def halo_members(means, members, blocks, b, dims, origin, side, margin):
+    """The halo of block b: {other block q: positions, in q's member list, of q's Gaussians
+    whose means lie within `margin` of b's cell (the closed box widened by margin on every
+    side)}.  Cells are numbered x + dims[0] (y + dims[1] z)."""
+    gx, gy, _ = dims
+    ix, iy, iz = b % gx, (b // gx) % gy, b // (gx * gy)
+    lo = np.asarray(origin, np.float64) + side * np.array([ix, iy, iz], np.float64)
+    hi = lo + side
+    out = {}
+    for q in blocks:
+        if q == b:
+            continue
+        mq = np.asarray(means, np.float64)[members[q]]
+        near = np.all((mq >= lo - margin) & (mq <= hi + margin), axis=1)
+        if near.any():
+            out[q] = np.nonzero(near)[0]
+    return out
+
+
 class BCD:
     """Cyclic block coordinate descent over the cells of a regular grid.
 
@@ -95,20 +114,8 @@ class BCD:
         self.measure_visibility()
 
     def _halo(self, b, means):
-        """Other blocks' Gaussians whose means lie within self.overlap of block b's cell."""
-        gx, gy, _ = self.dims
-        ix, iy, iz = b % gx, (b // gx) % gy, b // (gx * gy)
-        lo = np.asarray(self.origin) + self.side * np.array([ix, iy, iz], np.float64)
-        hi = lo + self.side
-        out = {}
-        for q in self.blocks:
-            if q == b:
-                continue
-            mq = means[self.members[q]]
-            near = np.all((mq >= lo - self.overlap) & (mq <= hi + self.overlap), axis=1)
-            if near.any():
-                out[q] = np.nonzero(near)[0]
-        return out
+        return halo_members(means, self.members, self.blocks, b, self.dims, self.origin,
+                            self.side, self.overlap)
 
     def _take(self, g, pos):
         """Gaussians at positions pos (host int array) of g, as new device tensors."""
