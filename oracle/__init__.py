@@ -4,8 +4,9 @@ Plain fp64 C++ (``abcd_oracle.cpp``) behind ctypes, with numpy-friendly wrappers
 what the CUDA path is checked against; it shares no code with it.  Only ``tests/``,
 ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg may import it.
 
-Parity unpinned: nothing here is unpinned except what the design doc lists (the difference between
-the partition-layered render and a single global depth sort, which is only reported).
+Parity unpinned: none of the functions here (each is pinned by tests/test_oracle_pins.py).
+Only reported, not pinned: the difference between the partition-layered render and a single
+global depth sort of every Gaussian.
 """
 from __future__ import annotations
 
