@@ -268,8 +268,9 @@ abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_ma
  * every channel of every pixel by at most the sum over D of alpha_j T_j (premultiplied colours
  * at most alpha), so the sum of the dropped layers' visible shares bounds the mean error of
  * the culled composite.  layers: host array of L device pointers to fp16 [H][W][4]
- * premultiplied RGBA (8-byte aligned); visible, coverage: device double [L] (coverage may be
- * NULL), overwritten.  The sums are exact in 24-bit fixed point per pixel value (result
+ * premultiplied RGBA with alpha in [0, 1] (8-byte aligned; entries of layers not in the order
+ * are not read and may be NULL); visible, coverage: device double [L] (coverage may be NULL),
+ * overwritten.  The sums are exact in 24-bit fixed point per pixel value (result
  * independent of the order of the additions); they use the context's workspace (ABCD_ERR_WORKSPACE
  * without one).  L <= 256; ABCD_ERR_INVALID_ARG for a repeated or out-of-range index, a NULL
  * or misaligned layer or output. */
