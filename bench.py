@@ -449,12 +449,13 @@ def algorithmic(st: Stage, name, avg_ms, pairs_mean):
         C = len(st.cams)
         byts = st.cache_bytes / C + (st.n_parts - 1) * st.n_t * 4 + 2 * 8 * npx
         return "hbm", byts / (avg_ms * 1e-3) / 1e9, "GB/s"
+    P = 4 * PARAM_FLOATS(D)     # bytes of one Gaussian's parameters (236 at SH degree 3)
     if name == "adam":
-        return "hbm", 7 * 4 * (14 + 3 * D) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
+        return "hbm", 7 * P * n / (avg_ms * 1e-3) / 1e9, "GB/s"
     if name == "project":
-        return "hbm", (4 * (14 + 3 * D) + 52) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
+        return "hbm", (P + 52) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
     if name == "project_bwd":
-        return "hbm", (2 * 4 * (14 + 3 * D) + 36) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
+        return "hbm", (2 * P + 36) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
     if name == "bin_sort":
         K = st.k_mean
         byts = 20 * n + 4 * 24 * n + 8 * K + 2 * 24 * K + 12 * K
@@ -462,10 +463,18 @@ def algorithmic(st: Stage, name, avg_ms, pairs_mean):
     return None
 
 
-def fp32_peak_tflops(peaks):
-    sms = 152
-    mhz = peaks.get("sm_max_mhz", 2070.0) if peaks else 2070.0
-    return sms * 128 * 2 * mhz * 1e6 / 1e12
+def PARAM_FLOATS(D):
+    """Floats per Gaussian: mean 3, log-scale 3, quaternion 4, opacity logit 1, SH 3 D."""
+    return 3 + 3 + 4 + 1 + 3 * D
+
+
+def measured_alu_peaks(device):
+    """fp32 FMA and ex2.approx peaks measured on this device by the library's microbenchmark
+    (SM count read from the device, CUDA events, no clock changes)."""
+    import paper_2608_27735_gb300 as ab
+    p = ab.abcd_measure_alu_peaks(device)
+    p["fp32_tflops"] = max(p["ffma_tflops"], p["ffma2_tflops"])
+    return p
 
 
 def load_peaks():
@@ -519,6 +528,9 @@ def run_ours(args):
     st.ctx.sync()
     st.reset_events()
     peaks = load_peaks()
+    alu = measured_alu_peaks(local)
+    log(f"[bench] measured fp32 FMA {alu['ffma_tflops']:.1f} TFLOP/s (FFMA2 {alu['ffma2_tflops']:.1f}), "
+        f"ex2 {alu['ex2_tops']:.2f} T/s on {alu['sms']} SMs")
 
     def barrier():
         if world > 1:
@@ -564,19 +576,26 @@ def run_ours(args):
     pairs_mean = float(torch.stack(st.pairs_sample).double().mean().item()) if st.pairs_sample else 0.0
     single = [k for k in ops if k not in ("bin_sort", "refresh")]
     dom = max(single, key=lambda k: share[k])
-    bound, achieved, unit = algorithmic(st, dom, ops[dom]["avg_ms"], pairs_mean)
-    if bound == "hbm":
-        peak = peaks["hbm_gbs"] if peaks else 6800.0
-        peak_note = "measured HBM copy" if peaks else "fallback"
-    else:
-        peak = fp32_peak_tflops(peaks)
-        peak_note = "FP32 FMA peak 152 SM x 128 lanes x 2 x sm_max_mhz"
+    hbm_peak = peaks["hbm_gbs"] if peaks else 6800.0
+    hbm_note = "of measured (HBM copy, MEASURED_PEAKS.json)" if peaks else "of fallback"
+    alu_note = (f"of measured (fp32 FMA microbenchmark on {alu['sms']} SMs: FFMA "
+                f"{alu['ffma_tflops']:.1f}, FFMA2 {alu['ffma2_tflops']:.1f} TFLOP/s; the larger)")
+
+    def roof(name):
+        r = algorithmic(st, name, ops[name]["avg_ms"], pairs_mean)
+        if r is None:
+            return None
+        bound, achieved, unit = r
+        peak, note = (hbm_peak, hbm_note) if bound == "hbm" else (alu["fp32_tflops"], alu_note)
+        return dict(bound=bound, achieved=round(achieved, 3), peak=round(peak, 1), unit=unit,
+                    frac=round(achieved / peak, 4), peak_source=note)
+
+    rf = roof(dom)
     kname = op_kernel_names()[dom]
-    roofline = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
-                "frac": round(achieved / peak, 4), "traffic": profile_traffic(kname),
-                "kernel": kname, "peak_source": peak_note,
-                "algorithmic_per_launch": (f"{pairs_mean:.0f} pixel-list pairs" if dom.startswith("render")
-                                           else None)}
+    roofline = dict(rf, traffic=profile_traffic(kname), kernel=kname,
+                    algorithmic_per_launch=(f"{pairs_mean:.0f} pixel-list pairs" if dom.startswith("render")
+                                            else None))
+    per_kernel = {k: roof(k) for k in ops if k != "refresh"}
     # ---- end to end through the C ABI with host buffers
     e2e = None
     if not args.no_e2e:
@@ -615,6 +634,8 @@ def run_ours(args):
         "gpu_launches": int(launches),
         "clocks": clocks,
         "ops": {k: {"avg_ms": round(v["avg_ms"], 4), "share": round(share[k], 4)} for k, v in ops.items()},
+        "rooflines": per_kernel,
+        "alu_peaks": {k: (round(v, 3) if isinstance(v, float) else v) for k, v in alu.items()},
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -627,7 +648,7 @@ TAU_VISIBLE = 1e-3
 
 
 def run_visibility(st: Stage, reps=3):
-    """Section 5's visibility threshold and occlusion culling on the stage's cache: every
+    """Section 4's visibility threshold and occlusion culling on the stage's cache: every
     observing camera's layers (the active one as last refreshed) in its depth order, one
     abcd_layer_visibility_packed call per camera, timed on the context's stream; the pairs
     whose visible share is below TAU_VISIBLE, the stored bytes they hold and the bound on the

@@ -32,7 +32,8 @@ typedef enum {
   ABCD_ERR_INVALID_ARG = 1,   /* bad pointer / size / option; nothing launched */
   ABCD_ERR_CUDA = 2,          /* a CUDA runtime call or launch failed (see abcd_last_error) */
   ABCD_ERR_CAPACITY = 3,      /* device: tile pairs K exceeded abcd_tiles.capacity */
-  ABCD_ERR_TIMEOUT = 4,       /* device: a bounded wait gave up (reserved) */
+  ABCD_ERR_TIMEOUT = 4,       /* device: a bounded wait gave up (the radix sort's look-back;
+                                 the results of that call are wrong, nothing hangs) */
   ABCD_ERR_WORKSPACE = 5      /* workspace missing or smaller than abcd_workspace_size() */
 } abcd_status;
 
@@ -120,17 +121,30 @@ abcd_status abcd_clear_status(abcd_ctx* ctx);
 const char* abcd_last_error(const abcd_ctx* ctx);
 /* Number of kernels this context has launched since creation (instrumentation). */
 long long abcd_launch_count(const abcd_ctx* ctx);
+/* Bound on the polls of a device-side wait (the radix sort's decoupled look-back waits for the
+ * tiles before its own, whose CTAs are already running) [2^20, about 40 ms]: a wait that
+ * reaches it gives up, the call's results are wrong and ABCD_ERR_TIMEOUT is set in the status
+ * word (abcd_sync); nothing hangs, and later calls run normally once the status is cleared. */
+abcd_status abcd_set_wait_limit(abcd_ctx* ctx, unsigned polls);
+/* Test hook for the bounded waits: in the next abcd_bin_sort call, tile `tile` of the first
+ * pass of the tile sort publishes nothing, so the waits of the tiles after it run out (after
+ * the wait limit).  -1 (the default) turns it off; it turns itself off after that pass. */
+abcd_status abcd_test_withhold_lookback(abcd_ctx* ctx, long long tile);
 
 /* ---- the hot path (Section 2: one step renders only the active block) ----------------- */
 
-/* K2. EWA projection of the active block for one camera (3DGS): camera-space mean, world
+/* K2. EWA projection of the active block for one camera.  Section 2 renders only the active
+ * partition at each step; the renderer is 3D Gaussian Splatting, which the paper instantiates
+ * by citation (Section 1, last paragraph), so the formulas are 3DGS's: camera-space mean, world
  * covariance R(q) diag(exp(2 log_scale)) R(q)^T, 2-D covariance J W Sigma W^T J^T +
  * dilation*I, its inverse, the 3-sigma radius, SH colour + 0.5 clamped at 0 and
  * opacity = sigmoid(logit).  Writes every field of out. */
 abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_camera* cam,
                          const abcd_render_opts* opts, abcd_projected* out);
 
-/* K3 + K4. Tile binning and depth sort: a visible Gaussian is listed in each tile its square
+/* K3 + K4. Tile binning and depth sort of the active block (the tile rasteriser of 3D Gaussian
+ * Splatting, Section 1 by citation; Section 2 renders the active partition alone, so only its
+ * Gaussians are binned).  A visible Gaussian is listed in each tile its square
  * [u-r, u+r] x [v-r, v+r] meets on which it can reach alpha >= alpha_min (the least sigma over
  * the box of the tile's pixel centres is at most ln(opacity / alpha_min), tested with a margin
  * of about 0.7% in sigma, so a list may hold a few entries that every pixel of the tile
@@ -143,7 +157,12 @@ abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_
 abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, int n,
                           const abcd_camera* cam, const abcd_render_opts* opts, abcd_tiles* out);
 
-/* K5. Front-to-back blend of the active block per pixel (alpha = min(alpha_max,
+/* K5. The active partition rendered and composited with the cached foreground and background
+ * (Section 2: the frozen partitions in front of / behind the active one collapse into F and B,
+ * and compositing with them equals rendering with every frozen parameter present).  The call
+ * takes the active block's projection (abcd_project) and tile lists (abcd_bin_sort) rather than
+ * theta itself, so that one projection serves the forward, the backward and the refresh.
+ * Front-to-back blend of the active block per pixel (alpha = min(alpha_max,
  * o exp(-sigma)), skip alpha < alpha_min, stop before T < t_min), giving the premultiplied
  * A = (sum T_i alpha_i c_i, 1 - T_final); then out = F over (A over B), over meaning
  * X + (1 - X.a) Y on premultiplied RGBA, and out.rgb += (1 - out.a) * bg.
@@ -156,14 +175,16 @@ abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camera* cam,
                                       int fb_dtype, const float* bg, float* out_rgba,
                                       abcd_fwd_state* state, void* refresh_f16);
 
-/* K6. Reconstruction loss (1 - lambda) mean|x - y| + lambda (1 - mean SSIM(x, y)) over the
+/* K6. The reconstruction loss each step of Section 2 evaluates, in the L1 + D-SSIM form of
+ * 3D Gaussian Splatting: (1 - lambda) mean|x - y| + lambda (1 - mean SSIM(x, y)) over the
  * rgb of out_rgba [H][W][4] against gt_rgb [H][W][3]; SSIM with an 11x11 Gaussian window
  * (sigma 1.5), zero padding, C1 = 0.01^2, C2 = 0.03^2.  loss_out: device float scalar.
  * dL_dout: [H][W][3] receives dL/d(out.rgb). */
 abcd_status abcd_loss(abcd_ctx* ctx, const float* out_rgba, const float* gt_rgb, int width,
                       int height, float lambda_ssim, float* loss_out, float* dL_dout);
 
-/* K7. Backward of the blend + composite for one image: given dL/d(final rgb) [H][W][3],
+/* K7. Backward of the blend + composite for one image (Section 2: gradients flow only into the
+ * active block; F and B are constants of the step): given dL/d(final rgb) [H][W][3],
  * writes grad2d [n][9] = dL/d(u, v, a, b, c, opacity, r, g, b) per Gaussian (overwritten).
  * The alpha of the active layer also receives -(1 - F.a) <g, B.rgb + (1 - B.a) bg>. */
 abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* cam,
@@ -172,8 +193,9 @@ abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* cam,
                                  int fb_dtype, const float* bg, const abcd_fwd_state* state,
                                  const float* dL_dout, int n, float* grad2d);
 
-/* K8. Chain rule from grad2d [n][9] to the parameters of theta (overwrites grads; culled
- * Gaussians get 0). */
+/* K8. Chain rule from grad2d [n][9] to the parameters of theta, the active block (Section 2:
+ * gradients reach theta_active only; the projection is 3DGS's, Section 1 by citation).
+ * Overwrites grads; culled Gaussians get 0. */
 abcd_status abcd_project_backward(abcd_ctx* ctx, const abcd_gaussians* theta,
                                   const abcd_camera* cam, const abcd_render_opts* opts,
                                   const float* grad2d, abcd_gaussians* grads);
@@ -188,7 +210,9 @@ abcd_status abcd_backward(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd
                           const float* gt_rgb, float lambda_ssim, float* loss_out,
                           const float* dL_dout, abcd_gaussians* grads);
 
-/* K9. Adam with bias correction (torch semantics), dense over the active block only:
+/* K9. The update of the T gradient steps of Section 2 on theta_active (the optimiser is Adam, as
+ * in 3D Gaussian Splatting; the paper names none).  Bias-corrected (torch semantics), dense
+ * over the active block only:
  * m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2; theta -= lr m/(1-b1^t) / (sqrt(v/(1-b2^t)) + eps).
  * lr[6] per group: means, log_scales, quats, opacity_logits, sh degree 0, sh degree >= 1.
  * step is 1-based. */
@@ -258,7 +282,7 @@ abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_ma
                                         void* B_out, int out_dtype);
 
 /* Visibility of the cached layers of one camera, for the visibility thresholds and occlusion
- * culling of camera-partition pairs that Section 5 proposes.  The layers are taken in `order`
+ * culling of camera-partition pairs that Section 4 proposes.  The layers are taken in `order`
  * (host, `count` distinct indices below L, front to back; a layer left out counts as absent).
  * For the layer at position k, with alpha_k its alpha and T_k the product of (1 - alpha) over
  * the layers before it:
@@ -293,11 +317,15 @@ abcd_status abcd_layer_visibility_packed(abcd_ctx* ctx, const int* const* tile_m
  * Its scratch (per-CTA partial sums and a completion counter, about 512 KB) is a static
  * device array of this library, held by every GPU that loads the library until the process
  * exits; images may have at most 65536 CTAs, one per channel of a 64x28-pixel tile (e.g.
- * 8192 x 4096), larger ones return ABCD_ERR_WORKSPACE.  The first call on a device looks up the array's address (with
- * that device current), so make it before any stream capture.  All calls on a device share
+ * 8192 x 4096), larger ones return ABCD_ERR_WORKSPACE.  The first call on a device (made with
+ * that device current) loads the library's device code there and looks up the array's
+ * address, so make it before any stream capture; later calls look the address up again (a
+ * host-side table read), so a device reset never leaves a stale address.  All calls on a device share
  * the array: calls whose kernels overlap on the GPU race and give wrong losses, so order them
  * (one stream, or events).  The counter is cleared at the start of every call.  Returns
- * ABCD_ERR_INVALID_ARG for bad pointers, sizes or lambda, ABCD_ERR_CUDA if a launch fails. */
+ * ABCD_ERR_INVALID_ARG for bad pointers, sizes or lambda, ABCD_ERR_CUDA if the address lookup,
+ * the counter's clear or the launch fails (the launch's own status; earlier errors of other
+ * work are not reported here).  loss_out and dL_dout may each be NULL. */
 abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba, const float* gt_rgb,
                              int width, int height, float lambda_ssim, float* loss_out,
                              float* dL_dout);
@@ -339,6 +367,24 @@ abcd_status abcd_cache_store(abcd_ctx* ctx, int slot, const void* dev_src, void*
 /* Waits until the context's queued fetches and stores are done (abcd_sync waits for its
  * compute stream only). */
 abcd_status abcd_cache_sync(abcd_ctx* ctx);
+
+/* ---- instrumentation: the arithmetic peaks the roofline fractions are taken against ----- */
+
+typedef struct {
+  int sms;                   /* multiprocessors, read from the device */
+  double clock_mhz_nominal;  /* the device's reported SM clock (the runs take whatever clock
+                                the GPU is at; nothing is locked or changed) */
+  double ffma_tflops;        /* fp32 FMA, scalar FFMA, 2 flops per FMA */
+  double ffma2_tflops;       /* fp32 FMA through the packed two-lane FFMA2 */
+  double ex2_tops;           /* ex2.approx.ftz.f32 (MUFU) results per second, 1e12 */
+  double ms_ffma, ms_ffma2, ms_ex2;   /* best timed launch of each kernel */
+} abcd_alu_peaks;
+
+/* Measures fp32 FMA and ex2.approx throughput on `device` with three short kernels of
+ * independent dependency chains over 4 CTAs of 256 threads per SM (about 10 ms each, timed with
+ * CUDA events on a private stream after a warm-up launch; best of five).  Synchronous; allocates
+ * nothing.  ABCD_ERR_CUDA if a launch or event fails. */
+abcd_status abcd_measure_alu_peaks(int device, abcd_alu_peaks* out);
 
 /* ---- host-side partition logic (Section 2: regular grid, assignment by mean) --------- */
 

@@ -165,7 +165,7 @@ int orc_backward_pixels(const orc_splats* s, const long long* offsets, const int
 int orc_composite_layers(int n_pixels, const double* layers, const int* order, int count,
                          double* out);
 
-/* Visibility of each layer of one camera's depth order (Section 5: visibility thresholds and
+/* Visibility of each layer of one camera's depth order (Section 4: visibility thresholds and
  * occlusion culling of camera-partition pairs).  For the layer at position k of the order,
  * with alpha_k its alpha and T_k the product of (1 - alpha) over the layers before it:
  * visible[order[k]] = mean over pixels of alpha_k T_k, coverage[order[k]] = mean of alpha_k;

@@ -65,6 +65,12 @@ class abcd_fwd_state(C.Structure):
     _fields_ = [("A_T", C.c_void_p), ("n_last", C.c_void_p)]
 
 
+class abcd_alu_peaks(C.Structure):
+    _fields_ = [("sms", C.c_int), ("clock_mhz_nominal", C.c_double), ("ffma_tflops", C.c_double),
+                ("ffma2_tflops", C.c_double), ("ex2_tops", C.c_double), ("ms_ffma", C.c_double),
+                ("ms_ffma2", C.c_double), ("ms_ex2", C.c_double)]
+
+
 _lock = threading.Lock()
 _lib = None
 
@@ -112,6 +118,9 @@ _SIGS = {
     "abcd_cache_release": [C.c_void_p, C.c_int],
     "abcd_cache_store": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
     "abcd_cache_sync": [C.c_void_p],
+    "abcd_measure_alu_peaks": [C.c_int, C.c_void_p],
+    "abcd_set_wait_limit": [C.c_void_p, C.c_uint],
+    "abcd_test_withhold_lookback": [C.c_void_p, C.c_longlong],
     "abcd_assign_cells": [C.c_void_p, C.c_int, C.c_void_p, C.c_double, C.c_void_p, C.c_void_p],
     "abcd_partition_split": [C.c_void_p, C.c_void_p, C.c_double, C.c_void_p, C.c_int,
                              C.c_void_p, C.POINTER(C.c_int), C.c_void_p, C.POINTER(C.c_int)],
@@ -461,7 +470,7 @@ def abcd_layer_visibility_tables(ctx: Context, pl, width, height, visible, cover
 
 
 def cull_pairs(visible, coverage, tau_visible, tau_area=0.0):
-    """Camera-partition pairs to keep (Section 5's visibility threshold and occlusion culling):
+    """Camera-partition pairs to keep (Section 4's visibility threshold and occlusion culling):
     a layer stays when its visible share of the composite is at least tau_visible and its
     image area at least tau_area.  The dropped layers' visible shares add up to a bound on the
     mean per-channel error of the culled composite.  Host arrays in, boolean mask out."""
@@ -582,3 +591,13 @@ def abcd_partition_split(dims, origin, side, campos, active):
     if st != ABCD_OK:
         raise AbcdError(st, "abcd_partition_split")
     return front[:nf.value].copy(), back[:nb.value].copy()
+
+
+def abcd_measure_alu_peaks(device=0) -> dict:
+    """Measured fp32 FMA (scalar and packed) and ex2.approx throughput of `device` (a few short
+    timed kernels; no clock or device setting is changed)."""
+    p = abcd_alu_peaks()
+    st = lib().abcd_measure_alu_peaks(int(device), C.byref(p))
+    if st != ABCD_OK:
+        raise AbcdError(st, "abcd_measure_alu_peaks")
+    return {k: getattr(p, k) for k, _ in abcd_alu_peaks._fields_}

@@ -49,12 +49,12 @@ class BCD:
     gaussians: scenegen.Gaussians of the whole scene; dims, origin, side: the grid; cameras:
     objects with R, t, fx, fy, cx, cy, width, height, position; targets: float32 [C][H][W][3];
     mode: "abcd" (F and B from the cache) or "ablated" (F = B = transparent).  cull_tau: the
-    visibility threshold of Section 5's culling of camera-partition pairs (None: no culling):
+    visibility threshold of Section 4's culling of camera-partition pairs (None: no culling):
     after every refresh each camera's layers are measured (abcd_layer_visibility) and a pair
     whose visible share of the camera's composite is below cull_tau is dropped, from F and B
     of the other blocks' stages and from the cameras its own block trains on, until a later
     measurement brings it back.  overlap: the width of the overlapping boundary region that
-    Section 5 proposes (0: none).  Membership stays by the mean, but a block's stage renders,
+    Section 4 proposes (0: none).  Membership stays by the mean, but a block's stage renders,
     with the block, the other blocks' Gaussians whose means lie within `overlap` of its cell
     (its halo: frozen, sorted by depth together with the block's own, no gradient step), and
     for every camera F and B take each donor block's layer re-rendered without them, so every
@@ -201,7 +201,11 @@ class BCD:
             self.queue = [allowed[i] for i in self.rng.permutation(len(allowed))]
         return int(self.queue.pop())
 
-    def stage(self, b):
+    def stage(self, b, trace=None):
+        """One stage of block b: composite F and B (abcd mode), T steps, refresh.  trace, if
+        given, is called after every step as trace(t, camera, theta, grads, m, v, loss) with the
+        block's device tensors as they are after the step's Adam update (an observer: it must
+        not change them)."""
         th = self.theta[b]
         grads, m, v = (Gaussians.zeros_like(th) for _ in range(3))   # Adam state per stage
         if self.mode == "abcd":
@@ -227,6 +231,8 @@ class BCD:
                               self.loss[t:t + 1], None, gs)
                 abcd_adam_active(self.ctx, head(ths), head(gs), m, v, self.lr, 0.9, 0.999,
                                  1e-15, t + 1)
+                if trace is not None:
+                    trace(t, ci, head(ths), head(gs), m, v, self.loss[t:t + 1])
             for a_, s_ in zip(th.tensors(), ths.tensors()):
                 a_.copy_(s_[:th.n])
         else:
@@ -237,6 +243,8 @@ class BCD:
                 F = self.F[ci] if self.mode == "abcd" else None
                 B = self.B[ci] if self.mode == "abcd" else None
                 step(self.cams[ci], F, B, self.gt[ci], self.loss[t:t + 1], t + 1)
+                if trace is not None:
+                    trace(t, ci, th, grads, m, v, self.loss[t:t + 1])
         self.steps_done += self.T if allowed else 0
         self.refresh(b)
 
@@ -289,8 +297,8 @@ def quality_experiment(T=100, cycles=3, per_cell=1000, n_cams=8, width=96, heigh
     0): full-scene training (one block, 4 T steps per cycle), ABCD and the ablated variant (4
     blocks, T steps each per cycle), the same number of steps in all three, against targets
     rendered from a perturbed copy of the scene; and ABCD with the camera-partition pairs
-    culled at visible share cull_tau (Section 5), which trains each block on the cameras that
-    see it, and ABCD with an overlapping boundary region of width `overlap` (Section 5).
+    culled at visible share cull_tau (Section 4), which trains each block on the cameras that
+    see it, and ABCD with an overlapping boundary region of width `overlap` (Section 4).
     Returns {name: [eval loss after 0..cycles]}; the eval renders every layer."""
     from . import scenegen as sg
     dims, side = (2, 2, 1), 5.0

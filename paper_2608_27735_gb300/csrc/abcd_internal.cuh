@@ -147,6 +147,8 @@ struct abcd_ctx {
   abcd::SHConst sh{};
   long long launches = 0;
   unsigned os_epoch = 0;                // last look-back epoch handed to a sort pass
+  unsigned wait_limit = 1u << 20;       // polls before a device-side wait gives up
+  long long withhold_tile = -1;         // test hook: a look-back tile that publishes nothing
   char err[512] = {0};
 };
 

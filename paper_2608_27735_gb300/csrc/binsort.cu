@@ -314,7 +314,6 @@ __device__ __forceinline__ void tile_digit_counts(unsigned t, unsigned c, const 
 
 constexpr int kOsWarps = 8;
 constexpr int kOsThreads = 32 * kOsWarps;
-constexpr unsigned kOsSpinLimit = 1u << 20;
 
 // Look-back state word: epoch (30 bits) | flag (2 bits: 1 aggregate, 2 inclusive) | count.
 // The epoch changes with every pass launch, so words left by earlier passes read as "not
@@ -367,12 +366,15 @@ sort_digits_kernel(const T* in, long long n_static, const long long* n_dev, long
 // One pass: stable scatter of the items of [0, n) by the BITS-bit digit at `shift`.  gh holds
 // this pass's digit counts; ctr[0] hands out tiles and ctr[1] counts finished CTAs (the last
 // one clears both); state holds kRadixBins words per tile.  On the last pass out_ids (when not
-// null) receives the bits id_mask of each item instead of the item.
+// null) receives the bits id_mask of each item instead of the item.  A look-back wait gives up
+// after spin_limit polls.  Tile `withhold` (a test hook; -1 in normal use) publishes nothing,
+// so the waits of the tiles after it run out.
 template <typename T, int BITS, bool MATCH>
 __global__ void __launch_bounds__(kOsThreads, 2)
 onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
                 const long long* n_dev, long long cap, int shift, const unsigned* gh, u64* state,
-                unsigned* ctr, unsigned epoch, unsigned* status) {
+                unsigned* ctr, unsigned epoch, unsigned* status, unsigned spin_limit,
+                long long withhold) {
   pdl_prologue();
   constexpr unsigned BINS = 1u << BITS, MASK = BINS - 1;
   constexpr int U = 64 / (int)sizeof(T);          // items per lane: 64 bytes in flight
@@ -421,7 +423,8 @@ onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long l
 #pragma unroll
       for (int k = 0; k < kOsWarps; ++k) { const unsigned c = cnt[k][d]; cnt[k][d] = run; run += c; }
       s_run[d] = run;
-      os_publish(state + (size_t)t * kRadixBins + d, os_word(epoch, t == 0 ? 2u : 1u, run));
+      if (t != withhold)
+        os_publish(state + (size_t)t * kRadixBins + d, os_word(epoch, t == 0 ? 2u : 1u, run));
     }
     __syncthreads();
     {
@@ -466,12 +469,13 @@ onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long l
         k0 -= consumed;
         if (res == 1) break;
         if (res == 2) {
-          if (++spins > kOsSpinLimit) { if (q == 0) atomicOr(status, kStatusTimeout); break; }
+          if (++spins > spin_limit) { if (q == 0) atomicOr(status, kStatusTimeout); break; }
           __nanosleep(32);
         }
       }
       if (q == 0) {
-        if (t > 0) os_publish(state + (size_t)t * kRadixBins + d, os_word(epoch, 2u, prefix + s_run[d]));
+        if (t > 0 && t != withhold)
+          os_publish(state + (size_t)t * kRadixBins + d, os_word(epoch, 2u, prefix + s_run[d]));
         s_off[d] = s_base[d] + prefix;
       }
     }
@@ -798,16 +802,17 @@ template <typename T>
 abcd_status launch_onesweep(abcd_ctx* ctx, cudaStream_t st, int bits, bool match, int G,
                             const T* src, T* dst, unsigned* ids, unsigned id_mask,
                             long long n_static, const long long* n_dev, long long cap, int shift,
-                            const unsigned* gh, unsigned* ctr) {
+                            const unsigned* gh, unsigned* ctr, long long withhold) {
   const unsigned epoch = ++ctx->os_epoch;
+  const unsigned spin = ctx->wait_limit;
 #define ABCD_PASS(B)                                                                              \
   case B:                                                                                         \
     e = match ? launch_pdl(onesweep_kernel<T, B, true>, dim3(G), dim3(kOsThreads), 0, st, src, dst, \
                            ids, id_mask, n_static, n_dev, cap, shift, gh, ctx->ws.os_state, ctr,   \
-                           epoch, ctx->ws.status)                                                  \
+                           epoch, ctx->ws.status, spin, withhold)                                  \
               : launch_pdl(onesweep_kernel<T, B, false>, dim3(G), dim3(kOsThreads), 0, st, src,    \
                            dst, ids, id_mask, n_static, n_dev, cap, shift, gh, ctx->ws.os_state,   \
-                           ctr, epoch, ctx->ws.status);                                            \
+                           ctr, epoch, ctx->ws.status, spin, withhold);                            \
     break;
   cudaError_t e = cudaSuccess;
   switch (bits) {
@@ -852,10 +857,13 @@ abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_s
   T* dst = b;
   for (int p = 0; p < sp.n; ++p) {
     const bool last = p == sp.n - 1;
+    // the test hook withholds a tile of the tile sort's first pass only
+    const long long withhold = (slot == 1 && p == 0) ? ctx->withhold_tile : -1;
     if ((s = launch_onesweep<T>(ctx, st, sp.bits[p], p >= match_from, G, src, dst,
                                 last ? ids_out : nullptr, id_mask, n_static, n_dev, cap,
-                                sp.shift[p], gh + p * kRadixBins, ctr)))
+                                sp.shift[p], gh + p * kRadixBins, ctr, withhold)))
       return s;
+    if (slot == 1 && p == 0) ctx->withhold_tile = -1;
     T* t = src; src = dst; dst = t;
   }
   if (result) *result = src;

@@ -344,7 +344,7 @@ extern "C" abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* con
                                  tiles_x, F_out, B_out, out_dtype == ABCD_F16 ? 1 : 0));
 }
 
-// ---- visibility of the layers of one camera's depth order (Section 5: visibility thresholds
+// ---- visibility of the layers of one camera's depth order (Section 4: visibility thresholds
 // and occlusion culling of camera-partition pairs).  For the layer at position k, with alpha_k
 // its alpha and T_k the product of (1 - alpha) over the layers before it, visible = mean over
 // pixels of alpha_k T_k and coverage = mean of alpha_k.  Leaving a set D of layers out of the

@@ -222,6 +222,18 @@ abcd_status abcd_sync(abcd_ctx* ctx) {
 
 const char* abcd_last_error(const abcd_ctx* ctx) { return ctx ? ctx->err : "null context"; }
 
+abcd_status abcd_set_wait_limit(abcd_ctx* ctx, unsigned polls) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  ctx->wait_limit = polls;
+  return ABCD_OK;
+}
+
+abcd_status abcd_test_withhold_lookback(abcd_ctx* ctx, long long tile) {
+  if (!ctx || tile < -1) return ABCD_ERR_INVALID_ARG;
+  ctx->withhold_tile = tile;
+  return ABCD_OK;
+}
+
 long long abcd_launch_count(const abcd_ctx* ctx) { return ctx ? ctx->launches : 0; }
 
 abcd_status abcd_assign_cells(const float* means, int n, const double origin[3], double side,

@@ -14,7 +14,6 @@
 // The scalar is reduced deterministically: per-CTA partial sums, then the last CTA to finish
 // adds them in a fixed order (no waiting on other CTAs).
 #include <cmath>
-#include <mutex>
 
 #include "abcd_internal.cuh"
 
@@ -357,20 +356,15 @@ constexpr int kStaticLossWords = 2 * kStaticLossMaxBlocks + 64;   // partial sum
 // Device scratch shared by every abcd_loss_static call on a device (held until exit).
 static __device__ __align__(256) unsigned g_loss_static_scratch[kStaticLossWords];
 
-constexpr int kMaxDevices = 256;
-std::mutex g_static_mu;
-unsigned* g_static_ptr[kMaxDevices] = {nullptr};
-
-// Device address of the static scratch on the current device, looked up once per device.
-cudaError_t static_scratch(int device, unsigned** out) {
-  std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_ptr[device]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_loss_static_scratch);
-    if (e != cudaSuccess) return e;
-    g_static_ptr[device] = static_cast<unsigned*>(p);
-  }
-  *out = g_static_ptr[device];
+// Device address of the static scratch on the current device.  The first lookup on a device
+// loads this library's device code there; every call looks the address up again (a host-side
+// table read once the code is loaded), so an address never outlives a device reset that moved
+// the array.
+cudaError_t static_scratch(unsigned** out) {
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_loss_static_scratch);
+  if (e != cudaSuccess) return e;
+  *out = static_cast<unsigned*>(p);
   return cudaSuccess;
 }
 
@@ -386,11 +380,8 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
     return ABCD_ERR_INVALID_ARG;
   const dim3 grid = loss_grid(width, height);
   if ((long long)grid.x * grid.y * grid.z > kStaticLossMaxBlocks) return ABCD_ERR_WORKSPACE;
-  int device = 0;
-  if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices)
-    return ABCD_ERR_CUDA;
   unsigned* scratch = nullptr;
-  if (static_scratch(device, &scratch) != cudaSuccess) return ABCD_ERR_CUDA;
+  if (static_scratch(&scratch) != cudaSuccess) return ABCD_ERR_CUDA;
   float* partials = reinterpret_cast<float*>(scratch);
   unsigned* ticket = scratch + 2 * kStaticLossMaxBlocks;
   cudaStream_t stream = (cudaStream_t)cuda_stream;
@@ -403,5 +394,5 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
   const cudaError_t e = launch_pdl(loss_kernel, grid, dim3(kThreads), smem, stream, out_rgba,
                                    gt_rgb, width, height, lambda_ssim, ssim_window(), dL_dout,
                                    partials, ticket, loss_out);
-  return e == cudaSuccess && cudaGetLastError() == cudaSuccess ? ABCD_OK : ABCD_ERR_CUDA;
+  return e == cudaSuccess ? ABCD_OK : ABCD_ERR_CUDA;   // the launch's own status, not a sticky one
 }

@@ -751,6 +751,38 @@ def test_capacity_overflow_reported(ctx, tiny):
     ctx.sync()
 
 
+def test_bin_sort_wait_timeout_reported(ctx, tiny):
+    """The radix sort's look-back waits are bounded: with tile 0 of the tile sort's first pass
+    withheld (a test hook: it publishes nothing) and a short wait limit, the tiles behind it give
+    up, abcd_sync reports ABCD_ERR_TIMEOUT and the call returns; once the status is cleared the
+    same context sorts correctly again."""
+    case = Case(tiny, 2, fb=False)
+    cam = ab.camera(case.cam)
+    theta = ab.Gaussians.from_numpy(case.g)
+    proj = ab.Projected.alloc(theta.n)
+    ab.abcd_project(ctx, theta, cam, None, proj)
+    tiles = ab.Tiles.alloc(1 << 20, case.cam.width, case.cam.height)
+    ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+    ctx.sync()
+    K = int(tiles.count.item())
+    assert K > 4096, K                # the first tile-sort pass spans more than one look-back tile
+    ref_ids = tiles.ids[:K].clone()
+    ref_rng = tiles.ranges.clone()
+    L = ab.lib()
+    assert L.abcd_set_wait_limit(ctx.h, 256) == ab.ABCD_OK
+    assert L.abcd_test_withhold_lookback(ctx.h, 0) == ab.ABCD_OK
+    ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+    with pytest.raises(ab.AbcdError) as ei:
+        ctx.sync()
+    assert ei.value.status == ab.ABCD_ERR_TIMEOUT
+    ctx.clear_status()
+    assert L.abcd_set_wait_limit(ctx.h, 1 << 20) == ab.ABCD_OK
+    ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+    ctx.sync()
+    assert int(tiles.count.item()) == K
+    assert torch.equal(tiles.ids[:K], ref_ids) and torch.equal(tiles.ranges, ref_rng)
+
+
 def test_invalid_arguments_rejected(ctx):
     cam = ab.abcd_camera()
     cam.width = 0
