@@ -166,10 +166,20 @@ def tiles_xy(width, height, tile=16):
     return (width + tile - 1) // tile, (height + tile - 1) // tile
 
 
-def tile_lists(proj, width, height, tile=16, rule="alpha", alpha_min=1.0 / 255.0):
-    """Returns (offsets[n_tiles + 1] int64, ids[K] int32).  rule="alpha" keeps a tile of the
-    3-sigma square only where the Gaussian can reach alpha_min (the renderer's listing rule);
-    rule="square" keeps the whole square (3DGS)."""
+# The renderer's listing reading (R1b): a tile is listed when the least sigma over its pixel
+# centres, in log2 units, is at most (thr (1 + LIST_REL) + LIST_ABS) (1 + LIST_REL), thr =
+# log2(opacity / alpha_min): the exact rule widened by a margin that keeps every tile the exact
+# rule keeps whatever the fp32 rounding of the extent computation.
+LIST_REL = 1e-3
+LIST_ABS = 0.01
+
+
+def tile_lists(proj, width, height, tile=16, rule="listing", alpha_min=1.0 / 255.0):
+    """Returns (offsets[n_tiles + 1] int64, ids[K] int32).  rule="listing" (the renderer's
+    listing rule, R1b) keeps a tile of the 3-sigma square where the least sigma over its pixel
+    centres is within the margin above ln(o / alpha_min); rule="alpha" keeps exactly the tiles
+    on which the Gaussian can reach alpha_min; rule="square" keeps the whole square (3DGS)."""
+    assert rule in ("listing", "alpha", "square"), rule
     tx, ty = tiles_xy(width, height, tile)
     vis = np.ascontiguousarray(proj["visible"], dtype=np.int32)
     rect = np.ascontiguousarray(proj["rect"], dtype=np.int32)
@@ -179,10 +189,11 @@ def tile_lists(proj, width, height, tile=16, rule="alpha", alpha_min=1.0 / 255.0
                      np.maximum(rect[:, 3] - rect[:, 1], 0)))
     offsets = np.zeros(tx * ty + 1, np.int64)
     ids = np.zeros(max(cap, 1), np.int32)
-    sp = SplatSet.from_proj(proj) if rule == "alpha" else None
+    sp = SplatSet.from_proj(proj) if rule != "square" else None
+    rel, ab_ = (LIST_REL, LIST_ABS) if rule == "listing" else (0.0, 0.0)
     K = lib().orc_tile_lists(n, _p(vis), _p(rect), _p(key), tx, ty, _p(offsets), _p(ids),
                              C.c_longlong(cap), C.byref(sp.s) if sp is not None else None,
-                             C.c_double(alpha_min), int(tile))
+                             C.c_double(alpha_min), int(tile), C.c_double(rel), C.c_double(ab_))
     assert 0 <= K <= cap, (K, cap)
     return offsets, ids[:K]
 

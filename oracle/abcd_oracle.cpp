@@ -246,11 +246,50 @@ void add_event(int* ev, int max_ev, int* n_ev, int id, int type) {
   ++*n_ev;
 }
 
-// Returns the contributors in order; fills A = (sum T a c, 1 - T_final).
+// The blend of one pixel, as 3D Gaussian Splatting defines it (Section 1 by citation): front
+// to back over the tile's list, sigma = 1/2 d^T conic d at the pixel centre, alpha =
+// min(alpha_max, o exp(-sigma)); an entry with sigma < 0 or alpha < alpha_min is skipped; the
+// pixel stops before an entry that would take T (1 - alpha) below t_min; otherwise
+// C += alpha T c and T *= 1 - alpha.  Returns the contributors in order and A = (C, 1 - T).
 void blend_pixel(const orc_splats* s, const int* list, int len, int px, int py,
-                 const orc_opts& op, const int* tg, int nt, const orc_margins* mg,
-                 std::vector<Added>& added, double A[4], double* T_final, int* n_used,
-                 int* ev, int max_ev, int* n_ev) {
+                 const orc_opts& op, std::vector<Added>& added, double A[4], double* T_final,
+                 int* n_used) {
+  const double cxp = px + 0.5, cyp = py + 0.5;
+  double T = 1.0, C[3] = {0, 0, 0};
+  int used = 0;
+  added.clear();
+  for (int k = 0; k < len; ++k) {
+    const int id = list[k];
+    const double dx = cxp - s->uv[2 * id], dy = cyp - s->uv[2 * id + 1];
+    const double ca = s->conic[3 * id], cb = s->conic[3 * id + 1], cc = s->conic[3 * id + 2];
+    const double sigma = 0.5 * (ca * dx * dx + cc * dy * dy) + cb * dx * dy;
+    const double ge = std::exp(-sigma);
+    const double araw = s->opacity[id] * ge;
+    const bool clamped = araw > op.alpha_max;
+    const double alpha = clamped ? op.alpha_max : araw;
+    if (sigma < 0.0 || alpha < op.alpha_min) continue;
+    const double test = T * (1.0 - alpha);
+    if (test < op.t_min) break;
+    for (int ch = 0; ch < 3; ++ch) C[ch] += alpha * T * s->rgb[3 * id + ch];
+    added.push_back(Added{id, alpha, araw, T, sigma, ge, dx, dy, clamped});
+    T = test;
+    used = k + 1;
+  }
+  A[0] = C[0]; A[1] = C[1]; A[2] = C[2]; A[3] = 1.0 - T;
+  *T_final = T;
+  *n_used = used;
+}
+
+// Test-harness form of blend_pixel, used only to compare an fp32 implementation with it: the
+// same loop, which also reports the decisions that lie within a stated uncertainty model's
+// reach of their thresholds (skip, stop, alpha clamp; mg), and takes the opposite branch of
+// the decisions listed in tg (pairs of Gaussian id, event), so that every combination of the
+// ambiguous decisions can be rendered.  With no toggles its result equals blend_pixel's (a
+// pinned property).
+void blend_pixel_probe(const orc_splats* s, const int* list, int len, int px, int py,
+                       const orc_opts& op, const int* tg, int nt, const orc_margins* mg,
+                       std::vector<Added>& added, double A[4], double* T_final, int* n_used,
+                       int* ev, int max_ev, int* n_ev) {
   const double cxp = px + 0.5, cyp = py + 0.5;
   double T = 1.0, C[3] = {0, 0, 0};
   double epsT = 0.0;   // running relative uncertainty of T (event reporting only)
@@ -302,6 +341,20 @@ void blend_pixel(const orc_splats* s, const int* list, int len, int px, int py,
   A[0] = C[0]; A[1] = C[1]; A[2] = C[2]; A[3] = 1.0 - T;
   *T_final = T;
   *n_used = used;
+}
+
+// The plain blend, or the harness form when toggles or margins are given.
+void blend_any(const orc_splats* s, const int* list, int len, int px, int py,
+               const orc_opts& op, const int* tg, int nt, const orc_margins* mg,
+               std::vector<Added>& added, double A[4], double* T_final, int* n_used,
+               int* ev, int max_ev, int* n_ev) {
+  if (nt == 0 && !mg) {
+    if (n_ev) *n_ev = 0;
+    blend_pixel(s, list, len, px, py, op, added, A, T_final, n_used);
+  } else {
+    blend_pixel_probe(s, list, len, px, py, op, tg, nt, mg, added, A, T_final, n_used, ev,
+                      max_ev, n_ev);
+  }
 }
 
 void over(const double* X, const double* Y, double* out) {   // X over Y, premultiplied
@@ -467,7 +520,8 @@ double orc_box_min_sigma(const double* q, double X0, double X1, double Y0, doubl
 
 long long orc_tile_lists(int n, const int* visible, const int* rect, const unsigned* depth_key,
                          int tiles_x, int tiles_y, long long* offsets, int* ids,
-                         long long capacity, const orc_splats* s, double alpha_min, int tile) {
+                         long long capacity, const orc_splats* s, double alpha_min, int tile,
+                         double margin_rel, double margin_abs) {
   struct Item { long long tile; unsigned key; int id; };
   std::vector<Item> items;
   for (int i = 0; i < n; ++i) {
@@ -482,7 +536,16 @@ long long orc_tile_lists(int n, const int* visible, const int* rect, const unsig
           const double m = orc_box_min_sigma(s->conic + 3 * i, x * tile + 0.5 - u,
                                              x * tile + tile - 0.5 - u, y * tile + 0.5 - v,
                                              y * tile + tile - 0.5 - v);
-          if (m > std::log(o / alpha_min)) continue;
+          // keep when m <= ln(o / alpha_min) (the Gaussian reaches alpha_min somewhere on the
+          // tile), or, with a margin, when m log2(e) <= (thr (1 + rel) + abs) (1 + rel) with
+          // thr = log2(o / alpha_min): a superset whose extra entries no pixel of t reaches
+          const double thr2 = std::log2(o / alpha_min);
+          const double lim2 = (thr2 * (1.0 + margin_rel) + margin_abs) * (1.0 + margin_rel);
+          if (margin_rel == 0.0 && margin_abs == 0.0) {
+            if (m > std::log(o / alpha_min)) continue;
+          } else if (m / std::log(2.0) > lim2) {
+            continue;
+          }
         }
         items.push_back(Item{(long long)y * tiles_x + x, depth_key[i], i});
       }
@@ -508,7 +571,7 @@ int orc_render_pixel(const orc_splats* s, const int* list, int len, int px, int 
                      int* ev, int max_ev, int* n_ev) {
   std::vector<Added> added;
   if (n_ev) *n_ev = 0;
-  blend_pixel(s, list, len, px, py, *o, toggles, n_toggles, mg, added, A4, T_final, n_used,
+  blend_any(s, list, len, px, py, *o, toggles, n_toggles, mg, added, A4, T_final, n_used,
               ev, max_ev, n_ev);
   composite_out(A4, F, B, bg, out4);
   return 0;
@@ -528,7 +591,7 @@ int orc_render_image(const orc_splats* s, const long long* offsets, const int* i
     std::vector<Added> added;
     double A4[4], o4[4], Tf;
     int nu, ne = 0;
-    blend_pixel(s, ids + b, (int)(e - b), px, py, *o, nullptr, 0, mg, added, A4, &Tf, &nu,
+    blend_any(s, ids + b, (int)(e - b), px, py, *o, nullptr, 0, mg, added, A4, &Tf, &nu,
                 ev ? ev + (size_t)p * max_ev * 2 : nullptr, max_ev, n_ev ? &ne : nullptr);
     composite_out(A4, F ? F + 4 * (size_t)p : nullptr, B ? B + 4 * (size_t)p : nullptr, bg, o4);
     for (int c = 0; c < 4; ++c) {
@@ -548,7 +611,7 @@ int orc_backward_pixel(const orc_splats* s, const int* list, int len, int px, in
   std::vector<Added> added;
   double A[4], Tf;
   int nu;
-  blend_pixel(s, list, len, px, py, *o, toggles, n_toggles, nullptr, added, A, &Tf, &nu,
+  blend_any(s, list, len, px, py, *o, toggles, n_toggles, nullptr, added, A, &Tf, &nu,
               nullptr, 0, nullptr);
   // d final / d A: out = F over (A over B), final.rgb = out.rgb + (1 - out.a) bg
   const double Fa = F ? F[3] : 0.0;

@@ -116,10 +116,14 @@ int orc_project_backward(const orc_gaussians* g, const orc_camera* cam, const or
  * Listing rule: tile t of Gaussian i's rectangle is kept when s (uv, conic, opacity) is NULL,
  * else only if the Gaussian can reach alpha >= alpha_min on t: o >= alpha_min and the minimum
  * of sigma over the box of t's pixel centres [16 tx + 0.5, 16 tx + 15.5] x [...] is
- * <= ln(o / alpha_min).  Dropped entries are skipped by every pixel of t anyway. */
+ * <= ln(o / alpha_min).  Dropped entries are skipped by every pixel of t anyway.
+ * With margin_rel or margin_abs non-zero (the renderer's listing reading, R1b), the test is
+ * m / ln 2 <= (thr (1 + margin_rel) + margin_abs) (1 + margin_rel), thr = log2(o / alpha_min):
+ * a superset of the exact rule's lists whose extra entries every pixel of their tile skips. */
 long long orc_tile_lists(int n, const int* visible, const int* rect, const unsigned* depth_key,
                          int tiles_x, int tiles_y, long long* offsets, int* ids,
-                         long long capacity, const orc_splats* s, double alpha_min, int tile);
+                         long long capacity, const orc_splats* s, double alpha_min, int tile,
+                         double margin_rel, double margin_abs);
 
 /* Minimum of sigma(d) = 1/2 (a dx^2 + c dy^2) + b dx dy over the box [X0, X1] x [Y0, Y1]
  * (convex: 0 if the box holds d = 0, else the least value on its four edges). */

@@ -116,35 +116,52 @@ def _in(rect, x, y):
 LOG2E = 1.4426950408889634
 
 
-def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, delta=1e-4, tiles=None):
+def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, tiles=None, m_uv=None):
     """Entries (Gaussian, tile) the GPU may list or not.
 
-    The oracle lists tile t of Gaussian g when t is in g's square and the least sigma over
-    t's pixel-centre box is <= ln(o / alpha_min).  The GPU tests the same quantity in fp32 in
-    log2 units with a margin: kept when sigma' * 0.999 <= (1.001 thr' + 0.01) * 1.001.
-    Returns (opt_list, opt_render): tile -> set of ids whose listing may differ, and the
-    subset where the Gaussian might still reach alpha_min at a pixel (render alternatives
-    needed); the rest of opt_list is skipped by every pixel either way.  tiles: only these
-    tiles (all if None)."""
+    Both sides list by the renderer's listing rule (R1b): tile t of Gaussian g's square is
+    listed when m, the least sigma over t's pixel-centre box in log2 units, is at most
+    lim = (thr (1 + LIST_REL) + LIST_ABS) (1 + LIST_REL), thr = log2(o / alpha_min).  The GPU
+    decides it in fp32 (the x-extent of the ellipse sigma' <= lim over the tile row's band), so
+    an entry is optional only when m lies within fp32 reach of lim:
+      |m - lim| <= delta_g (lim + 1) + |grad m| |d uv| + lambda |d uv|^2 / 2,
+    delta_g = 2 m_conic + 1e-5 (the conic's relative uncertainty of the model above and about
+    170 roundings of the extent arithmetic), |grad m| <= sqrt(2 lambda m) at the box minimum,
+    lambda the largest eigenvalue of the log2-scaled conic, d uv the mean's uncertainty; or when
+    the tile's place in the square is itself ambiguous (lo / hi rectangles).
+    Returns (opt_list, opt_render): tile -> set of ids whose listing may differ, and the subset
+    where the Gaussian might still reach alpha_min at a pixel (render alternatives needed; the
+    band around lim lies above thr, so only square-boundary entries can be in it).  tiles: only
+    these tiles (all if None)."""
     tx, ty = oracle.tiles_xy(cam.width, cam.height, tile)
     opt_list, opt_render = {}, {}
+    lam = P["eig"]
+    kappa = np.where(lam[:, 1] > 0, lam[:, 0] / np.maximum(lam[:, 1], 1e-30), 1.0)
+    m_conic = 64 * U * (1 + kappa)
+    duv = np.hypot(m_uv[:, 0], m_uv[:, 1]) if m_uv is not None else np.full(len(kappa), 1e-4)
 
     def visit(g, x, y):
         o = P["opacity"][g]
         u, v = P["uv"][g]
-        thr = math.log(o / alpha_min) * LOG2E if o >= alpha_min else -1.0
-        lim = (thr * 1.001 + 0.01) * 1.001 if thr >= 0 else -1.0
+        if not o >= alpha_min:
+            return
+        thr = math.log2(o / alpha_min)
+        lim = (thr * (1 + oracle.LIST_REL) + oracle.LIST_ABS) * (1 + oracle.LIST_REL)
+        a, b, c = P["conic"][g]
+        qmax = LOG2E * 0.5 * (a + c + math.hypot(a - c, 2 * b))
         m = LOG2E * oracle.box_min_sigma(P["conic"][g], x * tile + 0.5 - u,
                                          x * tile + tile - 0.5 - u,
                                          y * tile + 0.5 - v, y * tile + tile - 0.5 - v)
+        band = (2 * m_conic[g] + 1e-5) * (lim + 1) + math.sqrt(2 * qmax * max(m, 0.0)) * duv[g] + \
+            0.5 * qmax * duv[g] ** 2
         in_sq_certain = _in(lo[g], x, y)
-        keep_certain = thr >= 0 and m <= thr * (1 - delta) - delta
-        keep_possible = thr >= 0 and m * 0.999 <= lim * (1 + delta) + delta
+        keep_certain = m <= lim - band
+        keep_possible = m <= lim + band
         if (in_sq_certain and keep_certain) or not keep_possible:
             return
         t = y * tx + x
         opt_list.setdefault(t, set()).add(int(g))
-        if thr >= 0 and m <= thr * (1 + delta) + delta:
+        if m <= thr + band:
             opt_render.setdefault(t, set()).add(int(g))
 
     live = np.any(hi != 0, axis=1) & (P["depth"] > 0.2)
@@ -160,6 +177,12 @@ def listing_ambiguity(P, lo, hi, cam, alpha_min=1.0 / 255.0, tile=16, delta=1e-4
             for g in np.nonzero(cand)[0]:
                 visit(g, x, y)
     return opt_list, opt_render
+
+
+def optional_share(opt_list, K):
+    """Optional entries over the listed pairs, for the test output."""
+    n = sum(len(v) for v in opt_list.values())
+    return n, n / max(K, 1)
 
 
 def check_tile_lists(gpu_ranges, gpu_ids, off, ids, P, opt, n_tiles, tiles=None):

@@ -64,7 +64,7 @@ def sampled_block_check(ctx, g, cam_np, n_tiles_sampled, seed, max_pairs, min_cl
     off, ids = oracle.tile_lists(P, W, H)
     m_uv, _ = par.margins(gs, cam_np, P)
     lo, hi, _ = par.rect_bounds(P, cam_np, m_uv)
-    opt_list, opt = par.listing_ambiguity(P, lo, hi, cam_np, tiles=tiles)
+    opt_list, opt = par.listing_ambiguity(P, lo, hi, cam_np, tiles=tiles, m_uv=m_uv)
     Fh, Bh = sg.premultiplied_layers(2, H, W, seed=seed + 1).astype(np.float16)
     F64, B64 = Fh.astype(np.float64), Bh.astype(np.float64)
     # GPU: the whole block

@@ -202,15 +202,17 @@ def test_tile_lists_brute_force():
     assert np.all(np.abs(z32.astype(np.float64) - P["depth"][vis]) <= 4e-7 * P["depth"][vis])
 
 
-def test_alpha_listing_rule_drops_only_skipped_entries():
-    """The listing rule keeps a tile of the 3-sigma square only where the Gaussian can reach
-    alpha_min: every dropped entry is skipped by all 256 pixel centres of its tile, and the
+@pytest.mark.parametrize("rule", ["alpha", "listing"])
+def test_alpha_listing_rule_drops_only_skipped_entries(rule):
+    """The alpha rule keeps a tile of the 3-sigma square only where the Gaussian can reach
+    alpha_min, and the renderer's listing rule (R1b) only where it comes within the listing
+    margin of that: every dropped entry is skipped by all 256 pixel centres of its tile, and the
     rendered image is bit-identical to the one over the full squares."""
     s = sg.tiny_scene(per_cell=300, res=96, n_cams=2)
     for cam in s.cameras:
         P = oracle.project(s.gaussians, cam)
         oq, iq = oracle.tile_lists(P, cam.width, cam.height, rule="square")
-        oa, ia = oracle.tile_lists(P, cam.width, cam.height, rule="alpha")
+        oa, ia = oracle.tile_lists(P, cam.width, cam.height, rule=rule)
         tx, ty = oracle.tiles_xy(cam.width, cam.height)
         assert len(ia) < len(iq)
         ys, xs = np.mgrid[0:16, 0:16] + 0.5
@@ -229,6 +231,35 @@ def test_alpha_listing_rule_drops_only_skipped_entries():
         Ra = oracle.render(sp, oa, ia, cam.width, cam.height)
         np.testing.assert_array_equal(Ra["out"], Rq["out"])
         np.testing.assert_array_equal(Ra["T_final"], Rq["T_final"])
+
+
+def test_listing_margin_keeps_a_superset_of_the_alpha_rule():
+    """The listing rule's lists hold the alpha rule's in the same order; an entry it adds has
+    its least sigma over the tile's pixel centres above ln(o / alpha_min) (no pixel of the tile
+    reaches alpha_min) and at most the margin's limit, and the margin adds few entries."""
+    s = sg.tiny_scene(per_cell=600, res=128, n_cams=3)
+    for cam in s.cameras:
+        P = oracle.project(s.gaussians, cam)
+        oa, ia = oracle.tile_lists(P, cam.width, cam.height, rule="alpha")
+        ol, il = oracle.tile_lists(P, cam.width, cam.height, rule="listing")
+        tx, ty = oracle.tiles_xy(cam.width, cam.height)
+        extra = 0
+        for t in range(tx * ty):
+            kept = list(ia[oa[t]:oa[t + 1]])
+            listed = list(il[ol[t]:ol[t + 1]])
+            assert [g for g in listed if g in set(kept)] == kept, t
+            x, y = t % tx, t // tx
+            for g in set(listed) - set(kept):
+                extra += 1
+                u, v = P["uv"][g]
+                m = oracle.box_min_sigma(P["conic"][g], 16 * x + 0.5 - u, 16 * x + 15.5 - u,
+                                         16 * y + 0.5 - v, 16 * y + 15.5 - v)
+                thr = math.log(P["opacity"][g] * 255.0)
+                lim = (thr / math.log(2) * (1 + oracle.LIST_REL) + oracle.LIST_ABS) * \
+                    (1 + oracle.LIST_REL) * math.log(2)
+                assert thr < m <= lim, (t, g, m, thr, lim)
+        assert len(il) == len(ia) + extra
+        assert extra <= 0.02 * len(ia), (extra, len(ia))
 
 
 def test_box_min_sigma_against_dense_sampling():
@@ -631,3 +662,20 @@ def test_partition_order_consistent_with_rays():
                     assert c in fset, (campos, active, c)
                 else:
                     assert c not in fset, (campos, active, c)
+
+
+def test_blend_harness_form_equals_the_definition():
+    """The oracle's test-harness form of the blend (event reporting under an uncertainty model,
+    decisions inverted on request) gives, with no decision inverted, exactly the plain
+    definition's image."""
+    from tests import _parity as par
+    s = sg.tiny_scene(per_cell=300, res=64, n_cams=2)
+    for cam in s.cameras:
+        P = oracle.project(s.gaussians, cam)
+        off, ids = oracle.tile_lists(P, cam.width, cam.height)
+        plain = oracle.render(oracle.SplatSet.from_proj(P), off, ids, cam.width, cam.height)
+        probe = oracle.render(par.splats_with_margins(s.gaussians, cam, P), off, ids, cam.width,
+                              cam.height)
+        np.testing.assert_array_equal(plain["out"], probe["out"])
+        np.testing.assert_array_equal(plain["T_final"], probe["T_final"])
+        np.testing.assert_array_equal(plain["n_used"], probe["n_used"])
