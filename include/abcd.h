@@ -126,9 +126,10 @@ long long abcd_launch_count(const abcd_ctx* ctx);
  * reaches it gives up, the call's results are wrong and ABCD_ERR_TIMEOUT is set in the status
  * word (abcd_sync); nothing hangs, and later calls run normally once the status is cleared. */
 abcd_status abcd_set_wait_limit(abcd_ctx* ctx, unsigned polls);
-/* Test hook for the bounded waits: in the next abcd_bin_sort call, tile `tile` of the first
- * pass of the tile sort publishes nothing, so the waits of the tiles after it run out (after
- * the wait limit).  -1 (the default) turns it off; it turns itself off after that pass. */
+/* Test hook for the bounded waits: in the next abcd_bin_sort call, look-back tile `tile` (2048
+ * keys) of the first pass of the depth sort publishes nothing, so the waits of the tiles after
+ * it run out (after the wait limit).  -1 (the default) turns it off; it turns itself off after
+ * that pass. */
 abcd_status abcd_test_withhold_lookback(abcd_ctx* ctx, long long tile);
 
 /* ---- the hot path (Section 2: one step renders only the active block) ----------------- */
@@ -145,10 +146,11 @@ abcd_status abcd_project(abcd_ctx* ctx, const abcd_gaussians* theta, const abcd_
 /* K3 + K4. Tile binning and depth sort of the active block (the tile rasteriser of 3D Gaussian
  * Splatting, Section 1 by citation; Section 2 renders the active partition alone, so only its
  * Gaussians are binned).  A visible Gaussian is listed in each tile its square
- * [u-r, u+r] x [v-r, v+r] meets on which it can reach alpha >= alpha_min (the least sigma over
- * the box of the tile's pixel centres is at most ln(opacity / alpha_min), tested with a margin
- * of about 0.7% in sigma, so a list may hold a few entries that every pixel of the tile
- * skips); lists are ordered by the fp32 depth, ties by id.  Leaving out the tiles on which
+ * [u-r, u+r] x [v-r, v+r] meets on which it comes within a small margin of alpha_min: the least
+ * sigma over the box of the tile's pixel centres, in log2 units, is at most
+ * (1.001 log2(opacity / alpha_min) + 0.01) 1.001 (the exact rule, sigma <= ln(opacity /
+ * alpha_min), widened so that fp32 rounding never drops a tile it keeps; a list may hold a few
+ * entries that every pixel of the tile skips); lists are ordered by the fp32 depth, ties by id.  Leaving out the tiles on which
  * every pixel would skip the Gaussian does not change any pixel.  n must equal the n given
  * to abcd_project; opts as there (NULL = defaults; alpha_min is used).  Also leaves in the
  * context's workspace the tiles ordered by decreasing list length, tagged with out->ranges;
@@ -280,6 +282,20 @@ abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_ma
                                         const void* const* packed, int L, const int* order,
                                         int split, int width, int height, void* F_out,
                                         void* B_out, int out_dtype);
+
+/* One side of K1 in pieces, for devices that cannot hold every frozen layer of a camera at once
+ * (Section 2's memory hierarchy: the stored renders stay in host memory or on disk and pass
+ * through a device buffer of fixed size).  acc_out = acc_in over layer 0 over layer 1 ... over
+ * layer count-1 (packed layers as for abcd_composite_cache_packed, tile_maps[k] / packed[k] in
+ * fold order; acc_in NULL: from transparent), fp32 premultiplied RGBA [H][W][4]; out16, if not
+ * NULL, receives the fp16 (RNE) rounding of the result.  acc_in may equal acc_out.  The fp32
+ * operations and their order are those of abcd_composite_cache_packed, so folding F's (or B's)
+ * layers piece by piece into one accumulator and rounding at the end gives its F (B) bit for
+ * bit.  count <= 256. */
+abcd_status abcd_composite_fold_packed(abcd_ctx* ctx, const int* const* tile_maps,
+                                       const void* const* packed, int count, int width,
+                                       int height, const float* acc_in, float* acc_out,
+                                       void* out16);
 
 /* Visibility of the cached layers of one camera, for the visibility thresholds and occlusion
  * culling of camera-partition pairs that Section 4 proposes.  The layers are taken in `order`

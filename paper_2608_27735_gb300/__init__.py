@@ -118,6 +118,8 @@ _SIGS = {
     "abcd_cache_release": [C.c_void_p, C.c_int],
     "abcd_cache_store": [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_size_t],
     "abcd_cache_sync": [C.c_void_p],
+    "abcd_composite_fold_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_int,
+                                   C.c_void_p, C.c_void_p, C.c_void_p],
     "abcd_measure_alu_peaks": [C.c_int, C.c_void_p],
     "abcd_set_wait_limit": [C.c_void_p, C.c_uint],
     "abcd_test_withhold_lookback": [C.c_void_p, C.c_longlong],
@@ -438,6 +440,17 @@ def abcd_composite_cache_packed(ctx: Context, tile_maps, packed, order, split, w
     ordr = (C.c_int * max(1, L))(*[int(k) for k in order])
     ctx.check(lib().abcd_composite_cache_packed(ctx.h, maps, data, L, ordr, int(split), int(width),
                                                 int(height), _p(F_out), _p(B_out), int(out_dtype)))
+
+
+def abcd_composite_fold_packed(ctx: Context, tile_maps, packed, width, height, acc_in=None,
+                               acc_out=None, out16=None):
+    """One side of K1 in pieces: acc_out = acc_in over the given packed layers, in list order
+    (CUDA tensors; acc fp32 [H][W][4], out16 fp16 [H][W][4])."""
+    n = len(tile_maps)
+    maps = (C.c_void_p * max(1, n))(*[t.data_ptr() for t in tile_maps])
+    data = (C.c_void_p * max(1, n))(*[t.data_ptr() for t in packed])
+    ctx.check(lib().abcd_composite_fold_packed(ctx.h, maps, data, n, int(width), int(height),
+                                               _p(acc_in), _p(acc_out), _p(out16)))
 
 
 def abcd_layer_visibility(ctx: Context, layers, order, width, height, visible, coverage=None):

@@ -149,6 +149,10 @@ struct abcd_ctx {
   unsigned os_epoch = 0;                // last look-back epoch handed to a sort pass
   unsigned wait_limit = 1u << 20;       // polls before a device-side wait gives up
   long long withhold_tile = -1;         // test hook: a look-back tile that publishes nothing
+  // dynamic shared memory limits already raised on this context's device, per kernel (the
+  // attribute call costs host time on every step otherwise)
+  const void* smem_fn[16] = {nullptr};
+  int smem_set[16] = {0};
   char err[512] = {0};
 };
 
@@ -158,6 +162,8 @@ abcd_status fail(abcd_ctx* ctx, abcd_status code, const char* fmt, ...);
 void cache_destroy(abcd_ctx* ctx);            // copy streams and slot events (cache.cu)
 abcd_status check_launch(abcd_ctx* ctx, const char* what);
 abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched);
+// Raises kernel fn's dynamic shared-memory limit to at least `bytes` (once per context and size).
+cudaError_t ensure_smem(abcd_ctx* ctx, const void* fn, size_t bytes);
 bool has_workspace(const abcd_ctx* ctx);
 Cam make_cam(const abcd_camera* c, const abcd_render_opts* o);
 Opts make_opts(const abcd_render_opts* o);

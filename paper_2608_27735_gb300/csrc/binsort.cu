@@ -857,13 +857,13 @@ abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_s
   T* dst = b;
   for (int p = 0; p < sp.n; ++p) {
     const bool last = p == sp.n - 1;
-    // the test hook withholds a tile of the tile sort's first pass only
-    const long long withhold = (slot == 1 && p == 0) ? ctx->withhold_tile : -1;
+    // the test hook withholds a tile of the depth sort's first pass only
+    const long long withhold = (slot == 0 && p == 0) ? ctx->withhold_tile : -1;
     if ((s = launch_onesweep<T>(ctx, st, sp.bits[p], p >= match_from, G, src, dst,
                                 last ? ids_out : nullptr, id_mask, n_static, n_dev, cap,
                                 sp.shift[p], gh + p * kRadixBins, ctr, withhold)))
       return s;
-    if (slot == 1 && p == 0) ctx->withhold_tile = -1;
+    if (slot == 0 && p == 0) ctx->withhold_tile = -1;
     T* t = src; src = dst; dst = t;
   }
   if (result) *result = src;
@@ -939,8 +939,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   {
     const int cells = (tiles_x + 1) * (tiles_y + 1);
     const size_t smem = cells <= kSmemDiffCells ? sizeof(int) * cells : 0;
-    if (smem > 48 * 1024) {
-      const cudaError_t e2 = cudaFuncSetAttribute(tile_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    {
+      const cudaError_t e2 = ensure_smem(ctx, (const void*)tile_rows_kernel, smem);
       if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile_rows smem: %s", cudaGetErrorString(e2));
     }
     if ((s = check_launch(ctx, "tile_rows_kernel",
@@ -955,8 +955,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
     ctx->order_ranges = nullptr;
     if (cells <= kSmemDiffCells && n_tiles <= ctx->ws.max_tiles) {
       const size_t smem = sizeof(int) * cells + (size_t)n_tiles;
-      if (smem > 48 * 1024) {
-        const cudaError_t e2 = cudaFuncSetAttribute(ranges_order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      {
+        const cudaError_t e2 = ensure_smem(ctx, (const void*)ranges_order_kernel, smem);
         if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "ranges smem: %s", cudaGetErrorString(e2));
       }
       if ((s = check_launch(ctx, "ranges_order_kernel",

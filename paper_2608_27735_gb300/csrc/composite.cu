@@ -300,8 +300,71 @@ composite_packed_kernel(const __grid_constant__ PackedTable pt, int nf, int nb, 
   }
 }
 
+// One side's left fold continued from an fp32 accumulator: acc = acc over the listed layers, in
+// order (acc_in NULL: from transparent); the accumulator goes back in fp32 (acc_out) and/or as
+// its fp16 rounding (out16).  The fold runs the same fp32 operations in the same order as
+// composite_packed_kernel, so folding the layers in pieces gives its result bit for bit.
+__global__ void __launch_bounds__(kPackedThreads)
+fold_packed_kernel(const __grid_constant__ PackedTable pt, int n, int width, int height,
+                   int tiles_x, const float4* acc_in, float4* acc_out, uint2* out16) {
+  pdl_prologue();
+  __shared__ int s_map[kMaxLayers];
+  const int tile = blockIdx.x;
+  const int unit = threadIdx.x;
+  for (int k = threadIdx.x; k < n; k += blockDim.x) s_map[k] = __ldg(pt.map[k] + tile);
+  __syncthreads();
+  const int r = unit / (kTile / 2), c = 2 * (unit % (kTile / 2));
+  const int y = (tile / tiles_x) * kTile + r, x = (tile % tiles_x) * kTile + c;
+  const long long p0 = (long long)y * width + x;
+  const bool in0 = y < height && x < width, in1 = y < height && x + 1 < width;
+  float acc[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+  if (acc_in) {
+    if (in0) { const float4 a = acc_in[p0]; acc[0] = a.x; acc[1] = a.y; acc[2] = a.z; acc[3] = a.w; }
+    if (in1) { const float4 a = acc_in[p0 + 1]; acc[4] = a.x; acc[5] = a.y; acc[6] = a.z; acc[7] = a.w; }
+  }
+  fold_packed(pt, s_map, 0, n, unit, acc);
+  if (in0) {
+    if (acc_out) acc_out[p0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    if (out16) store_pixel_out(out16, 1, p0, acc);
+  }
+  if (in1) {
+    if (acc_out) acc_out[p0 + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    if (out16) store_pixel_out(out16, 1, p0 + 1, acc + 4);
+  }
+}
+
 }  // namespace
 }  // namespace abcd
+
+extern "C" abcd_status abcd_composite_fold_packed(abcd_ctx* ctx, const int* const* tile_maps,
+                                                  const void* const* packed, int count,
+                                                  int width, int height, const float* acc_in,
+                                                  float* acc_out, void* out16) {
+  if (!ctx) return ABCD_ERR_INVALID_ARG;
+  if (count < 0 || count > kMaxLayers || (count > 0 && (!tile_maps || !packed)) || width <= 0 ||
+      height <= 0)
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_fold_packed: bad layer list or size");
+  if (((uintptr_t)acc_in & 15) || ((uintptr_t)acc_out & 15) || ((uintptr_t)out16 & 7))
+    return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_fold_packed: misaligned accumulator or output");
+  PackedTable pt;
+  for (int k = 0; k < count; ++k) {
+    const int* m = tile_maps[k];
+    const void* d = packed[k];
+    if (!m || !d) return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_fold_packed: layer %d is NULL", k);
+    if (((uintptr_t)d & 15) || ((uintptr_t)m & 3))
+      return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_composite_fold_packed: layer %d misaligned", k);
+    pt.map[k] = m;
+    pt.data[k] = (const uint4*)d;
+  }
+  if (!acc_out && !out16) return ABCD_OK;
+  const int tiles_x = (width + kTile - 1) / kTile, tiles_y = (height + kTile - 1) / kTile;
+  return check_launch(ctx, "fold_packed_kernel",
+                      launch_pdl(fold_packed_kernel, dim3(tiles_x * tiles_y), dim3(kPackedThreads),
+                                 0, ctx->stream, pt, count, width, height, tiles_x,
+                                 (const float4*)acc_in, (float4*)acc_out, (uint2*)out16));
+}
 
 extern "C" abcd_status abcd_composite_cache_packed(abcd_ctx* ctx, const int* const* tile_maps,
                                                    const void* const* packed, int L,

@@ -38,6 +38,23 @@ abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched) 
 
 bool has_workspace(const abcd_ctx* ctx) { return ctx && ctx->ws_base != nullptr; }
 
+cudaError_t ensure_smem(abcd_ctx* ctx, const void* fn, size_t bytes) {
+  if (bytes <= 48 * 1024) return cudaSuccess;
+  int slot = -1;
+  for (int i = 0; i < 16; ++i) {
+    if (ctx->smem_fn[i] == fn) { slot = i; break; }
+    if (!ctx->smem_fn[i] && slot < 0) slot = i;
+  }
+  if (slot >= 0 && ctx->smem_fn[slot] == fn && ctx->smem_set[slot] >= (int)bytes) return cudaSuccess;
+  int prev = 0;
+  cudaGetDevice(&prev);
+  if (prev != ctx->device) cudaSetDevice(ctx->device);
+  const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (prev != ctx->device) cudaSetDevice(prev);
+  if (e == cudaSuccess && slot >= 0) { ctx->smem_fn[slot] = fn; ctx->smem_set[slot] = (int)bytes; }
+  return e;
+}
+
 Opts make_opts(const abcd_render_opts* o) {
   Opts r;
   r.near_z = o ? o->near_z : 0.2f;
@@ -194,6 +211,7 @@ abcd_status abcd_set_workspace(abcd_ctx* ctx, void* ptr, size_t bytes, int max_g
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.os_ctr, 0, 256, ctx->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.vis_sums, 0, 8ull * kVisSumCopies * 2 * kMaxLayers, ctx->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->ws.vis_ticket, 0, 256, ctx->stream);
+
   if (e == cudaSuccess)
     e = cudaMemsetAsync(ctx->ws.os_state, 0, 8ull * kRadixBins * (size_t)ctx->ws.os_tiles, ctx->stream);
   ctx->os_epoch = 0;

@@ -326,7 +326,7 @@ abcd_status loss_launch(abcd_ctx* ctx, const float* out_rgba, const float* gt_rg
   if ((long long)grid.x * grid.y * grid.z > kMaxLossBlocks)
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_loss: image too large (%d x %d)", width, height);
   const size_t smem = sizeof(float) * kSmemFloats;
-  cudaError_t e = cudaFuncSetAttribute(loss_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = ensure_smem(ctx, (const void*)loss_kernel, smem);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "loss smem attribute: %s", cudaGetErrorString(e));
   return check_launch(ctx, "loss_kernel",
                       launch_pdl(loss_kernel, grid, dim3(kThreads), smem, ctx->stream, out_rgba, gt_rgb,

@@ -61,7 +61,8 @@ class Case:
         self.off, self.ids = oracle.tile_lists(self.P, self.cam.width, self.cam.height)
         self.m_uv, _ = par.margins(self.g, self.cam, self.P)
         self.lo, self.hi, self.amb_r = par.rect_bounds(self.P, self.cam, self.m_uv)
-        self.opt_list, self.opt = par.listing_ambiguity(self.P, self.lo, self.hi, self.cam)
+        self.opt_list, self.opt = par.listing_ambiguity(self.P, self.lo, self.hi, self.cam,
+                                                             m_uv=self.m_uv)
         self.sp = par.splats_with_margins(self.g, self.cam, self.P)
 
     def F64(self):
@@ -144,8 +145,11 @@ def test_bin_sort_matches_oracle(ctx, tiny, cam_idx):
     ids = r["tiles"].ids.cpu().numpy()[:K]
     tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
     par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
-    n_opt = sum(len(v) for v in case.opt_list.values())
+    n_opt, share = par.optional_share(case.opt_list, K)
+    print(f"camera {cam_idx}: K = {K}, oracle {len(case.ids)}, optional entries {n_opt} "
+          f"({share:.2e} of K)")
     assert abs(K - len(case.ids)) <= n_opt
+    assert share <= 1e-3
 
 
 def test_bin_sort_ragged_and_sh3(ctx, ragged):
@@ -173,6 +177,24 @@ def test_bin_sort_many_gaussians(ctx):
     ids = r["tiles"].ids.cpu().numpy()[:K]
     tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
     par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
+
+
+def test_bin_sort_wide_image(ctx):
+    """A wide tile grid (4096x640: 10,240 tiles, 14 tile bits: the tile sort's passes take 7
+    bits each) with 3,000 Gaussians: the lists equal the oracle's."""
+    s = sg.grid_scene((1, 1, 1), 5.0, 3000, 0, seed=95)
+    s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 4096, 640, seed=95,
+                                height_jitter=1.0)
+    case = Case(s, 0, fb=False)
+    r = run_forward(ctx, case, want_state=False)
+    K = int(r["tiles"].count.item())
+    rng = r["tiles"].ranges.cpu().numpy().astype(np.int64)
+    ids = r["tiles"].ids.cpu().numpy()[:K]
+    tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
+    assert tx * ty == 10240
+    par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
+    n_opt, share = par.optional_share(case.opt_list, K)
+    print(f"wide image: K = {K}, optional entries {n_opt} ({share:.2e} of K)")
 
 
 @pytest.mark.parametrize("cam_idx,bg,fbdt", [(0, None, "f16"), (1, (0.2, 0.5, 0.9), "f16"),
@@ -751,21 +773,23 @@ def test_capacity_overflow_reported(ctx, tiny):
     ctx.sync()
 
 
-def test_bin_sort_wait_timeout_reported(ctx, tiny):
-    """The radix sort's look-back waits are bounded: with tile 0 of the tile sort's first pass
+def test_bin_sort_wait_timeout_reported(ctx):
+    """The radix sort's look-back waits are bounded: with tile 0 of the depth sort's first pass
     withheld (a test hook: it publishes nothing) and a short wait limit, the tiles behind it give
     up, abcd_sync reports ABCD_ERR_TIMEOUT and the call returns; once the status is cleared the
     same context sorts correctly again."""
-    case = Case(tiny, 2, fb=False)
-    cam = ab.camera(case.cam)
-    theta = ab.Gaussians.from_numpy(case.g)
+    s = sg.grid_scene((1, 1, 1), 5.0, 6000, 0, seed=97)
+    s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 96, 64, seed=97)
+    g = s.gaussians
+    assert g.n > 2 * 2048             # the depth sort's passes span three look-back tiles
+    cam = ab.camera(s.cameras[0])
+    theta = ab.Gaussians.from_numpy(g)
     proj = ab.Projected.alloc(theta.n)
     ab.abcd_project(ctx, theta, cam, None, proj)
-    tiles = ab.Tiles.alloc(1 << 20, case.cam.width, case.cam.height)
+    tiles = ab.Tiles.alloc(1 << 20, s.cameras[0].width, s.cameras[0].height)
     ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
     ctx.sync()
     K = int(tiles.count.item())
-    assert K > 4096, K                # the first tile-sort pass spans more than one look-back tile
     ref_ids = tiles.ids[:K].clone()
     ref_rng = tiles.ranges.clone()
     L = ab.lib()
