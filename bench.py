@@ -56,6 +56,8 @@ def parse(argv=None):
     ap.add_argument("--width", type=int, default=1237)
     ap.add_argument("--height", type=int, default=822)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the measurements of the other workload configurations")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sample-every", type=int, default=10, help="per-op event sampling stride")
     return ap.parse_args(argv)
@@ -177,8 +179,6 @@ class Stage:
         for c in scene.cameras:
             f, b = ab.abcd_partition_split(grid.dims, grid.origin, grid.side, c.position, self.active)
             self.splits.append((list(f), list(b)))
-        # cameras that observe the active partition (all of them on this ring)
-        self.observing = list(range(len(self.cams)))
         npx = self.W * self.H
         self.ctx.reserve(max(n_max, 1), 16_000_000, npx)
         self.theta = ab.Gaussians.from_numpy(g.subset(self.part_idx[self.active]), device)
@@ -231,6 +231,13 @@ class Stage:
         self.pk_active = torch.empty(C, self.n_t, 16, 16, 4, dtype=torch.float16, device=device)
         self.pk_count = torch.zeros(C, P, dtype=torch.int32, device=device)
         ths = [ab.Gaussians.from_numpy(g.subset(self.part_idx[p]), device) for p in range(P)]
+        # a0: the visible camera-partition pairs (frustum filter on each partition's cell and
+        # 3-sigma box); the cameras that observe the active partition train it
+        self.vis_pairs = ab.visible_pairs(self.ctx, {p: ths[p] for p in range(P)}, scene.cameras,
+                                          grid.dims, grid.origin, grid.side)
+        self.observing = [ci for ci in range(C) if self.vis_pairs[ci, a]]
+        log(f"[bench] visible camera-partition pairs {int(self.vis_pairs.sum())} of {C * P}; "
+            f"{len(self.observing)} cameras observe the active partition")
         tmp = torch.empty(P, self.n_t, 16, 16, 4, dtype=torch.float16, device=device)
         self.pk_frozen, self.pk_off = [], []
         for ci in range(C):
@@ -615,6 +622,19 @@ def run_ours(args):
                            "counts; full_scene = one block; abcd_culled = camera-partition pairs "
                            "below a 1% visible share dropped; abcd_overlap = overlapping "
                            "boundary region of width 1 (a fifth of a cell)")
+    configs = None
+    if not args.no_configs:
+        del st.pk_frozen, st.F, st.B, st.gt        # make room: the stage is measured
+        torch.cuda.empty_cache()
+        configs = {}
+        for name, fn in (("cache_sweep_64_layers_1080p", run_cache_sweep),
+                         ("stress_2M_1080p", run_stress),
+                         ("grid_3x3x3_20k_640x480_stage", run_medium_stage)):
+            t0 = time.time()
+            configs[name] = fn(local)
+            log(f"[bench] {name}: {configs[name]} ({time.time() - t0:.1f}s)")
+        cs = configs["cache_sweep_64_layers_1080p"]
+        cs["hbm_frac"] = round(cs["gbs"] / hbm_peak, 4)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, log)
@@ -631,10 +651,17 @@ def run_ours(args):
         "streaming_one_fb_pair": streaming,
         "bcd_quality": quality,
         "visibility_culling": visibility,
+        "frustum": {"pairs": int(st.vis_pairs.size), "visible_pairs": int(st.vis_pairs.sum()),
+                    "observing_cameras": len(st.observing),
+                    "note": "a camera-partition pair is kept when the partition's cell united "
+                            "with its Gaussians' 3-sigma box meets the guard-widened view "
+                            "frustum (abcd_block_bounds, abcd_pair_visible); ring cameras "
+                            "facing the grid see every partition"},
         "gpu_launches": int(launches),
         "clocks": clocks,
         "ops": {k: {"avg_ms": round(v["avg_ms"], 4), "share": round(share[k], 4)} for k, v in ops.items()},
         "rooflines": per_kernel,
+        "configs": configs,
         "alu_peaks": {k: (round(v, 3) if isinstance(v, float) else v) for k, v in alu.items()},
     }
     if rank == 0:
@@ -645,6 +672,154 @@ def run_ours(args):
 
 
 TAU_VISIBLE = 1e-3
+
+
+# ---------------------------------------------------------------------------------------
+# the other workload configurations, measured after the headline stage (each bounded to
+# seconds of GPU time)
+
+def run_cache_sweep(device, n_cams=200, L=64, width=1920, height=1080, sets=16, seed=404):
+    """K1 on the cache compositing sweep: per camera 64 fp16 premultiplied layers at 1080p in a
+    random depth order, folded into F and B for the split at every position 1..63; 16 distinct
+    layer sets (17 GB, far more than the L2) cycled over the 200 cameras with a fresh order
+    each.  GB/s of algorithmic bytes ((L - 1) layers read, F and B written, per split)."""
+    import torch
+    import paper_2608_27735_gb300 as ab
+    ctx = ab.Context(device)
+    P = width * height
+    g = torch.Generator(device=f"cuda:{device}")
+    g.manual_seed(seed)
+    layer_sets = []
+    for _ in range(sets):
+        a = torch.rand(L, height, width, 1, device=device, generator=g)
+        rgb = torch.rand(L, height, width, 3, device=device, generator=g) * a
+        layer_sets.append(torch.cat([rgb, a], -1).half())
+        del a, rgb
+    F = torch.empty(height, width, 4, dtype=torch.float16, device=device)
+    B = torch.empty_like(F)
+    rng = np.random.default_rng(seed)
+    orders = [list(rng.permutation(L)) for _ in range(n_cams)]
+    tables = []
+    for ci in range(n_cams):
+        st = layer_sets[ci % sets]
+        tables.append([st[k] for k in range(L)])
+    def sweep(cams):
+        for ci in cams:
+            for split in range(1, L):
+                lay = list(tables[ci])
+                lay[orders[ci][split]] = None
+                ab.abcd_composite_cache(ctx, lay, orders[ci], split, width, height, F, B)
+    sweep(range(2))
+    torch.cuda.synchronize()
+    e0 = torch_event(torch, ctx.stream)
+    sweep(range(n_cams))
+    e1 = torch_event(torch, ctx.stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    per = (L - 1) * 8 * P + 2 * 8 * P
+    calls = n_cams * (L - 1)
+    gbs = calls * per / (ms * 1e-3) / 1e9
+    del layer_sets, tables
+    torch.cuda.empty_cache()
+    return {"workload": f"{L} fp16 RGBA layers {width}x{height} per camera, {n_cams} cameras, "
+                        f"splits 1..{L - 1}, {sets} distinct layer sets ({sets * L * 8 * P / 1e9:.1f} GB)",
+            "calls": calls, "ms": round(ms, 1), "us_per_split": round(1e3 * ms / calls, 2),
+            "algorithmic_bytes_per_split": per, "gbs": round(gbs, 1), "kernel": "composite_kernel"}
+
+
+def run_stress(device, n=2_000_000, width=1920, height=1080, n_cams=200, sampled=12, seed=505):
+    """The stress block: 2M Gaussians (SH 3) from a 16-blob mixture, one dense block seen by 200
+    ring cameras at 1920x1080; per sampled camera one forward + backward step (project, bin +
+    sort, render, L1 + 0.2 D-SSIM against a target, backward to the parameters), timed with
+    events; list statistics from the tile ranges."""
+    import torch
+    import paper_2608_27735_gb300 as ab
+    from paper_2608_27735_gb300 import scenegen as sg
+    g = sg.mixture_block(n, 20.0, 16, 3, seed=seed)
+    cams_np = sg.ring_cameras(n_cams, 30.0, np.zeros(3), width, height, seed=seed, height_jitter=2.0)
+    cams = [ab.camera(c) for c in cams_np]
+    ctx = ab.Context(device)
+    theta = ab.Gaussians.from_numpy(g)
+    grads = ab.Gaussians.zeros_like(theta)
+    proj = ab.Projected.alloc(n)
+    cap = 450_000_000
+    ctx.reserve(n, cap, width * height)
+    tiles = ab.Tiles.alloc(cap, width, height)
+    out = torch.empty(height, width, 4, device=device)
+    state = ab.FwdState.alloc(width, height)
+    gt = torch.rand(height, width, 3, device=device)
+    loss = torch.zeros(sampled, device=device)
+    pick = list(range(0, n_cams, max(1, n_cams // sampled)))[:sampled]
+    def step(k, ci):
+        ab.abcd_project(ctx, theta, cams[ci], None, proj)
+        ab.abcd_bin_sort(ctx, proj, n, cams[ci], tiles)
+        ab.abcd_render_composite_fwd(ctx, cams[ci], None, proj, tiles, None, None, ab.ABCD_F16,
+                                     None, out, state)
+        ab.abcd_backward(ctx, theta, cams[ci], None, proj, tiles, None, None, ab.ABCD_F16, None,
+                         out, state, gt, 0.2, loss[k:k + 1], None, grads)
+    step(0, pick[0])
+    ctx.sync()
+    Ks, lmean, lmax, walked, ms_all = [], [], [], [], []
+    for k, ci in enumerate(pick):
+        e0 = torch_event(torch, ctx.stream)
+        step(k, ci)
+        e1 = torch_event(torch, ctx.stream)
+        ctx.sync()
+        ms_all.append(e0.elapsed_time(e1))
+        K = int(tiles.count.item())
+        r = tiles.ranges.long()
+        lens = (r[:, 1] - r[:, 0]).clamp(min=0)
+        Ks.append(K)
+        lmean.append(float(lens.double().mean()))
+        lmax.append(int(lens.max()))
+        walked.append(int(state.n_last.sum(dtype=torch.int64)))
+    ms = float(np.mean(ms_all))
+    res = {"workload": f"one block of {n} Gaussians (SH 3, 16-blob mixture), {width}x{height}, "
+                       f"{len(pick)} of {n_cams} ring cameras",
+           "fwd_bwd_steps_per_s": round(1e3 / ms, 2), "ms_per_step": round(ms, 3),
+           "K_mean": int(np.mean(Ks)), "list_len_mean": round(float(np.mean(lmean)), 1),
+           "list_len_max": int(np.max(lmax)), "pixel_list_pairs_walked_mean": int(np.mean(walked)),
+           "pairs_per_s": round(float(np.mean(walked)) / (ms * 1e-3), 1)}
+    del theta, grads, proj, tiles
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_medium_stage(device, T=100, seed=1002):
+    """The 3x3x3 grid x 20,000 Gaussians (SH 3) workload, 50 hemisphere cameras at 640x480: one
+    ABCD stage of the centre partition through the BCD driver (F/B composited from the cached
+    layers of the visible pairs, T = 100 Adam steps, refresh), timed with events."""
+    import torch
+    import paper_2608_27735_gb300 as ab
+    from paper_2608_27735_gb300 import scenegen as sg
+    from paper_2608_27735_gb300.bcd import BCD, default_lr
+    s = sg.medium_scene(seed=seed)
+    tgt = sg.perturbed(s.gaussians, s.grid.side, seed=seed + 1)
+    ref = BCD(tgt, (1, 1, 1), s.grid.origin, 3 * s.grid.side, s.cameras,
+              np.zeros((len(s.cameras), 480, 640, 3), np.float32), 0, default_lr(15.0),
+              max_pairs=40_000_000)
+    targets = np.stack([ref.render_full(ci)[..., :3].cpu().numpy() for ci in range(len(s.cameras))])
+    del ref
+    run = BCD(s.gaussians, s.grid.dims, s.grid.origin, s.grid.side, s.cameras, targets, T,
+              default_lr(15.0), seed=seed, max_pairs=8_000_000)
+    centre = 13
+    run.stage(centre)
+    run.ctx.sync()
+    e0 = torch_event(torch, run.ctx.stream)
+    run.stage(centre)
+    e1 = torch_event(torch, run.ctx.stream)
+    run.ctx.sync()
+    ms = e0.elapsed_time(e1)
+    res = {"workload": "3x3x3 grid x 20000 Gaussians (SH 3), 50 hemisphere cameras 640x480, "
+                       f"centre partition, T={T} steps per stage",
+           "stage_ms": round(ms, 2), "active_steps_per_s": round(T / (ms * 1e-3), 1),
+           "observing_cameras": len(run.cameras_of(centre)),
+           "visible_pairs": int(run.frustum.sum()), "pairs": int(run.frustum.size),
+           "loss_mean_first_last_10_steps": [round(float(run.loss[:10].mean()), 5),
+                                             round(float(run.loss[T - 10:].mean()), 5)]}
+    del run
+    torch.cuda.empty_cache()
+    return res
 
 
 def run_visibility(st: Stage, reps=3):

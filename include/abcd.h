@@ -402,6 +402,25 @@ typedef struct {
  * nothing.  ABCD_ERR_CUDA if a launch or event fails. */
 abcd_status abcd_measure_alu_peaks(int device, abcd_alu_peaks* out);
 
+/* ---- visible camera-partition pairs (Section 2 caches renders of the visible pairs and
+ * trains a block on the cameras observing its partition; Section 3 speaks of the cameras left
+ * after frustum filtering) ------------------------------------------------------------------ */
+
+/* The axis-aligned box holding every Gaussian's 3-sigma ellipsoid of theta: box[0..2] lowest
+ * x, y, z, box[3..5] highest (device float [6], written; for Sigma = R(q) diag(exp(2 log_scale))
+ * R(q)^T the ellipsoid reaches mean_k +- 3 sqrt(Sigma_kk) along axis k, widened by 1e-6 relative
+ * for fp32 rounding).  An empty block gives lowest > highest.  One CTA (a per-stage call). */
+abcd_status abcd_block_bounds(abcd_ctx* ctx, const abcd_gaussians* theta, float* box);
+
+/* Whether a partition whose extent is the box (host double [6], as abcd_block_bounds; take the
+ * union with the cell) may be seen by the camera: the camera-space view frustum is
+ * {z >= near_z, |x| <= gx z, |y| <= gy z}, gx = guard * (width / 2) / fx, gy likewise; the
+ * pair is not visible (*visible = 0) only when the whole box lies outside one of those five
+ * half-spaces, so a box that meets the frustum is never culled (a few boxes near the frustum's
+ * edges that miss it are kept).  An empty box is not visible.  Host only. */
+abcd_status abcd_pair_visible(const abcd_camera* cam, const abcd_render_opts* opts,
+                              const double box[6], int* visible);
+
 /* ---- host-side partition logic (Section 2: regular grid, assignment by mean) --------- */
 
 /* cell[i] = linear id (i + gx (j + gy k)) of the grid cell holding means[i] (host array,

@@ -389,6 +389,22 @@ def partition_split(dims, origin, side, campos, active):
     return front[:nf.value].copy(), back[:nb.value].copy()
 
 
+def block_bounds(g) -> np.ndarray:
+    """Box (lowest x, y, z, highest x, y, z) of the Gaussians' 3-sigma ellipsoids."""
+    k = _GaussKeep(g)
+    box = np.zeros(6)
+    assert lib().orc_block_bounds(C.byref(k.s), _p(box)) == 0
+    return box
+
+
+def pair_visible(cam, box, opts=None) -> bool:
+    opts = opts or default_opts()
+    b = _f64(box)
+    v = C.c_int()
+    assert lib().orc_pair_visible(C.byref(camera(cam)), C.byref(opts), _p(b), C.byref(v)) == 0
+    return bool(v.value)
+
+
 def sh_basis(l, m, x, y, z):
     return lib().orc_sh_basis(l, m, x, y, z)
 

@@ -856,3 +856,60 @@ int orc_partition_split(const int* dims, const double* origin, double side,
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------
+// Visible camera-partition pairs (Section 2: the visible pairs are cached; Section 3: the
+// cameras left after frustum filtering).
+
+int orc_block_bounds(const orc_gaussians* g, double* box) {
+  for (int k = 0; k < 3; ++k) { box[k] = HUGE_VAL; box[3 + k] = -HUGE_VAL; }
+  for (int i = 0; i < g->n; ++i) {
+    const double* q = g->quats + 4 * i;
+    const double qn = std::sqrt(q[0] * q[0] + q[1] * q[1] + q[2] * q[2] + q[3] * q[3]);
+    const double w = q[0] / qn, x = q[1] / qn, y = q[2] / qn, z = q[3] / qn;
+    const double R[3][3] = {{1 - 2 * (y * y + z * z), 2 * (x * y - w * z), 2 * (x * z + w * y)},
+                            {2 * (x * y + w * z), 1 - 2 * (x * x + z * z), 2 * (y * z - w * x)},
+                            {2 * (x * z - w * y), 2 * (y * z + w * x), 1 - 2 * (x * x + y * y)}};
+    double S2[3];
+    for (int j = 0; j < 3; ++j) S2[j] = std::exp(2.0 * g->log_scales[3 * i + j]);
+    for (int k = 0; k < 3; ++k) {
+      // Sigma_kk = sum_j R_kj^2 s_j^2: the ellipsoid's half-width along axis k is 3 sqrt(Sigma_kk)
+      double v = 0.0;
+      for (int j = 0; j < 3; ++j) v += R[k][j] * R[k][j] * S2[j];
+      const double e = 3.0 * std::sqrt(v), m = g->means[3 * i + k];
+      box[k] = std::min(box[k], m - e);
+      box[3 + k] = std::max(box[3 + k], m + e);
+    }
+  }
+  return 0;
+}
+
+int orc_pair_visible(const orc_camera* cam, const orc_opts* o, const double* box, int* visible) {
+  if (!(box[0] <= box[3] && box[1] <= box[4] && box[2] <= box[5])) { *visible = 0; return 0; }
+  const double gx = o->guard * 0.5 * cam->width / cam->fx;
+  const double gy = o->guard * 0.5 * cam->height / cam->fy;
+  // the box's eight corners in camera space
+  double pc[8][3];
+  for (int c = 0; c < 8; ++c) {
+    const double p[3] = {box[(c & 1) ? 3 : 0], box[(c & 2) ? 4 : 1], box[(c & 4) ? 5 : 2]};
+    for (int i = 0; i < 3; ++i) {
+      pc[c][i] = cam->t[i];
+      for (int j = 0; j < 3; ++j) pc[c][i] += cam->R[3 * i + j] * p[j];
+    }
+  }
+  // culled when all corners lie outside one bounding plane of the frustum (a linear function
+  // is largest over the box at a corner)
+  auto all_out = [&](auto outside) {
+    for (int c = 0; c < 8; ++c)
+      if (!outside(pc[c][0], pc[c][1], pc[c][2])) return false;
+    return true;
+  };
+  const bool culled =
+      all_out([&](double, double, double z) { return z < o->near_z; }) ||
+      all_out([&](double x, double, double z) { return x > gx * z; }) ||
+      all_out([&](double x, double, double z) { return -x > gx * z; }) ||
+      all_out([&](double, double y, double z) { return y > gy * z; }) ||
+      all_out([&](double, double y, double z) { return -y > gy * z; });
+  *visible = culled ? 0 : 1;
+  return 0;
+}

@@ -27,6 +27,10 @@
  *   orc_loss               SSIM(x,x)=1, scipy 2-D correlation, finite differences
  *   orc_adam               first-step closed form, hand-computed second step
  *   orc_assign_cells / orc_partition_split   brute-force ray sampling of the depth order
+ *   orc_block_bounds       sampled points of every 3-sigma ellipsoid inside the box, its
+ *                          faces touched
+ *   orc_pair_visible       dense sampling of boxes: a box with a sampled point inside the
+ *                          frustum is never culled; closed-form cases
  */
 #ifndef ABCD_ORACLE_H
 #define ABCD_ORACLE_H
@@ -202,6 +206,15 @@ int orc_assign_cells(int n, const double* means, const double* origin, double si
 int orc_partition_split(const int* dims, const double* origin, double side,
                         const double* campos, int active, int* front, int* nf, int* back,
                         int* nb);
+
+/* Axis-aligned box of the 3-sigma ellipsoids of g: box[0..2] lowest, box[3..5] highest corner
+ * (half-width along axis k: 3 sqrt(Sigma_kk), Sigma = R(q) diag(exp(2 log_scale)) R(q)^T). */
+int orc_block_bounds(const orc_gaussians* g, double* box);
+
+/* Whether the box may be seen by the camera (reading R14): it is culled only when all eight
+ * corners lie, in camera space, on the outer side of one bounding plane of the view frustum
+ * {z >= near_z, |x| <= gx z, |y| <= gy z}, gx = guard * (width / 2) / fx (gy likewise). */
+int orc_pair_visible(const orc_camera* cam, const orc_opts* o, const double* box, int* visible);
 
 /* Real spherical harmonic Y_lm (Condon-Shortley phase) at a unit direction (for pins). */
 double orc_sh_basis(int l, int m, double x, double y, double z);

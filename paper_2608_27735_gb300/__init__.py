@@ -121,6 +121,8 @@ _SIGS = {
     "abcd_composite_fold_packed": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_int,
                                    C.c_void_p, C.c_void_p, C.c_void_p],
     "abcd_measure_alu_peaks": [C.c_int, C.c_void_p],
+    "abcd_block_bounds": [C.c_void_p, C.c_void_p, C.c_void_p],
+    "abcd_pair_visible": [C.c_void_p, C.c_void_p, C.c_void_p, C.POINTER(C.c_int)],
     "abcd_set_wait_limit": [C.c_void_p, C.c_uint],
     "abcd_test_withhold_lookback": [C.c_void_p, C.c_longlong],
     "abcd_assign_cells": [C.c_void_p, C.c_int, C.c_void_p, C.c_double, C.c_void_p, C.c_void_p],
@@ -614,3 +616,47 @@ def abcd_measure_alu_peaks(device=0) -> dict:
     if st != ABCD_OK:
         raise AbcdError(st, "abcd_measure_alu_peaks")
     return {k: getattr(p, k) for k, _ in abcd_alu_peaks._fields_}
+
+
+def abcd_block_bounds(ctx: Context, theta: Gaussians, box):
+    """box: CUDA float tensor [6] (lowest x, y, z, highest x, y, z of the 3-sigma ellipsoids)."""
+    g = theta.c()
+    ctx.check(lib().abcd_block_bounds(ctx.h, C.byref(g), _p(box)))
+
+
+def abcd_pair_visible(cam: abcd_camera, box, opts=None) -> bool:
+    """Whether the partition with extent `box` (6 floats: lowest, highest corner) may be seen."""
+    b = (C.c_double * 6)(*[float(v) for v in box])
+    v = C.c_int()
+    st = lib().abcd_pair_visible(C.byref(cam), _opt(opts), b, C.byref(v))
+    if st != ABCD_OK:
+        raise AbcdError(st, "abcd_pair_visible")
+    return bool(v.value)
+
+
+def visible_pairs(ctx: Context, blocks, cameras, dims, origin, side, opts=None):
+    """Visibility of every (camera, block) pair: [C][n_blocks] bool; a block's extent is its
+    cell united with its Gaussians' 3-sigma box (blocks: {block id: Gaussians on the device};
+    absent or empty blocks are not visible)."""
+    import numpy as np
+    torch = _torch()
+    n_blocks = int(np.prod(dims))
+    out = np.zeros((len(cameras), n_blocks), bool)
+    boxes = {}
+    for b, th in blocks.items():
+        if th.n == 0:
+            continue
+        dev = torch.empty(6, device="cuda")
+        abcd_block_bounds(ctx, th, dev)
+        boxes[b] = dev
+    ctx.sync()
+    gx, gy = int(dims[0]), int(dims[1])
+    cams = [c if isinstance(c, abcd_camera) else camera(c) for c in cameras]
+    for b, dev in boxes.items():
+        bx = dev.cpu().numpy().astype(np.float64)
+        ijk = np.array([b % gx, (b // gx) % gy, b // (gx * gy)], np.float64)
+        lo = np.asarray(origin, np.float64) + side * ijk
+        box = np.concatenate([np.minimum(bx[:3], lo), np.maximum(bx[3:], lo + side)])
+        for ci, cam in enumerate(cams):
+            out[ci, b] = abcd_pair_visible(cam, box, opts)
+    return out

@@ -16,7 +16,8 @@ import numpy as np
 from . import (ABCD_F16, ABCD_F32, Context, FwdState, Gaussians, Projected, Tiles, TrainStep,
                abcd_adam_active, abcd_assign_cells, abcd_backward, abcd_composite_cache,
                abcd_layer_visibility, abcd_loss, abcd_partition_split, abcd_project,
-               abcd_bin_sort, abcd_render_composite_fwd, camera, cull_pairs, _torch)
+               abcd_bin_sort, abcd_render_composite_fwd, camera, cull_pairs, visible_pairs,
+               _torch)
 
 # Adam learning rates per group (means, log-scales, quaternions, opacity logits, SH degree 0,
 # higher SH degrees): 3DGS-style defaults, the means' scaled by the scene extent.
@@ -109,6 +110,8 @@ class BCD:
         self.cull_tau = cull_tau
         self.keep = np.ones((C, n_blocks), bool)     # camera-partition pairs in use
         self.visible = np.zeros((C, n_blocks))
+        self.frustum = np.ones((C, n_blocks), bool)  # pairs that pass the frustum filter
+        self.update_frustum()
         for b in self.blocks:
             self.refresh(b, measure=False)
         self.measure_visibility()
@@ -149,6 +152,9 @@ class BCD:
         (with culling) measures the cameras' layers again."""
         th = self.theta[b]
         for ci, cam in enumerate(self.cams):
+            if not self.frustum[ci, b]:           # outside the frustum: transparent
+                self.layers[ci, b].zero_()
+                continue
             abcd_project(self.ctx, th, cam, None, self.proj)
             abcd_bin_sort(self.ctx, self.proj, th.n, cam, self.tiles)
             abcd_render_composite_fwd(self.ctx, cam, None, self.proj, self.tiles,
@@ -156,9 +162,20 @@ class BCD:
         if measure:
             self.measure_visibility()
 
+    def update_frustum(self):
+        """a0: the camera-partition pairs whose partition (cell united with its Gaussians'
+        3-sigma box) meets the camera's frustum; the others are never cached, composited or
+        trained on (their layers are transparent)."""
+        self.frustum = visible_pairs(self.ctx, self.theta, self.cams, self.dims, self.origin,
+                                     self.side)
+        if self.cull_tau is None:
+            self.keep = self.frustum.copy()
+        else:
+            self.keep &= self.frustum
+
     def measure_visibility(self):
         """Visible share of every camera-partition pair in its camera's composite of all
-        cached layers, and the pairs kept at the threshold."""
+        cached layers, and the pairs kept at the threshold (within the frustum's pairs)."""
         if self.cull_tau is None:
             return
         torch = self.torch
@@ -170,7 +187,7 @@ class BCD:
             abcd_layer_visibility(self.ctx, [self.layers[ci, k] for k in range(n_blocks)], order,
                                   self.W, self.H, vis[ci], cov[ci])
         self.visible = vis.cpu().numpy()
-        self.keep = cull_pairs(self.visible, cov.cpu().numpy(), self.cull_tau)
+        self.keep = cull_pairs(self.visible, cov.cpu().numpy(), self.cull_tau) & self.frustum
 
     def composite(self, b):
         """F and B of every camera around active block b, from the cached layers of the pairs
@@ -246,6 +263,7 @@ class BCD:
                 if trace is not None:
                     trace(t, ci, th, grads, m, v, self.loss[t:t + 1])
         self.steps_done += self.T if allowed else 0
+        self.update_frustum()                  # the block's Gaussians moved
         self.refresh(b)
 
     def stage_render(self, b, ci):

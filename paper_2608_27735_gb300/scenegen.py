@@ -127,6 +127,21 @@ def ring_cameras(n, radius, center, width, height, seed, height_jitter=0.0, fov=
     return cams
 
 
+def inside_cameras(grid, n, width, height, seed, fov=60.0):
+    """n cameras inside the grid's box (walk-through views): positions uniform in the middle
+    80% of the box, looking horizontally in a uniform direction."""
+    rng = _rng(seed, 7)
+    lo = np.asarray(grid.origin, np.float64)
+    hi = lo + grid.side * np.asarray(grid.dims, np.float64)
+    cams = []
+    for _ in range(n):
+        p = lo + (0.1 + 0.8 * rng.random(3)) * (hi - lo)
+        yaw = rng.uniform(0.0, 2.0 * np.pi)
+        cams.append(look_at(p, p + np.array([np.cos(yaw), np.sin(yaw), 0.0]), width, height,
+                            fov_x_deg=fov))
+    return cams
+
+
 def hemisphere_cameras(n, radius, center, width, height, fov=60.0):
     cams = []
     golden = math.pi * (3.0 - math.sqrt(5.0))

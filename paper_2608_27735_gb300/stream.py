@@ -30,7 +30,7 @@ import numpy as np
 from . import (Context, FwdState, Gaussians, Projected, RefreshLayer, Tiles, TrainStep, TILE,
                abcd_assign_cells, abcd_cache_fetch, abcd_cache_release, abcd_cache_store,
                abcd_cache_sync, abcd_cache_wait, abcd_composite_fold_packed,
-               abcd_partition_split, camera, _torch)
+               abcd_partition_split, camera, visible_pairs, _torch)
 
 BLOCK_TILE = (TILE, TILE, 4)          # one stored tile of a packed layer: 16 x 16 fp16 RGBA
 MAX_PIECE_LAYERS = 64                 # layers folded per call (tile maps staged at once)
@@ -155,6 +155,9 @@ class StreamingABCD:
         self.back_map = torch.empty(self.n_t, dtype=torch.int32).pin_memory()
         self.back_cnt = torch.empty(2, dtype=torch.int32).pin_memory()
         self.loss_host = torch.empty(max(1, self.T), dtype=torch.float32).pin_memory()
+        # a0: pairs whose partition meets the camera's frustum (the others are transparent:
+        # stored empty, not rendered, not trained on)
+        self.frustum = np.zeros((C, n_blocks), bool)
         for b in self.blocks:                   # the initial cache: every block's layers
             self._load(b)
             self.refresh(b)
@@ -181,10 +184,17 @@ class StreamingABCD:
             dst.copy_(src, non_blocking=True)
 
     def refresh(self, b):
-        """Block b's layer for every camera, rendered into a packed layer and stored."""
+        """Block b's layer for every camera that sees it, rendered into a packed layer and
+        stored (an empty layer for the others)."""
         th = self._view(b)[0]
+        self.frustum[:, b] = visible_pairs(self.ctx, {b: th}, self.cams, self.dims, self.origin,
+                                           self.side)[:, b]
         rl = RefreshLayer(self.ctx, th, self.proj, self.tiles)
         for ci, cam in enumerate(self.cams):
+            if not self.frustum[ci, b]:
+                self.store.put(ci, b, self.torch.full((self.n_t,), -1, dtype=self.torch.int32),
+                               self.torch.empty(0, *BLOCK_TILE, dtype=self.torch.float16))
+                continue
             rl(cam, self.ref_maps[0], self.ref_tiles[0], self.ref_cnt[0:1])
             self.back_cnt.copy_(self.ref_cnt, non_blocking=True)
             self.ctx.sync()
@@ -244,11 +254,13 @@ class StreamingABCD:
                 keep.clear()
         abcd_cache_sync(ctx)
 
-    def next_camera(self):
-        """Shuffle without replacement over the cameras, reshuffled when used up."""
+    def next_camera(self, allowed=None):
+        """Shuffle without replacement over the allowed cameras, reshuffled when used up."""
+        allowed = list(range(len(self.cams))) if allowed is None else list(allowed)
+        self.queue = [ci for ci in self.queue if ci in allowed]
         if not self.queue:
-            self.queue = [int(i) for i in self.rng.permutation(len(self.cams))]
-        return self.queue.pop()
+            self.queue = [allowed[i] for i in self.rng.permutation(len(allowed))]
+        return int(self.queue.pop())
 
     def stage(self, b, trace=None):
         """One stage of block b (see the module docstring).  trace, if given, is called after
@@ -259,7 +271,8 @@ class StreamingABCD:
         th, gr, m, v = self._view(b)
         step = TrainStep(ctx, th, gr, m, v, self.proj, self.tiles, self.out, self.state, self.lr,
                          lambda_ssim=self.lam)
-        order = [self.next_camera() for _ in range(self.T)]
+        allowed = [ci for ci in range(len(self.cams)) if self.frustum[ci, b]]
+        order = [self.next_camera(allowed) for _ in range(self.T)] if allowed else []
 
         def fetch(k, ci):
             s = self.slots[k]

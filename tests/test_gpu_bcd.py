@@ -108,3 +108,47 @@ def test_overlap_region_draws_every_gaussian_once():
                 side_gap["wide"] += (w_ - ref).abs().mean().item()
     assert side_gap["plain"] > 1e-3              # beside the split the layering departs
     print("side-camera gap (mean |composite - one-sort render|, 4 renders):", side_gap)
+
+
+def test_frustum_filter_of_camera_partition_pairs():
+    """a0 (reading R14) with walk-through cameras inside a 4x4x2 grid: abcd_block_bounds holds
+    the oracle's 3-sigma box of every block (to fp32 rounding), the driver's pair mask is the
+    oracle's frustum rule on the cells united with those boxes, culled pairs are never cached,
+    composited or trained on (their layers stay transparent), and a stage of a block trains on
+    the cameras that see it only."""
+    import oracle
+    ab.build()
+    from paper_2608_27735_gb300.bcd import BCD, default_lr
+    s = sg.grid_scene((4, 4, 2), 5.0, 300, 0, seed=72)
+    cams = sg.inside_cameras(s.grid, 8, 80, 54, seed=5)
+    tg = np.stack([sg.random_image(54, 80, 3, seed=60 + k) for k in range(8)]).astype(np.float32)
+    run = BCD(s.gaussians, s.grid.dims, s.grid.origin, s.grid.side, cams, tg, 6, default_lr(10.0),
+              seed=2)
+    cells = oracle.assign_cells(s.gaussians.means, s.grid.origin, s.grid.side, s.grid.dims)
+    for b in run.blocks:
+        gb = s.gaussians.subset(np.nonzero(cells == b)[0])
+        ref = oracle.block_bounds(gb)
+        box = torch.empty(6, device="cuda")
+        ab.abcd_block_bounds(run.ctx, run.theta[b], box)
+        run.ctx.sync()
+        got = box.cpu().numpy().astype(np.float64)
+        slack = 1e-5 * (1.0 + np.abs(ref))
+        assert np.all(got[:3] <= ref[:3] + slack[:3]) and np.all(got[3:] >= ref[3:] - slack[3:])
+        assert np.all(np.abs(got - ref) <= slack), (b, got, ref)
+        ijk = np.array([b % 4, (b // 4) % 4, b // 16], np.float64)
+        lo = np.asarray(s.grid.origin) + 5.0 * ijk
+        full = np.concatenate([np.minimum(ref[:3], lo), np.maximum(ref[3:], lo + 5.0)])
+        for ci, cam in enumerate(cams):
+            assert run.frustum[ci, b] == oracle.pair_visible(cam, full), (ci, b)
+    assert (~run.frustum).sum() >= 0.3 * run.frustum.size
+    layers = run.layers.cpu()
+    for ci in range(len(cams)):
+        for b in run.blocks:
+            if not run.frustum[ci, b]:
+                assert int(layers[ci, b].abs().sum()) == 0
+    b = max(run.blocks, key=lambda q: (0 < run.frustum[:, q].sum() < len(cams), run.frustum[:, q].sum()))
+    allowed = set(run.cameras_of(b))
+    assert allowed == {ci for ci in range(len(cams)) if run.frustum[ci, b]}
+    seen = []
+    run.stage(b, trace=lambda t, ci, *a: seen.append(ci))
+    assert seen and set(seen) <= allowed

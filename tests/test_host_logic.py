@@ -50,3 +50,25 @@ def test_cull_pairs_thresholds():
     assert ab.cull_pairs(v, c, 1e-3).tolist() == [True, False, True, False, True]
     assert ab.cull_pairs(v, c, 1e-3, tau_area=0.02).tolist() == [True, False, False, False, True]
     assert ab.cull_pairs(v, c, 0.25).tolist() == [False, False, False, False, True]
+
+
+def test_pair_visible_matches_oracle():
+    """abcd_pair_visible (host code of libabcd) decides every pair as the oracle's restatement
+    of the frustum rule does: walk-through and ring cameras, random boxes of every size."""
+    import oracle
+    from paper_2608_27735_gb300 import scenegen as sg
+    ab.build()
+    grid = sg.Grid(origin=np.array([-10.0, -10.0, -5.0]), side=5.0, dims=(4, 4, 2))
+    cams = sg.inside_cameras(grid, 6, 160, 107, seed=3) + \
+        sg.ring_cameras(6, 25.0, np.zeros(3), 160, 107, seed=3, height_jitter=1.0)
+    rng = np.random.default_rng(12)
+    agree = 0
+    for cam in cams:
+        c = ab.camera(cam)
+        for _ in range(300):
+            mid = rng.uniform(-20, 20, 3)
+            h = rng.uniform(0.01, 6.0, 3)
+            box = np.concatenate([mid - h, mid + h])
+            assert ab.abcd_pair_visible(c, box) == oracle.pair_visible(cam, box), (mid, h)
+            agree += 1
+    assert agree == 12 * 300

@@ -679,3 +679,89 @@ def test_blend_harness_form_equals_the_definition():
         np.testing.assert_array_equal(plain["out"], probe["out"])
         np.testing.assert_array_equal(plain["T_final"], probe["T_final"])
         np.testing.assert_array_equal(plain["n_used"], probe["n_used"])
+
+
+def _rot(q):
+    w, x, y, z = np.asarray(q, np.float64) / np.linalg.norm(q)
+    return np.array([[1 - 2 * (y * y + z * z), 2 * (x * y - w * z), 2 * (x * z + w * y)],
+                     [2 * (x * y + w * z), 1 - 2 * (x * x + z * z), 2 * (y * z - w * x)],
+                     [2 * (x * z - w * y), 2 * (y * z + w * x), 1 - 2 * (x * x + y * y)]])
+
+
+def test_block_bounds_hold_every_3sigma_ellipsoid():
+    """Points on every Gaussian's 3-sigma ellipsoid (mu + 3 R S u for unit u) lie in the box,
+    and each face of the box is touched (up to the sampling) by one of them."""
+    s = sg.grid_scene((1, 1, 1), 5.0, 40, 0, seed=61)
+    g = s.gaussians
+    box = oracle.block_bounds(g)
+    rng = np.random.default_rng(3)
+    u = rng.normal(size=(4000, 3))
+    u /= np.linalg.norm(u, axis=1, keepdims=True)
+    pts = []
+    for i in range(g.n):
+        M = _rot(g.quats[i]) @ np.diag(np.exp(g.log_scales[i].astype(np.float64)))
+        pts.append(g.means[i].astype(np.float64) + 3.0 * u @ M.T)
+    pts = np.concatenate(pts)
+    assert np.all(pts >= box[:3] - 1e-12) and np.all(pts <= box[3:] + 1e-12)
+    span = box[3:] - box[:3]
+    assert np.all(pts.min(0) - box[:3] <= 2e-2 * span) and np.all(box[3:] - pts.max(0) <= 2e-2 * span)
+
+
+def test_pair_visibility_never_culls_a_seen_box():
+    """Dense samples of random boxes: a box with a sample point inside the view frustum is
+    always visible; a box reported not visible has every sample outside; closed-form cases."""
+    cam = sg.look_at(np.array([0.0, -10.0, 0.0]), np.zeros(3), 160, 120)
+    rng = np.random.default_rng(8)
+    g = np.linspace(0.0, 1.0, 9)
+    gx = 1.3 * 0.5 * cam.width / cam.fx
+    gy = 1.3 * 0.5 * cam.height / cam.fy
+    R, t = cam.R.astype(np.float64), cam.t.astype(np.float64)
+    n_vis = n_cul = 0
+    for _ in range(400):
+        c = rng.uniform(-15, 15, 3)
+        h = rng.uniform(0.2, 4.0, 3)
+        box = np.concatenate([c - h, c + h])
+        P = np.stack(np.meshgrid(g, g, g, indexing="ij"), -1).reshape(-1, 3)
+        P = box[:3] + P * (box[3:] - box[:3])
+        pc = P @ R.T + t
+        inside = (pc[:, 2] >= 0.2) & (np.abs(pc[:, 0]) <= gx * pc[:, 2]) & \
+            (np.abs(pc[:, 1]) <= gy * pc[:, 2])
+        v = oracle.pair_visible(cam, box)
+        if inside.any():
+            assert v
+        n_vis += v
+        n_cul += not v
+    assert n_vis > 50 and n_cul > 50
+    pos = cam.position
+    ahead = pos + 6.0 * (R.T @ np.array([0.0, 0.0, 1.0]))
+    assert oracle.pair_visible(cam, np.concatenate([ahead - 0.1, ahead + 0.1]))
+    behind = pos - 6.0 * (R.T @ np.array([0.0, 0.0, 1.0]))
+    assert not oracle.pair_visible(cam, np.concatenate([behind - 0.1, behind + 0.1]))
+    side = pos + 6.0 * (R.T @ np.array([0.0, 0.0, 1.0])) + 6.0 * gx * 1.5 * (R.T @ np.array([1.0, 0, 0]))
+    assert not oracle.pair_visible(cam, np.concatenate([side - 0.1, side + 0.1]))
+    assert not oracle.pair_visible(cam, np.array([1.0, 1.0, 1.0, 0.0, 0.0, 0.0]))   # empty
+
+
+def test_culled_pairs_render_transparent():
+    """Walk-through cameras inside a 4x4x2 grid: every camera-partition pair the rule culls
+    lists no Gaussian on any tile in the oracle, so its layer is transparent (the reading loses
+    nothing), and the rule culls a good share of the pairs."""
+    s = sg.grid_scene((4, 4, 2), 5.0, 200, 0, seed=72)
+    cams = sg.inside_cameras(s.grid, 8, 160, 107, seed=5)
+    cells = oracle.assign_cells(s.gaussians.means, s.grid.origin, s.grid.side, s.grid.dims)
+    culled = 0
+    for cam in cams:
+        for b in range(32):
+            gb = s.gaussians.subset(np.nonzero(cells == b)[0])
+            bx = oracle.block_bounds(gb)
+            ijk = np.array([b % 4, (b // 4) % 4, b // 16], np.float64)
+            lo = np.asarray(s.grid.origin) + s.grid.side * ijk
+            box = np.concatenate([np.minimum(bx[:3], lo), np.maximum(bx[3:], lo + s.grid.side)])
+            if oracle.pair_visible(cam, box):
+                continue
+            culled += 1
+            P = oracle.project(gb, cam)
+            off, ids = oracle.tile_lists(P, cam.width, cam.height)
+            assert len(ids) == 0
+    assert culled >= 0.3 * 32 * len(cams), culled
+    print(f"culled pairs: {culled} of {32 * len(cams)}")
