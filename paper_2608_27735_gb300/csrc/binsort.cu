@@ -929,11 +929,9 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->side, ctx->ev_fork, 0);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort fork: %s", cudaGetErrorString(e));
   u64* by_depth = nullptr;
-  {
-    if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, n,
-                             32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom)))
-      return s;
-  }
+  if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, n,
+                           32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom)))
+    return s;
   e = cudaEventRecord(ctx->ev_join, ctx->side);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
   {
