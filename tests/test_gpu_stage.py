@@ -147,6 +147,74 @@ def group_lr(lr, k, shape):
     return out
 
 
+def check_steps(run, rec, theta0, halo, cams, F64, B64, targets, lr, min_kept=0.3):
+    """Every recorded step of a stage against the oracle at the parameters the GPU held before
+    it: the loss, the gradient of the trained rows (element-wise, or with the pixels near an
+    ambiguous decision left out of both sides plus in relative L2 norm) and the Adam update.
+    halo: frozen Gaussians rendered after the trained ones (scenegen.Gaussians) or None;
+    min_kept: the least share of pixels an ambiguous step may keep for its element-wise check."""
+    W, H = cams[0].width, cams[0].height
+    n = theta0.n
+    th = [a.astype(np.float64) for a in theta0.arrays()]
+    m_prev = [np.zeros_like(a) for a in th]
+    v_prev = [np.zeros_like(a) for a in th]
+    strict_steps = 0
+    kept_share = []
+    for t, r in enumerate(rec):
+        ci = r["ci"]
+        cam = cams[ci]
+        parts = [a.astype(np.float32) for a in th]
+        if halo is not None:
+            parts = [np.concatenate([a, h]) for a, h in zip(parts, halo.arrays())]
+        g = sg.Gaussians(*parts, theta0.sh_degree)
+        P, off, ids, sp, R = oracle_render(g, cam, F64[ci], B64[ci])
+        L, dL = oracle.loss(R["out"][..., :3], targets[ci].astype(np.float64), LAM)
+        g2 = oracle.backward(sp, off, ids, W, H, dL, F=F64[ci], B=B64[ci])
+        ref = {k: v[:n] for k, v in oracle.project_backward(g, cam, g2).items()}
+        amb, opt, _ = ambiguous(g, cam, P, R)
+        assert abs(r["loss"] - L) <= 1e-5 * L, (t, r["loss"], L)
+        if amb:
+            gm, refm, kept = masked_gradients(run, g, ci, cam, F64[ci], B64[ci], targets[ci], P, off,
+                                              ids, sp, R, opt)
+            gm = [x[:n] for x in gm]
+            refm = {k: v[:n] for k, v in refm.items()}
+            assert kept > min_kept, (t, kept)
+            kept_share.append(kept)
+        for k, name in enumerate(GROUPS):
+            got = r["grad"][k].astype(np.float64)
+            if not amb:
+                atol = min(1e-5, 1e-5 * float(np.abs(ref[name]).max()))
+                par.assert_grad_close(got, ref[name], rtol=1e-3, atol=atol, what=f"step {t} {name}")
+            else:
+                rel = np.linalg.norm(got - ref[name]) / max(np.linalg.norm(ref[name]), 1e-30)
+                assert rel < 1e-3, (t, name, rel)
+                atol = min(1e-5, 1e-5 * float(np.abs(refm[name]).max()))
+                par.assert_grad_close(gm[k], refm[name], rtol=1e-3, atol=atol,
+                                      what=f"step {t} {name} (unambiguous pixels)")
+        strict_steps += not amb
+        # the update: the oracle's Adam on the GPU's gradient from the GPU's state
+        a, mm, vv = [x.copy() for x in th], [x.copy() for x in m_prev], [x.copy() for x in v_prev]
+        oracle_adam(a, [x.astype(np.float64) for x in r["grad"]], mm, vv, lr, t + 1)
+        for k in range(5):
+            np.testing.assert_allclose(r["m"][k], mm[k], rtol=2e-6, atol=1e-12)
+            np.testing.assert_allclose(r["v"][k], vv[k], rtol=4e-6, atol=1e-18)
+            np.testing.assert_allclose(r["theta"][k], a[k], rtol=2e-6, atol=2e-7)
+        th, m_prev, v_prev = r["theta"], r["m"], r["v"]
+    print(f"stage: {strict_steps} of {len(rec)} steps free of ambiguous decisions (whole gradient "
+          f"element-wise); the others element-wise on the pixels kept ({np.mean(kept_share or [1]):.0%}"
+          f" on average) and in relative L2 norm on all")
+
+
+def recorder(rec):
+    def trace(t, ci, th, grads, m, v, loss):
+        rec.append(dict(ci=ci, theta=[x.cpu().numpy().astype(np.float64) for x in th.tensors()],
+                        grad=[x.cpu().numpy() for x in grads.tensors()],
+                        m=[x.cpu().numpy().astype(np.float64) for x in m.tensors()],
+                        v=[x.cpu().numpy().astype(np.float64) for x in v.tensors()],
+                        loss=float(loss.item())))
+    return trace
+
+
 def test_stage_matches_oracle():
     scene = sg.tiny_scene()
     dims, side, origin = scene.grid.dims, scene.grid.side, scene.grid.origin
@@ -205,51 +273,7 @@ def test_stage_matches_oracle():
             dst[ci] = got[ci].astype(np.float64)
 
     # ---- every step at the GPU's own parameters
-    th = [a.astype(np.float64) for a in theta0.arrays()]
-    m_prev = [np.zeros_like(a) for a in th]
-    v_prev = [np.zeros_like(a) for a in th]
-    strict_steps = 0
-    kept_share = []
-    for t, r in enumerate(rec):
-        ci = r["ci"]
-        cam = cams[ci]
-        g = sg.Gaussians(*[a.astype(np.float32) for a in th], theta0.sh_degree)
-        P, off, ids, sp, R = oracle_render(g, cam, F64[ci], B64[ci])
-        L, dL = oracle.loss(R["out"][..., :3], targets[ci].astype(np.float64), LAM)
-        g2 = oracle.backward(sp, off, ids, W, H, dL, F=F64[ci], B=B64[ci])
-        ref = oracle.project_backward(g, cam, g2)
-        amb, opt, _ = ambiguous(g, cam, P, R)
-        assert abs(r["loss"] - L) <= 1e-5 * L, (t, r["loss"], L)
-        if amb:
-            # the step's own gradient in relative L2 norm, and element-wise with the pixels
-            # near an ambiguous decision left out of both sides
-            gm, refm, kept = masked_gradients(run, g, ci, cam, F64[ci], B64[ci], targets[ci], P, off,
-                                              ids, sp, R, opt)
-            assert kept > 0.3, (t, kept)
-            kept_share.append(kept)
-        for k, name in enumerate(GROUPS):
-            got = r["grad"][k].astype(np.float64)
-            if not amb:
-                atol = min(1e-5, 1e-5 * float(np.abs(ref[name]).max()))
-                par.assert_grad_close(got, ref[name], rtol=1e-3, atol=atol, what=f"step {t} {name}")
-            else:
-                rel = np.linalg.norm(got - ref[name]) / max(np.linalg.norm(ref[name]), 1e-30)
-                assert rel < 1e-3, (t, name, rel)
-                atol = min(1e-5, 1e-5 * float(np.abs(refm[name]).max()))
-                par.assert_grad_close(gm[k], refm[name], rtol=1e-3, atol=atol,
-                                      what=f"step {t} {name} (unambiguous pixels)")
-        strict_steps += not amb
-        # the update: the oracle's Adam on the GPU's gradient from the GPU's state
-        a, mm, vv = [x.copy() for x in th], [x.copy() for x in m_prev], [x.copy() for x in v_prev]
-        oracle_adam(a, [x.astype(np.float64) for x in r["grad"]], mm, vv, lr, t + 1)
-        for k in range(5):
-            np.testing.assert_allclose(r["m"][k], mm[k], rtol=2e-6, atol=1e-12)
-            np.testing.assert_allclose(r["v"][k], vv[k], rtol=4e-6, atol=1e-18)
-            np.testing.assert_allclose(r["theta"][k], a[k], rtol=2e-6, atol=2e-7)
-        th, m_prev, v_prev = r["theta"], r["m"], r["v"]
-    print(f"stage: {strict_steps} of {T_STAGE} steps free of ambiguous decisions (whole gradient "
-          f"element-wise); the others element-wise on the pixels kept ({np.mean(kept_share or [1]):.0%}"
-          f" on average) and in relative L2 norm on all")
+    check_steps(run, rec, theta0, None, cams, F64, B64, targets, lr)
 
     # ---- the refresh: the block's layers rendered from the parameters the stage ended with
     thetaT = host_gaussians(run.theta[active])
@@ -317,3 +341,65 @@ def test_stage_matches_oracle():
         worst = max(worst, float((d / np.maximum(moved, 1e-12))[moved > 1e-6].max(initial=0.0)))
     print(f"independent oracle stage: losses within {max_loss_rel:.2e} relative; parameters "
           f"within {worst:.2e} of their movement over the stage")
+
+
+def test_overlap_stage_matches_oracle():
+    """A stage with an overlapping boundary region (reading R17): block 0 of a 2x1x1 grid is
+    trained together with its halo (block 1's Gaussians within 1.0 of its cell, rendered in the
+    same depth sort, frozen), against F and B folded from block 1's layer re-rendered without
+    them.  Checked against the oracle: the re-rendered donor layers, F and B as the fold of the
+    layers the stage uses, every step (loss, the block's gradient, Adam on the block's rows
+    only) at the parameters the GPU held, the block's refreshed layers, and the donor block
+    bit-identical afterwards."""
+    s = sg.grid_scene((2, 1, 1), 5.0, 300, 0, seed=11)
+    g = s.gaussians
+    cams = sg.ring_cameras(4, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 160, 120, seed=11)
+    W, H = 160, 120
+    tgt = sg.perturbed(g, 5.0, seed=12)
+    targets = []
+    for cam in cams:
+        Pt = oracle.project(tgt, cam)
+        ot, it = oracle.tile_lists(Pt, W, H)
+        targets.append(oracle.render(oracle.SplatSet.from_proj(Pt), ot, it, W, H)["out"][..., :3])
+    targets = np.stack(targets).astype(np.float32)
+    lr = [float(np.float32(x)) for x in default_lr(10.0)]
+    run = BCD(g, (2, 1, 1), s.grid.origin, 5.0, cams, targets, 6, lr, seed=4, lambda_ssim=LAM,
+              overlap=1.0)
+    b, q = 0, 1
+    pos = run.halo[b][q]
+    assert len(pos) > 10
+    donor = host_gaussians(run.theta[q])
+    halo = donor.subset(pos)
+    core = donor.subset(np.setdiff1d(np.arange(donor.n), pos))
+    theta0 = host_gaussians(run.theta[b])
+    donor_before = [t.cpu().clone() for t in run.theta[q].tensors()]
+    # the donor's layer without its halo members, as the stage's composite takes it
+    cores = torch.empty(len(cams), H, W, 4, dtype=torch.float16, device="cuda")
+    for ci in range(len(cams)):
+        run._core_layer(q, pos, ci, cores[ci])
+    run.ctx.sync()
+    cores_np = cores.cpu().numpy()
+    left_out = [refresh_ok(cores_np[ci], core, cams[ci]) for ci in range(len(cams))]
+    assert max(left_out) < 0.05, left_out
+    rec = []
+    run.stage(b, trace=recorder(rec))
+    run.ctx.sync()
+    assert len(rec) == 6
+    F16, B16 = run.F.cpu().numpy(), run.B.cpu().numpy()
+    F64, B64 = {}, {}
+    for ci in range(len(cams)):
+        order, split = run.order[ci, b]
+        for lst, got, dst in ((order[:split], F16, F64), (order[split + 1:], B16, B64)):
+            if lst:
+                assert list(lst) == [q]
+                fb16_ok(got[ci], cores_np[ci].astype(np.float64), 1)
+            else:
+                assert not np.any(got[ci])
+            dst[ci] = got[ci].astype(np.float64)
+    check_steps(run, rec, theta0, halo, cams, F64, B64, targets, lr, min_kept=0.2)
+    thetaT = host_gaussians(run.theta[b])
+    layersT = run.layers.cpu().numpy()
+    left_out = [refresh_ok(layersT[ci, b], thetaT, cams[ci]) for ci in range(len(cams))]
+    assert max(left_out) < 0.05, left_out
+    for a_, b_ in zip(donor_before, run.theta[q].tensors()):
+        assert torch.equal(a_, b_.cpu())
