@@ -58,15 +58,20 @@ __device__ __forceinline__ float4 scaled_conic(float4 c) {
 
 // sigma * log2(e) = dx (a/2 dx + b dy) + c/2 dy^2 at the lane's two pixels (fx0, fy) and
 // (fx1, fy); the dy terms are shared.  Both kernels take every branch decision from these bits.
+// The two pixels go through the packed two-lane fp32 instructions, whose every component is
+// rounded exactly as the scalar instruction would round it.
 __device__ __forceinline__ void sigma_pair(float4 s, float2 m, float fx0, float fx1, float fy,
                                            float& dx0, float& dx1, float& dy, float& s0, float& s1) {
   dy = __fsub_rn(fy, m.y);
-  dx0 = __fsub_rn(fx0, m.x);
-  dx1 = __fsub_rn(fx1, m.x);
+  const float2 dx = __fadd2_rn(make_float2(fx0, fx1), make_float2(-m.x, -m.x));
+  dx0 = dx.x;
+  dx1 = dx.y;
   const float bdy = __fmul_rn(s.y, dy);
   const float cdy2 = __fmul_rn(__fmul_rn(s.z, dy), dy);
-  s0 = __fmaf_rn(dx0, __fmaf_rn(s.x, dx0, bdy), cdy2);
-  s1 = __fmaf_rn(dx1, __fmaf_rn(s.x, dx1, bdy), cdy2);
+  const float2 in = __ffma2_rn(make_float2(s.x, s.x), dx, make_float2(bdy, bdy));
+  const float2 sg = __ffma2_rn(dx, in, make_float2(cdy2, cdy2));
+  s0 = sg.x;
+  s1 = sg.y;
 }
 
 // Lower bound of sigma * log2(e) over the box [X0, X1] x [Y0, Y1] of offsets d = pixel - uv:
@@ -243,6 +248,13 @@ struct PixF {
   bool done;
 };
 
+// Blend state of the lane's two pixels, the first in .x, the second in .y.
+struct PixF2 {
+  float2 T, c0, c1, c2;
+  unsigned last0, last1;
+  bool done0, done1;
+};
+
 // One staged list entry as the blend loops read it.
 struct Entry {
   float4 s;            // scaled conic, opacity
@@ -273,20 +285,28 @@ __device__ __forceinline__ void alpha_pair(const Entry& e, float fx0, float fx1,
   ok1 = sg1 >= 0.f && a1 >= op.alpha_min;
 }
 
-// Front-to-back step of one pixel (selects, no branches): a passing entry either ends the
-// pixel (T (1 - alpha) < t_min; it does not contribute) or is blended in.
-__device__ __forceinline__ void blend(PixF& p, float alpha, bool ok, float4 col, const Opts& op) {
-  ok = ok && !p.done;
-  const float test = __fmul_rn(p.T, __fsub_rn(1.f, alpha));
-  const bool term = ok && test < op.t_min;
-  const bool use = ok && !term;
-  const float w = __fmul_rn(alpha, p.T);
-  p.done = p.done || term;
-  p.c0 = use ? __fmaf_rn(w, col.x, p.c0) : p.c0;
-  p.c1 = use ? __fmaf_rn(w, col.y, p.c1) : p.c1;
-  p.c2 = use ? __fmaf_rn(w, col.z, p.c2) : p.c2;
-  p.T = use ? test : p.T;
-  p.last = use ? __float_as_uint(col.w) + 1u : p.last;
+// Front-to-back step of the lane's two pixels for one entry (selects, no branches): a passing
+// entry either ends a pixel (T (1 - alpha) < t_min; it does not contribute) or is blended in.
+// A pixel the entry does not reach gets a zero weight, and fma(0, c, C) leaves C as it was.
+__device__ __forceinline__ void blend2(PixF2& p, float a0, float a1, bool ok0, bool ok1,
+                                       float4 col, const Opts& op) {
+  ok0 = ok0 && !p.done0;
+  ok1 = ok1 && !p.done1;
+  const float2 al = make_float2(a0, a1);
+  const float2 test = __fmul2_rn(p.T, __fadd2_rn(make_float2(1.f, 1.f), make_float2(-a0, -a1)));
+  const bool term0 = ok0 && test.x < op.t_min, term1 = ok1 && test.y < op.t_min;
+  const bool use0 = ok0 && !term0, use1 = ok1 && !term1;
+  const float2 w = __fmul2_rn(al, p.T);
+  const float2 wu = make_float2(use0 ? w.x : 0.f, use1 ? w.y : 0.f);
+  p.done0 = p.done0 || term0;
+  p.done1 = p.done1 || term1;
+  p.c0 = __ffma2_rn(wu, make_float2(col.x, col.x), p.c0);
+  p.c1 = __ffma2_rn(wu, make_float2(col.y, col.y), p.c1);
+  p.c2 = __ffma2_rn(wu, make_float2(col.z, col.z), p.c2);
+  p.T = make_float2(use0 ? test.x : p.T.x, use1 ? test.y : p.T.y);
+  const unsigned nxt = __float_as_uint(col.w) + 1u;
+  p.last0 = use0 ? nxt : p.last0;
+  p.last1 = use1 ? nxt : p.last1;
 }
 
 __device__ __forceinline__ void store_pixel(const FwdArgs& a, long long p, const PixF& s, int qx,
@@ -334,14 +354,18 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
   const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
   const float fx0 = (float)bk.qx0 + 0.5f, fx1 = (float)bk.qx1 + 0.5f, fy = (float)bk.py + 0.5f;
   const float bx0 = (float)bk.px0 + 0.5f, by0 = (float)bk.py0 + 0.5f;
-  PixF p0 = {1.f, 0.f, 0.f, 0.f, 0u, !bk.in0};
-  PixF p1 = {1.f, 0.f, 0.f, 0.f, 0u, !bk.in1};
+  PixF2 pp;
+  pp.T = make_float2(1.f, 1.f);
+  pp.c0 = pp.c1 = pp.c2 = make_float2(0.f, 0.f);
+  pp.last0 = pp.last1 = 0u;
+  pp.done0 = !bk.in0;
+  pp.done1 = !bk.in1;
   int next = 0;
   bool ck_on = a.ckpt != nullptr;          // warp-uniform
   int n_items = 0;
   unsigned my_slot = 0u;                   // lane k: the slot of this block's item k
   while (next < n) {
-    if (__all_sync(0xffffffffu, p0.done && p1.done)) break;
+    if (__all_sync(0xffffffffu, pp.done0 && pp.done1)) break;
     __syncwarp();
     // with checkpoints, a batch ends at the next multiple of kCkChunk
     const int lim = ck_on ? min(n, (next / kCkChunk + 1) * kCkChunk) : n;
@@ -356,13 +380,11 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
       alpha_pair(e0, fx0, fx1, fy, a.op, a00, a01, k00, k01);
       alpha_pair(e1, fx0, fx1, fy, a.op, a10, a11, k10, k11);
       const bool v1 = j + 1 < cnt;
-      blend(p0, a00, k00, e0.col, a.op);
-      blend(p1, a01, k01, e0.col, a.op);
-      blend(p0, a10, k10 && v1, e1.col, a.op);
-      blend(p1, a11, k11 && v1, e1.col, a.op);
-      if ((j & 30) == 30 && __all_sync(0xffffffffu, p0.done && p1.done)) break;
+      blend2(pp, a00, a01, k00, k01, e0.col, a.op);
+      blend2(pp, a10, a11, k10 && v1, k11 && v1, e1.col, a.op);
+      if ((j & 30) == 30 && __all_sync(0xffffffffu, pp.done0 && pp.done1)) break;
     }
-    if (ck_on && next == lim && lim < n && !__all_sync(0xffffffffu, p0.done && p1.done)) {
+    if (ck_on && next == lim && lim < n && !__all_sync(0xffffffffu, pp.done0 && pp.done1)) {
       // the state after every position below lim, for the backward's chunk starting there
       unsigned slot = 0u;
       if (lane == 0) slot = atomicAdd(a.ck_count, 1u);
@@ -370,8 +392,8 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
       if (slot < (unsigned)a.ck_cap) {
         float4* ck = a.ckpt + (size_t)slot * (kSub * kSub);
         const int k0 = block_pixel(lane);
-        ck[k0] = make_float4(p0.c0, p0.c1, p0.c2, p0.T);
-        ck[k0 + 4] = make_float4(p1.c0, p1.c1, p1.c2, p1.T);
+        ck[k0] = make_float4(pp.c0.x, pp.c1.x, pp.c2.x, pp.T.x);
+        ck[k0 + 4] = make_float4(pp.c0.y, pp.c1.y, pp.c2.y, pp.T.y);
         if (lane == n_items) my_slot = slot;
         ++n_items;
       }
@@ -379,6 +401,8 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
       ck_on = slot < (unsigned)a.ck_cap && n_items < 32;
     }
   }
+  const PixF p0 = {pp.T.x, pp.c0.x, pp.c1.x, pp.c2.x, pp.last0, pp.done0};
+  const PixF p1 = {pp.T.y, pp.c0.y, pp.c1.y, pp.c2.y, pp.last1, pp.done1};
   if (a.ckpt) {
     if (lane == 0) a.ck_first[blk] = n_items > 0 ? (unsigned)kCkChunk : 0xffffffffu;
     if (lane < n_items) {
@@ -440,38 +464,62 @@ __device__ __forceinline__ void load_pixel_grad(const BwdArgs& a, long long p, i
   q.K = q.Gr * at.x + q.Gg * at.y + q.Gb * at.z - Ga * at.w;
 }
 
-// Backward of one pixel for one list entry (selects, no branches): when the entry contributed
-// to the pixel (live: a position below the pixel's last contributor; sigma >= 0; alpha >=
-// alpha_min) adds to v the opacity and colour gradients (v[5..8]) and the moments of d =
-// pixel - uv weighted by dL/dsigma, (sum w dx, w dy, w dx^2, w dx dy, w dy^2) in v[0..4] (the
-// conic and mean gradients follow from them once per entry), and advances the replayed
-// transmittance exactly as the forward did.  Returns whether the entry contributed.
-__device__ __forceinline__ bool pixel_backward(PixB& p, float4 s, float4 col, float sg, float dx,
-                                               float dy, bool live, const Opts& op, float* v) {
-  const float G = ex2_approx(-sg);
-  const float raw = __fmul_rn(s.w, G);
-  const float alpha = fminf(op.alpha_max, raw);
-  const bool ok = live && sg >= 0.f && alpha >= op.alpha_min;
-  const float w = __fmul_rn(alpha, p.T);
-  const float gcol = p.Gr * col.x + p.Gg * col.y + p.Gb * col.z;
-  const float gc = fmaf(w, gcol, p.Gc);               // G . C including this entry
-  const float ioma = __fdividef(1.f, 1.f - alpha);   // gradient scale only
-  const float dalpha = p.T * gcol - (p.K - gc) * ioma;
-  const bool grad_a = ok && raw <= op.alpha_max;      // derivative of min() is 0 once clamped
-  const float wk = ok ? w : 0.f;
-  const float dop = grad_a ? dalpha * G : 0.f;        // d alpha / d opacity = exp(-sigma)
-  const float dsig = grad_a ? -dalpha * raw : 0.f;    // d alpha / d sigma = -alpha
-  v[6] = fmaf(p.Gr, wk, v[6]); v[7] = fmaf(p.Gg, wk, v[7]); v[8] = fmaf(p.Gb, wk, v[8]);
-  v[5] += dop;
-  const float t = dsig * dx, u = dsig * dy;
-  v[0] += t;
-  v[1] += u;
-  v[2] = fmaf(t, dx, v[2]);
-  v[3] = fmaf(t, dy, v[3]);
-  v[4] = fmaf(u, dy, v[4]);
-  p.Gc = ok ? gc : p.Gc;
-  p.T = ok ? __fmul_rn(p.T, __fsub_rn(1.f, alpha)) : p.T;
-  return ok;
+// Backward of the lane's two pixels for one list entry (selects, no branches): when the entry
+// contributed to a pixel (live: a position below the pixel's last contributor; sigma >= 0;
+// alpha >= alpha_min) adds to v the opacity and colour gradients (v[5..8]) and the moments of
+// d = pixel - uv weighted by dL/dsigma, (sum w dx, w dy, w dx^2, w dx dy, w dy^2) in v[0..4]
+// (the conic and mean gradients follow from them once per entry), and advances the replayed
+// transmittance exactly as the forward did.  With G = dL/dA.rgb and G_a = dL/dA.a, the
+// derivative of the loss w.r.t. an entry's alpha is
+//   T (G . col) - (K - G . C) / (1 - alpha),   K = G . A - G_a T_final,
+// C the colour accumulated up to and including the entry.  The two pixels' arithmetic is paired through the packed two-lane fp32 instructions and the shared row
+// offset dy factored out of the moment sums (sum t dy = (t0 + t1) dy).  The decisions (alpha,
+// the skip tests, the replayed transmittance) are rounded exactly as the forward rounds them;
+// the gradient terms only round in a different order.  who0 / who1: whether the entry
+// contributed to each pixel.
+struct PixB2 {
+  float2 T, Gc, Gr, Gg, Gb, K;
+};
+
+__device__ __forceinline__ void pixel_backward2(PixB2& p, float4 s, float4 col, float sg0,
+                                                float sg1, float dx0, float dx1, float dy,
+                                                bool live0, bool live1, const Opts& op, float* v,
+                                                bool& who0, bool& who1) {
+  const float2 G = make_float2(ex2_approx(-sg0), ex2_approx(-sg1));
+  const float2 raw = __fmul2_rn(make_float2(s.w, s.w), G);
+  const float a0 = fminf(op.alpha_max, raw.x), a1 = fminf(op.alpha_max, raw.y);
+  const bool ok0 = live0 && sg0 >= 0.f && a0 >= op.alpha_min;
+  const bool ok1 = live1 && sg1 >= 0.f && a1 >= op.alpha_min;
+  const float2 w = __fmul2_rn(make_float2(a0, a1), p.T);
+  const float2 gcol = __ffma2_rn(p.Gb, make_float2(col.z, col.z),
+                                 __ffma2_rn(p.Gg, make_float2(col.y, col.y),
+                                            __fmul2_rn(p.Gr, make_float2(col.x, col.x))));
+  const float2 gc = __ffma2_rn(w, gcol, p.Gc);                     // G . C including the entry
+  const float2 oma = __fadd2_rn(make_float2(1.f, 1.f), make_float2(-a0, -a1));
+  const float2 ioma = make_float2(__fdividef(1.f, oma.x), __fdividef(1.f, oma.y));
+  const float2 km = __fadd2_rn(p.K, make_float2(-gc.x, -gc.y));
+  const float2 dalpha = __ffma2_rn(make_float2(-km.x, -km.y), ioma, __fmul2_rn(p.T, gcol));
+  const bool ga0 = ok0 && raw.x <= op.alpha_max, ga1 = ok1 && raw.y <= op.alpha_max;
+  const float2 dg = __fmul2_rn(dalpha, G);                          // d alpha / d opacity = G
+  const float2 dr = __fmul2_rn(dalpha, raw);                        // d alpha / d sigma = -alpha
+  const float wk0 = ok0 ? w.x : 0.f, wk1 = ok1 ? w.y : 0.f;
+  const float ds0 = ga0 ? -dr.x : 0.f, ds1 = ga1 ? -dr.y : 0.f;
+  v[5] += (ga0 ? dg.x : 0.f) + (ga1 ? dg.y : 0.f);
+  v[6] = fmaf(p.Gr.x, wk0, fmaf(p.Gr.y, wk1, v[6]));
+  v[7] = fmaf(p.Gg.x, wk0, fmaf(p.Gg.y, wk1, v[7]));
+  v[8] = fmaf(p.Gb.x, wk0, fmaf(p.Gb.y, wk1, v[8]));
+  const float2 t = __fmul2_rn(make_float2(ds0, ds1), make_float2(dx0, dx1));
+  const float ts = t.x + t.y, us = (ds0 + ds1) * dy;
+  v[0] += ts;
+  v[1] += us;
+  v[2] = fmaf(t.x, dx0, fmaf(t.y, dx1, v[2]));
+  v[3] = fmaf(ts, dy, v[3]);
+  v[4] = fmaf(us, dy, v[4]);
+  p.Gc = make_float2(ok0 ? gc.x : p.Gc.x, ok1 ? gc.y : p.Gc.y);
+  const float2 Tn = __fmul2_rn(p.T, oma);
+  p.T = make_float2(ok0 ? Tn.x : p.T.x, ok1 ? Tn.y : p.T.y);
+  who0 = ok0;
+  who1 = ok1;
 }
 
 // Warp sum of 27 per-lane values through shared memory: each lane writes its row, lane l < 27
@@ -518,6 +566,14 @@ __device__ __forceinline__ void bwd_chunk(const BwdArgs& a, int blk, int start, 
     p1.T = c1.w; p1.Gc = p1.Gr * c1.x + p1.Gg * c1.y + p1.Gb * c1.z;
   }
   const int span = (int)min((unsigned)__reduce_max_sync(0xffffffffu, max(p0.last, p1.last)), end);
+  PixB2 pp;
+  pp.T = make_float2(p0.T, p1.T);
+  pp.Gc = make_float2(p0.Gc, p1.Gc);
+  pp.Gr = make_float2(p0.Gr, p1.Gr);
+  pp.Gg = make_float2(p0.Gg, p1.Gg);
+  pp.Gb = make_float2(p0.Gb, p1.Gb);
+  pp.K = make_float2(p0.K, p1.K);
+  const unsigned last0 = p0.last, last1 = p1.last;
   int next = start;
   while (next < span) {
     __syncwarp();
@@ -537,8 +593,9 @@ __device__ __forceinline__ void bwd_chunk(const BwdArgs& a, int blk, int start, 
         const bool valid = j + i < cnt;
         float dx0, dx1, dy, sg0, sg1;
         sigma_pair(e.s, e.m, fx0, fx1, fy, dx0, dx1, dy, sg0, sg1);
-        const bool c0 = pixel_backward(p0, e.s, e.col, sg0, dx0, dy, valid && pos < p0.last, a.op, x + 9 * i);
-        const bool c1 = pixel_backward(p1, e.s, e.col, sg1, dx1, dy, valid && pos < p1.last, a.op, x + 9 * i);
+        bool c0, c1;
+        pixel_backward2(pp, e.s, e.col, sg0, sg1, dx0, dx1, dy, valid && pos < last0,
+                        valid && pos < last1, a.op, x + 9 * i, c0, c1);
         who[i] = __ballot_sync(0xffffffffu, c0 || c1);
       }
       if ((who[0] | who[1] | who[2]) == 0) continue;
