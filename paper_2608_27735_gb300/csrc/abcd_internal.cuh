@@ -19,6 +19,8 @@ constexpr int kMaxRadixBlocks = 1024;     // upper bound used to size the histog
 constexpr int kMaxLossBlocks = 1 << 16;
 constexpr int kMaxLayers = 256;
 constexpr long long kMaxDiffCells = 1LL << 20;   // (tiles_x + 1) * (tiles_y + 1)
+constexpr int kMaxRunRows = 1024;     // tile grids that bin through tile-row runs: rows ...
+constexpr int kMaxRunCols = 256;      // ... and columns at most
 constexpr int kVisSumCopies = 8;          // copies of the layer visibility sums
 
 // Device status bits (OR-ed into the status word; abcd_sync reports the lowest set code).
@@ -48,7 +50,9 @@ struct Workspace {
   unsigned long long* os_state;     // [os_tiles][kRadixBins] look-back words
   long long os_tiles;
   int4* rects;                      // [max_g] tile rectangle per Gaussian
-  unsigned* counts;                 // [max_g] listed tiles per Gaussian
+  unsigned* counts;                 // [max_g] listed tiles (or tile-row runs) per Gaussian
+  unsigned* row_runs;               // [kMaxRunRows] tile-row runs per tile row
+  long long* n_runs;                // tile-row runs of the last binning
   int* diff;                        // 2-D difference array over the tile grid
   size_t diff_bytes;
   unsigned long long* block_sums;   // [kMaxRadixBlocks + 1]

@@ -11,19 +11,25 @@
 // How (GB300 design, different from sorting 64-bit (tile | depth) keys):
 //   1. per Gaussian: its tile rectangle (kept in the workspace) and a sort key (fp32 depth
 //      bits, all ones when culled); then, one thread per Gaussian: the contiguous run of kept
-//      tiles in each of its tile rows (the kept set is convex), its pair count, and +-1 at the
-//      run's ends in a per-row difference array over the tile grid (block-local first);
+//      tiles in each of its tile rows (the kept set is convex), its pair (or run) count, and
+//      +-1 at the run's ends in a per-row difference array over the tile grid (block-local
+//      first);
 //   2. stable LSD radix sort of the n Gaussians by the 32 depth bits, on the context's side
 //      stream, while the main stream makes the row runs and then, in one block, the tile
 //      ranges (row prefix sums of the difference array, an exclusive scan, K) and the tiles
 //      ordered by decreasing pair count (the order the render kernels launch them in);
-//   3. exclusive scan of the pair counts in depth order: every Gaussian's output offset;
-//   4. emission of (tile << id_bits | id) items in depth order, 32-bit when tile and id bits
-//      fit (else 64-bit); the runs are recomputed with the same round-to-nearest arithmetic,
-//      so they match step 1 bit for bit; each warp writes its Gaussians' contiguous output in
-//      order, consecutive lanes on consecutive pairs;
-//   5. stable LSD radix sort of the K items on the tile bits only, in passes of equal width,
-//      which keeps depth order inside each tile; the last pass writes ids.
+//   3. exclusive scan of the pair (run) counts in depth order: every Gaussian's output offset;
+//   4. for tile grids up to 256 x 1024 tiles: emission of one item per non-empty (Gaussian,
+//      tile row) run in depth order (row, x0, x1, id; the runs are recomputed with the same
+//      round-to-nearest arithmetic, so they match step 1 bit for bit), a stable LSD radix sort
+//      of the runs on the row bits, and the placement of every run's id in the ranges of the
+//      tiles it covers (per row, chunks of runs count their runs per tile column, add the
+//      counts of the row's earlier chunks by decoupled look-back and write one column per
+//      lane, in run order): no pass over the K pairs but the final write;
+//   5. for larger grids: emission of (tile << id_bits | id) items in depth order, 32-bit when
+//      tile and id bits fit (else 64-bit), each warp writing its Gaussians' contiguous output
+//      in order, then a stable LSD radix sort of the K items on the tile bits only, in passes
+//      of equal width, which keeps depth order inside each tile; the last pass writes ids.
 // Radix sorts are one-sweep: one kernel counts the digits of all passes, then each pass is a
 // single kernel whose CTAs take tiles of items in order and find the offsets of their digits
 // by decoupled look-back over the tiles before theirs (bounded waits on CTAs that are already
@@ -67,10 +73,13 @@ __device__ __forceinline__ int4 tile_rect(float2 m, int r, int tiles_x, int tile
 // rectangle of its square
 __global__ void keys_rects_kernel(const float* depth, const int* radius, const float2* uv, int n,
                                   int tiles_x, int tiles_y, u64* items, int4* rects,
-                                  unsigned* gh_zero, int gh_words) {
+                                  unsigned* gh_zero, int gh_words, unsigned* rows_zero,
+                                  int rows_words) {
   pdl_prologue();
-  if (blockIdx.x == 0)                    // the radix sorts' digit counts start from zero
+  if (blockIdx.x == 0) {                  // the radix sorts' digit counts start from zero
     for (int k = threadIdx.x; k < gh_words; k += blockDim.x) gh_zero[k] = 0u;
+    for (int k = threadIdx.x; k < rows_words; k += blockDim.x) rows_zero[k] = 0u;
+  }
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   int4 q = make_int4(0, 0, 0, 0);
@@ -159,22 +168,27 @@ __device__ __forceinline__ int2 row_run(const Splat& s, int4 q, int ty) {
   return make_int2(xa, xb);
 }
 
-// ---- one thread per Gaussian, looping over its tile rows: the pair count and +1 / -1 at the
-// ends of every row's run in the per-row difference array.  The +-1 go to a block-local copy of
-// the difference array in shared memory first (the same few thousand cells are hit by every
-// block), then only its non-zero cells to the global array.
+// ---- one thread per Gaussian, looping over its tile rows: +1 / -1 at the ends of every row's
+// run in the per-row difference array, and the Gaussian's count: its pairs, or (RUNS) its
+// non-empty row runs, with the runs of every tile row added up in row_runs.  The +-1 go to a
+// block-local copy of the difference array in shared memory first (the same few thousand cells
+// are hit by every block), then only its non-zero cells to the global array.
 constexpr int kSmemDiffCells = 12288;      // 48 KB: tile grids up to ~1900x1500 pixels
 
+template <bool RUNS>
 __global__ void __launch_bounds__(256)
 tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, int tiles_x,
-                 int tiles_y, float alpha_min, unsigned* counts, int* diff) {
+                 int tiles_y, float alpha_min, unsigned* counts, int* diff, unsigned* row_runs) {
   pdl_prologue();
   extern __shared__ int sdiff[];
   const int W1 = tiles_x + 1;
   const int cells = W1 * (tiles_y + 1);
-  const bool local = cells <= kSmemDiffCells;
+  const bool local = cells <= kSmemDiffCells;      // always, with RUNS
+  unsigned* srows = reinterpret_cast<unsigned*>(sdiff + cells);   // RUNS: [tiles_y]
   if (local) {
     for (int k = threadIdx.x; k < cells; k += blockDim.x) sdiff[k] = 0;
+    if (RUNS)
+      for (int k = threadIdx.x; k < tiles_y; k += blockDim.x) srows[k] = 0u;
     __syncthreads();
   }
   int* dst = local ? sdiff : diff;
@@ -187,9 +201,10 @@ tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, i
       for (int ty = q.y; ty < q.w; ++ty) {
         const int2 r = row_run(s, q, ty);
         if (r.y > r.x) {
-          c += (unsigned)(r.y - r.x);
+          c += RUNS ? 1u : (unsigned)(r.y - r.x);
           atomicAdd(&dst[ty * W1 + r.x], 1);
           atomicAdd(&dst[ty * W1 + r.y], -1);
+          if (RUNS) atomicAdd(&srows[ty], 1u);
         }
       }
     }
@@ -201,6 +216,11 @@ tile_rows_kernel(const float2* uv, const float4* co, const int4* rects, int n, i
       const int v = sdiff[k];
       if (v != 0) atomicAdd(&diff[k], v);
     }
+    if (RUNS)
+      for (int k = threadIdx.x; k < tiles_y; k += blockDim.x) {
+        const unsigned v = srows[k];
+        if (v != 0u) atomicAdd(&row_runs[k], v);
+      }
   }
 }
 
@@ -428,9 +448,11 @@ onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long l
     }
     __syncthreads();
     {
-      // look-back: R threads per digit read 8 tiles each, nearest first, per round
+      // look-back: R threads per digit read LB tiles each, nearest first, per round.  At least
+      // 16 tiles per digit and round: when every CTA of a short pass starts at once, the
+      // inclusive prefixes move back along the tiles by that many tiles per round trip.
       constexpr int R = kOsThreads / (int)BINS;
-      constexpr int LB = 4;
+      constexpr int LB = 16 / R > 4 ? 16 / R : 4;
       const unsigned d = threadIdx.x / R;
       const int q = threadIdx.x % R;
       const unsigned gmask = R == 32 ? 0xffffffffu : (((1u << R) - 1u) << (lane & ~(R - 1)));
@@ -519,8 +541,10 @@ count_kernel(const u64* sorted, int n, const unsigned* counts, unsigned long lon
   long long lo, hi;
   block_range(n, G, &lo, &hi);
   unsigned long long s = 0;
-  for (long long i = lo + threadIdx.x; i < hi; i += blockDim.x)
-    s += counts[(unsigned)sorted[i]];
+  for (long long i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+    const unsigned id = (unsigned)sorted[i];
+    if (id < (unsigned)n) s += counts[id];           // (a timed-out sort may leave stale items)
+  }
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   __shared__ unsigned long long ws[8];
   if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = s;
@@ -602,9 +626,12 @@ __device__ __forceinline__ unsigned count_bucket(unsigned c) {
   return (unsigned)(kOrderBuckets - 1 - min(b, kOrderBuckets - 1));
 }
 
+// With row_runs (binning through tile-row runs) the digit counts are those of the runs' row
+// sort, and K goes to k_out (an overflow is flagged in status).
 __global__ void __launch_bounds__(1024)
 ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, long long cap, unsigned* ranges,
-                    unsigned* tile_order, SortPasses tp, unsigned* gh) {
+                    unsigned* tile_order, SortPasses tp, unsigned* gh, const unsigned* row_runs,
+                    long long* k_out, unsigned* status) {
   pdl_prologue();
   extern __shared__ int sd[];              // [(tiles_x + 1) (tiles_y + 1)] cells, then [nt] keys
   __shared__ unsigned hist[kOrderBuckets];
@@ -656,8 +683,16 @@ ranges_order_kernel(const int* diff, int tiles_x, int tiles_y, long long cap, un
     ranges[2 * t] = ok ? (unsigned)run : 0u;
     ranges[2 * t + 1] = ok ? (unsigned)(run + c) : 0u;
     skey[t] = (unsigned char)count_bucket(ok ? c : 0u);
-    tile_digit_counts((unsigned)t, c, tp, dh);
+    if (!row_runs) tile_digit_counts((unsigned)t, c, tp, dh);
     run += c;
+  }
+  if (row_runs) {
+    for (int y = threadIdx.x; y < tiles_y; y += blockDim.x)
+      tile_digit_counts((unsigned)y, row_runs[y], tp, dh);
+    if (threadIdx.x == 0) {
+      *k_out = (long long)total;
+      if (!ok) atomicOr(status, kStatusCapacity);
+    }
   }
   __syncthreads();
   for (int k = threadIdx.x; k < tp.n * kRadixBins; k += blockDim.x) gh[k] = (&dh[0][0])[k];
@@ -747,7 +782,7 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
     Splat sm_ = {};
     if (i < hi) {
       id = (unsigned)sorted[i];
-      t = counts[id];
+      t = id < (unsigned)n ? counts[id] : 0u;
       if (t > 0) { qm = rects[id]; sm_ = load_splat(uv, co, id, alpha_min); }
     }
     unsigned long long tot = 0;
@@ -794,6 +829,252 @@ emit_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const 
       done += total;
     }
     __syncthreads();                                 // s_sp, s_q, s_id are refilled next round
+  }
+}
+
+// ---- binning through tile-row runs (tile grids up to kMaxRunCols x kMaxRunRows).  Each
+// Gaussian's kept tiles in a tile row form one run [x0, x1) (the kept set is convex), so instead
+// of emitting every (tile, Gaussian) pair and sorting the pairs by tile, the runs (about a
+// seventh as many) are emitted in depth order, sorted stably by row, and each run's Gaussian
+// is written straight into the tiles' ranges: within a row, the pairs of tile column x come
+// from the row's runs that cover x, in order, so the position of a run's entry in column x is
+// the column's range start + the runs before it in the row that cover x.  The row's runs are
+// cut into chunks of kPlaceRuns; a chunk counts its runs per column (a difference array),
+// adds the counts of the row's earlier chunks by decoupled look-back over the columns, and
+// writes its entries one column per lane.
+
+// Run item: row (16 bits) | x0 (8) | x1 - 1 (8) | Gaussian id (32).
+constexpr int kRunRowShift = 48;
+
+__device__ __forceinline__ u64 run_item(int ty, int2 r, unsigned id) {
+  return ((u64)ty << kRunRowShift) | ((u64)r.x << 40) | ((u64)(r.y - 1) << 32) | id;
+}
+
+// The same traversal as emit_kernel, one item per non-empty (Gaussian, tile row) run, in depth
+// order then row order; run offsets from the scan of the per-Gaussian run counts.
+__global__ void __launch_bounds__(kEmitThreads)
+emit_runs_kernel(const u64* sorted, int n, const float2* uv, const float4* co, const int4* rects,
+                 const unsigned* counts, const unsigned long long* block_off, const long long* K,
+                 long long cap, float alpha_min, u64* runs, int G) {
+  pdl_prologue();
+  __shared__ Splat s_sp[kEmitThreads];
+  __shared__ int4 s_q[kEmitThreads];
+  __shared__ unsigned s_id[kEmitThreads];
+  if (*K > cap) return;
+  long long lo, hi;
+  block_range(n, G, &lo, &hi);
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const unsigned lt = (1u << lane) - 1u;
+  unsigned long long run = block_off[blockIdx.x];
+  for (long long base = lo; base < hi; base += blockDim.x) {
+    const long long i = base + threadIdx.x;
+    unsigned id = 0, t = 0;
+    int4 qm = make_int4(0, 0, 0, 0);
+    Splat sm_ = {};
+    if (i < hi) {
+      id = (unsigned)sorted[i];
+      t = id < (unsigned)n ? counts[id] : 0u;
+      if (t > 0) { qm = rects[id]; sm_ = load_splat(uv, co, id, alpha_min); }
+    }
+    unsigned long long tot = 0;
+    const unsigned long long off = run + block_exclusive_scan(t, &tot);
+    run += tot;
+    s_sp[threadIdx.x] = sm_;
+    s_q[threadIdx.x] = qm;
+    s_id[threadIdx.x] = id;
+    const unsigned long long off0 = __shfl_sync(0xffffffffu, off, 0);   // the warp's first run
+    const unsigned rows = t > 0 ? (unsigned)(qm.w - qm.y) : 0u;
+    const unsigned rincl = warp_inclusive_scan(rows, lane);
+    const unsigned P = __shfl_sync(0xffffffffu, rincl, 31);
+    __syncwarp();
+    unsigned long long at = off0;
+    for (unsigned p0 = 0; p0 < P; p0 += 32) {
+      const unsigned pr = p0 + lane;                 // this lane's (Gaussian, row) pair
+      const int j = scan_search(rincl, pr);
+      const unsigned jfirst = __shfl_sync(0xffffffffu, rincl - rows, j);
+      int2 r = make_int2(0, 0);
+      int ty = 0;
+      unsigned idj = 0;
+      if (pr < P) {
+        const int slot = w * 32 + j;
+        const int4 q = s_q[slot];
+        ty = q.y + (int)(pr - jfirst);
+        r = row_run(s_sp[slot], q, ty);
+        idj = s_id[slot];
+      }
+      const bool ne = r.y > r.x;
+      const unsigned b = __ballot_sync(0xffffffffu, ne);
+      const unsigned long long dst = at + __popc(b & lt);
+      if (ne && dst < (unsigned long long)cap) runs[dst] = run_item(ty, r, idj);
+      at += __popc(b);
+    }
+    __syncthreads();                                 // s_sp, s_q, s_id are refilled next round
+  }
+}
+
+constexpr int kPlaceThreads = 128;
+constexpr int kPlaceRuns = 512;                      // runs per chunk: 4 per thread
+constexpr int kPlaceWords = kPlaceRuns / 32;         // words of a column's run mask
+constexpr int kPlacePitch = kPlaceWords + 1;         // odd pitch: a column per thread, no conflicts
+constexpr int kPlaceLB = 8;                          // look-back words read per column and round
+static_assert(kMaxRunRows % kPlaceThreads == 0 && kPlaceRuns % kPlaceThreads == 0, "tiling");
+
+// Runs sorted by row (depth order inside a row) -> ids in the tile ranges.  row_runs: runs per
+// row; chunks are claimed in order through ctr (the last CTA clears it); state: tiles_x look-back
+// words per chunk.  Inside a chunk, column x keeps a bit mask of the runs that cover it and the
+// number of covering runs before each mask word, so the rank of run j in column x is a
+// popcount.  A wait gives up after spin_limit polls (status gets ABCD_ERR_TIMEOUT).
+__global__ void __launch_bounds__(kPlaceThreads)
+place_kernel(const u64* runs, const long long* n_runs, long long cap, const unsigned* row_runs,
+             int rows, int tiles_x, const unsigned* ranges, const long long* K, unsigned* ids,
+             u64* state, unsigned* ctr, unsigned epoch, unsigned* status, unsigned spin_limit) {
+  pdl_prologue();
+  __shared__ unsigned s_rs[kMaxRunRows + 1];         // first run of each row
+  __shared__ unsigned s_cs[kMaxRunRows + 1];         // first chunk of each row
+  __shared__ unsigned s_mask[kMaxRunCols * kPlacePitch];          // [column][word]
+  __shared__ unsigned short s_pc[kMaxRunCols * kPlacePitch];      // covering runs before a word
+  __shared__ unsigned s_cnt[kMaxRunCols];            // the chunk's runs per column
+  __shared__ unsigned s_base[kMaxRunCols];           // where the chunk's entries of a column start
+  __shared__ unsigned s_c, s_row;
+  if (*K > cap) return;                              // the ranges are empty: nothing to place
+  const long long nr = dev_count(0, n_runs, cap);
+  {
+    constexpr int PER = kMaxRunRows / kPlaceThreads;
+    unsigned a[PER], b[PER], sa = 0, sb = 0;
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+      const int y = threadIdx.x * PER + k;
+      a[k] = y < rows ? row_runs[y] : 0u;
+      b[k] = (a[k] + kPlaceRuns - 1) / kPlaceRuns;
+      sa += a[k];
+      sb += b[k];
+    }
+    unsigned long long ta = 0, tb = 0;
+    unsigned long long ea = block_exclusive_scan(sa, &ta);
+    unsigned long long eb = block_exclusive_scan(sb, &tb);
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+      const int y = threadIdx.x * PER + k;
+      if (y < rows) { s_rs[y] = (unsigned)ea; s_cs[y] = (unsigned)eb; }
+      ea += a[k];
+      eb += b[k];
+    }
+    if (threadIdx.x == 0) { s_rs[rows] = (unsigned)ta; s_cs[rows] = (unsigned)tb; }
+  }
+  __syncthreads();
+  const unsigned n_chunks = s_cs[rows];
+  for (;;) {
+    if (threadIdx.x == 0) {
+      const unsigned c = atomicAdd(ctr, 1u);
+      unsigned y = 0;
+      if (c < n_chunks) {                            // the row with s_cs[y] <= c < s_cs[y + 1]
+        int lo = 0, hi = rows;
+        while (hi - lo > 1) {
+          const int mid = (lo + hi) >> 1;
+          if (s_cs[mid] <= c) lo = mid; else hi = mid;
+        }
+        y = (unsigned)lo;
+      }
+      s_c = c;
+      s_row = y;
+    }
+    for (int k = threadIdx.x; k < tiles_x * kPlacePitch; k += kPlaceThreads) s_mask[k] = 0u;
+    __syncthreads();
+    const unsigned c = s_c;
+    if (c >= n_chunks) break;                        // block-uniform
+    const int ty = (int)s_row;
+    const unsigned c0 = s_cs[ty], k = c - c0;
+    const unsigned r0 = s_rs[ty] + k * kPlaceRuns;
+    const unsigned r1 = min(s_rs[ty + 1], r0 + (unsigned)kPlaceRuns);
+    // this thread's runs j = threadIdx.x + 128 q, kept in registers for the placement
+    unsigned rx0[kPlaceRuns / kPlaceThreads], rxm[kPlaceRuns / kPlaceThreads];
+    unsigned rid[kPlaceRuns / kPlaceThreads];
+#pragma unroll
+    for (int q = 0; q < kPlaceRuns / kPlaceThreads; ++q) {
+      const int j = threadIdx.x + q * kPlaceThreads;
+      rx0[q] = 1u;
+      rxm[q] = 0u;                                   // empty
+      rid[q] = 0u;
+      if (r0 + j < r1 && (long long)(r0 + j) < nr) {
+        const u64 v = runs[r0 + j];
+        rx0[q] = (unsigned)(v >> 40) & 255u;
+        rxm[q] = min((unsigned)(v >> 32) & 255u, (unsigned)tiles_x - 1u);
+        rid[q] = (unsigned)v;
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kPlaceRuns / kPlaceThreads; ++q) {
+      const int j = threadIdx.x + q * kPlaceThreads;
+      const unsigned bit = 1u << (j & 31);
+      for (unsigned x = rx0[q]; x <= rxm[q]; ++x) atomicOr(&s_mask[x * kPlacePitch + (j >> 5)], bit);
+    }
+    __syncthreads();
+    // per column: covering runs before each word, and in all
+    for (int x = threadIdx.x; x < tiles_x; x += kPlaceThreads) {
+      unsigned run = 0;
+#pragma unroll
+      for (int w = 0; w < kPlaceWords; ++w) {
+        s_pc[x * kPlacePitch + w] = (unsigned short)run;
+        run += __popc(s_mask[x * kPlacePitch + w]);
+      }
+      s_cnt[x] = run;
+    }
+    // publish the chunk's counts (the row's first chunk: as inclusive prefixes) ...
+    for (int x = threadIdx.x; x < tiles_x; x += kPlaceThreads)
+      os_publish(state + (size_t)c * tiles_x + x, os_word(epoch, k == 0 ? 2u : 1u, s_cnt[x]));
+    // ... then add up the row's earlier chunks per column, nearest first
+    for (int x = threadIdx.x; x < tiles_x; x += kPlaceThreads) {
+      unsigned prefix = 0;
+      if (k > 0) {
+        long long j0 = (long long)c - 1;             // nearest chunk not summed yet
+        unsigned spins = 0;
+        for (;;) {
+          u64 v[kPlaceLB];
+#pragma unroll
+          for (int q = 0; q < kPlaceLB; ++q) {
+            const long long idx = j0 - q;
+            v[q] = idx >= (long long)c0 ? os_peek(state + (size_t)idx * tiles_x + x)
+                                        : os_word(epoch, 2u, 0u);
+          }
+          unsigned sum = 0;
+          int used = kPlaceLB, kind = 0;             // 0: all aggregates, 1: inclusive, 2: blocked
+#pragma unroll
+          for (int q = 0; q < kPlaceLB; ++q) {
+            if (kind != 0) continue;
+            const unsigned flag = (unsigned)(v[q] >> 32) & 3u;
+            if ((unsigned)(v[q] >> 34) != epoch || flag == 0u) { kind = 2; used = q; continue; }
+            sum += (unsigned)v[q];
+            if (flag == 2u) { kind = 1; used = q + 1; }
+          }
+          prefix += sum;
+          j0 -= used;
+          if (kind == 1) break;
+          if (kind == 2) {
+            if (++spins > spin_limit) { atomicOr(status, kStatusTimeout); break; }
+            __nanosleep(32);
+          }
+        }
+        os_publish(state + (size_t)c * tiles_x + x, os_word(epoch, 2u, prefix + s_cnt[x]));
+      }
+      s_base[x] = ranges[2 * (ty * tiles_x + x)] + prefix;
+    }
+    __syncthreads();
+    // entries: run j in column x goes to base(x) + the runs before j that cover x
+#pragma unroll
+    for (int q = 0; q < kPlaceRuns / kPlaceThreads; ++q) {
+      const int j = threadIdx.x + q * kPlaceThreads;
+      const unsigned below = (1u << (j & 31)) - 1u;
+      for (unsigned x = rx0[q]; x <= rxm[q]; ++x) {
+        const int at = (int)x * kPlacePitch + (j >> 5);
+        const unsigned pos = s_base[x] + s_pc[at] + __popc(s_mask[at] & below);
+        if ((long long)pos < cap) ids[pos] = rid[q];
+      }
+    }
+    __syncthreads();                                 // before the next chunk reuses the arrays
+  }
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(ctr + 1, 1u) == gridDim.x - 1) { ctr[0] = 0u; ctr[1] = 0u; }
   }
 }
 
@@ -914,14 +1195,25 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   const float alpha_min = make_opts(opts).alpha_min;
   int tile_bits = 1;
   while ((1LL << tile_bits) < n_tiles) ++tile_bits;
-  // digit counts of the tile sort's passes, made with the tile ranges
-  const SortPasses tile_passes = make_passes(0, tile_bits);
+  int row_bits = 1;
+  while ((1 << row_bits) < tiles_y) ++row_bits;
+  const int cells = (tiles_x + 1) * (tiles_y + 1);
+  // tile grids up to kMaxRunCols x kMaxRunRows bin through tile-row runs (the run placement's
+  // look-back words must fit the workspace); larger ones sort (tile, Gaussian) pairs
+  const long long max_chunks = cap / kPlaceRuns + tiles_y + 1;
+  const bool by_runs = tiles_x <= kMaxRunCols && tiles_y <= kMaxRunRows &&
+                       cells <= kSmemDiffCells && n_tiles <= ctx->ws.max_tiles &&
+                       max_chunks * tiles_x <= ctx->ws.os_tiles * kRadixBins;
+  // digit counts of the tile sort's passes (or of the runs' row sort), made with the ranges;
+  // the passes count from the tile (row) bits' lowest, the sorts' own from the items' field
+  const SortPasses tile_passes = make_passes(0, by_runs ? row_bits : tile_bits);
   unsigned* tile_gh = ctx->ws.os_gh + 4 * kRadixBins;
   if ((s = check_launch(ctx, "keys_rects_kernel",
                         launch_pdl(keys_rects_kernel, dim3((n + 255) / 256), dim3(256), 0, ctx->stream,
                                    (const float*)proj->depth, (const int*)proj->radius,
                                    (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
-                                   ctx->ws.rects, ctx->ws.os_gh, 2 * 4 * kRadixBins))))
+                                   ctx->ws.rects, ctx->ws.os_gh, 2 * 4 * kRadixBins,
+                                   ctx->ws.row_runs, by_runs ? tiles_y : 0))))
     return s;
   // the depth sort only needs the keys: it runs on the side stream while the tile rows and
   // ranges are made here
@@ -935,21 +1227,23 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   e = cudaEventRecord(ctx->ev_join, ctx->side);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
   {
-    const int cells = (tiles_x + 1) * (tiles_y + 1);
-    const size_t smem = cells <= kSmemDiffCells ? sizeof(int) * cells : 0;
+    const size_t smem = cells <= kSmemDiffCells
+                            ? sizeof(int) * cells + (by_runs ? sizeof(unsigned) * tiles_y : 0)
+                            : 0;
+    auto kern = by_runs ? tile_rows_kernel<true> : tile_rows_kernel<false>;
     {
-      const cudaError_t e2 = ensure_smem(ctx, (const void*)tile_rows_kernel, smem);
+      const cudaError_t e2 = ensure_smem(ctx, (const void*)kern, smem);
       if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile_rows smem: %s", cudaGetErrorString(e2));
     }
     if ((s = check_launch(ctx, "tile_rows_kernel",
-                          launch_pdl(tile_rows_kernel, dim3((n + 255) / 256), dim3(256), smem,
+                          launch_pdl(kern, dim3((n + 255) / 256), dim3(256), smem,
                                      ctx->stream, (const float2*)proj->uv,
                                      (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
-                                     n, tiles_x, tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff))))
+                                     n, tiles_x, tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff,
+                                     ctx->ws.row_runs))))
       return s;
   }
   {
-    const int cells = (tiles_x + 1) * (tiles_y + 1);
     ctx->order_ranges = nullptr;
     if (cells <= kSmemDiffCells && n_tiles <= ctx->ws.max_tiles) {
       const size_t smem = sizeof(int) * cells + (size_t)n_tiles;
@@ -960,7 +1254,9 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       if ((s = check_launch(ctx, "ranges_order_kernel",
                             launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->stream,
                                        (const int*)ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges,
-                                       ctx->ws.tile_order, tile_passes, tile_gh))))
+                                       ctx->ws.tile_order, tile_passes, tile_gh,
+                                       by_runs ? (const unsigned*)ctx->ws.row_runs : nullptr,
+                                       by_runs ? (long long*)out->count : nullptr, ctx->ws.status))))
         return s;
       ctx->order_ranges = out->ranges;           // the order belongs to these ranges
       ctx->order_tiles = n_tiles;
@@ -982,8 +1278,35 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
     return s;
   if ((s = check_launch(ctx, "scan_blocks_kernel",
                         launch_pdl(scan_blocks_kernel, dim3(1), dim3(1024), 0, ctx->stream,
-                                   ctx->ws.block_sums, Ge, out->count, cap, ctx->ws.status))))
+                                   ctx->ws.block_sums, Ge,
+                                   by_runs ? ctx->ws.n_runs : (long long*)out->count, cap,
+                                   ctx->ws.status))))
     return s;
+  if (by_runs) {
+    u64* runs = ctx->ws.pairs[0];
+    if ((s = check_launch(ctx, "emit_runs_kernel",
+                          launch_pdl(emit_runs_kernel, dim3(Ge), dim3(kEmitThreads), 0, ctx->stream,
+                                     (const u64*)by_depth, n, (const float2*)proj->uv,
+                                     (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
+                                     (const unsigned*)ctx->ws.counts,
+                                     (const unsigned long long*)ctx->ws.block_sums,
+                                     (const long long*)out->count, cap, alpha_min, runs, Ge))))
+      return s;
+    u64* by_row = nullptr;
+    if ((s = radix_sort<u64>(ctx, ctx->stream, runs, ctx->ws.pairs[1], 0, ctx->ws.n_runs, cap, cap,
+                             kRunRowShift, kRunRowShift + row_bits, 1, true, &by_row, nullptr,
+                             0xffffffffu, 1)))
+      return s;
+    const unsigned epoch = ++ctx->os_epoch;
+    const int Gp = (int)std::max<long long>(1, std::min<long long>(max_chunks, 8LL * ctx->num_sms));
+    return check_launch(ctx, "place_kernel",
+                        launch_pdl(place_kernel, dim3(Gp), dim3(kPlaceThreads), 0, ctx->stream,
+                                   (const u64*)by_row, (const long long*)ctx->ws.n_runs, cap,
+                                   (const unsigned*)ctx->ws.row_runs, tiles_y, tiles_x,
+                                   (const unsigned*)out->ranges, (const long long*)out->count,
+                                   (unsigned*)out->ids, ctx->ws.os_state, ctx->ws.os_ctr + 4, epoch,
+                                   ctx->ws.status, ctx->wait_limit));
+  }
   int id_bits = 1;
   while ((1LL << id_bits) < n) ++id_bits;
   // K lives on the device: the tile passes take the largest grid; blocks past K exit at once.

@@ -163,11 +163,15 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.pairs[1] = (unsigned long long*)take(8ull * (size_t)max_pairs);
   w.os_gh = (unsigned*)take(4ull * 2 * 4 * kRadixBins);
   w.os_ctr = (unsigned*)take(256);
-  // sort tiles hold 2048 32-bit or 1024 64-bit items
-  w.os_tiles = (std::max<long long>(max_pairs, max_g) + 1023) / 1024 + 1;
+  // look-back words: a sort tile holds at least 1024 items; the run placement publishes one
+  // word per tile column for each chunk of 512 runs (runs <= pairs) and row
+  w.os_tiles = std::max<long long>((std::max<long long>(max_pairs, max_g) + 1023) / 1024,
+                                   (max_pairs + 511) / 512 + kMaxRunRows) + 1;
   w.os_state = (unsigned long long*)take(8ull * kRadixBins * (size_t)w.os_tiles);
   w.rects = (int4*)take(16ull * (size_t)max_g);
   w.counts = (unsigned*)take(4ull * (size_t)max_g);
+  w.row_runs = (unsigned*)take(4ull * kMaxRunRows);
+  w.n_runs = (long long*)take(8);
   w.diff_bytes = 4ull * kMaxDiffCells;
   w.diff = (int*)take(w.diff_bytes);
   w.block_sums = (unsigned long long*)take(8ull * (kMaxRadixBlocks + 1));

@@ -239,6 +239,8 @@ struct FwdArgs {
   unsigned* ck_count;
   unsigned* ck_first;
   int ck_cap;
+  const unsigned* status;       // the context's status word: after a timed-out wait the lists
+                                // may hold stale ids, so every list reads as empty
 };
 
 // Blend state of one pixel.
@@ -351,7 +353,7 @@ __global__ void __launch_bounds__(kSubThreads) render_fwd_kernel(FwdArgs a) {
   const Block bk = block_of(a.cam, blk);
   const int lane = threadIdx.x & 31;
   const uint2 rg = a.ranges[bk.tile];
-  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
+  const int n = (rg.y > rg.x && !(*a.status & kStatusTimeout)) ? (int)(rg.y - rg.x) : 0;
   const float fx0 = (float)bk.qx0 + 0.5f, fx1 = (float)bk.qx1 + 0.5f, fy = (float)bk.py + 0.5f;
   const float bx0 = (float)bk.px0 + 0.5f, by0 = (float)bk.py0 + 0.5f;
   PixF2 pp;
@@ -437,6 +439,7 @@ struct BwdArgs {
   const unsigned* ck_first;
   int ck_cap;
   int n_item_ctas;              // the first CTAs of the launch replay the listed chunks
+  const unsigned* status;       // as in FwdArgs
 };
 
 // Backward state of one pixel.  With G = dL/dA.rgb and G_a = dL/dA.a, the derivative of the
@@ -552,7 +555,7 @@ __device__ __forceinline__ void bwd_chunk(const BwdArgs& a, int blk, int start, 
   const Block bk = block_of(a.cam, blk);
   const int lane = threadIdx.x & 31;
   const uint2 rg = a.ranges[bk.tile];
-  const int n = rg.y > rg.x ? (int)(rg.y - rg.x) : 0;
+  const int n = (rg.y > rg.x && !(*a.status & kStatusTimeout)) ? (int)(rg.y - rg.x) : 0;
   const float fx0 = (float)bk.qx0 + 0.5f, fx1 = (float)bk.qx1 + 0.5f, fy = (float)bk.py + 0.5f;
   const float bx0 = (float)bk.px0 + 0.5f, by0 = (float)bk.py0 + 0.5f;
   PixB p0 = {}, p1 = {};
@@ -696,6 +699,7 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   if (((uintptr_t)out_rgba & 15) || ((uintptr_t)refresh_f16 & 7))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_composite_fwd: misaligned output");
   FwdArgs a;
+  a.status = ctx->ws.status;
   a.cam = make_cam(cam, opts);
   a.op = make_opts(opts);
   a.uv = (const float2*)proj->uv;
@@ -747,6 +751,7 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   cudaError_t e = cudaMemsetAsync(grad2d, 0, sizeof(float) * 9 * (size_t)n, ctx->stream);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "grad2d memset: %s", cudaGetErrorString(e));
   BwdArgs a;
+  a.status = ctx->ws.status;
   a.cam = make_cam(cam, opts);
   a.op = make_opts(opts);
   a.uv = (const float2*)proj->uv;
@@ -834,6 +839,7 @@ extern "C" abcd_status abcd_render_refresh_packed(abcd_ctx* ctx, const abcd_came
   if (!tile_map || !packed || !count || ((uintptr_t)packed & 15) || ((uintptr_t)tile_map & 3))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_refresh_packed: bad or misaligned output");
   FwdArgs a;
+  a.status = ctx->ws.status;
   a.cam = make_cam(cam, opts);
   a.op = make_opts(opts);
   a.uv = (const float2*)proj->uv;

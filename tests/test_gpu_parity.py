@@ -179,22 +179,26 @@ def test_bin_sort_many_gaussians(ctx):
     par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
 
 
-def test_bin_sort_wide_image(ctx):
-    """A wide tile grid (4096x640: 10,240 tiles, 14 tile bits: the tile sort's passes take 7
-    bits each) with 3,000 Gaussians: the lists equal the oracle's."""
+@pytest.mark.parametrize("W,H", [(4096, 640), (4200, 96), (64, 4200)])
+def test_bin_sort_wide_image(ctx, W, H):
+    """Large tile grids with 3,000 Gaussians; the lists equal the oracle's.  4096x640: 256 tile
+    columns, the most that bin through tile-row runs; 4200x96: 263 columns, binned through
+    sorted (tile, Gaussian) pairs (11 tile bits: passes of 6 and 5 bits); 64x4200: 263 tile
+    rows, the runs sorted by row in two passes (5 and 4 bits)."""
     s = sg.grid_scene((1, 1, 1), 5.0, 3000, 0, seed=95)
-    s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 4096, 640, seed=95,
+    s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), W, H, seed=95,
                                 height_jitter=1.0)
+    ctx.reserve(3000, 2_000_000, W * H)
     case = Case(s, 0, fb=False)
     r = run_forward(ctx, case, want_state=False)
     K = int(r["tiles"].count.item())
     rng = r["tiles"].ranges.cpu().numpy().astype(np.int64)
     ids = r["tiles"].ids.cpu().numpy()[:K]
     tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
-    assert tx * ty == 10240
+    assert tx * ty == ((W + 15) // 16) * ((H + 15) // 16)
     par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
     n_opt, share = par.optional_share(case.opt_list, K)
-    print(f"wide image: K = {K}, optional entries {n_opt} ({share:.2e} of K)")
+    print(f"{W}x{H}: K = {K}, optional entries {n_opt} ({share:.2e} of K)")
 
 
 @pytest.mark.parametrize("cam_idx,bg,fbdt", [(0, None, "f16"), (1, (0.2, 0.5, 0.9), "f16"),
@@ -777,7 +781,8 @@ def test_bin_sort_wait_timeout_reported(ctx):
     """The radix sort's look-back waits are bounded: with tile 0 of the depth sort's first pass
     withheld (a test hook: it publishes nothing) and a short wait limit, the tiles behind it give
     up, abcd_sync reports ABCD_ERR_TIMEOUT and the call returns; once the status is cleared the
-    same context sorts correctly again."""
+    same context sorts correctly again.  A render queued behind the timed-out sort reads every
+    list as empty (the lists may hold stale ids): its image is the empty one."""
     s = sg.grid_scene((1, 1, 1), 5.0, 6000, 0, seed=97)
     s.cameras = sg.ring_cameras(1, 1.5 * sg.half_diagonal(s.grid), np.zeros(3), 96, 64, seed=97)
     g = s.gaussians
@@ -796,9 +801,14 @@ def test_bin_sort_wait_timeout_reported(ctx):
     assert L.abcd_set_wait_limit(ctx.h, 256) == ab.ABCD_OK
     assert L.abcd_test_withhold_lookback(ctx.h, 0) == ab.ABCD_OK
     ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
+    H, W = s.cameras[0].height, s.cameras[0].width
+    out = torch.full((H, W, 4), 7.0, device="cuda")
+    ab.abcd_render_composite_fwd(ctx, cam, None, proj, tiles, None, None, ab.ABCD_F16, None, out,
+                                 None)
     with pytest.raises(ab.AbcdError) as ei:
         ctx.sync()
     assert ei.value.status == ab.ABCD_ERR_TIMEOUT
+    assert torch.count_nonzero(out).item() == 0
     ctx.clear_status()
     assert L.abcd_set_wait_limit(ctx.h, 1 << 20) == ab.ABCD_OK
     ab.abcd_bin_sort(ctx, proj, theta.n, cam, tiles)
