@@ -236,6 +236,7 @@ class Stage:
         self.vis_pairs = ab.visible_pairs(self.ctx, {p: ths[p] for p in range(P)}, scene.cameras,
                                           grid.dims, grid.origin, grid.side)
         self.observing = [ci for ci in range(C) if self.vis_pairs[ci, a]]
+        self.runs_mean = self.count_runs(self.theta, 4)
         log(f"[bench] visible camera-partition pairs {int(self.vis_pairs.sum())} of {C * P}; "
             f"{len(self.observing)} cameras observe the active partition")
         tmp = torch.empty(P, self.n_t, 16, 16, 4, dtype=torch.float16, device=device)
@@ -331,6 +332,23 @@ class Stage:
             self.gt[ci].copy_(full[..., :3])
         self.ctx.sync()
         self.tgt_dev = None
+
+    def count_runs(self, th, n_cams):
+        """Mean number of (Gaussian, tile row) runs of the active block over a few observing
+        cameras: the distinct ids of each tile row's lists (one run per Gaussian and row)."""
+        ab = self.ab
+        tx, ty = (self.W + 15) // 16, (self.H + 15) // 16
+        out = []
+        for ci in list(self.observing)[:n_cams]:
+            ab.abcd_project(self.ctx, th, self.cams[ci], None, self.proj)
+            ab.abcd_bin_sort(self.ctx, self.proj, th.n, self.cams[ci], self.tiles)
+            self.ctx.sync()
+            K = int(self.tiles.count.item())
+            rg = self.tiles.ranges[:tx * ty].cpu().numpy().astype(np.int64)
+            ids = self.tiles.ids[:K].cpu().numpy()
+            out.append(sum(len(np.unique(ids[rg[y * tx, 0]:rg[y * tx + tx - 1, 1]]))
+                           for y in range(ty)))
+        return float(np.mean(out)) if out else 0.0
 
     # ---- timing helpers
     def _mark(self, name, sampled, fn, *a, **k):
@@ -464,9 +482,13 @@ def algorithmic(st: Stage, name, avg_ms, pairs_mean):
     if name == "project_bwd":
         return "hbm", (2 * P + 36) * n / (avg_ms * 1e-3) / 1e9, "GB/s"
     if name == "bin_sort":
-        K = st.k_mean
-        byts = 20 * n + 4 * 24 * n + 8 * K + 2 * 24 * K + 12 * K
-        return "hbm", byts / (avg_ms * 1e-3) / 1e9, "GB/s"
+        # keys and rectangles 20 B per Gaussian, four depth passes over 8-B items (16 B each);
+        # runs: 8 B emitted, one row pass (16 B), 8 B read and a 4-B id written per pair by
+        # the placement.  The working set stays in L2 and the passes are latency-bound, so the
+        # HBM copy rate is a yardstick here, not the bound.
+        K, R = st.k_mean, st.runs_mean
+        byts = 20 * n + 4 * 16 * n + 8 * R + 16 * R + 8 * R + 4 * K
+        return "latency", byts / (avg_ms * 1e-3) / 1e9, "GB/s"
     return None
 
 
@@ -593,7 +615,9 @@ def run_ours(args):
         if r is None:
             return None
         bound, achieved, unit = r
-        peak, note = (hbm_peak, hbm_note) if bound == "hbm" else (alu["fp32_tflops"], alu_note)
+        peak, note = ((hbm_peak, hbm_note) if bound == "hbm" else
+                      (hbm_peak, "HBM copy rate as a yardstick: " + hbm_note) if bound == "latency"
+                      else (alu["fp32_tflops"], alu_note))
         return dict(bound=bound, achieved=round(achieved, 3), peak=round(peak, 1), unit=unit,
                     frac=round(achieved / peak, 4), peak_source=note)
 
@@ -645,6 +669,7 @@ def run_ours(args):
         "data": "synthetic (seeded scenegen, shaped like the paper's 200-camera grid scenes)",
         "config": stage_config(args, st.n, world),
         "pairs_mean": round(st.k_mean),
+        "runs_mean": round(st.runs_mean),
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
