@@ -332,8 +332,8 @@ abcd_status abcd_layer_visibility_packed(abcd_ctx* ctx, const int* const* tile_m
  * for those callers.  Same arguments and results as abcd_loss, with an explicit stream.
  * Its scratch (per-CTA partial sums and a completion counter, about 512 KB) is a static
  * device array of this library, held by every GPU that loads the library until the process
- * exits; images may have at most 65536 CTAs, one per channel of a 64x28-pixel tile (e.g.
- * 8192 x 4096), larger ones return ABCD_ERR_WORKSPACE.  The first call on a device (made with
+ * exits; images may have at most 8192 x 4096 pixels (and 65536 CTAs, one per channel of a
+ * 64x28-pixel tile), larger ones return ABCD_ERR_WORKSPACE before any launch.  The first call on a device (made with
  * that device current) loads the library's device code there and looks up the array's
  * address, so make it before any stream capture; later calls look the address up again (a
  * host-side table read), so a device reset never leaves a stale address.  All calls on a device share

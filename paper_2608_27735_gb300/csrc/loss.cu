@@ -351,6 +351,7 @@ namespace abcd {
 namespace {
 
 constexpr int kStaticLossMaxBlocks = 65536;            // CTAs (64x28 pixels, one channel): 8192 x 4096
+constexpr long long kStaticLossMaxPixels = 8192LL * 4096;   // the image size the header states
 constexpr int kStaticLossWords = 2 * kStaticLossMaxBlocks + 64;   // partial sums, then the ticket
 
 // Device scratch shared by every abcd_loss_static call on a device (held until exit).
@@ -379,7 +380,11 @@ extern "C" abcd_status abcd_loss_static(void* cuda_stream, const float* out_rgba
       !(lambda_ssim >= 0.f && lambda_ssim <= 1.f))
     return ABCD_ERR_INVALID_ARG;
   const dim3 grid = loss_grid(width, height);
-  if ((long long)grid.x * grid.y * grid.z > kStaticLossMaxBlocks) return ABCD_ERR_WORKSPACE;
+  // the stated limit is on the image (whatever the tile shape), and the scratch must hold a
+  // partial sum per CTA
+  if ((long long)width * height > kStaticLossMaxPixels ||
+      (long long)grid.x * grid.y * grid.z > kStaticLossMaxBlocks)
+    return ABCD_ERR_WORKSPACE;
   unsigned* scratch = nullptr;
   if (static_scratch(&scratch) != cudaSuccess) return ABCD_ERR_CUDA;
   float* partials = reinterpret_cast<float*>(scratch);
