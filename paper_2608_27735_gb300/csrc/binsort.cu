@@ -924,17 +924,26 @@ static_assert(kMaxRunRows % kPlaceThreads == 0 && kPlaceRuns % kPlaceThreads == 
 // words per chunk.  Inside a chunk, column x keeps a bit mask of the runs that cover it and the
 // number of covering runs before each mask word, so the rank of run j in column x is a
 // popcount.  A wait gives up after spin_limit polls (status gets ABCD_ERR_TIMEOUT).
-__global__ void __launch_bounds__(kPlaceThreads)
+// Dynamic shared memory of place_kernel, sized for the grid (so that, with at most 64
+// registers, eight CTAs fit on an SM): the rows' run and chunk starts, then per tile column the
+// run mask, the chunk's count and base, and the popcounts before each mask word.
+inline size_t place_smem_bytes(int rows, int tiles_x) {
+  return sizeof(unsigned) * (2 * (size_t)(rows + 1) + (size_t)tiles_x * (kPlacePitch + 2)) +
+         sizeof(unsigned short) * (size_t)tiles_x * kPlacePitch;
+}
+
+__global__ void __launch_bounds__(kPlaceThreads, 8)
 place_kernel(const u64* runs, const long long* n_runs, long long cap, const unsigned* row_runs,
              int rows, int tiles_x, const unsigned* ranges, const long long* K, unsigned* ids,
              u64* state, unsigned* ctr, unsigned epoch, unsigned* status, unsigned spin_limit) {
   pdl_prologue();
-  __shared__ unsigned s_rs[kMaxRunRows + 1];         // first run of each row
-  __shared__ unsigned s_cs[kMaxRunRows + 1];         // first chunk of each row
-  __shared__ unsigned s_mask[kMaxRunCols * kPlacePitch];          // [column][word]
-  __shared__ unsigned short s_pc[kMaxRunCols * kPlacePitch];      // covering runs before a word
-  __shared__ unsigned s_cnt[kMaxRunCols];            // the chunk's runs per column
-  __shared__ unsigned s_base[kMaxRunCols];           // where the chunk's entries of a column start
+  extern __shared__ __align__(16) unsigned place_sm[];
+  unsigned* s_rs = place_sm;                                  // [rows + 1] first run of a row
+  unsigned* s_cs = s_rs + (rows + 1);                         // [rows + 1] first chunk of a row
+  unsigned* s_mask = s_cs + (rows + 1);                       // [column][word]
+  unsigned* s_cnt = s_mask + tiles_x * kPlacePitch;           // the chunk's runs per column
+  unsigned* s_base = s_cnt + tiles_x;                         // where a column's entries start
+  unsigned short* s_pc = reinterpret_cast<unsigned short*>(s_base + tiles_x);   // before a word
   __shared__ unsigned s_c, s_row;
   if (*K > cap) return;                              // the ranges are empty: nothing to place
   const long long nr = dev_count(0, n_runs, cap);
@@ -1299,8 +1308,13 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       return s;
     const unsigned epoch = ++ctx->os_epoch;
     const int Gp = (int)std::max<long long>(1, std::min<long long>(max_chunks, 8LL * ctx->num_sms));
+    const size_t psm = place_smem_bytes(tiles_y, tiles_x);
+    {
+      const cudaError_t e2 = ensure_smem(ctx, (const void*)place_kernel, psm);
+      if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "place smem: %s", cudaGetErrorString(e2));
+    }
     return check_launch(ctx, "place_kernel",
-                        launch_pdl(place_kernel, dim3(Gp), dim3(kPlaceThreads), 0, ctx->stream,
+                        launch_pdl(place_kernel, dim3(Gp), dim3(kPlaceThreads), psm, ctx->stream,
                                    (const u64*)by_row, (const long long*)ctx->ws.n_runs, cap,
                                    (const unsigned*)ctx->ws.row_runs, tiles_y, tiles_x,
                                    (const unsigned*)out->ranges, (const long long*)out->count,
