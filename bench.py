@@ -534,7 +534,7 @@ def profile_traffic(kernel):
 
 def op_kernel_names():
     return {"render_fwd": "render_fwd_kernel", "render_bwd": "render_bwd_kernel",
-            "loss": "loss_kernel", "composite": "composite_kernel", "adam": "adam_kernel",
+            "loss": "ssim_fwd_kernel", "composite": "composite_kernel", "adam": "adam_kernel",
             "project": "project_fwd_kernel", "project_bwd": "project_bwd_kernel",
             "bin_sort": "binsort"}
 

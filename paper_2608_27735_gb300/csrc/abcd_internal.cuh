@@ -59,6 +59,8 @@ struct Workspace {
   float* grad2d;                    // [max_g][9]
   float* dl_dout;                   // [max_pixels][3]
   float* loss_partials;             // [kMaxLossBlocks][2]
+  float2* ssim_ab;                  // [3][max_pixels] SSIM partials (A, B) per channel and pixel
+  float* ssim_c;                    // [3][max_pixels] SSIM partial C
   unsigned* tile_order;             // [max_tiles] tiles by decreasing list length (bin_sort)
   long long max_tiles;
   // render checkpoints: the forward saves each pixel's (colour, T) where a block's walk crosses

@@ -178,6 +178,8 @@ static size_t layout(char* base, int max_g, long long max_pairs, long long max_p
   w.grad2d = (float*)take(4ull * 9 * (size_t)max_g);
   w.dl_dout = (float*)take(4ull * 3 * (size_t)max_pixels);
   w.loss_partials = (float*)take(4ull * 2 * kMaxLossBlocks);
+  w.ssim_ab = (float2*)take(8ull * 3 * (size_t)max_pixels);
+  w.ssim_c = (float*)take(4ull * 3 * (size_t)max_pixels);
   w.max_tiles = max_order_tiles(max_pixels);
   w.tile_order = (unsigned*)take(4ull * (size_t)w.max_tiles);
   w.ck_cap = (int)std::max<long long>(1024, max_pixels / 128);

@@ -363,7 +363,10 @@ def test_project_backward_matches_oracle(ctx, ragged):
 
 
 def test_loss_matches_oracle(ctx):
-    for (H, W, lam, seed) in [(64, 64, 0.2, 1), (100, 150, 0.2, 2), (37, 53, 0.0, 3), (128, 96, 1.0, 4)]:
+    # sizes below, at and across the 118x16 tiles of the two loss kernels (ragged tails in both
+    # directions, several tiles in each) and of the fused kernel's 64x28 tiles
+    for (H, W, lam, seed) in [(64, 64, 0.2, 1), (100, 150, 0.2, 2), (37, 53, 0.0, 3), (128, 96, 1.0, 4),
+                              (70, 300, 0.2, 5), (9, 13, 0.2, 6), (33, 237, 0.5, 7)]:
         x = sg.random_image(H, W, 4, seed)
         y = np.clip(x[..., :3] + sg.random_image(H, W, 3, seed + 50, -0.2, 0.2), 0, 1).astype(np.float32)
         L, g = oracle.loss(x[..., :3].astype(np.float64), y.astype(np.float64), lam)
