@@ -330,7 +330,7 @@ constexpr int QPM = QC | 1;                  // pitch of the vertical-window row
 constexpr int QPO = QW | 1;                  // pitch of the per-pixel results staged for the copy-out
 static_assert(QC * (QH / QRUN) == kQThreads && QH % QRUN == 0, "one vertical run per thread");
 static_assert(QH * QHSEG <= kQThreads, "one horizontal round");
-static_assert((QR * QC) % kQThreads == 0, "staging rounds");
+static_assert(kQThreads == 2 * QC && QR % 2 == 0 && QH % 2 == 0, "a thread stages one column, every other row");
 static_assert(QW - QRUN + QRUN + 10 <= QC, "horizontal runs stay in the staged columns");
 constexpr int kQFwdFloats = 2 * QR * QC + 5 * QH * QPM;
 constexpr int kQBwdFloats = 3 * QR * QC + 3 * QH * QPM;
@@ -357,30 +357,32 @@ ssim_fwd_kernel(const float* __restrict__ xin, const float* __restrict__ yin, in
   const int ox = blockIdx.x * QW, oy = blockIdx.y * QH, ch = blockIdx.z;
   const float C1 = 0.01f * 0.01f, C2 = 0.03f * 0.03f;
   float l1 = 0.f, ssim = 0.f;
-  // ---- x, y on the tile + 5, zero outside the image (all loads before the first store)
+  // ---- x, y on the tile + 5, zero outside the image (all loads before the first store); a
+  // thread stages one column, every other row
   {
-    constexpr int kLoads = QR * QC / kQThreads;
-    float xv[kLoads], yv[kLoads];
+    constexpr int kRows = QR / 2;
+    const int c = threadIdx.x % QC, rb = threadIdx.x / QC;
+    const int gx = ox - 5 + c;
+    const bool col_in = gx >= 0 && gx < W;
+    const bool col_own = c >= 5 && c < 5 + QW;     // a column of the tile itself
+    float xv[kRows], yv[kRows];
 #pragma unroll
-    for (int j = 0; j < kLoads; ++j) {
-      const int k = threadIdx.x + j * kQThreads;
-      const int r = k / QC, c = k - r * QC;
-      const int gy = oy - 5 + r, gx = ox - 5 + c;
+    for (int j = 0; j < kRows; ++j) {
+      const int gy = oy - 5 + rb + 2 * j;
       xv[j] = 0.f;
       yv[j] = 0.f;
-      if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
+      if (col_in && gy >= 0 && gy < H) {
         const int p = gy * W + gx;   // at most 65536 CTAs: about 41M pixels, 4p fits an int
         xv[j] = __ldg(xin + 4 * p + ch);
         yv[j] = __ldg(yin + 3 * p + ch);
       }
     }
 #pragma unroll
-    for (int j = 0; j < kLoads; ++j) {
-      const int k = threadIdx.x + j * kQThreads;
-      const int r = k / QC, c = k - r * QC;
-      sXY[k] = make_float2(xv[j], yv[j]);
+    for (int j = 0; j < kRows; ++j) {
+      const int r = rb + 2 * j;
+      sXY[r * QC + c] = make_float2(xv[j], yv[j]);
       // |x - y| of the tile's own pixels (zero off the image, where both are zero)
-      if (r >= 5 && r < 5 + QH && c >= 5 && c < 5 + QW) l1 += fabsf(xv[j] - yv[j]);
+      if (col_own && r >= 5 && r < 5 + QH) l1 += fabsf(xv[j] - yv[j]);
     }
   }
   __syncthreads();
@@ -454,13 +456,18 @@ ssim_fwd_kernel(const float* __restrict__ xin, const float* __restrict__ yin, in
   }
   if (abc_ab) {
     __syncthreads();
-    for (int k = threadIdx.x; k < QH * QW; k += kQThreads) {
-      const int r = k / QW, c = k - r * QW;
-      const int gy = oy + r, gx = ox + c;
-      if (gx >= W || gy >= H) continue;
-      const int q = (ch * H + gy) * W + gx;
-      abc_ab[q] = make_float2(oA[r * QPO + c], oB[r * QPO + c]);
-      abc_c[q] = oC[r * QPO + c];
+    // a thread copies one column of the tile, every other row (coalesced along the rows)
+    const int c = threadIdx.x % QC, rb = threadIdx.x / QC;
+    const int gx = ox + c;
+    if (c < QW && gx < W) {
+#pragma unroll
+      for (int j = 0; j < QH / 2; ++j) {
+        const int r = rb + 2 * j, gy = oy + r;
+        if (gy >= H) break;
+        const int q = (ch * H + gy) * W + gx;
+        abc_ab[q] = make_float2(oA[r * QPO + c], oB[r * QPO + c]);
+        abc_c[q] = oC[r * QPO + c];
+      }
     }
   }
   // block partial sums -> the last block finishes the scalar
@@ -518,45 +525,48 @@ ssim_bwd_kernel(const float* __restrict__ xin, const float* __restrict__ yin, in
   float* gC = reinterpret_cast<float*>(gAB + QH * QPM);    // [QH][QPM] windows of C
   const int ox = blockIdx.x * QW, oy = blockIdx.y * QH, ch = blockIdx.z;
   const float inv = 1.f / (3.f * (float)W * (float)H);
-  // x and y of the pixels this thread finishes in the last pass, loaded first so that their
-  // latency hides behind the window passes
-  constexpr int kOut = (QH * QW + kQThreads - 1) / kQThreads;
-  float xq[kOut], yq[kOut];
+  // x and y of the pixels this thread finishes in the last pass (one column of the tile, every
+  // other row), loaded first so that their latency hides behind the window passes
+  const int fc = threadIdx.x % QC, fr = threadIdx.x / QC;
+  const int fx = ox + fc;
+  const bool f_col = fc < QW && fx < W;
+  float xq[QH / 2], yq[QH / 2];
 #pragma unroll
-  for (int j = 0; j < kOut; ++j) {
-    const int k = threadIdx.x + j * kQThreads;
-    const int r = k / QW, c = k - r * QW;
-    const int gy = oy + r, gx = ox + c;
+  for (int j = 0; j < QH / 2; ++j) {
+    const int gy = oy + fr + 2 * j;
     xq[j] = 0.f;
     yq[j] = 0.f;
-    if (k < QH * QW && gx < W && gy < H) {
-      const int q = gy * W + gx;
+    if (f_col && gy < H) {
+      const int q = gy * W + fx;
       xq[j] = __ldg(xin + 4 * q + ch);
       yq[j] = __ldg(yin + 3 * q + ch);
     }
   }
-  // ---- A, B, C on the tile + 5, zero outside the image (no pixel there contributes)
+  // ---- A, B, C on the tile + 5, zero outside the image (no pixel there contributes); a thread
+  // stages one column, every other row
   {
-    constexpr int kLoads = QR * QC / kQThreads;
-    float2 ab[kLoads];
-    float cv[kLoads];
+    constexpr int kRows = QR / 2;
+    const int c = threadIdx.x % QC, rb = threadIdx.x / QC;
+    const int gx = ox - 5 + c;
+    const bool col_in = gx >= 0 && gx < W;
+    float2 ab[kRows];
+    float cv[kRows];
 #pragma unroll
-    for (int j = 0; j < kLoads; ++j) {
-      const int k = threadIdx.x + j * kQThreads;
-      const int r = k / QC, c = k - r * QC;
-      const int gy = oy - 5 + r, gx = ox - 5 + c;
+    for (int j = 0; j < kRows; ++j) {
+      const int gy = oy - 5 + rb + 2 * j;
       ab[j] = make_float2(0.f, 0.f);
       cv[j] = 0.f;
-      if (gx >= 0 && gx < W && gy >= 0 && gy < H) {
+      if (col_in && gy >= 0 && gy < H) {
         const int q = (ch * H + gy) * W + gx;
         ab[j] = __ldcg(abc_ab + q);
         cv[j] = __ldcg(abc_c + q);
       }
     }
 #pragma unroll
-    for (int j = 0; j < kLoads; ++j) {
-      sAB[threadIdx.x + j * kQThreads] = ab[j];
-      sC[threadIdx.x + j * kQThreads] = cv[j];
+    for (int j = 0; j < kRows; ++j) {
+      const int r = rb + 2 * j;
+      sAB[r * QC + c] = ab[j];
+      sC[r * QC + c] = cv[j];
     }
   }
   __syncthreads();
@@ -606,18 +616,17 @@ ssim_bwd_kernel(const float* __restrict__ xin, const float* __restrict__ yin, in
     }
   }
   __syncthreads();
+  if (!f_col) return;
 #pragma unroll
-  for (int j = 0; j < kOut; ++j) {
-    const int k = threadIdx.x + j * kQThreads;
-    const int r = k / QW, c = k - r * QW;
-    const int gy = oy + r, gx = ox + c;
-    if (k >= QH * QW || gx >= W || gy >= H) continue;
-    const int q = gy * W + gx;
+  for (int j = 0; j < QH / 2; ++j) {
+    const int r = fr + 2 * j, gy = oy + r;
+    if (gy >= H) break;
+    const int q = gy * W + fx;
     const float xv = xq[j], yv = yq[j];
     const float d = xv - yv;
     const float sgn = (d > 0.f) ? 1.f : ((d < 0.f) ? -1.f : 0.f);
-    const float2 wab = oAB[r * QPO + c];
-    const float dS = wab.x + 2.f * xv * wab.y + yv * oC[r * QPO + c];
+    const float2 wab = oAB[r * QPO + fc];
+    const float dS = wab.x + 2.f * xv * wab.y + yv * oC[r * QPO + fc];
     grad[3 * q + ch] = ((1.f - lam) * sgn - lam * dS) * inv;
   }
 }
