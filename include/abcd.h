@@ -180,8 +180,11 @@ abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camera* cam,
 /* K6. The reconstruction loss each step of Section 2 evaluates, in the L1 + D-SSIM form of
  * 3D Gaussian Splatting: (1 - lambda) mean|x - y| + lambda (1 - mean SSIM(x, y)) over the
  * rgb of out_rgba [H][W][4] against gt_rgb [H][W][3]; SSIM with an 11x11 Gaussian window
- * (sigma 1.5), zero padding, C1 = 0.01^2, C2 = 0.03^2.  loss_out: device float scalar.
- * dL_dout: [H][W][3] receives dL/d(out.rgb). */
+ * (sigma 1.5), zero padding, C1 = 0.01^2, C2 = 0.03^2.  loss_out: device float scalar (may
+ * be NULL).  dL_dout: [H][W][3] receives dL/d(out.rgb) (may be NULL: the loss alone).  The
+ * SSIM's per-pixel partials pass between its two kernels through the workspace, so the image
+ * may have at most the workspace's max_pixels pixels (ABCD_ERR_WORKSPACE otherwise, before any
+ * launch); ABCD_ERR_INVALID_ARG for null inputs, non-positive sizes or lambda outside [0, 1]. */
 abcd_status abcd_loss(abcd_ctx* ctx, const float* out_rgba, const float* gt_rgb, int width,
                       int height, float lambda_ssim, float* loss_out, float* dL_dout);
 
