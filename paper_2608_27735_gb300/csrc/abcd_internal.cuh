@@ -170,6 +170,9 @@ abcd_status check_launch(abcd_ctx* ctx, const char* what);
 abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched);
 // Raises kernel fn's dynamic shared-memory limit to at least `bytes` (once per context and size).
 cudaError_t ensure_smem(abcd_ctx* ctx, const void* fn, size_t bytes);
+// Zeroes bytes at p on the context's stream with a programmatically serialised kernel (a memset
+// when p or bytes is not a multiple of 4).
+abcd_status zero_async(abcd_ctx* ctx, void* p, size_t bytes, const char* what);
 bool has_workspace(const abcd_ctx* ctx);
 Cam make_cam(const abcd_camera* c, const abcd_render_opts* o);
 Opts make_opts(const abcd_render_opts* o);

@@ -74,12 +74,16 @@ __device__ __forceinline__ int4 tile_rect(float2 m, int r, int tiles_x, int tile
 __global__ void keys_rects_kernel(const float* depth, const int* radius, const float2* uv, int n,
                                   int tiles_x, int tiles_y, u64* items, int4* rects,
                                   unsigned* gh_zero, int gh_words, unsigned* rows_zero,
-                                  int rows_words) {
+                                  int rows_words, int* diff_zero, int diff_cells) {
   pdl_prologue();
   if (blockIdx.x == 0) {                  // the radix sorts' digit counts start from zero
     for (int k = threadIdx.x; k < gh_words; k += blockDim.x) gh_zero[k] = 0u;
     for (int k = threadIdx.x; k < rows_words; k += blockDim.x) rows_zero[k] = 0u;
   }
+  // and so does the tile rows' difference array (here rather than by a memset, which would
+  // end the programmatic overlap of the launches before and after it)
+  for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < diff_cells; k += gridDim.x * blockDim.x)
+    diff_zero[k] = 0;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   int4 q = make_int4(0, 0, 0, 0);
@@ -1198,8 +1202,6 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   const size_t diff_bytes = sizeof(int) * (size_t)(tiles_x + 1) * (tiles_y + 1);
   if (diff_bytes > ctx->ws.diff_bytes)
     return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_bin_sort: tile grid exceeds the workspace");
-  e = cudaMemsetAsync(ctx->ws.diff, 0, diff_bytes, ctx->stream);
-  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "diff memset: %s", cudaGetErrorString(e));
   abcd_status s;
   const float alpha_min = make_opts(opts).alpha_min;
   int tile_bits = 1;
@@ -1218,11 +1220,13 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   const SortPasses tile_passes = make_passes(0, by_runs ? row_bits : tile_bits);
   unsigned* tile_gh = ctx->ws.os_gh + 4 * kRadixBins;
   if ((s = check_launch(ctx, "keys_rects_kernel",
-                        launch_pdl(keys_rects_kernel, dim3((n + 255) / 256), dim3(256), 0, ctx->stream,
+                        launch_pdl(keys_rects_kernel,
+                                   dim3((unsigned)std::max<size_t>((n + 255) / 256, (cells + 4095) / 4096)),
+                                   dim3(256), 0, ctx->stream,
                                    (const float*)proj->depth, (const int*)proj->radius,
                                    (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
                                    ctx->ws.rects, ctx->ws.os_gh, 2 * 4 * kRadixBins,
-                                   ctx->ws.row_runs, by_runs ? tiles_y : 0))))
+                                   ctx->ws.row_runs, by_runs ? tiles_y : 0, ctx->ws.diff, cells))))
     return s;
   // the depth sort only needs the keys: it runs on the side stream while the tile rows and
   // ranges are made here

@@ -38,6 +38,33 @@ abcd_status check_launch(abcd_ctx* ctx, const char* what, cudaError_t launched) 
 
 bool has_workspace(const abcd_ctx* ctx) { return ctx && ctx->ws_base != nullptr; }
 
+// Zeroes `words` 4-byte words at p (4-byte aligned): 16-byte stores over the aligned body, 4-byte
+// ones around it.  A kernel rather than a memset: launched with programmatic serialisation, it
+// keeps the launches of a call overlapping the tails of the kernels before them.
+__global__ void __launch_bounds__(256) zero_kernel(unsigned* p, long long words) {
+  pdl_prologue();
+  const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  const long long head = min((long long)(((16u - ((uintptr_t)p & 15u)) & 15u) / 4u), words);
+  const long long body = (words - head) / 4;
+  for (long long i = tid; i < head; i += stride) p[i] = 0u;
+  uint4* q = reinterpret_cast<uint4*>(p + head);
+  for (long long i = tid; i < body; i += stride) q[i] = make_uint4(0u, 0u, 0u, 0u);
+  for (long long i = head + 4 * body + tid; i < words; i += stride) p[i] = 0u;
+}
+
+abcd_status zero_async(abcd_ctx* ctx, void* p, size_t bytes, const char* what) {
+  if (bytes == 0) return ABCD_OK;
+  if (((uintptr_t)p & 3) || (bytes & 3)) {
+    const cudaError_t e = cudaMemsetAsync(p, 0, bytes, ctx->stream);
+    return e == cudaSuccess ? ABCD_OK : fail(ctx, ABCD_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+  }
+  const long long words = (long long)(bytes / 4);
+  const long long blocks = std::min<long long>((words / 4 + 255) / 256 + 1, 4LL * ctx->num_sms);
+  return check_launch(ctx, what, launch_pdl(zero_kernel, dim3((unsigned)blocks), dim3(256), 0,
+                                            ctx->stream, (unsigned*)p, words));
+}
+
 cudaError_t ensure_smem(abcd_ctx* ctx, const void* fn, size_t bytes) {
   if (bytes <= 48 * 1024) return cudaSuccess;
   int slot = -1;

@@ -720,8 +720,8 @@ extern "C" abcd_status abcd_render_composite_fwd(abcd_ctx* ctx, const abcd_camer
   a.ckpt = nullptr; a.ck_items = nullptr; a.ck_count = nullptr; a.ck_first = nullptr;
   a.ck_cap = 0;
   if (state && ckpt_ok(ctx, n_blocks)) {
-    const cudaError_t e = cudaMemsetAsync(ctx->ws.ck_count, 0, sizeof(unsigned), ctx->stream);
-    if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "checkpoint count memset: %s", cudaGetErrorString(e));
+    const abcd_status z = zero_async(ctx, ctx->ws.ck_count, sizeof(unsigned), "checkpoint count clear");
+    if (z != ABCD_OK) return z;
     a.ckpt = ctx->ws.ckpt; a.ck_items = ctx->ws.ck_items; a.ck_count = ctx->ws.ck_count;
     a.ck_first = ctx->ws.ck_first; a.ck_cap = ctx->ws.ck_cap;
     ctx->ck_state = state->A_T;
@@ -748,8 +748,10 @@ extern "C" abcd_status abcd_render_backward(abcd_ctx* ctx, const abcd_camera* ca
   if (!state || !state->A_T || !state->n_last || !dL_dout || n < 0 || (n > 0 && !grad2d))
     return fail(ctx, ABCD_ERR_INVALID_ARG, "abcd_render_backward: null state, gradient or output");
   if (n == 0) return ABCD_OK;
-  cudaError_t e = cudaMemsetAsync(grad2d, 0, sizeof(float) * 9 * (size_t)n, ctx->stream);
-  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "grad2d memset: %s", cudaGetErrorString(e));
+  {
+    const abcd_status z = zero_async(ctx, grad2d, sizeof(float) * 9 * (size_t)n, "grad2d clear");
+    if (z != ABCD_OK) return z;
+  }
   BwdArgs a;
   a.status = ctx->ws.status;
   a.cam = make_cam(cam, opts);
