@@ -153,6 +153,7 @@ struct abcd_ctx {
   abcd::SHConst sh{};
   long long launches = 0;
   unsigned os_epoch = 0;                // last look-back epoch handed to a sort pass
+  unsigned krange_parity = 0;           // which pair of depth-key range words bin_sort uses next
   unsigned wait_limit = 1u << 20;       // polls before a device-side wait gives up
   long long withhold_tile = -1;         // test hook: a look-back tile that publishes nothing
   // dynamic shared memory limits already raised on this context's device, per kernel (the

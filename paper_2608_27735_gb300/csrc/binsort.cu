@@ -74,26 +74,48 @@ __device__ __forceinline__ int4 tile_rect(float2 m, int r, int tiles_x, int tile
 __global__ void keys_rects_kernel(const float* depth, const int* radius, const float2* uv, int n,
                                   int tiles_x, int tiles_y, u64* items, int4* rects,
                                   unsigned* gh_zero, int gh_words, unsigned* rows_zero,
-                                  int rows_words, int* diff_zero, int diff_cells) {
+                                  int rows_words, int* diff_zero, int diff_cells, unsigned* krange,
+                                  unsigned* krange_next) {
   pdl_prologue();
   if (blockIdx.x == 0) {                  // the radix sorts' digit counts start from zero
     for (int k = threadIdx.x; k < gh_words; k += blockDim.x) gh_zero[k] = 0u;
     for (int k = threadIdx.x; k < rows_words; k += blockDim.x) rows_zero[k] = 0u;
+    // the key range words of the next call (two pairs used in turn, so no memset is needed)
+    if (threadIdx.x < 2) krange_next[threadIdx.x] = 0u;
   }
   // and so does the tile rows' difference array (here rather than by a memset, which would
   // end the programmatic overlap of the launches before and after it)
   for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < diff_cells; k += gridDim.x * blockDim.x)
     diff_zero[k] = 0;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
   int4 q = make_int4(0, 0, 0, 0);
-  const int r = radius[i];
-  if (r > 0) q = tile_rect(uv[i], r, tiles_x, tiles_y);
-  const bool vis = r > 0 && q.x < q.z && q.y < q.w;
-  if (!vis) q = make_int4(0, 0, 0, 0);
-  rects[i] = q;
-  const unsigned key = vis ? __float_as_uint(depth[i]) : 0xFFFFFFFFu;
-  items[i] = ((u64)key << 32) | (unsigned)i;
+  bool vis = false;
+  unsigned key = 0xFFFFFFFFu;
+  if (i < n) {
+    const int r = radius[i];
+    if (r > 0) q = tile_rect(uv[i], r, tiles_x, tiles_y);
+    vis = r > 0 && q.x < q.z && q.y < q.w;
+    if (!vis) q = make_int4(0, 0, 0, 0);
+    rects[i] = q;
+    if (vis) key = __float_as_uint(depth[i]);
+    items[i] = ((u64)key << 32) | (unsigned)i;
+  }
+  // the range of the visible keys, for the depth sort's digits: the warps' extremes, then one
+  // pair of atomics per block
+  __shared__ unsigned s_kr[2][32];
+  const unsigned kmax = __reduce_max_sync(0xffffffffu, vis ? key : 0u);
+  const unsigned kcmin = __reduce_max_sync(0xffffffffu, vis ? ~key : 0u);
+  if ((threadIdx.x & 31) == 0) { s_kr[0][threadIdx.x >> 5] = kcmin; s_kr[1][threadIdx.x >> 5] = kmax; }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int nw = blockDim.x >> 5;
+    const unsigned a = __reduce_max_sync(0xffffffffu, (int)threadIdx.x < nw ? s_kr[0][threadIdx.x] : 0u);
+    const unsigned b = __reduce_max_sync(0xffffffffu, (int)threadIdx.x < nw ? s_kr[1][threadIdx.x] : 0u);
+    if (threadIdx.x == 0 && b != 0u) {
+      atomicMax(krange, a);
+      atomicMax(krange + 1, b);
+    }
+  }
 }
 
 // The tiles of row ty kept for a Gaussian are those whose pixel-centre box meets the ellipse
@@ -246,6 +268,39 @@ __device__ __forceinline__ unsigned digit_of(T x, long long i, long long wh, int
   return i < wh ? ((unsigned)(x >> shift) & mask) : 0x100u;
 }
 
+// The depth sort ranks keys relative to the smallest visible one (the positive depths' float
+// bits keep their order under the subtraction), with the culled items' all-ones keys mapped
+// just above the largest: when the visible keys span fewer than 2^24 - 1 values, every item's
+// top byte is then zero and the last 8-bit pass has a single digit, so it runs as a copy.  The
+// order is the one of the keys themselves.  krange: [0] the largest complement of a visible
+// key, [1] the largest visible key (both zero when none is visible).  Its first pass writes the
+// items with their keys mapped; only the id bits are read after the sort.
+struct KeyMap {
+  unsigned lo, sat;
+  bool on;
+};
+
+__device__ __forceinline__ KeyMap key_map(const unsigned* kr) {
+  KeyMap m{0u, 0xFFFFFFFFu, kr != nullptr};
+  if (kr) {
+    const unsigned lo = ~kr[0], hi = kr[1];
+    m.lo = lo;
+    m.sat = (hi >= lo && hi - lo < 0xFFFFFFu) ? 0xFFFFFFu : 0xFFFFFFFFu;
+  }
+  return m;
+}
+
+template <typename T>
+__device__ __forceinline__ T map_item(T x, const KeyMap& m) {
+  if constexpr (sizeof(T) == 8) {
+    const unsigned k = (unsigned)(x >> 32);
+    const unsigned kk = k == 0xFFFFFFFFu ? m.sat : k - m.lo;
+    return ((T)kk << 32) | (x & 0xFFFFFFFFull);
+  } else {
+    return x;
+  }
+}
+
 // Lanes holding the same BITS-bit digit as this lane, among the lanes of valid_mask: one
 // ballot per bit (a cost independent of how many distinct digits the warp holds).
 template <int BITS>
@@ -360,7 +415,7 @@ __device__ __forceinline__ u64 os_peek(const u64* p) {
 template <typename T>
 __global__ void __launch_bounds__(256)
 sort_digits_kernel(const T* in, long long n_static, const long long* n_dev, long long cap,
-                   SortPasses sp, int match_from, unsigned* gh) {
+                   SortPasses sp, int match_from, unsigned* gh, const unsigned* krange) {
   pdl_prologue();
   __shared__ unsigned h[4][kRadixBins];
   for (int k = threadIdx.x; k < 4 * kRadixBins; k += blockDim.x) (&h[0][0])[k] = 0;
@@ -369,11 +424,12 @@ sort_digits_kernel(const T* in, long long n_static, const long long* n_dev, long
   const int lane = threadIdx.x & 31;
   const unsigned lt = (1u << lane) - 1u;
   const long long stride = (long long)gridDim.x * blockDim.x;
+  const KeyMap km = key_map(krange);
   // the loop runs while any lane of the warp has an item (the ranking is warp-collective)
   for (long long b = (long long)blockIdx.x * blockDim.x + (threadIdx.x & ~31); b < n; b += stride) {
     const long long i = b + lane;
     const bool valid = i < n;
-    const T x = valid ? in[i] : (T)0;
+    const T x = valid ? (km.on ? map_item(in[i], km) : in[i]) : (T)0;
     for (int p = 0; p < sp.n; ++p) {
       const unsigned d = valid ? (unsigned)(x >> sp.shift[p]) & ((1u << sp.bits[p]) - 1u) : 0x100u;
       const unsigned peers = p >= match_from ? __match_any_sync(0xffffffffu, d) : match_byte(d);
@@ -398,7 +454,7 @@ __global__ void __launch_bounds__(kOsThreads, 2)
 onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long long n_static,
                 const long long* n_dev, long long cap, int shift, const unsigned* gh, u64* state,
                 unsigned* ctr, unsigned epoch, unsigned* status, unsigned spin_limit,
-                long long withhold) {
+                long long withhold, const unsigned* krange) {
   pdl_prologue();
   constexpr unsigned BINS = 1u << BITS, MASK = BINS - 1;
   constexpr int U = 64 / (int)sizeof(T);          // items per lane: 64 bytes in flight
@@ -410,16 +466,43 @@ onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long l
   __shared__ unsigned s_loc[BINS];                // start of each digit inside the tile
   __shared__ T s_items[TILE];                     // the tile's items in digit order
   __shared__ unsigned s_tile;
+  __shared__ int s_copy;
+  const long long n = dev_count(n_static, n_dev, cap);
+  if (threadIdx.x == 0) s_copy = 0;
+  __syncthreads();
   {
     const unsigned v = threadIdx.x < BINS ? gh[threadIdx.x] : 0u;
+    // every item holds the same digit: the stable scatter is the identity, a copy
+    if (n > 0 && (long long)v == n) s_copy = 1;
     const unsigned long long ex = block_exclusive_scan(v, nullptr);
     if (threadIdx.x < BINS) s_base[threadIdx.x] = (unsigned)ex;
   }
-  const long long n = dev_count(n_static, n_dev, cap);
   const long long n_tiles = (n + TILE - 1) / TILE;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const unsigned lt = (1u << lane) - 1u;
-  for (;;) {
+  const KeyMap km = key_map(krange);
+  while (s_copy) {                                   // block-uniform (set before the scan's barriers)
+    if (threadIdx.x == 0) s_tile = atomicAdd(ctr, 1u);
+    __syncthreads();
+    const long long t = s_tile;
+    __syncthreads();                                 // s_tile is read before the next claim
+    if (t >= n_tiles) break;
+    T xs[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {                    // all loads in flight together
+      const long long i = t * TILE + j * kOsThreads + threadIdx.x;
+      xs[j] = i < n ? in[i] : (T)0;
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const long long i = t * TILE + j * kOsThreads + threadIdx.x;
+      if (i >= n) continue;
+      const T x = km.on ? map_item(xs[j], km) : xs[j];
+      if (out_ids) out_ids[i] = (unsigned)x & id_mask;
+      else out[i] = x;
+    }
+  }
+  for (; !s_copy;) {
     if (threadIdx.x == 0) s_tile = atomicAdd(ctr, 1u);
     for (int k = threadIdx.x; k < kOsWarps * (int)BINS; k += kOsThreads) (&cnt[0][0])[k] = 0;
     __syncthreads();
@@ -429,6 +512,10 @@ onesweep_kernel(const T* in, T* out, unsigned* out_ids, unsigned id_mask, long l
     T xs[U];
     unsigned rk[U];
     load_items(in, b0, n, lane, xs);
+    if (km.on) {
+#pragma unroll
+      for (int j = 0; j < U; ++j) xs[j] = map_item(xs[j], km);
+    }
 #pragma unroll
     for (int j = 0; j < U; ++j) {
       const unsigned d = digit_of(xs[j], b0 + 32 * j + lane, n, shift, MASK);
@@ -1096,17 +1183,18 @@ template <typename T>
 abcd_status launch_onesweep(abcd_ctx* ctx, cudaStream_t st, int bits, bool match, int G,
                             const T* src, T* dst, unsigned* ids, unsigned id_mask,
                             long long n_static, const long long* n_dev, long long cap, int shift,
-                            const unsigned* gh, unsigned* ctr, long long withhold) {
+                            const unsigned* gh, unsigned* ctr, long long withhold,
+                            const unsigned* krange) {
   const unsigned epoch = ++ctx->os_epoch;
   const unsigned spin = ctx->wait_limit;
 #define ABCD_PASS(B)                                                                              \
   case B:                                                                                         \
     e = match ? launch_pdl(onesweep_kernel<T, B, true>, dim3(G), dim3(kOsThreads), 0, st, src, dst, \
                            ids, id_mask, n_static, n_dev, cap, shift, gh, ctx->ws.os_state, ctr,   \
-                           epoch, ctx->ws.status, spin, withhold)                                  \
+                           epoch, ctx->ws.status, spin, withhold, krange)                          \
               : launch_pdl(onesweep_kernel<T, B, false>, dim3(G), dim3(kOsThreads), 0, st, src,    \
                            dst, ids, id_mask, n_static, n_dev, cap, shift, gh, ctx->ws.os_state,   \
-                           ctr, epoch, ctx->ws.status, spin, withhold);                            \
+                           ctr, epoch, ctx->ws.status, spin, withhold, krange);                    \
     break;
   cudaError_t e = cudaSuccess;
   switch (bits) {
@@ -1131,7 +1219,7 @@ template <typename T>
 abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_static,
                        const long long* n_dev, long long cap, long long n_max, int bit_lo,
                        int bit_hi, int slot, bool counted, T** result, unsigned* ids_out,
-                       unsigned id_mask, int match_from) {
+                       unsigned id_mask, int match_from, const unsigned* krange = nullptr) {
   const SortPasses sp = make_passes(bit_lo, bit_hi);
   if (sp.n < 1 || sp.n > 4) return fail(ctx, ABCD_ERR_INVALID_ARG, "radix sort of %d bits", bit_hi - bit_lo);
   unsigned* gh = ctx->ws.os_gh + (size_t)slot * 4 * kRadixBins;
@@ -1145,7 +1233,7 @@ abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_s
   if (!counted &&                              // the tile sort's counts come with the ranges
       (s = check_launch(ctx, "sort_digits_kernel",
                         launch_pdl(sort_digits_kernel<T>, dim3(Gd), dim3(256), 0, st, (const T*)a,
-                                   n_static, n_dev, cap, sp, match_from, gh))))
+                                   n_static, n_dev, cap, sp, match_from, gh, krange))))
     return s;
   T* src = a;
   T* dst = b;
@@ -1155,7 +1243,8 @@ abcd_status radix_sort(abcd_ctx* ctx, cudaStream_t st, T* a, T* b, long long n_s
     const long long withhold = (slot == 0 && p == 0) ? ctx->withhold_tile : -1;
     if ((s = launch_onesweep<T>(ctx, st, sp.bits[p], p >= match_from, G, src, dst,
                                 last ? ids_out : nullptr, id_mask, n_static, n_dev, cap,
-                                sp.shift[p], gh + p * kRadixBins, ctr, withhold)))
+                                sp.shift[p], gh + p * kRadixBins, ctr, withhold,
+                                p == 0 ? krange : nullptr)))
       return s;
     if (slot == 0 && p == 0) ctx->withhold_tile = -1;
     T* t = src; src = dst; dst = t;
@@ -1203,6 +1292,10 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (diff_bytes > ctx->ws.diff_bytes)
     return fail(ctx, ABCD_ERR_WORKSPACE, "abcd_bin_sort: tile grid exceeds the workspace");
   abcd_status s;
+  // the visible depth keys' range: two pairs of words used in turn, each call's keys_rects
+  // clearing the other pair for the next call (zero initially: the workspace set-up clears them)
+  unsigned* krange = ctx->ws.os_ctr + 8 + 2 * (int)(ctx->krange_parity & 1u);
+  unsigned* krange_next = ctx->ws.os_ctr + 8 + 2 * (int)((ctx->krange_parity + 1u) & 1u);
   const float alpha_min = make_opts(opts).alpha_min;
   int tile_bits = 1;
   while ((1LL << tile_bits) < n_tiles) ++tile_bits;
@@ -1226,8 +1319,10 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    (const float*)proj->depth, (const int*)proj->radius,
                                    (const float2*)proj->uv, n, tiles_x, tiles_y, ctx->ws.dsort[0],
                                    ctx->ws.rects, ctx->ws.os_gh, 2 * 4 * kRadixBins,
-                                   ctx->ws.row_runs, by_runs ? tiles_y : 0, ctx->ws.diff, cells))))
+                                   ctx->ws.row_runs, by_runs ? tiles_y : 0, ctx->ws.diff, cells,
+                                   krange, krange_next))))
     return s;
+  ++ctx->krange_parity;                              // the next call's pair is being cleared
   // the depth sort only needs the keys: it runs on the side stream while the tile rows and
   // ranges are made here
   e = cudaEventRecord(ctx->ev_fork, ctx->stream);
@@ -1235,7 +1330,8 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort fork: %s", cudaGetErrorString(e));
   u64* by_depth = nullptr;
   if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, n,
-                           32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom)))
+                           32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom,
+                           krange)))
     return s;
   e = cudaEventRecord(ctx->ev_join, ctx->side);
   if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
