@@ -182,6 +182,36 @@ def test_bin_sort_many_gaussians(ctx):
     par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
 
 
+def test_bin_sort_depth_key_range(ctx):
+    """The depth sort ranks keys relative to the smallest visible one, and a pass whose digit
+    counts put every item in one bin runs as a copy (on ring cameras the last pass does).  The
+    lists equal the oracle's where the visible keys span more than 2^24 values (a camera inside
+    the block, depths from the near plane on: all four passes rank, the culled keys kept above
+    the visible ones) and where nothing is visible (a camera looking away: no pair listed)."""
+    s = sg.grid_scene((1, 1, 1), 5.0, 3000, 0, seed=97)
+    c = np.asarray(s.grid.origin, dtype=np.float64) + 2.5
+    s.cameras = [sg.look_at(c, c + np.array([1.0, 0.2, 0.1]), 96, 64),
+                 sg.look_at(c - np.array([10.0, 0.0, 0.0]), c - np.array([20.0, 0.0, 0.0]), 96, 64)]
+    ctx.reserve(3000, 2_000_000, 96 * 64)
+    for ci in range(2):
+        case = Case(s, ci, fb=False)
+        vis = np.asarray(case.P["radius"]) > 0
+        if ci == 0:
+            bits = np.asarray(case.P["depth"], dtype=np.float32)[vis].view(np.uint32).astype(np.int64)
+            assert bits.max() - bits.min() >= (1 << 24) and not vis.all()
+        else:
+            assert not vis.any() and len(case.ids) == 0
+        r = run_forward(ctx, case, want_state=False)
+        K = int(r["tiles"].count.item())
+        rng = r["tiles"].ranges.cpu().numpy().astype(np.int64)
+        ids = r["tiles"].ids.cpu().numpy()[:K]
+        tx, ty = oracle.tiles_xy(case.cam.width, case.cam.height)
+        par.check_tile_lists(rng, ids, case.off, case.ids, case.P, case.opt_list, tx * ty)
+        if ci == 1:
+            assert K == 0 and not rng.any()
+            assert torch.count_nonzero(r["out"]).item() == 0
+
+
 @pytest.mark.parametrize("W,H", [(4096, 640), (4200, 96), (64, 4200)])
 def test_bin_sort_wide_image(ctx, W, H):
     """Large tile grids with 3,000 Gaussians; the lists equal the oracle's.  4096x640: 256 tile
