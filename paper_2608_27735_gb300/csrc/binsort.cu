@@ -1323,18 +1323,12 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
                                    krange, krange_next))))
     return s;
   ++ctx->krange_parity;                              // the next call's pair is being cleared
-  // the depth sort only needs the keys: it runs on the side stream while the tile rows and
-  // ranges are made here
+  // the tile rows and ranges only need the rectangles: they run on the side stream while the
+  // depth sort, the longer branch, runs here (its launches chained to keys_rects_kernel's
+  // without the fork's event wait)
   e = cudaEventRecord(ctx->ev_fork, ctx->stream);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->side, ctx->ev_fork, 0);
-  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort fork: %s", cudaGetErrorString(e));
-  u64* by_depth = nullptr;
-  if ((s = radix_sort<u64>(ctx, ctx->side, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, n,
-                           32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom,
-                           krange)))
-    return s;
-  e = cudaEventRecord(ctx->ev_join, ctx->side);
-  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile rows fork: %s", cudaGetErrorString(e));
   {
     const size_t smem = cells <= kSmemDiffCells
                             ? sizeof(int) * cells + (by_runs ? sizeof(unsigned) * tiles_y : 0)
@@ -1346,7 +1340,7 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
     }
     if ((s = check_launch(ctx, "tile_rows_kernel",
                           launch_pdl(kern, dim3((n + 255) / 256), dim3(256), smem,
-                                     ctx->stream, (const float2*)proj->uv,
+                                     ctx->side, (const float2*)proj->uv,
                                      (const float4*)proj->conic_opacity, (const int4*)ctx->ws.rects,
                                      n, tiles_x, tiles_y, alpha_min, ctx->ws.counts, ctx->ws.diff,
                                      ctx->ws.row_runs))))
@@ -1361,7 +1355,7 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
         if (e2 != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "ranges smem: %s", cudaGetErrorString(e2));
       }
       if ((s = check_launch(ctx, "ranges_order_kernel",
-                            launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->stream,
+                            launch_pdl(ranges_order_kernel, dim3(1), dim3(1024), smem, ctx->side,
                                        (const int*)ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges,
                                        ctx->ws.tile_order, tile_passes, tile_gh,
                                        by_runs ? (const unsigned*)ctx->ws.row_runs : nullptr,
@@ -1371,14 +1365,21 @@ extern "C" abcd_status abcd_bin_sort(abcd_ctx* ctx, const abcd_projected* proj, 
       ctx->order_tiles = n_tiles;
     } else {
       if ((s = check_launch(ctx, "ranges_from_diff_kernel",
-                            launch_pdl(ranges_from_diff_kernel, dim3(1), dim3(1024), 0, ctx->stream,
+                            launch_pdl(ranges_from_diff_kernel, dim3(1), dim3(1024), 0, ctx->side,
                                        ctx->ws.diff, tiles_x, tiles_y, cap, out->ranges,
                                        tile_passes, tile_gh))))
         return s;
     }
   }
+  e = cudaEventRecord(ctx->ev_join, ctx->side);
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile rows join: %s", cudaGetErrorString(e));
+  u64* by_depth = nullptr;
+  if ((s = radix_sort<u64>(ctx, ctx->stream, ctx->ws.dsort[0], ctx->ws.dsort[1], n, nullptr, n, n,
+                           32, 64, 0, false, &by_depth, nullptr, 0xffffffffu, kDepthMatchFrom,
+                           krange)))
+    return s;
   e = cudaStreamWaitEvent(ctx->stream, ctx->ev_join, 0);
-  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "depth sort join: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) return fail(ctx, ABCD_ERR_CUDA, "tile rows join: %s", cudaGetErrorString(e));
   const int Ge = std::min(kMaxRadixBlocks, 6 * ctx->num_sms);   // blocks of count / emit
   if ((s = check_launch(ctx, "count_kernel",
                         launch_pdl(count_kernel, dim3(Ge), dim3(256), 0, ctx->stream,
